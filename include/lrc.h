@@ -1,0 +1,198 @@
+/*
+ * lrc.h -- C ABI of the GB300 (sm_103a) rank-compensation hot path.
+ *
+ * The library implements the resident downstream kernels of "Low-Precision
+ * Rank Compensation for Matrices and Tensor Trains": factor rounding, the
+ * batched low-rank apply, dense Tensor-Train reconstruction, and the
+ * Frobenius-difference reduction that measures the storage perturbation eta
+ * used by the certificates of Thm 4.1 and Thm 6.1.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - All arrays are C order (row-major).  "Device" pointers are CUDA global
+ *    memory addresses of the current device; "host" pointers are ordinary
+ *    process memory.  The caller owns every buffer; the library keeps no
+ *    pointer after a call returns.
+ *  - `stream` is a cudaStream_t passed as an opaque pointer (NULL = the
+ *    legacy default stream).  Calls are asynchronous on it unless stated.
+ *  - Every argument is validated before anything is launched; on a
+ *    validation error nothing is written and the call returns a negative
+ *    lrc_status.  A failed launch returns LRC_ERR_CUDA.  Faults of a kernel
+ *    that already ran surface at the next synchronising call, as in CUDA.
+ *    lrc_last_error() gives a message for the last failure of the calling
+ *    thread.
+ *  - Sizes are int64_t; products of sizes must not overflow int64.
+ *  - The library never traps, never allocates on the apply / TT / rounding
+ *    paths, and has no CPU fallback: it needs an sm_103a GPU.
+ */
+#ifndef LRC_H
+#define LRC_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define LRC_API __attribute__((visibility("default")))
+#else
+#define LRC_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Storage / arithmetic formats (Sec. 3.2, Table "precision comparison";
+ * Sec. 3.4: FP16 products accumulate in FP32, TF32 is never used). */
+typedef enum {
+    LRC_F64 = 0,      /* binary64 storage, binary64 arithmetic, binary64 output             */
+    LRC_F32 = 1,      /* binary32 storage, binary32 FMA arithmetic, binary32 output         */
+    LRC_F16 = 2,      /* binary16 storage, binary32 accumulation, binary32 output           */
+    LRC_F16_O16 = 3   /* binary16 storage, binary32 accumulation, binary16 workspaces and
+                         output: the method-precision FP16 path of Sec. 3.4                 */
+} lrc_fmt;
+
+typedef enum {
+    LRC_OK = 0,
+    LRC_ERR_INVALID_ARG = -1,   /* null pointer, size <= 0, overflow, bad rank vector ... */
+    LRC_ERR_ALIGNMENT = -2,     /* a pointer is not 16-byte aligned                       */
+    LRC_ERR_UNSUPPORTED = -3,   /* valid request outside what this build implements       */
+    LRC_ERR_CUDA = -4,          /* a CUDA call or launch failed                           */
+    LRC_ERR_NOMEM = -5,         /* library scratch could not be allocated                 */
+    LRC_ERR_TIMEOUT = -6        /* a bounded device-side wait gave up                     */
+} lrc_status;
+
+typedef void* lrc_stream_t;     /* cudaStream_t */
+
+/* Row pitch (in elements) of a packed factor with `cols` logical columns:
+ * cols rounded up to a multiple of 16, so that every row starts on a
+ * 16-byte boundary in every format.  Returns -1 for cols < 0. */
+LRC_API int64_t lrc_packed_ld(int64_t cols);
+
+/*
+ * lrc_round_factors -- store a factor in a lower precision (Sec. 3.2-3.3;
+ * the remark after Thm 4.1: U, Sigma and V^T are rounded individually, and
+ * Alg. 1 step 4 rounds TT cores).
+ *
+ *   src     device, binary64, rows x cols with row pitch ld_src (>= cols)
+ *   dst     device, rows x ld_dst elements of the format `fmt`
+ *           (LRC_F64: binary64 copy; LRC_F32: binary32; LRC_F16 and
+ *           LRC_F16_O16: binary16)
+ *   ld_dst  row pitch of dst in elements, >= cols
+ *
+ * Each element is converted directly from binary64 with IEEE 754
+ * round-to-nearest, ties to even (no intermediate format), subnormals kept,
+ * overflow to +-infinity, NaN to a quiet NaN of the same sign.  Columns
+ * [cols, ld_dst) of every dst row are written with +0.  src and dst must be
+ * 16-byte aligned; rows*ld of either may be zero only if rows or cols is 0
+ * (then nothing happens).
+ */
+LRC_API lrc_status lrc_round_factors(const double* src, int64_t rows, int64_t cols, int64_t ld_src,
+                             void* dst, int64_t ld_dst, lrc_fmt fmt, lrc_stream_t stream);
+
+/*
+ * lrc_widen_factors -- exact binary64 value of a stored factor, so that the
+ * rounded factors can be contracted in FP64 as the paper does for eta
+ * (remark after Thm 4.1; Sec. 6.1: rounded cores reconstructed in FP64).
+ *
+ *   src     device, rows x cols, row pitch ld_src, format `fmt`
+ *   dst     device, binary64, rows x ld_dst; columns [cols, ld_dst) get +0
+ */
+LRC_API lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows, int64_t cols,
+                             int64_t ld_src, double* dst, int64_t ld_dst, lrc_stream_t stream);
+
+/*
+ * lrc_apply -- batched low-rank apply (Sec. 4.4, Eq. gpu_matrix_apply):
+ *
+ *     Y = [(X V) diag(s)] U^T,   i.e. Y^T = U (diag(s) (V^T X^T)),
+ *
+ * with the factors of a rank-k approximation A_k = U diag(s) V^T of an
+ * m x n matrix, applied to b queries at once.  The k x b intermediate
+ * V^T X^T never leaves the chip.
+ *
+ *   U    device, m x k, row pitch lrc_packed_ld(k)
+ *   S    device, k singular values s_1..s_k
+ *   Vt   device, V^T: k x n, row pitch lrc_packed_ld(n)
+ *   X    device, b x n queries (one per row), row pitch lrc_packed_ld(n)
+ *   Y    device, b x m results, row pitch m
+ *
+ * Element types: LRC_F64 -> U, S, Vt, X, Y binary64; LRC_F32 -> all
+ * binary32; LRC_F16 -> U, S, Vt, X binary16 and Y binary32; LRC_F16_O16 ->
+ * all binary16 (the intermediate is rounded to binary16 as well).  Pad
+ * columns of U, Vt and X are never read.  All five pointers must be 16-byte
+ * aligned.  k may exceed min(m, n).  Asynchronous on `stream`.
+ */
+LRC_API lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X, void* Y,
+                     int64_t m, int64_t n, int64_t k, int64_t b, lrc_fmt fmt,
+                     lrc_stream_t stream);
+
+/*
+ * tt_reconstruct -- dense Tensor-Train reconstruction (Sec. 5.1:
+ * T(i_1..i_d) = G_1(i_1) ... G_d(i_d); Sec. 7.5, Eq. gpu_tt_reconstruction:
+ * the chain B_l = Z_{l-1} K_l, Z_l = reshape(B_l)).
+ *
+ *   cores   HOST array of d DEVICE pointers; cores[l] holds G_{l+1}, an
+ *           unpadded C-order ranks[l] x dims[l] x ranks[l+1] array
+ *   dims    host, d mode sizes n_1..n_d (> 0)
+ *   ranks   host, d+1 TT ranks with ranks[0] = ranks[d] = 1 (> 0)
+ *   d       number of cores, 2 <= d <= 16
+ *   out     device, prod(dims) entries in C order (i_1 slowest): the
+ *           vectorised tensor of Eq. gpu_tt_reconstruction
+ *
+ * Element types: LRC_F64 cores/out binary64; LRC_F32 binary32; LRC_F16
+ * binary16 cores, binary32 out; LRC_F16_O16 binary16 cores, workspaces and
+ * out.  Cores must be aligned to their element size, out to 16 bytes.
+ * Intermediate products Z_l stay on chip.  Asynchronous on `stream`.
+ */
+LRC_API lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims, const int64_t* ranks,
+                          int d, lrc_fmt fmt, void* out, lrc_stream_t stream);
+
+/*
+ * lrc_fro_diff -- Frobenius norm of a difference (Sec. 5.1 "Frobenius norm";
+ * eta of Thm 4.1 and eta_TT of Thm 6.1 are ||A_k' - Ahat_k'||_F and
+ * ||T_R+ - That_R+||_F of the FP64 reconstructions).
+ *
+ *   A, B        device arrays of `count` elements in formats fa, fb
+ *               (LRC_F64, LRC_F32, or LRC_F16 / LRC_F16_O16 = binary16);
+ *               B may be NULL, meaning B = 0
+ *   diff_out    host: sqrt(sum_i (A_i - B_i)^2), differences and squares in
+ *               binary64
+ *   normA_out   host, may be NULL: sqrt(sum_i A_i^2)
+ *
+ * Summation is deterministic: fixed per-block partial sums reduced in a
+ * fixed order, so repeated calls on the same data give identical bits.
+ * Uses library-held device scratch (allocated on first use per device,
+ * released by lrc_shutdown), so concurrent calls on different streams of
+ * the same device must not overlap.  SYNCHRONISES `stream`.
+ */
+LRC_API lrc_status lrc_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
+                        double* diff_out, double* normA_out, lrc_stream_t stream);
+
+/* Thm 4.1 Eq. matrix_condition and Thm 6.1 Eq. tt_condition:
+ * returns 1 if e_aug + eta <= e_base (certified non-increase), else 0. */
+LRC_API int lrc_certified(double e_base, double e_aug, double eta);
+
+/* Sec. 4: E_k = (sum_{j>k} sigma_j^2)^(1/2) for host sigma[0..len) (sigma_1
+ * first), summed from the smallest term up.  Returns -1 on bad arguments. */
+LRC_API double lrc_tail_error(const double* sigma, int64_t len, int64_t k);
+
+/* Eq. matrix_storage_ratio generalised to k_aug >= k_base: storage of the
+ * rank-k_aug factors in `fmt` over the FP64 rank-k_base factors. */
+LRC_API double lrc_matrix_storage_ratio(int64_t m, int64_t n, int64_t k_base, int64_t k_aug, lrc_fmt fmt);
+
+/* Sec. 5.1: TT storage in bytes, sum_l R_{l-1} n_l R_l scalars of `fmt`. */
+LRC_API double lrc_tt_storage_bytes(const int64_t* dims, const int64_t* ranks, int d, lrc_fmt fmt);
+
+/* Message for a status code, and the last error message of this thread. */
+LRC_API const char* lrc_status_string(lrc_status status);
+LRC_API const char* lrc_last_error(void);
+
+/* Number of kernels this library has launched in this process. */
+LRC_API uint64_t lrc_launch_count(void);
+
+/* Release library-held scratch on every device; the library stays usable. */
+LRC_API lrc_status lrc_shutdown(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LRC_H */

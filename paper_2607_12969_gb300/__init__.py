@@ -1,0 +1,205 @@
+"""Python binding of liblrc.so, the GB300 rank-compensation hot path.
+
+Argument marshalling only: every entry point forwards device pointers of
+torch tensors (torch is used for device memory and streams) and sizes to the
+C ABI declared in include/lrc.h, where every step runs in the library's own
+CUDA kernels.  There is no CPU fallback: if the library is missing or fails
+to load, every call raises.
+
+Names follow the C ABI: lrc_round_factors, lrc_widen_factors, lrc_apply,
+tt_reconstruct, lrc_fro_diff, plus the host helpers lrc_certified,
+lrc_tail_error, lrc_matrix_storage_ratio and lrc_tt_storage_bytes.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence, Tuple
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "liblrc.so")
+
+F64, F32, F16, F16_O16 = 0, 1, 2, 3
+FORMATS = {"f64": F64, "f32": F32, "f16": F16, "f16_o16": F16_O16}
+STATUS = {0: "ok", -1: "invalid argument", -2: "misaligned pointer", -3: "unsupported",
+          -4: "CUDA error", -5: "out of memory", -6: "device wait timed out"}
+
+
+class LrcError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS.get(status, status)}: {message}")
+        self.status = status
+
+
+_lib: Optional[ctypes.CDLL] = None
+
+
+def load() -> ctypes.CDLL:
+    """Load liblrc.so (built by build.py); raises if it is absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                           "`python -c 'import __graft_entry__ as g; g.build()'`")
+    L = ctypes.CDLL(LIB_PATH)
+    i64, i32, vp, dbl = ctypes.c_int64, ctypes.c_int, ctypes.c_void_p, ctypes.c_double
+    L.lrc_packed_ld.argtypes = [i64]
+    L.lrc_packed_ld.restype = i64
+    L.lrc_round_factors.argtypes = [vp, i64, i64, i64, vp, i64, i32, vp]
+    L.lrc_round_factors.restype = i32
+    L.lrc_widen_factors.argtypes = [vp, i32, i64, i64, i64, vp, i64, vp]
+    L.lrc_widen_factors.restype = i32
+    L.lrc_apply.argtypes = [vp, vp, vp, vp, vp, i64, i64, i64, i64, i32, vp]
+    L.lrc_apply.restype = i32
+    L.tt_reconstruct.argtypes = [vp, vp, vp, i32, i32, vp, vp]
+    L.tt_reconstruct.restype = i32
+    L.lrc_fro_diff.argtypes = [vp, i32, vp, i32, i64, vp, vp, vp]
+    L.lrc_fro_diff.restype = i32
+    L.lrc_certified.argtypes = [dbl, dbl, dbl]
+    L.lrc_certified.restype = i32
+    L.lrc_tail_error.argtypes = [vp, i64, i64]
+    L.lrc_tail_error.restype = dbl
+    L.lrc_matrix_storage_ratio.argtypes = [i64, i64, i64, i64, i32]
+    L.lrc_matrix_storage_ratio.restype = dbl
+    L.lrc_tt_storage_bytes.argtypes = [vp, vp, i32, i32]
+    L.lrc_tt_storage_bytes.restype = dbl
+    L.lrc_status_string.argtypes = [i32]
+    L.lrc_status_string.restype = ctypes.c_char_p
+    L.lrc_last_error.restype = ctypes.c_char_p
+    L.lrc_launch_count.restype = ctypes.c_uint64
+    L.lrc_shutdown.restype = i32
+    _lib = L
+    return L
+
+
+def _fmt(fmt) -> int:
+    if isinstance(fmt, str):
+        return FORMATS[fmt]
+    return int(fmt)
+
+
+def storage_dtype(fmt):
+    import torch
+    f = _fmt(fmt)
+    return {F64: torch.float64, F32: torch.float32, F16: torch.float16, F16_O16: torch.float16}[f]
+
+
+def output_dtype(fmt):
+    import torch
+    f = _fmt(fmt)
+    return {F64: torch.float64, F32: torch.float32, F16: torch.float32, F16_O16: torch.float16}[f]
+
+
+def _check(status: int) -> None:
+    if status != 0:
+        msg = load().lrc_last_error().decode(errors="replace")
+        raise LrcError(status, msg)
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _ptr(t) -> int:
+    return 0 if t is None else t.data_ptr()
+
+
+# --------------------------------------------------------------------------
+# entry points (same names and argument order as include/lrc.h)
+# --------------------------------------------------------------------------
+
+def lrc_packed_ld(cols: int) -> int:
+    return int(load().lrc_packed_ld(int(cols)))
+
+
+def lrc_round_factors(src, rows: int, cols: int, ld_src: int, dst, ld_dst: int, fmt, stream=None):
+    _check(load().lrc_round_factors(_ptr(src), rows, cols, ld_src, _ptr(dst), ld_dst, _fmt(fmt),
+                                    _stream(stream)))
+
+
+def lrc_widen_factors(src, fmt, rows: int, cols: int, ld_src: int, dst, ld_dst: int, stream=None):
+    _check(load().lrc_widen_factors(_ptr(src), _fmt(fmt), rows, cols, ld_src, _ptr(dst), ld_dst,
+                                    _stream(stream)))
+
+
+def lrc_apply(U, S, Vt, X, Y, m: int, n: int, k: int, b: int, fmt, stream=None):
+    _check(load().lrc_apply(_ptr(U), _ptr(S), _ptr(Vt), _ptr(X), _ptr(Y), m, n, k, b, _fmt(fmt),
+                            _stream(stream)))
+
+
+def tt_reconstruct(cores: Sequence, dims: Sequence[int], ranks: Sequence[int], fmt, out, stream=None):
+    d = len(cores)
+    ptrs = (ctypes.c_void_p * d)(*[c.data_ptr() for c in cores])
+    dd = (ctypes.c_int64 * d)(*[int(x) for x in dims])
+    rr = (ctypes.c_int64 * (d + 1))(*[int(x) for x in ranks])
+    _check(load().tt_reconstruct(ctypes.cast(ptrs, ctypes.c_void_p), ctypes.cast(dd, ctypes.c_void_p),
+                                 ctypes.cast(rr, ctypes.c_void_p), d, _fmt(fmt), _ptr(out),
+                                 _stream(stream)))
+
+
+def lrc_fro_diff(A, fa, B, fb, count: int, stream=None) -> Tuple[float, float]:
+    """Returns (||A - B||_F, ||A||_F); B may be None."""
+    diff = ctypes.c_double(0.0)
+    norm = ctypes.c_double(0.0)
+    _check(load().lrc_fro_diff(_ptr(A), _fmt(fa), _ptr(B), _fmt(fb) if B is not None else 0, count,
+                               ctypes.addressof(diff), ctypes.addressof(norm), _stream(stream)))
+    return diff.value, norm.value
+
+
+def lrc_certified(e_base: float, e_aug: float, eta: float) -> bool:
+    return bool(load().lrc_certified(float(e_base), float(e_aug), float(eta)))
+
+
+def lrc_tail_error(sigma, k: int) -> float:
+    import numpy as np
+    s = np.ascontiguousarray(sigma, dtype=np.float64)
+    return float(load().lrc_tail_error(s.ctypes.data, s.size, int(k)))
+
+
+def lrc_matrix_storage_ratio(m: int, n: int, k_base: int, k_aug: int, fmt) -> float:
+    return float(load().lrc_matrix_storage_ratio(m, n, k_base, k_aug, _fmt(fmt)))
+
+
+def lrc_tt_storage_bytes(dims: Sequence[int], ranks: Sequence[int], fmt) -> float:
+    d = len(dims)
+    dd = (ctypes.c_int64 * d)(*[int(x) for x in dims])
+    rr = (ctypes.c_int64 * (d + 1))(*[int(x) for x in ranks])
+    return float(load().lrc_tt_storage_bytes(ctypes.cast(dd, ctypes.c_void_p),
+                                             ctypes.cast(rr, ctypes.c_void_p), d, _fmt(fmt)))
+
+
+def lrc_launch_count() -> int:
+    return int(load().lrc_launch_count())
+
+
+def lrc_shutdown() -> None:
+    _check(load().lrc_shutdown())
+
+
+# --------------------------------------------------------------------------
+# convenience helpers built only from the entry points above
+# --------------------------------------------------------------------------
+
+def round_matrix(src64, fmt, ld: Optional[int] = None, stream=None):
+    """Round a 2-D CUDA float64 tensor into a new packed tensor (lrc_round_factors)."""
+    import torch
+    rows, cols = src64.shape
+    ld = lrc_packed_ld(cols) if ld is None else ld
+    dst = torch.empty((rows, ld), dtype=storage_dtype(fmt), device=src64.device)
+    lrc_round_factors(src64, rows, cols, src64.stride(0), dst, ld, fmt, stream)
+    return dst
+
+
+def widen_matrix(src, fmt, cols: int, stream=None):
+    """Exact float64 copy (rows x packed ld) of a packed tensor (lrc_widen_factors)."""
+    import torch
+    rows, ld = src.shape
+    dst = torch.empty((rows, lrc_packed_ld(cols)), dtype=torch.float64, device=src.device)
+    lrc_widen_factors(src, fmt, rows, cols, ld, dst, dst.shape[1], stream)
+    return dst

@@ -1,0 +1,243 @@
+// abi.cu -- the extern "C" entry points of liblrc.so: argument validation,
+// dispatch to the kernels, and the host-side certificate / storage helpers.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <atomic>
+#include <mutex>
+
+#include "common.cuh"
+
+namespace lrc {
+
+static thread_local char g_msg[512] = "";
+static std::atomic<uint64_t> g_launches{0};
+
+void set_error(const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_msg, sizeof g_msg, fmt, ap);
+    va_end(ap);
+}
+
+lrc_status cuda_fail(cudaError_t e, const char* what) {
+    set_error("%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+    return LRC_ERR_CUDA;
+}
+
+lrc_status after_launch(const char* what) {
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, what);
+    return LRC_OK;
+}
+
+int sm_count() {
+    static std::mutex mu;
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+    std::lock_guard<std::mutex> lock(mu);
+    if (cache[dev] == 0) {
+        int v = 0;
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+        cache[dev] = v > 0 ? v : 1;
+    }
+    return cache[dev];
+}
+
+static lrc_status invalid(const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_msg, sizeof g_msg, fmt, ap);
+    va_end(ap);
+    return LRC_ERR_INVALID_ARG;
+}
+
+static lrc_status misaligned(const char* name) {
+    set_error("%s is not 16-byte aligned", name);
+    return LRC_ERR_ALIGNMENT;
+}
+
+}  // namespace lrc
+
+using namespace lrc;
+
+extern "C" {
+
+int64_t lrc_packed_ld(int64_t cols) {
+    if (cols < 0 || cols > INT64_MAX - 15) return -1;
+    return (cols + 15) / 16 * 16;
+}
+
+lrc_status lrc_round_factors(const double* src, int64_t rows, int64_t cols, int64_t ld_src,
+                             void* dst, int64_t ld_dst, lrc_fmt fmt, lrc_stream_t stream) {
+    if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    if (rows < 0 || cols < 0) return invalid("negative size (rows=%lld cols=%lld)", (long long)rows, (long long)cols);
+    if (ld_src < cols || ld_dst < cols) return invalid("leading dimension below cols");
+    if (rows == 0 || cols == 0) return LRC_OK;
+    int64_t t;
+    if (!mul_ok(rows, ld_src, &t) || !mul_ok(rows, ld_dst, &t) || !mul_ok(t, 8, &t))
+        return invalid("size overflow");
+    if (!src || !dst) return invalid("null pointer");
+    if (!aligned16(src)) return misaligned("src");
+    if (!aligned16(dst)) return misaligned("dst");
+    return launch_round(src, rows, cols, ld_src, dst, ld_dst, fmt, as_stream(stream));
+}
+
+lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows, int64_t cols,
+                             int64_t ld_src, double* dst, int64_t ld_dst, lrc_stream_t stream) {
+    if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    if (rows < 0 || cols < 0) return invalid("negative size");
+    if (ld_src < cols || ld_dst < cols) return invalid("leading dimension below cols");
+    if (rows == 0 || cols == 0) return LRC_OK;
+    int64_t t;
+    if (!mul_ok(rows, ld_src, &t) || !mul_ok(rows, ld_dst, &t) || !mul_ok(t, 8, &t))
+        return invalid("size overflow");
+    if (!src || !dst) return invalid("null pointer");
+    if (!aligned16(src)) return misaligned("src");
+    if (!aligned16(dst)) return misaligned("dst");
+    return launch_widen(src, fmt, rows, cols, ld_src, dst, ld_dst, as_stream(stream));
+}
+
+lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X, void* Y,
+                     int64_t m, int64_t n, int64_t k, int64_t b, lrc_fmt fmt,
+                     lrc_stream_t stream) {
+    if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    if (m <= 0 || n <= 0 || k <= 0 || b <= 0)
+        return invalid("sizes must be positive (m=%lld n=%lld k=%lld b=%lld)", (long long)m,
+                       (long long)n, (long long)k, (long long)b);
+    int64_t t;
+    const int64_t ldk = lrc_packed_ld(k), ldn = lrc_packed_ld(n);
+    if (ldk < 0 || ldn < 0 || !mul_ok(m, ldk, &t) || !mul_ok(t, 8, &t) || !mul_ok(k, ldn, &t) ||
+        !mul_ok(t, 8, &t) || !mul_ok(b, ldn, &t) || !mul_ok(t, 8, &t) || !mul_ok(b, m, &t) ||
+        !mul_ok(t, 8, &t))
+        return invalid("size overflow");
+    if (!U || !S || !Vt || !X || !Y) return invalid("null pointer");
+    if (!aligned16(U)) return misaligned("U");
+    if (!aligned16(S)) return misaligned("S");
+    if (!aligned16(Vt)) return misaligned("Vt");
+    if (!aligned16(X)) return misaligned("X");
+    if (!aligned16(Y)) return misaligned("Y");
+    cudaStream_t s = as_stream(stream);
+    switch (fmt) {
+        case LRC_F64:
+            return launch_apply_f64((const double*)U, (const double*)S, (const double*)Vt,
+                                    (const double*)X, (double*)Y, m, n, k, b, s);
+        case LRC_F32:
+            return launch_apply_f32((const float*)U, (const float*)S, (const float*)Vt,
+                                    (const float*)X, (float*)Y, m, n, k, b, s);
+        case LRC_F16:
+        case LRC_F16_O16:
+            return launch_apply_f16(U, S, Vt, X, Y, m, n, k, b, fmt == LRC_F16_O16, s);
+    }
+    return invalid("unknown format");
+}
+
+lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims, const int64_t* ranks,
+                          int d, lrc_fmt fmt, void* out, lrc_stream_t stream) {
+    if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    if (!cores || !dims || !ranks || !out) return invalid("null pointer");
+    if (d < 2 || d > 16) return invalid("d must be in [2, 16] (d=%d)", d);
+    if (ranks[0] != 1 || ranks[d] != 1) return invalid("ranks[0] and ranks[d] must be 1");
+    TTShape sh;
+    sh.d = d;
+    int64_t numel = 1;
+    const int64_t es = storage_bytes(fmt);
+    for (int l = 0; l < d; ++l) {
+        if (dims[l] <= 0) return invalid("dims[%d] = %lld must be positive", l, (long long)dims[l]);
+        if (ranks[l] <= 0 || ranks[l] > 4096) return invalid("ranks[%d] out of range", l);
+        if (!cores[l]) return invalid("cores[%d] is null", l);
+        if ((reinterpret_cast<uintptr_t>(cores[l]) % (uintptr_t)es) != 0) {
+            set_error("cores[%d] is not aligned to its element size", l);
+            return LRC_ERR_ALIGNMENT;
+        }
+        int64_t c;
+        if (!mul_ok(ranks[l], dims[l], &c) || !mul_ok(c, ranks[l + 1], &c) || !mul_ok(c, 8, &c))
+            return invalid("core %d size overflow", l);
+        if (!mul_ok(numel, dims[l], &numel)) return invalid("tensor size overflow");
+        sh.dims[l] = dims[l];
+        sh.ranks[l] = ranks[l];
+        sh.cores[l] = cores[l];
+    }
+    sh.ranks[d] = 1;
+    int64_t t;
+    if (!mul_ok(numel, 8, &t)) return invalid("tensor size overflow");
+    sh.numel = numel;
+    if (!aligned16(out)) return misaligned("out");
+    cudaStream_t s = as_stream(stream);
+    if (fmt == LRC_F16 || fmt == LRC_F16_O16) return launch_tt_f16(sh, fmt == LRC_F16_O16, out, s);
+    return launch_tt_cc(sh, fmt, out, s);
+}
+
+lrc_status lrc_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
+                        double* diff_out, double* normA_out, lrc_stream_t stream) {
+    if (!valid_fmt(fa) || !valid_fmt(fb)) return invalid("unknown format");
+    if (count < 0) return invalid("negative count");
+    if (!diff_out) return invalid("null diff_out");
+    int64_t t;
+    if (!mul_ok(count, 8, &t)) return invalid("size overflow");
+    if (count > 0 && !A) return invalid("null A");
+    if (count > 0 && !aligned16(A)) return misaligned("A");
+    if (B && !aligned16(B)) return misaligned("B");
+    if (count == 0) {
+        *diff_out = 0.0;
+        if (normA_out) *normA_out = 0.0;
+        return LRC_OK;
+    }
+    return run_fro_diff(A, fa, B, fb, count, diff_out, normA_out, as_stream(stream));
+}
+
+int lrc_certified(double e_base, double e_aug, double eta) { return (e_aug + eta <= e_base) ? 1 : 0; }
+
+double lrc_tail_error(const double* sigma, int64_t len, int64_t k) {
+    if (!sigma || len < 0 || k < 0) return -1.0;
+    // ascending order (smallest singular values first), compensated
+    double s = 0.0, c = 0.0;
+    for (int64_t j = len - 1; j >= k; --j) {
+        const double term = sigma[j] * sigma[j];
+        const double u = s + term;
+        c += (fabs(s) >= fabs(term)) ? ((s - u) + term) : ((term - u) + s);
+        s = u;
+    }
+    return sqrt(s + c);
+}
+
+double lrc_matrix_storage_ratio(int64_t m, int64_t n, int64_t k_base, int64_t k_aug, lrc_fmt fmt) {
+    if (m <= 0 || n <= 0 || k_base <= 0 || k_aug <= 0 || !valid_fmt(fmt)) return -1.0;
+    const double per = (double)(m + n + 1);
+    return ((double)storage_bytes(fmt) * (double)k_aug * per) / (8.0 * (double)k_base * per);
+}
+
+double lrc_tt_storage_bytes(const int64_t* dims, const int64_t* ranks, int d, lrc_fmt fmt) {
+    if (!dims || !ranks || d < 1 || !valid_fmt(fmt)) return -1.0;
+    double s = 0.0;
+    for (int l = 0; l < d; ++l) s += (double)ranks[l] * (double)dims[l] * (double)ranks[l + 1];
+    return s * (double)storage_bytes(fmt);
+}
+
+const char* lrc_status_string(lrc_status st) {
+    switch (st) {
+        case LRC_OK: return "ok";
+        case LRC_ERR_INVALID_ARG: return "invalid argument";
+        case LRC_ERR_ALIGNMENT: return "misaligned pointer";
+        case LRC_ERR_UNSUPPORTED: return "unsupported";
+        case LRC_ERR_CUDA: return "CUDA error";
+        case LRC_ERR_NOMEM: return "out of memory";
+        case LRC_ERR_TIMEOUT: return "device wait timed out";
+    }
+    return "unknown status";
+}
+
+const char* lrc_last_error(void) { return g_msg; }
+
+uint64_t lrc_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+lrc_status lrc_shutdown(void) {
+    release_scratch();
+    return LRC_OK;
+}
+
+}  // extern "C"

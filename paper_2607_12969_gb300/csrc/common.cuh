@@ -1,0 +1,74 @@
+// common.cuh -- internal helpers shared by the translation units of liblrc.so.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "lrc.h"
+
+namespace lrc {
+
+// Records a message for lrc_last_error() on the calling thread.
+void set_error(const char* fmt, ...);
+
+// Maps a CUDA error to LRC_ERR_CUDA with a message naming `what`.
+lrc_status cuda_fail(cudaError_t e, const char* what);
+
+// Checks cudaGetLastError() after a launch; counts the launch.
+lrc_status after_launch(const char* what);
+
+// Multiprocessor count of the current device (cached per device).
+int sm_count();
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+inline cudaStream_t as_stream(lrc_stream_t s) { return reinterpret_cast<cudaStream_t>(s); }
+
+// Bytes of one stored element of a format (binary16 for both F16 variants).
+inline int64_t storage_bytes(lrc_fmt f) {
+    switch (f) {
+        case LRC_F64: return 8;
+        case LRC_F32: return 4;
+        case LRC_F16:
+        case LRC_F16_O16: return 2;
+    }
+    return 0;
+}
+
+inline bool valid_fmt(int f) { return f >= LRC_F64 && f <= LRC_F16_O16; }
+
+// a * b with overflow detection (both >= 0).
+inline bool mul_ok(int64_t a, int64_t b, int64_t* out) {
+    if (a < 0 || b < 0) return false;
+    if (a != 0 && b > INT64_MAX / a) return false;
+    *out = a * b;
+    return true;
+}
+
+// ---- launchers (implemented in the .cu files) ----------------------------
+lrc_status launch_round(const double* src, int64_t rows, int64_t cols, int64_t ld_src, void* dst,
+                        int64_t ld_dst, lrc_fmt fmt, cudaStream_t s);
+lrc_status launch_widen(const void* src, lrc_fmt fmt, int64_t rows, int64_t cols, int64_t ld_src,
+                        double* dst, int64_t ld_dst, cudaStream_t s);
+lrc_status launch_apply_f64(const double* U, const double* S, const double* Vt, const double* X,
+                            double* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
+lrc_status launch_apply_f32(const float* U, const float* S, const float* Vt, const float* X,
+                            float* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
+lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y,
+                            int64_t m, int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s);
+
+struct TTShape {
+    int d;
+    int64_t dims[16];
+    int64_t ranks[17];
+    const void* cores[16];
+    int64_t numel;
+};
+lrc_status launch_tt_cc(const TTShape& sh, lrc_fmt fmt, void* out, cudaStream_t s);
+lrc_status launch_tt_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s);
+
+lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
+                        double* diff_out, double* normA_out, cudaStream_t s);
+void release_scratch();
+
+}  // namespace lrc

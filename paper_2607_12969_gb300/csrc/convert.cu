@@ -1,0 +1,176 @@
+// convert.cu -- factor rounding / packing (binary64 -> binary32 / binary16)
+// and exact widening back to binary64.
+//
+// Rounding is the hardware conversion cvt.rn.{f32,f16}.f64: IEEE 754
+// round-to-nearest-even directly from binary64 (no intermediate format),
+// subnormals kept (no .ftz), overflow to infinity.  The kernels are
+// HBM-bound streams: each thread converts a group of 8 consecutive elements
+// of one row with 128-bit loads and stores where the row pitch allows it.
+#include <cuda_fp16.h>
+
+#include "common.cuh"
+
+namespace lrc {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kGroup = 8;
+
+__device__ __forceinline__ uint16_t cvt_f16(double x) {
+    uint16_t h;
+    asm("cvt.rn.f16.f64 %0, %1;" : "=h"(h) : "d"(x));
+    return h;
+}
+__device__ __forceinline__ float cvt_f32(double x) {
+    float f;
+    asm("cvt.rn.f32.f64 %0, %1;" : "=f"(f) : "d"(x));
+    return f;
+}
+__device__ __forceinline__ double widen_f16(uint16_t h) {
+    double d;
+    asm("cvt.f64.f16 %0, %1;" : "=d"(d) : "h"(h));
+    return d;
+}
+
+// FMT: 0 = binary64 copy, 1 = binary32, 2 = binary16
+template <int FMT>
+__global__ void __launch_bounds__(kThreads)
+round_pack_kernel(const double* __restrict__ src, int64_t cols, int64_t ld_src,
+                  void* __restrict__ dst, int64_t ld_dst, int64_t groups_per_row,
+                  int64_t total_groups, bool vec_src, bool vec_dst) {
+    const int64_t stride = (int64_t)gridDim.x * kThreads;
+    for (int64_t g = (int64_t)blockIdx.x * kThreads + threadIdx.x; g < total_groups; g += stride) {
+        const int64_t r = g / groups_per_row;
+        const int64_t c0 = (g - r * groups_per_row) * kGroup;
+        const double* srow = src + r * ld_src;
+        double v[kGroup];
+        if (vec_src && c0 + kGroup <= cols) {
+#pragma unroll
+            for (int j = 0; j < kGroup; j += 2) {
+                const double2 p = __ldcs(reinterpret_cast<const double2*>(srow + c0 + j));
+                v[j] = p.x;
+                v[j + 1] = p.y;
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < kGroup; ++j) v[j] = (c0 + j < cols) ? __ldcs(srow + c0 + j) : 0.0;
+        }
+        const bool full = vec_dst && (c0 + kGroup <= ld_dst);
+        if (FMT == 2) {
+            uint16_t* drow = static_cast<uint16_t*>(dst) + r * ld_dst;
+            uint16_t h[kGroup];
+#pragma unroll
+            for (int j = 0; j < kGroup; ++j) h[j] = cvt_f16(v[j]);
+            if (full) {
+                uint4 q;
+                q.x = (uint32_t)h[0] | ((uint32_t)h[1] << 16);
+                q.y = (uint32_t)h[2] | ((uint32_t)h[3] << 16);
+                q.z = (uint32_t)h[4] | ((uint32_t)h[5] << 16);
+                q.w = (uint32_t)h[6] | ((uint32_t)h[7] << 16);
+                __stcs(reinterpret_cast<uint4*>(drow + c0), q);
+            } else {
+                for (int j = 0; j < kGroup; ++j)
+                    if (c0 + j < ld_dst) drow[c0 + j] = h[j];
+            }
+        } else if (FMT == 1) {
+            float* drow = static_cast<float*>(dst) + r * ld_dst;
+            float f[kGroup];
+#pragma unroll
+            for (int j = 0; j < kGroup; ++j) f[j] = cvt_f32(v[j]);
+            if (full) {
+                __stcs(reinterpret_cast<float4*>(drow + c0), make_float4(f[0], f[1], f[2], f[3]));
+                __stcs(reinterpret_cast<float4*>(drow + c0 + 4), make_float4(f[4], f[5], f[6], f[7]));
+            } else {
+                for (int j = 0; j < kGroup; ++j)
+                    if (c0 + j < ld_dst) drow[c0 + j] = f[j];
+            }
+        } else {
+            double* drow = static_cast<double*>(dst) + r * ld_dst;
+            if (full) {
+#pragma unroll
+                for (int j = 0; j < kGroup; j += 2)
+                    __stcs(reinterpret_cast<double2*>(drow + c0 + j), make_double2(v[j], v[j + 1]));
+            } else {
+                for (int j = 0; j < kGroup; ++j)
+                    if (c0 + j < ld_dst) drow[c0 + j] = v[j];
+            }
+        }
+    }
+}
+
+// FMT as above; dst is binary64.
+template <int FMT>
+__global__ void __launch_bounds__(kThreads)
+widen_kernel(const void* __restrict__ src, int64_t cols, int64_t ld_src, double* __restrict__ dst,
+             int64_t ld_dst, int64_t groups_per_row, int64_t total_groups) {
+    const int64_t stride = (int64_t)gridDim.x * kThreads;
+    for (int64_t g = (int64_t)blockIdx.x * kThreads + threadIdx.x; g < total_groups; g += stride) {
+        const int64_t r = g / groups_per_row;
+        const int64_t c0 = (g - r * groups_per_row) * kGroup;
+        double* drow = dst + r * ld_dst;
+#pragma unroll
+        for (int j = 0; j < kGroup; ++j) {
+            const int64_t c = c0 + j;
+            if (c >= ld_dst) break;
+            double v = 0.0;
+            if (c < cols) {
+                if (FMT == 2) v = widen_f16(static_cast<const uint16_t*>(src)[r * ld_src + c]);
+                else if (FMT == 1) v = (double)static_cast<const float*>(src)[r * ld_src + c];
+                else v = static_cast<const double*>(src)[r * ld_src + c];
+            }
+            drow[c] = v;
+        }
+    }
+}
+
+int grid_for(int64_t groups) {
+    const int64_t want = (groups + kThreads - 1) / kThreads;
+    const int64_t cap = (int64_t)sm_count() * 8;
+    return (int)(want < cap ? (want > 0 ? want : 1) : cap);
+}
+
+}  // namespace
+
+lrc_status launch_round(const double* src, int64_t rows, int64_t cols, int64_t ld_src, void* dst,
+                        int64_t ld_dst, lrc_fmt fmt, cudaStream_t s) {
+    const int64_t gpr = (ld_dst + kGroup - 1) / kGroup;
+    const int64_t total = rows * gpr;
+    const bool vec_src = (ld_src % 2) == 0;
+    const int grid = grid_for(total);
+    switch (fmt) {
+        case LRC_F64:
+            round_pack_kernel<0><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total,
+                                                            vec_src, (ld_dst % 2) == 0);
+            break;
+        case LRC_F32:
+            round_pack_kernel<1><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total,
+                                                            vec_src, (ld_dst % 4) == 0);
+            break;
+        default:
+            round_pack_kernel<2><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total,
+                                                            vec_src, (ld_dst % 8) == 0);
+            break;
+    }
+    return after_launch("round_pack_kernel");
+}
+
+lrc_status launch_widen(const void* src, lrc_fmt fmt, int64_t rows, int64_t cols, int64_t ld_src,
+                        double* dst, int64_t ld_dst, cudaStream_t s) {
+    const int64_t gpr = (ld_dst + kGroup - 1) / kGroup;
+    const int64_t total = rows * gpr;
+    const int grid = grid_for(total);
+    switch (fmt) {
+        case LRC_F64:
+            widen_kernel<0><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total);
+            break;
+        case LRC_F32:
+            widen_kernel<1><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total);
+            break;
+        default:
+            widen_kernel<2><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total);
+            break;
+    }
+    return after_launch("widen_kernel");
+}
+
+}  // namespace lrc

@@ -1,0 +1,226 @@
+// fro_diff.cu -- ||A - B||_F and ||A||_F in binary64 (Sec. 5.1), the
+// reduction behind eta (Thm 4.1) and eta_TT (Thm 6.1).
+//
+// Pass 1: a fixed grid of blocks streams the arrays (128-bit loads, groups of
+// 8 elements per thread and step), accumulates (a-b)^2 and a^2 in binary64
+// per thread, reduces each block with a fixed shuffle tree, and writes one
+// partial pair per block.  Pass 2: one block reduces the partials in a fixed
+// order.  The assignment of elements to threads depends only on `count` and
+// the device's SM count, so results are bitwise reproducible on a device.
+#include <cuda_fp16.h>
+
+#include <mutex>
+
+#include "common.cuh"
+
+namespace lrc {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kGroup = 8;
+constexpr int kMaxBlocks = 4096;
+
+struct Scratch {
+    double* partial = nullptr;   // 2 * kMaxBlocks + 2 doubles
+};
+std::mutex g_mu;
+Scratch g_scratch[64];
+
+__device__ __forceinline__ double widen_h(uint16_t h) {
+    double d;
+    asm("cvt.f64.f16 %0, %1;" : "=d"(d) : "h"(h));
+    return d;
+}
+
+// Loads elements [8g, 8g+8) of an array of format F as binary64.
+template <int F>
+__device__ __forceinline__ void load8(const void* p, int64_t g, double v[kGroup]) {
+    if (F == 0) {
+        const double2* q = reinterpret_cast<const double2*>(p) + g * 4;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const double2 t = __ldcs(q + j);
+            v[2 * j] = t.x;
+            v[2 * j + 1] = t.y;
+        }
+    } else if (F == 1) {
+        const float4* q = reinterpret_cast<const float4*>(p) + g * 2;
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+            const float4 t = __ldcs(q + j);
+            v[4 * j] = t.x;
+            v[4 * j + 1] = t.y;
+            v[4 * j + 2] = t.z;
+            v[4 * j + 3] = t.w;
+        }
+    } else {
+        const uint4 t = __ldcs(reinterpret_cast<const uint4*>(p) + g);
+        const uint32_t w[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            v[2 * j] = widen_h((uint16_t)(w[j] & 0xffffu));
+            v[2 * j + 1] = widen_h((uint16_t)(w[j] >> 16));
+        }
+    }
+}
+
+template <int F>
+__device__ __forceinline__ double load1(const void* p, int64_t i) {
+    if (F == 0) return static_cast<const double*>(p)[i];
+    if (F == 1) return (double)static_cast<const float*>(p)[i];
+    return widen_h(static_cast<const uint16_t*>(p)[i]);
+}
+
+__device__ __forceinline__ void block_sum2(double& a, double& b, double* sh) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        a += __shfl_xor_sync(0xffffffffu, a, o);
+        b += __shfl_xor_sync(0xffffffffu, b, o);
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        sh[warp] = a;
+        sh[32 + warp] = b;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        const int nw = blockDim.x >> 5;
+        a = lane < nw ? sh[lane] : 0.0;
+        b = lane < nw ? sh[32 + lane] : 0.0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            a += __shfl_xor_sync(0xffffffffu, a, o);
+            b += __shfl_xor_sync(0xffffffffu, b, o);
+        }
+    }
+}
+
+// FB = -1: B absent (treated as zero).
+template <int FA, int FB>
+__global__ void __launch_bounds__(kThreads)
+fro_partial_kernel(const void* __restrict__ A, const void* __restrict__ B, int64_t count,
+                   double* __restrict__ partial) {
+    __shared__ double sh[64];
+    double sd = 0.0, sa = 0.0;
+    const int64_t groups = count / kGroup;
+    const int64_t stride = (int64_t)gridDim.x * kThreads;
+    for (int64_t g = (int64_t)blockIdx.x * kThreads + threadIdx.x; g < groups; g += stride) {
+        double a[kGroup], b[kGroup];
+        load8<FA>(A, g, a);
+        if (FB >= 0) load8<FB>(B, g, b);
+#pragma unroll
+        for (int j = 0; j < kGroup; ++j) {
+            const double d = (FB >= 0) ? a[j] - b[j] : a[j];
+            sd = fma(d, d, sd);
+            sa = fma(a[j], a[j], sa);
+        }
+    }
+    if (blockIdx.x == 0) {  // ragged tail, fixed owner
+        for (int64_t i = groups * kGroup + threadIdx.x; i < count; i += kThreads) {
+            const double a = load1<FA>(A, i);
+            const double d = (FB >= 0) ? a - load1<FB < 0 ? 0 : FB>(B, i) : a;
+            sd = fma(d, d, sd);
+            sa = fma(a, a, sa);
+        }
+    }
+    block_sum2(sd, sa, sh);
+    if (threadIdx.x == 0) {
+        partial[blockIdx.x] = sd;
+        partial[gridDim.x + blockIdx.x] = sa;
+    }
+}
+
+__global__ void __launch_bounds__(1024)
+fro_final_kernel(const double* __restrict__ partial, int nblocks, double* __restrict__ result) {
+    __shared__ double sh[64];
+    double sd = 0.0, sa = 0.0;
+    for (int i = threadIdx.x; i < nblocks; i += blockDim.x) {
+        sd += partial[i];
+        sa += partial[nblocks + i];
+    }
+    block_sum2(sd, sa, sh);
+    if (threadIdx.x == 0) {
+        result[0] = sqrt(sd);
+        result[1] = sqrt(sa);
+    }
+}
+
+int fcode(lrc_fmt f) { return f == LRC_F64 ? 0 : (f == LRC_F32 ? 1 : 2); }
+
+template <int FA>
+void launch_partial(int fb, int grid, const void* A, const void* B, int64_t count, double* partial,
+                    cudaStream_t s) {
+    switch (fb) {
+        case 0: fro_partial_kernel<FA, 0><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
+        case 1: fro_partial_kernel<FA, 1><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
+        case 2: fro_partial_kernel<FA, 2><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
+        default: fro_partial_kernel<FA, -1><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
+    }
+}
+
+}  // namespace
+
+lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
+                        double* diff_out, double* normA_out, cudaStream_t s) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= 64) {
+        set_error("device ordinal %d out of range", dev);
+        return LRC_ERR_UNSUPPORTED;
+    }
+    double* partial;
+    {
+        std::lock_guard<std::mutex> lock(g_mu);
+        if (!g_scratch[dev].partial) {
+            e = cudaMalloc(&g_scratch[dev].partial, (2 * kMaxBlocks + 2) * sizeof(double));
+            if (e != cudaSuccess) {
+                g_scratch[dev].partial = nullptr;
+                set_error("scratch allocation failed: %s", cudaGetErrorString(e));
+                return LRC_ERR_NOMEM;
+            }
+        }
+        partial = g_scratch[dev].partial;
+    }
+    const int64_t groups = count / kGroup;
+    int64_t want = (groups + kThreads - 1) / kThreads;
+    const int64_t cap = (int64_t)sm_count() * 4;
+    int grid = (int)(want < cap ? (want > 0 ? want : 1) : cap);
+    if (grid > kMaxBlocks) grid = kMaxBlocks;
+    const int a = fcode(fa), b = B ? fcode(fb) : -1;
+    switch (a) {
+        case 0: launch_partial<0>(b, grid, A, B, count, partial, s); break;
+        case 1: launch_partial<1>(b, grid, A, B, count, partial, s); break;
+        default: launch_partial<2>(b, grid, A, B, count, partial, s); break;
+    }
+    lrc_status st = after_launch("fro_partial_kernel");
+    if (st != LRC_OK) return st;
+    double* result = partial + 2 * kMaxBlocks;
+    fro_final_kernel<<<1, 1024, 0, s>>>(partial, grid, result);
+    st = after_launch("fro_final_kernel");
+    if (st != LRC_OK) return st;
+    double host[2];
+    e = cudaMemcpyAsync(host, result, sizeof host, cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (fro_diff result)");
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize (fro_diff)");
+    *diff_out = host[0];
+    if (normA_out) *normA_out = host[1];
+    return LRC_OK;
+}
+
+void release_scratch() {
+    std::lock_guard<std::mutex> lock(g_mu);
+    int prev = -1;
+    cudaGetDevice(&prev);
+    for (int d = 0; d < 64; ++d) {
+        if (g_scratch[d].partial) {
+            cudaSetDevice(d);
+            cudaFree(g_scratch[d].partial);
+            g_scratch[d].partial = nullptr;
+        }
+    }
+    if (prev >= 0) cudaSetDevice(prev);
+}
+
+}  // namespace lrc

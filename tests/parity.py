@@ -1,0 +1,40 @@
+"""Shared helpers for the GPU parity tests: move seeded FP64 inputs to the
+device, round them through the library, and compare with the oracle."""
+import numpy as np
+
+import oracle
+
+# relative Frobenius tolerances per path
+TOL = {"f64": 1e-12, "f32": 1e-5, "f16": 1e-5, "f16_o16": 2e-3}
+BITS_DTYPE = {"f64": np.float64, "f32": np.uint32, "f16": np.uint16}
+
+
+def base_fmt(fmt: str) -> str:
+    return "f16" if fmt.startswith("f16") else fmt
+
+
+def rel_fro(got: np.ndarray, want: np.ndarray) -> float:
+    got = np.asarray(got, dtype=np.float64).reshape(-1)
+    want = np.asarray(want, dtype=np.float64).reshape(-1)
+    nw = float(np.linalg.norm(want))
+    return float(np.linalg.norm(got - want)) / (nw if nw > 0 else 1.0)
+
+
+def to_dev(a, dev):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+
+def packed(lrc, a64: np.ndarray, fmt: str, dev):
+    """Round a host FP64 matrix through lrc_round_factors into a packed tensor."""
+    a = a64 if a64.ndim == 2 else a64[None, :]
+    return lrc.round_matrix(to_dev(a, dev), fmt)
+
+
+def bits(t, fmt: str) -> np.ndarray:
+    return t.cpu().numpy().view(BITS_DTYPE[base_fmt(fmt)])
+
+
+def oracle_inputs(U, s, Vt, X, fmt):
+    b = base_fmt(fmt)
+    return (oracle.rounded(U, b), oracle.rounded(s, b), oracle.rounded(Vt, b), oracle.rounded(X, b))

@@ -1,0 +1,104 @@
+"""GPU batched low-rank apply (lrc_apply, Sec. 4.4 Eq. gpu_matrix_apply)
+against the oracle evaluated on the same rounded inputs."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads as W
+from parity import TOL, base_fmt, oracle_inputs, packed, rel_fro
+
+pytestmark = pytest.mark.gpu
+
+FMTS = ["f64", "f32", "f16", "f16_o16"]
+
+
+def run_apply(lrc, dev, U, s, Vt, X, fmt):
+    m, k = U.shape
+    n = Vt.shape[1]
+    b = X.shape[0]
+    Ud, Sd, Vd, Xd = (packed(lrc, a, fmt, dev) for a in (U, s, Vt, X))
+    Y = torch.full((b, m), float("nan"), dtype=lrc.output_dtype(fmt), device=dev)
+    lrc.lrc_apply(Ud, Sd, Vd, Xd, Y, m, n, k, b, fmt)
+    torch.cuda.synchronize()
+    return Y.double().cpu().numpy()
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("m,n,k,b", [(40, 24, 5, 3), (130, 70, 33, 17), (257, 129, 144, 129)])
+def test_integer_inputs_exact(lrc, cuda, fmt, m, n, k, b):
+    # small integers: every product and partial sum is exact in every format
+    U = W.integer_valued((m, k), 1, -2, 2)
+    s = W.integer_valued((k,), 2, 1, 2)
+    Vt = W.integer_valued((k, n), 3, -2, 2)
+    X = W.integer_valued((b, n), 4, -2, 2)
+    got = run_apply(lrc, cuda, U, s, Vt, X, fmt)
+    want = oracle.apply(U, s, Vt, X)
+    if fmt == "f16_o16":
+        # binary16 intermediate and output are exact below 2048
+        assert np.max(np.abs(want)) < 2048
+    assert np.array_equal(got, want), fmt
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("m,n,k,b", [
+    (512, 512, 34, 64),        # tiny workload shape
+    (100, 300, 1, 1),          # rank 1, single query
+    (1000, 136, 136, 7),       # k = n
+    (48, 40, 60, 5),           # k > min(m, n)
+    (777, 1029, 272, 250),     # ragged everything, rank of the sweep workload
+    (2048, 1536, 144, 300),
+])
+def test_random_factors_vs_oracle(lrc, cuda, fmt, m, n, k, b):
+    f = W.random_factors(m, n, k, seed=m + n + k)
+    X = W.gaussian((b, n), b + 5)
+    got = run_apply(lrc, cuda, f.U, f.s, f.Vt, X, fmt)
+    want = oracle.apply(*oracle_inputs(f.U, f.s, f.Vt, X, fmt))
+    err = rel_fro(got, want)
+    assert err <= TOL[fmt], (fmt, err)
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+def test_tiny_workload_full(lrc, cuda, fmt):
+    cfg = W.MATRIX_CONFIGS["tiny"]
+    f = W.matrix_factors(cfg, base_fmt(fmt))
+    X = W.queries(cfg)
+    got = run_apply(lrc, cuda, f.U, f.s, f.Vt, X, fmt)
+    want = oracle.apply(*oracle_inputs(f.U, f.s, f.Vt, X, fmt))
+    assert rel_fro(got, want) <= TOL[fmt]
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+def test_large_workload_sampled_rows(lrc, cuda, fmt):
+    """m = 16384, n = 8192, b = 8192 in the bench's launch configuration;
+    256 seeded query rows are checked against the oracle."""
+    cfg = W.MATRIX_CONFIGS["large"]
+    f = W.matrix_factors(cfg, base_fmt(fmt))
+    X = W.queries(cfg)
+    got = run_apply(lrc, cuda, f.U, f.s, f.Vt, X, fmt)
+    rows = W.sample_indices(256, cfg.b, 99)
+    Ur, sr, Vr, Xr = oracle_inputs(f.U, f.s, f.Vt, X, fmt)
+    want = oracle.apply_rows(Ur, sr, Vr, Xr, rows)
+    err = rel_fro(got[rows], want)
+    assert err <= TOL[fmt], (fmt, err)
+    assert np.isfinite(got).all()
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("b", [1, 16, 256])
+def test_sweep_workload_small_batches(lrc, cuda, fmt, b):
+    cfg = W.sweep_config(b)
+    f = W.matrix_factors(cfg, base_fmt(fmt))
+    X = W.queries(cfg)
+    got = run_apply(lrc, cuda, f.U, f.s, f.Vt, X, fmt)
+    rows = W.sample_indices(min(b, 32), b, 7)
+    want = oracle.apply_rows(*oracle_inputs(f.U, f.s, f.Vt, X, fmt), rows)
+    assert rel_fro(got[rows], want) <= TOL[fmt]
+
+
+def test_identity_queries_reconstruct_dense_f64(lrc, cuda):
+    # X = I_n gives A_k^T: the dense FP64 reconstruction used for eta
+    f = W.random_factors(300, 200, 20, seed=3)
+    got = run_apply(lrc, cuda, f.U, f.s, f.Vt, np.eye(200), "f64")
+    want = (f.Vt.T * f.s) @ f.U.T
+    assert np.max(np.abs(got - want)) <= 1e-14 * np.max(np.abs(want))

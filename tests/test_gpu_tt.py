@@ -1,0 +1,72 @@
+"""GPU dense TT reconstruction (tt_reconstruct; Sec. 5.1 and Sec. 7.5
+Eq. gpu_tt_reconstruction) against the oracle on the same rounded cores."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads as W
+from parity import TOL, base_fmt, rel_fro, to_dev
+
+pytestmark = pytest.mark.gpu
+
+FMTS = ["f64", "f32", "f16", "f16_o16"]
+
+
+def run_tt(lrc, dev, cores64, fmt):
+    b = base_fmt(fmt)
+    rc = [oracle.rounded(c, b) for c in cores64]
+    dc = [to_dev(c, dev).to(lrc.storage_dtype(fmt)).contiguous() for c in rc]
+    dims = [c.shape[1] for c in cores64]
+    ranks = [1] + [c.shape[2] for c in cores64]
+    out = torch.full((int(np.prod(dims)),), float("nan"), dtype=lrc.output_dtype(fmt), device=dev)
+    lrc.tt_reconstruct(dc, dims, ranks, fmt, out)
+    torch.cuda.synchronize()
+    return out.double().cpu().numpy(), rc
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("dims,ranks", [
+    ((3, 4), (1, 2, 1)),
+    ((5, 7, 3), (1, 2, 3, 1)),
+    ((2, 3, 2, 3, 2), (1, 2, 3, 3, 2, 1)),
+    ((1, 9, 1, 4), (1, 1, 2, 2, 1)),
+    ((300, 5), (1, 4, 1)),
+])
+def test_integer_cores_exact(lrc, cuda, fmt, dims, ranks):
+    cores = [W.integer_valued((ranks[l], dims[l], ranks[l + 1]), 50 + l, -2, 2) for l in range(len(dims))]
+    got, rc = run_tt(lrc, cuda, cores, fmt)
+    want = oracle.tt_full(rc).reshape(-1)
+    assert np.array_equal(got, want)
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("dims,r,kind", [
+    ((37, 29, 41), 9, "gauss_geo"),
+    ((8, 9, 7, 6, 5), 11, "gauss_alg"),
+    ((130, 70), 33, "gauss_geo"),
+    ((64, 48, 224), 52, "smooth"),
+    ((16,) * 5, 28, "gauss_alg"),
+])
+def test_random_cores_vs_oracle(lrc, cuda, fmt, dims, r, kind):
+    cores = W.make_tt(dims, W.capped_ranks(dims, r), kind, 17)
+    got, rc = run_tt(lrc, cuda, cores, fmt)
+    want = oracle.tt_full(rc).reshape(-1)
+    err = rel_fro(got, want)
+    assert err <= TOL[fmt], (fmt, err)
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("name", ["tt3", "tt6", "tt_hsi"])
+def test_workloads_sampled_entries(lrc, cuda, fmt, name):
+    """The three TT workloads at full size, in the bench's launch
+    configuration; 20000 seeded entries checked with the oracle's
+    independent entry evaluator."""
+    cfg = W.TT_CONFIGS[name]
+    cores = W.tt_cores(cfg, base_fmt(fmt))
+    got, rc = run_tt(lrc, cuda, cores, fmt)
+    idx = W.sample_indices(20000, got.size, 3)
+    want = oracle.tt_entries(rc, idx)
+    err = rel_fro(got[idx], want)
+    assert err <= TOL[fmt], (name, fmt, err)
+    assert np.isfinite(got).all()
