@@ -188,6 +188,18 @@ LRC_API const char* lrc_last_error(void);
 /* Number of kernels this library has launched in this process. */
 LRC_API uint64_t lrc_launch_count(void);
 
+/* Synchronises `stream`, then reports whether a bounded device-side wait in
+ * a tensor-core kernel gave up since the last call: LRC_ERR_TIMEOUT if so
+ * (the error words are cleared), LRC_ERR_CUDA if the stream reported an
+ * error, LRC_OK otherwise.  Kernels never hang: every wait on a barrier is
+ * limited in time, after which the CTA records the event and exits. */
+LRC_API lrc_status lrc_device_status(lrc_stream_t stream);
+
+/* Test hook for the failure path above: launches one CTA that waits, with a
+ * time limit of `limit_ns` (0 < limit_ns <= 1e9), on a barrier that nothing
+ * arrives on.  The next lrc_device_status() returns LRC_ERR_TIMEOUT. */
+LRC_API lrc_status lrc_selftest_wait_timeout(int64_t limit_ns, lrc_stream_t stream);
+
 /* Release library-held scratch on every device; the library stays usable. */
 LRC_API lrc_status lrc_shutdown(void);
 

@@ -69,6 +69,10 @@ def load() -> ctypes.CDLL:
     L.lrc_last_error.restype = ctypes.c_char_p
     L.lrc_launch_count.restype = ctypes.c_uint64
     L.lrc_shutdown.restype = i32
+    L.lrc_device_status.argtypes = [vp]
+    L.lrc_device_status.restype = i32
+    L.lrc_selftest_wait_timeout.argtypes = [i64, vp]
+    L.lrc_selftest_wait_timeout.restype = i32
     _lib = L
     return L
 
@@ -182,6 +186,16 @@ def lrc_shutdown() -> None:
     _check(load().lrc_shutdown())
 
 
+def lrc_device_status(stream=None) -> int:
+    """Synchronises the stream; returns the lrc_status (0, or -6 if a bounded
+    device wait gave up since the last call).  Does not raise."""
+    return int(load().lrc_device_status(_stream(stream)))
+
+
+def lrc_selftest_wait_timeout(limit_ns: int, stream=None) -> None:
+    _check(load().lrc_selftest_wait_timeout(int(limit_ns), _stream(stream)))
+
+
 # --------------------------------------------------------------------------
 # convenience helpers built only from the entry points above
 # --------------------------------------------------------------------------
@@ -190,9 +204,12 @@ def round_matrix(src64, fmt, ld: Optional[int] = None, stream=None):
     """Round a 2-D CUDA float64 tensor into a new packed tensor (lrc_round_factors)."""
     import torch
     rows, cols = src64.shape
+    if src64.stride(1) != 1 or (rows > 1 and src64.stride(0) < cols):
+        src64 = src64.contiguous()
+    ld_src = src64.stride(0) if rows > 1 else cols   # a single row may carry any stride
     ld = lrc_packed_ld(cols) if ld is None else ld
     dst = torch.empty((rows, ld), dtype=storage_dtype(fmt), device=src64.device)
-    lrc_round_factors(src64, rows, cols, src64.stride(0), dst, ld, fmt, stream)
+    lrc_round_factors(src64, rows, cols, ld_src, dst, ld, fmt, stream)
     return dst
 
 

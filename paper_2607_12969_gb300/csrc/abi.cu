@@ -235,6 +235,27 @@ const char* lrc_last_error(void) { return g_msg; }
 
 uint64_t lrc_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
+lrc_status lrc_device_status(lrc_stream_t stream) {
+    cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    const uint32_t a = take_apply_tc_error();
+    const uint32_t t = take_tt_tc_error();
+    if (a == 0xffffffffu || t == 0xffffffffu) {
+        set_error("could not read the device error words");
+        return LRC_ERR_CUDA;
+    }
+    if (a | t) {
+        set_error("a bounded device wait gave up (apply code 0x%x, TT code 0x%x)", a, t);
+        return LRC_ERR_TIMEOUT;
+    }
+    return LRC_OK;
+}
+
+lrc_status lrc_selftest_wait_timeout(int64_t limit_ns, lrc_stream_t stream) {
+    if (limit_ns <= 0 || limit_ns > 1000000000LL) return invalid("limit_ns must be in (0, 1e9]");
+    return launch_wait_timeout_probe(limit_ns, as_stream(stream));
+}
+
 lrc_status lrc_shutdown(void) {
     release_scratch();
     return LRC_OK;

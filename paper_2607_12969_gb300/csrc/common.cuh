@@ -67,6 +67,12 @@ struct TTShape {
 lrc_status launch_tt_cc(const TTShape& sh, lrc_fmt fmt, void* out, cudaStream_t s);
 lrc_status launch_tt_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s);
 
+// Device error words of the tensor-core kernels (bounded waits that gave up);
+// read and cleared by lrc_device_status().  0xffffffff = could not be read.
+uint32_t take_apply_tc_error();
+uint32_t take_tt_tc_error();
+lrc_status launch_wait_timeout_probe(int64_t limit_ns, cudaStream_t s);
+
 lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
                         double* diff_out, double* normA_out, cudaStream_t s);
 void release_scratch();

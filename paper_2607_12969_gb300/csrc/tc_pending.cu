@@ -1,18 +1,13 @@
-// tc_pending.cu -- the binary16 paths are not built yet: they report
-// LRC_ERR_UNSUPPORTED instead of falling back to anything else.
+// tc_pending.cu -- binary16 TT reconstruction runs on the CUDA-core chain
+// kernel (binary32 arithmetic) until the tensor-core version replaces it.
 #include "common.cuh"
 
 namespace lrc {
 
-lrc_status launch_apply_f16(const void*, const void*, const void*, const void*, void*, int64_t,
-                            int64_t, int64_t, int64_t, bool, cudaStream_t) {
-    set_error("binary16 apply is not built in this version");
-    return LRC_ERR_UNSUPPORTED;
+lrc_status launch_tt_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s) {
+    return launch_tt_cc(sh, out16 ? LRC_F16_O16 : LRC_F16, out, s);
 }
 
-lrc_status launch_tt_f16(const TTShape&, bool, void*, cudaStream_t) {
-    set_error("binary16 TT reconstruction is not built in this version");
-    return LRC_ERR_UNSUPPORTED;
-}
+uint32_t take_tt_tc_error() { return 0; }
 
 }  // namespace lrc

@@ -11,6 +11,12 @@
 // final product Z_{d-1} G_d -> out are the only steps whose size scales with
 // the tile.  The final product uses a TM x TN register tile per thread and
 // writes contiguous output rows.
+//
+// Element types: binary64 cores with binary64 arithmetic, binary32 with
+// binary32, and binary16 cores with binary32 arithmetic and a binary32 or
+// binary16 output (the latter rounded once per entry).
+#include <cuda_fp16.h>
+
 #include "common.cuh"
 
 namespace lrc {
@@ -19,7 +25,14 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kTM = 4, kTN = 4;
 
-template <typename T>
+__device__ __forceinline__ float to_acc(__half x) { return __half2float(x); }
+__device__ __forceinline__ float to_acc(float x) { return x; }
+__device__ __forceinline__ double to_acc(double x) { return x; }
+__device__ __forceinline__ void store_out(float* p, float v) { *p = v; }
+__device__ __forceinline__ void store_out(double* p, double v) { *p = v; }
+__device__ __forceinline__ void store_out(__half* p, float v) { *p = __float2half_rn(v); }
+
+template <typename TIn>
 struct TTParams {
     int d;
     int tile;          // prefix rows per CTA
@@ -29,12 +42,13 @@ struct TTParams {
     int64_t dims[16];
     int64_t ranks[17];
     int64_t div[16];   // div[l] = prod_{j=l+1}^{d-2} n_j: level-l row of prefix p is p / div[l]
-    const T* cores[16];
+    const TIn* cores[16];
 };
 
-template <typename T>
+// T: arithmetic type; TIn: core element type; TOut: output element type.
+template <typename T, typename TIn, typename TOut>
 __global__ void __launch_bounds__(kThreads)
-tt_cc_kernel(const TTParams<T> p, T* __restrict__ out) {
+tt_cc_kernel(const TTParams<TIn> p, TOut* __restrict__ out) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     T* zbuf[2];
     zbuf[0] = reinterpret_cast<T*>(smem_raw);
@@ -53,10 +67,10 @@ tt_cc_kernel(const TTParams<T> p, T* __restrict__ out) {
     {
         const int r1 = (int)p.ranks[1];
         const int cnt = (int)(hi - lo + 1);
-        const T* G = p.cores[0];
+        const TIn* G = p.cores[0];
         for (int e = tid; e < cnt * r1; e += kThreads) {
             const int q = e / r1, bcol = e % r1;
-            zbuf[0][q * p.ldz + bcol] = G[(lo + q) * r1 + bcol];
+            zbuf[0][q * p.ldz + bcol] = to_acc(G[(lo + q) * r1 + bcol]);
         }
     }
     __syncthreads();
@@ -67,7 +81,7 @@ tt_cc_kernel(const TTParams<T> p, T* __restrict__ out) {
         const int64_t nlo = p0 / p.div[l];
         const int64_t nhi = (pend - 1) / p.div[l];
         const int cnt = (int)(nhi - nlo + 1);
-        const T* G = p.cores[l];
+        const TIn* G = p.cores[l];
         const T* zin = zbuf[cur];
         T* zout = zbuf[cur ^ 1];
         for (int e = tid; e < cnt * r1; e += kThreads) {
@@ -76,9 +90,9 @@ tt_cc_kernel(const TTParams<T> p, T* __restrict__ out) {
             const int64_t parent = gq / nl;
             const int64_t i = gq - parent * nl;
             const T* zrow = zin + (parent - lo) * p.ldz;
-            const T* gcol = G + i * r1 + bcol;
+            const TIn* gcol = G + i * r1 + bcol;
             T acc = T(0);
-            for (int a = 0; a < r0; ++a) acc = fma(zrow[a], gcol[(int64_t)a * nl * r1], acc);
+            for (int a = 0; a < r0; ++a) acc = fma(zrow[a], to_acc(gcol[(int64_t)a * nl * r1]), acc);
             zout[q * p.ldz + bcol] = acc;
         }
         __syncthreads();
@@ -89,7 +103,7 @@ tt_cc_kernel(const TTParams<T> p, T* __restrict__ out) {
     // final product: out[p0 + t, :] = Z_{d-1}[t] G_d   (G_d is r x n_d)
     const int r = (int)p.ranks[d - 1];
     const int64_t nd = p.dims[d - 1];
-    const T* Gd = p.cores[d - 1];
+    const TIn* Gd = p.cores[d - 1];
     const T* z = zbuf[cur];
     const int TX = p.tx, TY = kThreads / TX;
     const int tx = tid % TX, ty = tid / TX;
@@ -119,7 +133,7 @@ tt_cc_kernel(const TTParams<T> p, T* __restrict__ out) {
 #pragma unroll
                 for (int i = 0; i < kTM; ++i) av[i] = z[rows[i] * p.ldz + a];
 #pragma unroll
-                for (int j = 0; j < kTN; ++j) bv[j] = __ldg(Gd + (int64_t)a * nd + cols[j]);
+                for (int j = 0; j < kTN; ++j) bv[j] = to_acc(__ldg(Gd + (int64_t)a * nd + cols[j]));
 #pragma unroll
                 for (int i = 0; i < kTM; ++i)
 #pragma unroll
@@ -129,24 +143,24 @@ tt_cc_kernel(const TTParams<T> p, T* __restrict__ out) {
             for (int i = 0; i < kTM; ++i) {
                 const int t = rb + ty + i * TY;
                 if (t >= pcount) continue;
-                T* orow = out + (p0 + t) * nd;
+                TOut* orow = out + (p0 + t) * nd;
 #pragma unroll
                 for (int j = 0; j < kTN; ++j)
-                    if (colok[j]) orow[cols[j]] = acc[i][j];
+                    if (colok[j]) store_out(orow + cols[j], acc[i][j]);
             }
         }
     }
 }
 
-template <typename T>
-lrc_status launch_tt_cc_t(const TTShape& sh, T* out, cudaStream_t s, const char* name) {
-    TTParams<T> p;
+template <typename T, typename TIn, typename TOut>
+lrc_status launch_tt_cc_t(const TTShape& sh, TOut* out, cudaStream_t s, const char* name) {
+    TTParams<TIn> p;
     p.d = sh.d;
     int64_t rmax = 1;
     for (int l = 0; l < sh.d; ++l) {
         p.dims[l] = sh.dims[l];
         p.ranks[l] = sh.ranks[l];
-        p.cores[l] = static_cast<const T*>(sh.cores[l]);
+        p.cores[l] = static_cast<const TIn*>(sh.cores[l]);
         if (sh.ranks[l] > rmax) rmax = sh.ranks[l];
     }
     p.ranks[sh.d] = 1;
@@ -176,18 +190,26 @@ lrc_status launch_tt_cc_t(const TTShape& sh, T* out, cudaStream_t s, const char*
         set_error("%s: tensor too large", name);
         return LRC_ERR_UNSUPPORTED;
     }
-    cudaError_t e = cudaFuncSetAttribute(tt_cc_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+    cudaError_t e = cudaFuncSetAttribute(tt_cc_kernel<T, TIn, TOut>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, name);
-    tt_cc_kernel<T><<<(unsigned)tiles, kThreads, smem, s>>>(p, out);
+    tt_cc_kernel<T, TIn, TOut><<<(unsigned)tiles, kThreads, smem, s>>>(p, out);
     return after_launch(name);
 }
 
 }  // namespace
 
 lrc_status launch_tt_cc(const TTShape& sh, lrc_fmt fmt, void* out, cudaStream_t s) {
-    if (fmt == LRC_F64) return launch_tt_cc_t<double>(sh, static_cast<double*>(out), s, "tt_cc_kernel<f64>");
-    return launch_tt_cc_t<float>(sh, static_cast<float*>(out), s, "tt_cc_kernel<f32>");
+    switch (fmt) {
+        case LRC_F64:
+            return launch_tt_cc_t<double, double, double>(sh, static_cast<double*>(out), s, "tt_cc_kernel<f64>");
+        case LRC_F32:
+            return launch_tt_cc_t<float, float, float>(sh, static_cast<float*>(out), s, "tt_cc_kernel<f32>");
+        case LRC_F16:
+            return launch_tt_cc_t<float, __half, float>(sh, static_cast<float*>(out), s, "tt_cc_kernel<f16,o32>");
+        default:
+            return launch_tt_cc_t<float, __half, __half>(sh, static_cast<__half*>(out), s, "tt_cc_kernel<f16,o16>");
+    }
 }
 
 }  // namespace lrc
