@@ -166,6 +166,32 @@ LRC_API lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims,
 LRC_API lrc_status lrc_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
                         double* diff_out, double* normA_out, lrc_stream_t stream);
 
+/*
+ * lrc_fro_diff_noalloc -- the same reduction as lrc_fro_diff for callers that
+ * must not allocate device memory.  The paper has no counterpart: this is a
+ * deployment variant.  Callers that run under a fixed device-memory budget
+ * whose memory is owned by another allocator (a serving framework's caching
+ * pool, say), or that cannot afford the implicit device synchronisation a
+ * cudaMalloc can cause in the middle of a latency-critical loop, can use it:
+ * it calls no cudaMalloc, cudaFree or other allocating routine.
+ *
+ * Arguments and results are those of lrc_fro_diff; A and B are still the
+ * caller's buffers.  The per-block partial sums live in a fixed array of
+ * 8194 doubles (about 64 KB) compiled into the library, which every GPU that
+ * loads the library keeps until the process exits.  That array bounds the
+ * input: count <= 268435456 (4096 blocks x 65536 elements); a larger count
+ * returns LRC_ERR_INVALID_ARG without launching.  The first call on each
+ * device looks up the array's device address (cudaGetSymbolAddress) with that
+ * device current; make that first call before any stream capture.  All calls
+ * share the one array and every call overwrites the entries it uses, so no
+ * state carries over between calls, but calls whose kernels overlap on the
+ * GPU (different streams, other threads) race on it and must be serialised by
+ * the caller.  Synchronises `stream`.
+ */
+LRC_API lrc_status lrc_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb,
+                                        int64_t count, double* diff_out, double* normA_out,
+                                        lrc_stream_t stream);
+
 /* Thm 4.1 Eq. matrix_condition and Thm 6.1 Eq. tt_condition:
  * returns 1 if e_aug + eta <= e_base (certified non-increase), else 0. */
 LRC_API int lrc_certified(double e_base, double e_aug, double eta);

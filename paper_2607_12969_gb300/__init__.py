@@ -56,6 +56,8 @@ def load() -> ctypes.CDLL:
     L.tt_reconstruct.restype = i32
     L.lrc_fro_diff.argtypes = [vp, i32, vp, i32, i64, vp, vp, vp]
     L.lrc_fro_diff.restype = i32
+    L.lrc_fro_diff_noalloc.argtypes = [vp, i32, vp, i32, i64, vp, vp, vp]
+    L.lrc_fro_diff_noalloc.restype = i32
     L.lrc_certified.argtypes = [dbl, dbl, dbl]
     L.lrc_certified.restype = i32
     L.lrc_tail_error.argtypes = [vp, i64, i64]
@@ -153,6 +155,16 @@ def lrc_fro_diff(A, fa, B, fb, count: int, stream=None) -> Tuple[float, float]:
     norm = ctypes.c_double(0.0)
     _check(load().lrc_fro_diff(_ptr(A), _fmt(fa), _ptr(B), _fmt(fb) if B is not None else 0, count,
                                ctypes.addressof(diff), ctypes.addressof(norm), _stream(stream)))
+    return diff.value, norm.value
+
+
+def lrc_fro_diff_noalloc(A, fa, B, fb, count: int, stream=None) -> Tuple[float, float]:
+    """lrc_fro_diff without any device allocation (scratch is a fixed array
+    inside the library); at most 268435456 elements.  Returns (||A - B||_F, ||A||_F)."""
+    diff = ctypes.c_double(0.0)
+    norm = ctypes.c_double(0.0)
+    _check(load().lrc_fro_diff_noalloc(_ptr(A), _fmt(fa), _ptr(B), _fmt(fb) if B is not None else 0, count,
+                                       ctypes.addressof(diff), ctypes.addressof(norm), _stream(stream)))
     return diff.value, norm.value
 
 

@@ -190,6 +190,25 @@ lrc_status lrc_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, in
     return run_fro_diff(A, fa, B, fb, count, diff_out, normA_out, as_stream(stream));
 }
 
+lrc_status lrc_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
+                                double* diff_out, double* normA_out, lrc_stream_t stream) {
+    if (!valid_fmt(fa) || !valid_fmt(fb)) return invalid("unknown format");
+    if (count < 0) return invalid("negative count");
+    if (!diff_out) return invalid("null diff_out");
+    if (count > fro_diff_noalloc_max_count())
+        return invalid("lrc_fro_diff_noalloc handles at most %lld elements (got %lld)",
+                       (long long)fro_diff_noalloc_max_count(), (long long)count);
+    if (count > 0 && !A) return invalid("null A");
+    if (count > 0 && !aligned16(A)) return misaligned("A");
+    if (B && !aligned16(B)) return misaligned("B");
+    if (count == 0) {
+        *diff_out = 0.0;
+        if (normA_out) *normA_out = 0.0;
+        return LRC_OK;
+    }
+    return run_fro_diff_noalloc(A, fa, B, fb, count, diff_out, normA_out, as_stream(stream));
+}
+
 int lrc_certified(double e_base, double e_aug, double eta) { return (e_aug + eta <= e_base) ? 1 : 0; }
 
 double lrc_tail_error(const double* sigma, int64_t len, int64_t k) {

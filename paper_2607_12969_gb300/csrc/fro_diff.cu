@@ -209,6 +209,73 @@ lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, in
     return LRC_OK;
 }
 
+// ---------------------------------------------------------------------------
+// Allocation-free variant.  The per-block partial sums go to a fixed array in
+// device memory that is part of the loaded library image, so the call never
+// allocates.  Its size caps the element count: one block per
+// kStaticElemsPerBlock elements, at most kStaticBlocks blocks.
+// ---------------------------------------------------------------------------
+namespace {
+constexpr int kStaticBlocks = 4096;
+constexpr int64_t kStaticElemsPerBlock = 65536;   // 256 threads x 32 groups of 8
+static __device__ __align__(256) double g_fro_static_scratch[2 * kStaticBlocks + 2];
+std::mutex g_static_mu;
+double* g_static_ptr[64] = {nullptr};             // device address of the array, per device
+}  // namespace
+
+int64_t fro_diff_noalloc_max_count() { return (int64_t)kStaticBlocks * kStaticElemsPerBlock; }
+
+lrc_status run_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
+                                double* diff_out, double* normA_out, cudaStream_t s) {
+    if (count > fro_diff_noalloc_max_count()) {
+        set_error("lrc_fro_diff_noalloc handles at most %lld elements (got %lld)",
+                  (long long)fro_diff_noalloc_max_count(), (long long)count);
+        return LRC_ERR_INVALID_ARG;
+    }
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= 64) {
+        set_error("device ordinal %d out of range", dev);
+        return LRC_ERR_UNSUPPORTED;
+    }
+    double* partial;
+    {
+        // one-time set-up per device, with that device current: the host-side
+        // name of the array is not a device address, so look the address up
+        std::lock_guard<std::mutex> lock(g_static_mu);
+        if (!g_static_ptr[dev]) {
+            void* p = nullptr;
+            e = cudaGetSymbolAddress(&p, g_fro_static_scratch);
+            if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress (fro_diff scratch)");
+            g_static_ptr[dev] = static_cast<double*>(p);
+        }
+        partial = g_static_ptr[dev];
+    }
+    int grid = (int)((count + kStaticElemsPerBlock - 1) / kStaticElemsPerBlock);
+    if (grid < 1) grid = 1;
+    const int a = fcode(fa), b = B ? fcode(fb) : -1;
+    switch (a) {
+        case 0: launch_partial<0>(b, grid, A, B, count, partial, s); break;
+        case 1: launch_partial<1>(b, grid, A, B, count, partial, s); break;
+        default: launch_partial<2>(b, grid, A, B, count, partial, s); break;
+    }
+    lrc_status st = after_launch("fro_partial_kernel (no-alloc)");
+    if (st != LRC_OK) return st;
+    double* result = partial + 2 * kStaticBlocks;
+    fro_final_kernel<<<1, 1024, 0, s>>>(partial, grid, result);
+    st = after_launch("fro_final_kernel (no-alloc)");
+    if (st != LRC_OK) return st;
+    double host[2];
+    e = cudaMemcpyAsync(host, result, sizeof host, cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (fro_diff no-alloc result)");
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize (fro_diff no-alloc)");
+    *diff_out = host[0];
+    if (normA_out) *normA_out = host[1];
+    return LRC_OK;
+}
+
 void release_scratch() {
     std::lock_guard<std::mutex> lock(g_mu);
     int prev = -1;
