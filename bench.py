@@ -493,6 +493,59 @@ def run_oracle_timing(steps: int, warmup: int):
 # main
 # ---------------------------------------------------------------------------
 
+def run_case(args):
+    """One call type at chosen sizes, launched `--reps` times after one warm-up
+    (the command ncu captures)."""
+    import torch
+    import paper_2607_12969_gb300 as lrc
+    lrc.load()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    fmt = args.fmt
+    base = "f16" if fmt.startswith("f16") else fmt
+    if args.case == "apply":
+        m, n, b, k = args.m, args.n, args.b, args.k
+        f = W.random_factors(m, n, k, seed=7)
+        X = W.gaussian((b, n), 8)
+        mk = lambda a: lrc.round_matrix(torch.from_numpy(a if a.ndim == 2 else a[None, :]).to(dev), fmt)  # noqa: E731
+        U, S, V, Xd = mk(f.U), mk(f.s), mk(f.Vt), mk(X)
+        Y = torch.empty((b, m), dtype=lrc.output_dtype(fmt), device=dev)
+        call = lambda: lrc.lrc_apply(U, S, V, Xd, Y, m, n, k, b, fmt)  # noqa: E731
+        work = work_apply(m, n, k, b, fmt)
+    elif args.case == "tt":
+        cfg = W.TT_CONFIGS[args.tt]
+        cores = [torch.from_numpy(c).to(dev).to(lrc.storage_dtype(fmt)).contiguous() for c in W.tt_cores(cfg, base)]
+        ranks = cfg.ranks[base]
+        out = torch.empty(int(np.prod(cfg.dims)), dtype=lrc.output_dtype(fmt), device=dev)
+        call = lambda: lrc.tt_reconstruct(cores, cfg.dims, ranks, fmt, out)  # noqa: E731
+        work = work_tt(cfg.dims, ranks, fmt)
+    elif args.case == "fro":
+        a = torch.randn(args.count, dtype=torch.float64, device=dev)
+        b2 = torch.randn(args.count, dtype=torch.float64, device=dev)
+        call = lambda: lrc.lrc_fro_diff(a, "f64", b2, "f64", args.count)  # noqa: E731
+        work = work_fro(args.count, "f64", "f64")
+    else:  # round
+        src = torch.randn(args.b, args.n, dtype=torch.float64, device=dev)
+        dst = torch.empty(args.b, args.n, dtype=lrc.storage_dtype(fmt), device=dev)
+        call = lambda: lrc.lrc_round_factors(src, args.b, args.n, args.n, dst, args.n, fmt)  # noqa: E731
+        work = work_round(args.b, args.n, args.n, fmt)
+    call()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.reps):
+        call()
+    e1.record()
+    torch.cuda.synchronize()
+    st = lrc.lrc_device_status()
+    ms = e0.elapsed_time(e1) / args.reps
+    print(json.dumps({"case": args.case, "fmt": fmt, "ms": ms, "status": st,
+                      "GBps": work["bytes"] / (ms * 1e-3) / 1e9,
+                      "TFLOPs": work["flops"] / (ms * 1e-3) / 1e12,
+                      "roofline_frac": roofline_time(work) / (ms * 1e-3)}))
+    return 0 if st == 0 else 1
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -500,7 +553,19 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--case", choices=["apply", "tt", "fro", "round"], default=None,
+                    help="time one call type instead of the step (profiling captures)")
+    ap.add_argument("--fmt", default="f16")
+    ap.add_argument("--m", type=int, default=16384)
+    ap.add_argument("--n", type=int, default=8192)
+    ap.add_argument("--b", type=int, default=2048)
+    ap.add_argument("--k", type=int, default=144)
+    ap.add_argument("--tt", default="tt3")
+    ap.add_argument("--count", type=int, default=1 << 26)
+    ap.add_argument("--reps", type=int, default=3)
     args = ap.parse_args()
+    if args.case:
+        return run_case(args)
     world, rank, local = dist_env()
 
     if args.impl == "reference":

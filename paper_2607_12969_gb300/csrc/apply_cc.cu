@@ -1,170 +1,201 @@
 // apply_cc.cu -- fused low-rank apply on the CUDA cores, binary64 and binary32
 // (Sec. 4.4, Eq. gpu_matrix_apply: Y = [(X V) diag(s)] U^T).
 //
-// One CTA owns BM query rows and a range of output columns of Y.
-//   phase 1: W = X[rows, :] V, reduced over n in BK-wide slabs staged in
-//            shared memory, in BN-wide chunks of the rank dimension;
+// A CTA owns BM query rows (a row tile) and a range of Y's columns; CTAs loop
+// over row tiles (persistent grid).
+//   phase 1: W = X[rows, :] V, reduced over n in BK1-wide slabs staged in
+//            shared memory, in BN-wide chunks of the rank dimension; the last
+//            chunk only computes the 16-wide column groups below k rounded
+//            up to 16, so no arithmetic is spent on rank padding.
 //            W <- W diag(s) is applied as each chunk finishes and the scaled
 //            chunk is kept (transposed) in shared memory -- it never reaches
 //            global memory;
 //   phase 2: Y[rows, m-tile] = W U[m-tile, :]^T for every BN-wide m-tile of
-//            the CTA's range, with U staged through shared memory.
-// Each thread owns a TM x TN register tile of the current output tile, with
-// rows strided by BM/TM and columns strided by BN/TN so that the shared-memory
+//            the CTA's range, with U staged through shared memory and the
+//            reduction running over k rounded up to 16 only.
+// Each thread owns a TM x TN register tile of the current output tile, rows
+// strided by BM/TM and columns strided by BN/TN, so that the shared-memory
 // reads of a warp are conflict-free; staging buffers are padded by one
 // element per row so that the transposing stores are conflict-free too.
-// binary32 adds each BK slab's partial sums to the running sums separately
-// (blocked accumulation) so the rounding error grows like sqrt(n / BK).
+//
+// binary64 (DFMA-bound: the GB300 issues about 2 DFMA per clock per SM) uses
+// thin 8-row tiles and many CTAs per SM, so the work spreads evenly over the
+// SMs; binary32 uses 64-row tiles with 4 x 4 register tiles and adds each
+// slab's partial sums to the running sums separately (blocked accumulation,
+// rounding error growing like sqrt(n / BK1)).
 #include "common.cuh"
 
 namespace lrc {
 namespace {
 
-constexpr int kThreads = 256;
-
 template <typename T>
-struct Tile;
+struct Cfg;
 template <>
-struct Tile<double> {  // binary64: BM x BN = 32 x 64, 2 x 4 per thread
-    static constexpr int BM = 32, BN = 64, BK = 16, TM = 2, TN = 4;
+struct Cfg<double> {
+    static constexpr int BM = 8, BN = 64, BK1 = 32, BK2 = 16, TM = 1, TN = 4, THREADS = 128;
     static constexpr bool kBlocked = false;
+    static constexpr int kCtasPerSm = 8;
 };
 template <>
-struct Tile<float> {   // binary32: 64 x 64, 4 x 4 per thread
-    static constexpr int BM = 64, BN = 64, BK = 32, TM = 4, TN = 4;
+struct Cfg<float> {
+    static constexpr int BM = 64, BN = 64, BK1 = 32, BK2 = 16, TM = 4, TN = 4, THREADS = 256;
     static constexpr bool kBlocked = true;
+    static constexpr int kCtasPerSm = 2;
 };
 
 template <typename T>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(Cfg<T>::THREADS)
 apply_cc_kernel(const T* __restrict__ U, const T* __restrict__ S, const T* __restrict__ Vt,
                 const T* __restrict__ X, T* __restrict__ Y, int64_t m, int64_t n, int k, int64_t b,
-                int64_t ldk, int64_t ldn, int kpad, int64_t m_chunk) {
-    using P = Tile<T>;
-    constexpr int BM = P::BM, BN = P::BN, BK = P::BK, TM = P::TM, TN = P::TN;
-    constexpr int TX = BN / TN;            // threads along columns
+                int64_t ldk, int64_t ldn, int kp16, int64_t ntiles, int64_t m_chunk) {
+    using P = Cfg<T>;
+    constexpr int BM = P::BM, BN = P::BN, BK1 = P::BK1, BK2 = P::BK2, TM = P::TM, TN = P::TN;
+    constexpr int NT = P::THREADS;
+    constexpr int TX = BN / TN;            // threads along columns (16)
     constexpr int TY = BM / TM;            // threads along rows
     constexpr int LDA = BM + 1, LDB = BN + 1;
-    static_assert(TY * TX == kThreads, "thread tile");
+    static_assert(TY * TX == NT, "thread tile");
+    static_assert(TX == 16, "16-wide column groups");
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    T* Ws = reinterpret_cast<T*>(smem_raw);            // [kpad][BM]   scaled W, transposed
-    T* As = Ws + (size_t)kpad * BM;                     // [BK][LDA]    X slab, transposed
-    T* Bs = As + BK * LDA;                              // [BK][LDB]    Vt / U slab, transposed
+    T* Ws = reinterpret_cast<T*>(smem_raw);            // [kp16][BM]   scaled W, transposed
+    T* As = Ws + (size_t)kp16 * BM;                     // [BK1][LDA]   X slab, transposed
+    T* Bs = As + BK1 * LDA;                             // [BK1][LDB]   Vt / U slab, transposed
 
     const int tid = threadIdx.x;
     const int tx = tid % TX, ty = tid / TX;
-    const int64_t row0 = (int64_t)blockIdx.x * BM;
     const int64_t mbeg = (int64_t)blockIdx.y * m_chunk;
     const int64_t mend = (mbeg + m_chunk < m) ? mbeg + m_chunk : m;
 
-    // ---------------- phase 1: W = X V, one BN-wide rank chunk at a time ----
-    for (int kc = 0; kc < kpad; kc += BN) {
-        T acc[TM][TN];
-#pragma unroll
-        for (int i = 0; i < TM; ++i)
-#pragma unroll
-            for (int j = 0; j < TN; ++j) acc[i][j] = T(0);
-        for (int64_t k0 = 0; k0 < n; k0 += BK) {
-            // X slab: BM rows x BK cols -> As[c][r]
-            for (int e = tid; e < BM * BK; e += kThreads) {
-                const int r = e / BK, c = e % BK;
-                const int64_t gr = row0 + r, gc = k0 + c;
-                As[c * LDA + r] = (gr < b && gc < n) ? X[gr * ldn + gc] : T(0);
-            }
-            // Vt slab: BN rank rows x BK cols -> Bs[c][j]
-            for (int e = tid; e < BN * BK; e += kThreads) {
-                const int j = e / BK, c = e % BK;
-                const int gj = kc + j;
-                const int64_t gc = k0 + c;
-                Bs[c * LDB + j] = (gj < k && gc < n) ? Vt[(int64_t)gj * ldn + gc] : T(0);
-            }
-            __syncthreads();
-            T part[TM][TN];
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int64_t row0 = tile * BM;
+        // ------------- phase 1: W = X V, one BN-wide rank chunk at a time --------
+        for (int kc = 0; kc < kp16; kc += BN) {
+            const int jmax = (kp16 - kc) / TX < TN ? (kp16 - kc) / TX : TN;   // 16-wide groups in use
+            const int rows_v = jmax * TX;
+            T acc[TM][TN];
 #pragma unroll
             for (int i = 0; i < TM; ++i)
 #pragma unroll
-                for (int j = 0; j < TN; ++j) part[i][j] = P::kBlocked ? T(0) : acc[i][j];
-#pragma unroll 4
-            for (int c = 0; c < BK; ++c) {
-                T a[TM], bb[TN];
-#pragma unroll
-                for (int i = 0; i < TM; ++i) a[i] = As[c * LDA + ty + i * TY];
-#pragma unroll
-                for (int j = 0; j < TN; ++j) bb[j] = Bs[c * LDB + tx + j * TX];
-#pragma unroll
-                for (int i = 0; i < TM; ++i)
-#pragma unroll
-                    for (int j = 0; j < TN; ++j) part[i][j] = fma(a[i], bb[j], part[i][j]);
-            }
-#pragma unroll
-            for (int i = 0; i < TM; ++i)
-#pragma unroll
-                for (int j = 0; j < TN; ++j) acc[i][j] = P::kBlocked ? acc[i][j] + part[i][j] : part[i][j];
-            __syncthreads();
-        }
-        // W <- W diag(s), kept transposed in shared memory
-#pragma unroll
-        for (int j = 0; j < TN; ++j) {
-            const int gj = kc + tx + j * TX;
-            const T sj = (gj < k) ? S[gj] : T(0);
-#pragma unroll
-            for (int i = 0; i < TM; ++i) Ws[(size_t)gj * BM + ty + i * TY] = acc[i][j] * sj;
-        }
-    }
-    __syncthreads();
-
-    // ---------------- phase 2: Y[rows, m-tile] = W U[m-tile, :]^T -----------
-    for (int64_t mt = mbeg; mt < mend; mt += BN) {
-        T acc[TM][TN];
-#pragma unroll
-        for (int i = 0; i < TM; ++i)
-#pragma unroll
-            for (int j = 0; j < TN; ++j) acc[i][j] = T(0);
-        for (int k0 = 0; k0 < kpad; k0 += BK) {
-            for (int e = tid; e < BN * BK; e += kThreads) {
-                const int j = e / BK, c = e % BK;
-                const int64_t gm = mt + j;
-                const int gc = k0 + c;
-                Bs[c * LDB + j] = (gm < mend && gc < k) ? U[gm * ldk + gc] : T(0);
-            }
-            __syncthreads();
-#pragma unroll 4
-            for (int c = 0; c < BK; ++c) {
-                T a[TM], bb[TN];
-#pragma unroll
-                for (int i = 0; i < TM; ++i) a[i] = Ws[(size_t)(k0 + c) * BM + ty + i * TY];
-#pragma unroll
-                for (int j = 0; j < TN; ++j) bb[j] = Bs[c * LDB + tx + j * TX];
+                for (int j = 0; j < TN; ++j) acc[i][j] = T(0);
+            for (int64_t k0 = 0; k0 < n; k0 += BK1) {
+                for (int e = tid; e < BM * BK1; e += NT) {
+                    const int r = e / BK1, c = e % BK1;
+                    const int64_t gr = row0 + r, gc = k0 + c;
+                    As[c * LDA + r] = (gr < b && gc < n) ? X[gr * ldn + gc] : T(0);
+                }
+                for (int e = tid; e < rows_v * BK1; e += NT) {
+                    const int j = e / BK1, c = e % BK1;
+                    const int gj = kc + j;
+                    const int64_t gc = k0 + c;
+                    Bs[c * LDB + j] = (gj < k && gc < n) ? Vt[(int64_t)gj * ldn + gc] : T(0);
+                }
+                __syncthreads();
+                T part[TM][TN];
 #pragma unroll
                 for (int i = 0; i < TM; ++i)
 #pragma unroll
-                    for (int j = 0; j < TN; ++j) acc[i][j] = fma(a[i], bb[j], acc[i][j]);
-            }
-            __syncthreads();
-        }
+                    for (int j = 0; j < TN; ++j) part[i][j] = P::kBlocked ? T(0) : acc[i][j];
+                if (jmax == TN) {
+#pragma unroll 4
+                    for (int c = 0; c < BK1; ++c) {
+                        T a[TM], bb[TN];
 #pragma unroll
-        for (int i = 0; i < TM; ++i) {
-            const int64_t gr = row0 + ty + i * TY;
-            if (gr >= b) continue;
+                        for (int i = 0; i < TM; ++i) a[i] = As[c * LDA + ty + i * TY];
+#pragma unroll
+                        for (int j = 0; j < TN; ++j) bb[j] = Bs[c * LDB + tx + j * TX];
+#pragma unroll
+                        for (int i = 0; i < TM; ++i)
+#pragma unroll
+                            for (int j = 0; j < TN; ++j) part[i][j] = fma(a[i], bb[j], part[i][j]);
+                    }
+                } else {
+                    for (int c = 0; c < BK1; ++c) {
+                        T a[TM];
+#pragma unroll
+                        for (int i = 0; i < TM; ++i) a[i] = As[c * LDA + ty + i * TY];
+#pragma unroll
+                        for (int j = 0; j < TN; ++j) {
+                            if (j < jmax) {
+                                const T bb = Bs[c * LDB + tx + j * TX];
+#pragma unroll
+                                for (int i = 0; i < TM; ++i) part[i][j] = fma(a[i], bb, part[i][j]);
+                            }
+                        }
+                    }
+                }
+#pragma unroll
+                for (int i = 0; i < TM; ++i)
+#pragma unroll
+                    for (int j = 0; j < TN; ++j)
+                        acc[i][j] = P::kBlocked ? acc[i][j] + part[i][j] : part[i][j];
+                __syncthreads();
+            }
+            // W <- W diag(s), kept transposed in shared memory
 #pragma unroll
             for (int j = 0; j < TN; ++j) {
-                const int64_t gm = mt + tx + j * TX;
-                if (gm < mend) Y[gr * m + gm] = acc[i][j];
+                if (j >= jmax) break;
+                const int gj = kc + tx + j * TX;
+                const T sj = (gj < k) ? S[gj] : T(0);
+#pragma unroll
+                for (int i = 0; i < TM; ++i) Ws[(size_t)gj * BM + ty + i * TY] = acc[i][j] * sj;
             }
         }
+        __syncthreads();
+
+        // ------------- phase 2: Y[rows, m-tile] = W U[m-tile, :]^T ---------------
+        for (int64_t mt = mbeg; mt < mend; mt += BN) {
+            T acc[TM][TN];
+#pragma unroll
+            for (int i = 0; i < TM; ++i)
+#pragma unroll
+                for (int j = 0; j < TN; ++j) acc[i][j] = T(0);
+            for (int k0 = 0; k0 < kp16; k0 += BK2) {
+                for (int e = tid; e < BN * BK2; e += NT) {
+                    const int j = e / BK2, c = e % BK2;
+                    const int64_t gm = mt + j;
+                    const int gc = k0 + c;
+                    Bs[c * LDB + j] = (gm < mend && gc < k) ? U[gm * ldk + gc] : T(0);
+                }
+                __syncthreads();
+#pragma unroll
+                for (int c = 0; c < BK2; ++c) {
+                    T a[TM], bb[TN];
+#pragma unroll
+                    for (int i = 0; i < TM; ++i) a[i] = Ws[(size_t)(k0 + c) * BM + ty + i * TY];
+#pragma unroll
+                    for (int j = 0; j < TN; ++j) bb[j] = Bs[c * LDB + tx + j * TX];
+#pragma unroll
+                    for (int i = 0; i < TM; ++i)
+#pragma unroll
+                        for (int j = 0; j < TN; ++j) acc[i][j] = fma(a[i], bb[j], acc[i][j]);
+                }
+                __syncthreads();
+            }
+#pragma unroll
+            for (int i = 0; i < TM; ++i) {
+                const int64_t gr = row0 + ty + i * TY;
+                if (gr >= b) continue;
+#pragma unroll
+                for (int j = 0; j < TN; ++j) {
+                    const int64_t gm = mt + tx + j * TX;
+                    if (gm < mend) Y[gr * m + gm] = acc[i][j];
+                }
+            }
+        }
+        __syncthreads();   // Ws is rewritten by the next row tile
     }
 }
 
 template <typename T>
 lrc_status launch_apply_cc(const T* U, const T* S, const T* Vt, const T* X, T* Y, int64_t m,
                            int64_t n, int64_t k, int64_t b, cudaStream_t s, const char* name) {
-    using P = Tile<T>;
+    using P = Cfg<T>;
     if (k > 4096) {
         set_error("%s: rank %lld above the supported 4096", name, (long long)k);
         return LRC_ERR_UNSUPPORTED;
     }
-    const int kpad = (int)((k + P::BN - 1) / P::BN * P::BN);
-    const size_t smem = ((size_t)kpad * P::BM + P::BK * (P::BM + 1) + P::BK * (P::BN + 1)) * sizeof(T);
+    const int kp16 = (int)((k + 15) / 16 * 16);
+    const size_t smem = ((size_t)kp16 * P::BM + P::BK1 * (P::BM + 1) + P::BK1 * (P::BN + 1)) * sizeof(T);
     if (smem > 227 * 1024) {
         set_error("%s: rank %lld needs %zu bytes of shared memory", name, (long long)k, smem);
         return LRC_ERR_UNSUPPORTED;
@@ -172,24 +203,26 @@ lrc_status launch_apply_cc(const T* U, const T* S, const T* Vt, const T* X, T* Y
     cudaError_t e = cudaFuncSetAttribute(apply_cc_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, name);
-    const int64_t row_tiles = (b + P::BM - 1) / P::BM;
+    const int64_t ntiles = (b + P::BM - 1) / P::BM;
     const int64_t m_tiles = (m + P::BN - 1) / P::BN;
-    // split the m range only when the batch alone cannot fill the GPU
-    const int64_t target = 2 * (int64_t)sm_count();
+    const int sms = sm_count();
+    int ctas_per_sm = P::kCtasPerSm;
+    while (ctas_per_sm > 1 && (size_t)ctas_per_sm * (smem + 1024) > 228 * 1024) --ctas_per_sm;
+    const int64_t slots = (int64_t)sms * ctas_per_sm;
+    // split Y's columns only when the row tiles alone leave most of the GPU idle
+    // (each split recomputes phase 1)
     int64_t splits = 1;
-    if (row_tiles < target) splits = (target + row_tiles - 1) / row_tiles;
+    if (ntiles * 2 < sms) splits = (sms + ntiles - 1) / ntiles;
     if (splits > m_tiles) splits = m_tiles;
     if (splits > 65535) splits = 65535;
     const int64_t tiles_per_split = (m_tiles + splits - 1) / splits;
     const int64_t m_chunk = tiles_per_split * P::BN;
     splits = (m + m_chunk - 1) / m_chunk;
-    if (row_tiles > 0x7fffffff) {
-        set_error("%s: batch too large", name);
-        return LRC_ERR_UNSUPPORTED;
-    }
-    dim3 grid((unsigned)row_tiles, (unsigned)splits);
-    apply_cc_kernel<T><<<grid, kThreads, smem, s>>>(U, S, Vt, X, Y, m, n, (int)k, b,
-                                                    lrc_packed_ld(k), lrc_packed_ld(n), kpad, m_chunk);
+    int64_t gx = ntiles < slots ? ntiles : slots;
+    if (gx > 0x7fffffff) gx = 0x7fffffff;
+    dim3 grid((unsigned)gx, (unsigned)splits);
+    apply_cc_kernel<T><<<grid, P::THREADS, smem, s>>>(U, S, Vt, X, Y, m, n, (int)k, b, lrc_packed_ld(k),
+                                                       lrc_packed_ld(n), kp16, ntiles, m_chunk);
     return after_launch(name);
 }
 
