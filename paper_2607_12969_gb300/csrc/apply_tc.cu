@@ -254,7 +254,7 @@ apply_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_const
         unsigned char* wlo = smem + a.wlo_off;
         for (int c = 0; c < a.nchunk && ok; ++c) {
             const int buf = c % a.acc1_bufs;
-            if (!(ok = mbar_wait(&B.acc1_full[buf], (c / a.acc1_bufs) & 1, abort, err, 4u))) break;
+            if (!(ok = group_wait(&B.acc1_full[buf], (c / a.acc1_bufs) & 1, abort, err, 4u, 1, 128))) break;
             tc_fence_after();
             const bool first = (c == 0), last = (c == a.nchunk - 1);
             for (int c0 = 0; c0 < a.kp; c0 += 32) {
@@ -312,7 +312,7 @@ apply_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_const
         int chunk = 0;
         for (int mt = mt_begin, t = 0; mt < mt_end && ok; ++mt, ++t) {
             const int ab = t & 1;
-            if (!(ok = mbar_wait(&B.acc2_full[ab], (t >> 1) & 1, abort, err, 4u))) break;
+            if (!(ok = group_wait(&B.acc2_full[ab], (t >> 1) & 1, abort, err, 4u, 1, 128))) break;
             tc_fence_after();
             for (int cc = 0; cc < a.n2; cc += ecols, ++chunk) {
                 uint32_t v[64];

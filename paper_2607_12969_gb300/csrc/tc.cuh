@@ -81,6 +81,19 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
 }
 
 // ---------------------------------------------------------------- fences / barriers
+__device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t threads);
+
+// A group of `threads` threads (named barrier `id`) waits for one phase: every
+// thread waits (bounded), then the group meets, so that the decision to go on
+// or to abort is the same for all of them and no thread is left waiting at a
+// later named barrier.
+__device__ __forceinline__ bool group_wait(uint64_t* bar, uint32_t parity, volatile int* abort, unsigned int* err,
+                                           unsigned int code, uint32_t id, uint32_t threads) {
+    mbar_wait(bar, parity, abort, err, code);
+    named_bar_sync(id, threads);
+    return *abort == 0;
+}
+
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
