@@ -253,7 +253,7 @@ class Step:
                 Wd["U"], Wd["S"], Wd["Vt"], self.d_I, self.dense_hat, m, n, k, n, "f64"))
             res = {}
             self.timed("fro_diff", work_fro(m * n, "f64", "f64"), lambda: res.update(
-                eta=lrc.lrc_fro_diff(self.dense, "f64", self.dense_hat, "f64", m * n)[0]))
+                eta=lrc.lrc_fro_diff(self.dense, "f64", self.dense_hat, "f64", m * n, want_norm=False)[0]))
             self.results[f"eta_matrix_{fmt}"] = res["eta"]
         # a6: eta for the TT
         N = int(np.prod(tt.dims))
@@ -269,7 +269,7 @@ class Step:
                 self.tt_wide[fmt], tt.dims, ranks, "f64", self.tt_That))
             res = {}
             self.timed("fro_diff", work_fro(N, "f64", "f64"), lambda: res.update(
-                eta=lrc.lrc_fro_diff(self.tt_T, "f64", self.tt_That, "f64", N)[0]))
+                eta=lrc.lrc_fro_diff(self.tt_T, "f64", self.tt_That, "f64", N, want_norm=False)[0]))
             self.results[f"eta_tt_{fmt}"] = res["eta"]
         # a7: certificate (Eq. matrix_condition)
         Ek = lrc.lrc_tail_error(self.sigma, cfg.ranks["f64"])

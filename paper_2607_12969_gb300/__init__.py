@@ -149,12 +149,14 @@ def tt_reconstruct(cores: Sequence, dims: Sequence[int], ranks: Sequence[int], f
                                  _stream(stream)))
 
 
-def lrc_fro_diff(A, fa, B, fb, count: int, stream=None) -> Tuple[float, float]:
-    """Returns (||A - B||_F, ||A||_F); B may be None."""
+def lrc_fro_diff(A, fa, B, fb, count: int, stream=None, want_norm: bool = True) -> Tuple[float, float]:
+    """Returns (||A - B||_F, ||A||_F); B may be None.  With want_norm=False
+    ||A||_F is not computed (NaN is returned in its place)."""
     diff = ctypes.c_double(0.0)
-    norm = ctypes.c_double(0.0)
+    norm = ctypes.c_double(float("nan"))
     _check(load().lrc_fro_diff(_ptr(A), _fmt(fa), _ptr(B), _fmt(fb) if B is not None else 0, count,
-                               ctypes.addressof(diff), ctypes.addressof(norm), _stream(stream)))
+                               ctypes.addressof(diff), ctypes.addressof(norm) if want_norm else None,
+                               _stream(stream)))
     return diff.value, norm.value
 
 

@@ -33,28 +33,33 @@ template <typename T>
 struct Cfg;
 template <>
 struct Cfg<double> {
-    static constexpr int BM = 8, BN = 64, BK1 = 32, BK2 = 16, TM = 1, TN = 4, THREADS = 128;
+    // phase 1 handles TN1 16-wide rank groups per pass (TN1 is a template
+    // parameter chosen so the passes divide k rounded up to 16 evenly, at most
+    // kMaxTN1 groups: predicated-off FMAs still occupy the FP64 pipe, so no
+    // pass may carry idle groups); phase 2 uses 64-wide column tiles
+    static constexpr int BM = 8, TN2 = 4, BK1 = 16, BK2 = 16, TM = 1, THREADS = 128;
+    static constexpr int kMaxTN1 = 12;
     static constexpr bool kBlocked = false;
     static constexpr int kCtasPerSm = 8;
 };
 
-template <typename T>
+template <typename T, int TN1>
 __global__ void __launch_bounds__(Cfg<T>::THREADS)
 apply_cc_kernel(const T* __restrict__ U, const T* __restrict__ S, const T* __restrict__ Vt,
                 const T* __restrict__ X, T* __restrict__ Y, int64_t m, int64_t n, int k, int64_t b,
                 int64_t ldk, int64_t ldn, int kp16, int64_t ntiles, int64_t m_chunk) {
     using P = Cfg<T>;
-    constexpr int BM = P::BM, BN = P::BN, BK1 = P::BK1, BK2 = P::BK2, TM = P::TM, TN = P::TN;
+    constexpr int BM = P::BM, BK1 = P::BK1, BK2 = P::BK2, TM = P::TM, TN2 = P::TN2;
     constexpr int NT = P::THREADS;
-    constexpr int TX = BN / TN;            // threads along columns (16)
+    constexpr int TX = 16;                 // threads along columns: 16-wide column groups
     constexpr int TY = BM / TM;            // threads along rows
-    constexpr int LDA = BM + 1, LDB = BN + 1;
+    constexpr int BN1 = TX * TN1, BN2 = TX * TN2;
+    constexpr int LDA = BM + 1, LDB = (BN1 > BN2 ? BN1 : BN2) + 1;
     static_assert(TY * TX == NT, "thread tile");
-    static_assert(TX == 16, "16-wide column groups");
     extern __shared__ __align__(16) unsigned char smem_raw[];
     T* Ws = reinterpret_cast<T*>(smem_raw);            // [kp16][BM]   scaled W, transposed
     T* As = Ws + (size_t)kp16 * BM;                     // [BK1][LDA]   X slab, transposed
-    T* Bs = As + BK1 * LDA;                             // [BK1][LDB]   Vt / U slab, transposed
+    T* Bs = As + BK1 * LDA;                             // [BK][LDB]    Vt / U slab, transposed
 
     const int tid = threadIdx.x;
     const int tx = tid % TX, ty = tid / TX;
@@ -63,15 +68,14 @@ apply_cc_kernel(const T* __restrict__ U, const T* __restrict__ S, const T* __res
 
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t row0 = tile * BM;
-        // ------------- phase 1: W = X V, one BN-wide rank chunk at a time --------
-        for (int kc = 0; kc < kp16; kc += BN) {
-            const int jmax = (kp16 - kc) / TX < TN ? (kp16 - kc) / TX : TN;   // 16-wide groups in use
-            const int rows_v = jmax * TX;
-            T acc[TM][TN];
+        // ------------- phase 1: W = X V, BN1 rank columns per pass ----------------
+        for (int kc = 0; kc < kp16; kc += BN1) {
+            const int rows_v = TN1 * TX;       // passes are full by construction
+            T acc[TM][TN1];
 #pragma unroll
             for (int i = 0; i < TM; ++i)
 #pragma unroll
-                for (int j = 0; j < TN; ++j) acc[i][j] = T(0);
+                for (int j = 0; j < TN1; ++j) acc[i][j] = T(0);
             for (int64_t k0 = 0; k0 < n; k0 += BK1) {
                 for (int e = tid; e < BM * BK1; e += NT) {
                     const int r = e / BK1, c = e % BK1;
@@ -85,50 +89,33 @@ apply_cc_kernel(const T* __restrict__ U, const T* __restrict__ S, const T* __res
                     Bs[c * LDB + j] = (gj < k && gc < n) ? Vt[(int64_t)gj * ldn + gc] : T(0);
                 }
                 __syncthreads();
-                T part[TM][TN];
+                T part[TM][TN1];
 #pragma unroll
                 for (int i = 0; i < TM; ++i)
 #pragma unroll
-                    for (int j = 0; j < TN; ++j) part[i][j] = P::kBlocked ? T(0) : acc[i][j];
-                if (jmax == TN) {
+                    for (int j = 0; j < TN1; ++j) part[i][j] = P::kBlocked ? T(0) : acc[i][j];
 #pragma unroll 4
-                    for (int c = 0; c < BK1; ++c) {
-                        T a[TM], bb[TN];
+                for (int c = 0; c < BK1; ++c) {
+                    T a[TM], bb[TN1];
 #pragma unroll
-                        for (int i = 0; i < TM; ++i) a[i] = As[c * LDA + ty + i * TY];
+                    for (int i = 0; i < TM; ++i) a[i] = As[c * LDA + ty + i * TY];
 #pragma unroll
-                        for (int j = 0; j < TN; ++j) bb[j] = Bs[c * LDB + tx + j * TX];
+                    for (int j = 0; j < TN1; ++j) bb[j] = Bs[c * LDB + tx + j * TX];
 #pragma unroll
-                        for (int i = 0; i < TM; ++i)
+                    for (int i = 0; i < TM; ++i)
 #pragma unroll
-                            for (int j = 0; j < TN; ++j) part[i][j] = fma(a[i], bb[j], part[i][j]);
-                    }
-                } else {
-                    for (int c = 0; c < BK1; ++c) {
-                        T a[TM];
-#pragma unroll
-                        for (int i = 0; i < TM; ++i) a[i] = As[c * LDA + ty + i * TY];
-#pragma unroll
-                        for (int j = 0; j < TN; ++j) {
-                            if (j < jmax) {
-                                const T bb = Bs[c * LDB + tx + j * TX];
-#pragma unroll
-                                for (int i = 0; i < TM; ++i) part[i][j] = fma(a[i], bb, part[i][j]);
-                            }
-                        }
-                    }
+                        for (int j = 0; j < TN1; ++j) part[i][j] = fma(a[i], bb[j], part[i][j]);
                 }
 #pragma unroll
                 for (int i = 0; i < TM; ++i)
 #pragma unroll
-                    for (int j = 0; j < TN; ++j)
+                    for (int j = 0; j < TN1; ++j)
                         acc[i][j] = P::kBlocked ? acc[i][j] + part[i][j] : part[i][j];
                 __syncthreads();
             }
             // W <- W diag(s), kept transposed in shared memory
 #pragma unroll
-            for (int j = 0; j < TN; ++j) {
-                if (j >= jmax) break;
+            for (int j = 0; j < TN1; ++j) {
                 const int gj = kc + tx + j * TX;
                 const T sj = (gj < k) ? S[gj] : T(0);
 #pragma unroll
@@ -138,14 +125,14 @@ apply_cc_kernel(const T* __restrict__ U, const T* __restrict__ S, const T* __res
         __syncthreads();
 
         // ------------- phase 2: Y[rows, m-tile] = W U[m-tile, :]^T ---------------
-        for (int64_t mt = mbeg; mt < mend; mt += BN) {
-            T acc[TM][TN];
+        for (int64_t mt = mbeg; mt < mend; mt += BN2) {
+            T acc[TM][TN2];
 #pragma unroll
             for (int i = 0; i < TM; ++i)
 #pragma unroll
-                for (int j = 0; j < TN; ++j) acc[i][j] = T(0);
+                for (int j = 0; j < TN2; ++j) acc[i][j] = T(0);
             for (int k0 = 0; k0 < kp16; k0 += BK2) {
-                for (int e = tid; e < BN * BK2; e += NT) {
+                for (int e = tid; e < BN2 * BK2; e += NT) {
                     const int j = e / BK2, c = e % BK2;
                     const int64_t gm = mt + j;
                     const int gc = k0 + c;
@@ -154,15 +141,15 @@ apply_cc_kernel(const T* __restrict__ U, const T* __restrict__ S, const T* __res
                 __syncthreads();
 #pragma unroll
                 for (int c = 0; c < BK2; ++c) {
-                    T a[TM], bb[TN];
+                    T a[TM], bb[TN2];
 #pragma unroll
                     for (int i = 0; i < TM; ++i) a[i] = Ws[(size_t)(k0 + c) * BM + ty + i * TY];
 #pragma unroll
-                    for (int j = 0; j < TN; ++j) bb[j] = Bs[c * LDB + tx + j * TX];
+                    for (int j = 0; j < TN2; ++j) bb[j] = Bs[c * LDB + tx + j * TX];
 #pragma unroll
                     for (int i = 0; i < TM; ++i)
 #pragma unroll
-                        for (int j = 0; j < TN; ++j) acc[i][j] = fma(a[i], bb[j], acc[i][j]);
+                        for (int j = 0; j < TN2; ++j) acc[i][j] = fma(a[i], bb[j], acc[i][j]);
                 }
                 __syncthreads();
             }
@@ -171,7 +158,7 @@ apply_cc_kernel(const T* __restrict__ U, const T* __restrict__ S, const T* __res
                 const int64_t gr = row0 + ty + i * TY;
                 if (gr >= b) continue;
 #pragma unroll
-                for (int j = 0; j < TN; ++j) {
+                for (int j = 0; j < TN2; ++j) {
                     const int64_t gm = mt + tx + j * TX;
                     if (gm < mend) Y[gr * m + gm] = acc[i][j];
                 }
@@ -341,25 +328,23 @@ apply_f32_kernel(const float* __restrict__ U, const float* __restrict__ S, const
     }
 }
 
-template <typename T>
-lrc_status launch_apply_cc(const T* U, const T* S, const T* Vt, const T* X, T* Y, int64_t m,
-                           int64_t n, int64_t k, int64_t b, cudaStream_t s, const char* name) {
+template <typename T, int TN1>
+lrc_status launch_apply_cc_n(const T* U, const T* S, const T* Vt, const T* X, T* Y, int64_t m, int64_t n,
+                             int64_t k, int64_t b, int kp16, int passes, cudaStream_t s, const char* name) {
     using P = Cfg<T>;
-    if (k > 4096) {
-        set_error("%s: rank %lld above the supported 4096", name, (long long)k);
-        return LRC_ERR_UNSUPPORTED;
-    }
-    const int kp16 = (int)((k + 15) / 16 * 16);
-    const size_t smem = ((size_t)kp16 * P::BM + P::BK1 * (P::BM + 1) + P::BK1 * (P::BN + 1)) * sizeof(T);
+    constexpr int LDB = 16 * (TN1 > P::TN2 ? TN1 : P::TN2) + 1;
+    const int kw = passes * 16 * TN1;                 // rank columns covered by the passes
+    const size_t smem = ((size_t)kw * P::BM + P::BK1 * (P::BM + 1) +
+                         (size_t)(P::BK1 > P::BK2 ? P::BK1 : P::BK2) * LDB) * sizeof(T);
     if (smem > 227 * 1024) {
         set_error("%s: rank %lld needs %zu bytes of shared memory", name, (long long)k, smem);
         return LRC_ERR_UNSUPPORTED;
     }
-    cudaError_t e = cudaFuncSetAttribute(apply_cc_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(apply_cc_kernel<T, TN1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, name);
     const int64_t ntiles = (b + P::BM - 1) / P::BM;
-    const int64_t m_tiles = (m + P::BN - 1) / P::BN;
+    const int64_t m_tiles = (m + 16 * P::TN2 - 1) / (16 * P::TN2);
     const int sms = sm_count();
     int ctas_per_sm = P::kCtasPerSm;
     while (ctas_per_sm > 1 && (size_t)ctas_per_sm * (smem + 1024) > 228 * 1024) --ctas_per_sm;
@@ -371,14 +356,44 @@ lrc_status launch_apply_cc(const T* U, const T* S, const T* Vt, const T* X, T* Y
     if (splits > m_tiles) splits = m_tiles;
     if (splits > 65535) splits = 65535;
     const int64_t tiles_per_split = (m_tiles + splits - 1) / splits;
-    const int64_t m_chunk = tiles_per_split * P::BN;
+    const int64_t m_chunk = tiles_per_split * 16 * P::TN2;
     splits = (m + m_chunk - 1) / m_chunk;
     int64_t gx = ntiles < slots ? ntiles : slots;
     if (gx > 0x7fffffff) gx = 0x7fffffff;
     dim3 grid((unsigned)gx, (unsigned)splits);
-    apply_cc_kernel<T><<<grid, P::THREADS, smem, s>>>(U, S, Vt, X, Y, m, n, (int)k, b, lrc_packed_ld(k),
-                                                       lrc_packed_ld(n), kp16, ntiles, m_chunk);
+    // the kernel's phase 1 walks kw rank columns (k rounded up to 16, then to the passes)
+    apply_cc_kernel<T, TN1><<<grid, P::THREADS, smem, s>>>(U, S, Vt, X, Y, m, n, (int)k, b, lrc_packed_ld(k),
+                                                            lrc_packed_ld(n), kw, ntiles, m_chunk);
+    (void)kp16;
     return after_launch(name);
+}
+
+template <typename T>
+lrc_status launch_apply_cc(const T* U, const T* S, const T* Vt, const T* X, T* Y, int64_t m,
+                           int64_t n, int64_t k, int64_t b, cudaStream_t s, const char* name) {
+    using P = Cfg<T>;
+    if (k > 4096) {
+        set_error("%s: rank %lld above the supported 4096", name, (long long)k);
+        return LRC_ERR_UNSUPPORTED;
+    }
+    const int kp16 = (int)((k + 15) / 16 * 16);
+    const int groups = kp16 / 16;
+    const int passes = (groups + P::kMaxTN1 - 1) / P::kMaxTN1;
+    const int tn1 = (groups + passes - 1) / passes;   // passes * tn1 >= groups, tn1 <= kMaxTN1
+    switch (tn1) {
+        case 1: return launch_apply_cc_n<T, 1>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+        case 2: return launch_apply_cc_n<T, 2>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+        case 3: return launch_apply_cc_n<T, 3>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+        case 4: return launch_apply_cc_n<T, 4>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+        case 5: return launch_apply_cc_n<T, 5>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+        case 6: return launch_apply_cc_n<T, 6>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+        case 7: return launch_apply_cc_n<T, 7>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+        case 8: return launch_apply_cc_n<T, 8>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+        case 9: return launch_apply_cc_n<T, 9>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+        case 10: return launch_apply_cc_n<T, 10>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+        case 11: return launch_apply_cc_n<T, 11>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+        default: return launch_apply_cc_n<T, 12>(U, S, Vt, X, Y, m, n, k, b, kp16, passes, s, name);
+    }
 }
 
 }  // namespace

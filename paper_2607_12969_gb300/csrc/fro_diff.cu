@@ -95,8 +95,10 @@ __device__ __forceinline__ void block_sum2(double& a, double& b, double* sh) {
     }
 }
 
-// FB = -1: B absent (treated as zero).
-template <int FA, int FB>
+// FB = -1: B absent (treated as zero).  NORM = false skips the ||A||
+// accumulation (the reduction is bound by FP64 issue on this GPU, so the
+// extra FMA per element costs time when nobody reads the norm).
+template <int FA, int FB, bool NORM>
 __global__ void __launch_bounds__(kThreads)
 fro_partial_kernel(const void* __restrict__ A, const void* __restrict__ B, int64_t count,
                    double* __restrict__ partial) {
@@ -112,7 +114,7 @@ fro_partial_kernel(const void* __restrict__ A, const void* __restrict__ B, int64
         for (int j = 0; j < kGroup; ++j) {
             const double d = (FB >= 0) ? a[j] - b[j] : a[j];
             sd = fma(d, d, sd);
-            sa = fma(a[j], a[j], sa);
+            if (NORM) sa = fma(a[j], a[j], sa);
         }
     }
     if (blockIdx.x == 0) {  // ragged tail, fixed owner
@@ -120,7 +122,7 @@ fro_partial_kernel(const void* __restrict__ A, const void* __restrict__ B, int64
             const double a = load1<FA>(A, i);
             const double d = (FB >= 0) ? a - load1<FB < 0 ? 0 : FB>(B, i) : a;
             sd = fma(d, d, sd);
-            sa = fma(a, a, sa);
+            if (NORM) sa = fma(a, a, sa);
         }
     }
     block_sum2(sd, sa, sh);
@@ -147,15 +149,22 @@ fro_final_kernel(const double* __restrict__ partial, int nblocks, double* __rest
 
 int fcode(lrc_fmt f) { return f == LRC_F64 ? 0 : (f == LRC_F32 ? 1 : 2); }
 
+template <int FA, bool NORM>
+void launch_partial_n(int fb, int grid, const void* A, const void* B, int64_t count, double* partial,
+                      cudaStream_t s) {
+    switch (fb) {
+        case 0: fro_partial_kernel<FA, 0, NORM><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
+        case 1: fro_partial_kernel<FA, 1, NORM><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
+        case 2: fro_partial_kernel<FA, 2, NORM><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
+        default: fro_partial_kernel<FA, -1, NORM><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
+    }
+}
+
 template <int FA>
 void launch_partial(int fb, int grid, const void* A, const void* B, int64_t count, double* partial,
-                    cudaStream_t s) {
-    switch (fb) {
-        case 0: fro_partial_kernel<FA, 0><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
-        case 1: fro_partial_kernel<FA, 1><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
-        case 2: fro_partial_kernel<FA, 2><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
-        default: fro_partial_kernel<FA, -1><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
-    }
+                    cudaStream_t s, bool norm = true) {
+    if (norm) launch_partial_n<FA, true>(fb, grid, A, B, count, partial, s);
+    else launch_partial_n<FA, false>(fb, grid, A, B, count, partial, s);
 }
 
 }  // namespace
@@ -188,10 +197,11 @@ lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, in
     int grid = (int)(want < cap ? (want > 0 ? want : 1) : cap);
     if (grid > kMaxBlocks) grid = kMaxBlocks;
     const int a = fcode(fa), b = B ? fcode(fb) : -1;
+    const bool norm = normA_out != nullptr;
     switch (a) {
-        case 0: launch_partial<0>(b, grid, A, B, count, partial, s); break;
-        case 1: launch_partial<1>(b, grid, A, B, count, partial, s); break;
-        default: launch_partial<2>(b, grid, A, B, count, partial, s); break;
+        case 0: launch_partial<0>(b, grid, A, B, count, partial, s, norm); break;
+        case 1: launch_partial<1>(b, grid, A, B, count, partial, s, norm); break;
+        default: launch_partial<2>(b, grid, A, B, count, partial, s, norm); break;
     }
     lrc_status st = after_launch("fro_partial_kernel");
     if (st != LRC_OK) return st;

@@ -42,6 +42,11 @@ def test_fro_diff_null_b_and_determinism(lrc, cuda):
     assert abs(r1[0] - oracle.fro_diff(a.cpu().numpy())[0]) <= 1e-12 * r1[0]
     z, _ = lrc.lrc_fro_diff(a, "f64", a, "f64", a.numel())
     assert z == 0.0
+    # without the norm: same difference, norm not computed
+    b = a * 0.5
+    d1, n1 = lrc.lrc_fro_diff(a, "f64", b, "f64", a.numel())
+    d2, n2 = lrc.lrc_fro_diff(a, "f64", b, "f64", a.numel(), want_norm=False)
+    assert d1 == d2 and np.isnan(n2) and n1 > 0
 
 
 U64_ROUNDOFF = 2.0 ** -53
