@@ -23,7 +23,9 @@
 // the method-precision workspace of Sec. 3.4.  W never reaches global memory.
 // Phase 2 computes Y tiles = W U^T with two tensor-memory accumulators in
 // flight, so the epilogue drains one tile (TMEM -> registers -> swizzled
-// shared memory -> TMA store) while the next is being multiplied.
+// shared memory -> TMA store) while the next is being multiplied; each
+// epilogue warp stages and stores its own 32 rows, without barriers across
+// the four warps.
 #include <cudaTypedefs.h>
 
 #include <mutex>
@@ -248,7 +250,6 @@ apply_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_const
         const int g = warp & 3;                 // TMEM lane quarter of this warp
         const int r = g * 32 + lane;            // tile row of this thread
         const uint32_t lane_base = (uint32_t)(g * 32) << 16;
-        const bool issuer = (threadIdx.x == 64);
         bool ok = true;
         unsigned char* whi = smem + a.w_off;
         unsigned char* wlo = smem + a.wlo_off;
@@ -331,21 +332,23 @@ apply_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_const
                 }
                 const int64_t col0 = (int64_t)mt * a.n2 + cc;
                 if (a.tma_store) {
-                    unsigned char* sb = smem + a.ystage_off + (chunk & 1) * 16384;
+                    // this warp's 32 rows: own staging pair, own TMA store, no
+                    // barrier across the four epilogue warps
+                    unsigned char* sb = smem + a.ystage_off + (size_t)g * (2 * 32 * 128) + (chunk & 1) * (32 * 128);
                     if (chunk >= 2) {
-                        if (issuer) bulk_wait_read<1>();
-                        named_bar_sync(1, 128);
+                        if (lane == 0) bulk_wait_read<1>();
+                        __syncwarp();
                     }
 #pragma unroll
                     for (int j = 0; j < 8; ++j) {
-                        const uint32_t off = (uint32_t)r * 128u + (uint32_t)((j ^ (r & 7)) * 16);
+                        const uint32_t off = (uint32_t)lane * 128u + (uint32_t)((j ^ (lane & 7)) * 16);
                         *reinterpret_cast<uint4*>(sb + off) =
                             make_uint4(packed[4 * j], packed[4 * j + 1], packed[4 * j + 2], packed[4 * j + 3]);
                     }
                     fence_proxy_async_smem();
-                    named_bar_sync(1, 128);
-                    if (issuer && col0 < a.m) {
-                        tma_store_2d(&tm_y, (int32_t)col0, (int32_t)row0, sb);
+                    __syncwarp();
+                    if (lane == 0 && col0 < a.m) {
+                        tma_store_2d(&tm_y, (int32_t)col0, (int32_t)(row0 + g * 32), sb);
                         bulk_commit();
                     }
                 } else {
@@ -366,7 +369,7 @@ apply_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_const
             tc_fence_before();
             mbar_arrive(&B.acc2_empty[ab]);
         }
-        if (issuer && a.tma_store) bulk_wait<0>();
+        if (lane == 0 && a.tma_store) bulk_wait<0>();
     }
     tc_fence_before();
     __syncthreads();
@@ -524,7 +527,7 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
         return st;
     if (a.tma_store) {
         if ((st = make_map(&ty, out16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, e_out, Y, m,
-                           b, m * e_out, out16 ? 64 : 32, BM, "Y")) != LRC_OK)
+                           b, m * e_out, out16 ? 64 : 32, 32, "Y")) != LRC_OK)
             return st;
     } else {
         ty = tu;   // unused by the kernel

@@ -71,6 +71,10 @@ lrc_status launch_tt_f16(const TTShape& sh, bool out16, void* out, cudaStream_t 
 // read and cleared by lrc_device_status().  0xffffffff = could not be read.
 uint32_t take_apply_tc_error();
 uint32_t take_tt_tc_error();
+uint32_t take_tt3_tc_error();
+// 3-way binary16 TT on the tensor cores; *handled = false when the shape is
+// outside the kernel (nothing launched).
+lrc_status launch_tt3_f16_tc(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled);
 lrc_status launch_wait_timeout_probe(int64_t limit_ns, cudaStream_t s);
 
 lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,

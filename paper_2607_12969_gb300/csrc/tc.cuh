@@ -132,6 +132,14 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int32_t x, 
                  : "memory");
 }
 
+// 3-D tiled store of a shared-memory box to (x, y, z); elements outside the
+// tensor are not written.  x, y, z >= 0.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, int32_t x, int32_t y, int32_t z, const void* src) {
+    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];"
+                 ::"l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(src))
+                 : "memory");
+}
+
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 
 template <int N>
