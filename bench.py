@@ -531,7 +531,16 @@ def run_case(args):
         work = work_round(args.b, args.n, args.n, fmt)
     call()
     torch.cuda.synchronize()
+    # host cost of one call (marshalling, planning, launch), GPU left busy
+    t0 = time.perf_counter()
+    for _ in range(args.reps):
+        call()
+    host_us = (time.perf_counter() - t0) / args.reps * 1e6
+    torch.cuda.synchronize()
+    # device time: the calls queue up behind a GPU-side sleep, so the host's
+    # per-call cost does not open gaps between them
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda._sleep(int(2e6 + 2500 * host_us * args.reps))   # cycles, about 2 GHz
     e0.record()
     for _ in range(args.reps):
         call()
@@ -539,7 +548,7 @@ def run_case(args):
     torch.cuda.synchronize()
     st = lrc.lrc_device_status()
     ms = e0.elapsed_time(e1) / args.reps
-    print(json.dumps({"case": args.case, "fmt": fmt, "ms": ms, "status": st,
+    print(json.dumps({"case": args.case, "fmt": fmt, "ms": ms, "host_us": host_us, "status": st,
                       "GBps": work["bytes"] / (ms * 1e-3) / 1e9,
                       "TFLOPs": work["flops"] / (ms * 1e-3) / 1e12,
                       "roofline_frac": roofline_time(work) / (ms * 1e-3)}))

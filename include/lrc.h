@@ -105,8 +105,7 @@ LRC_API lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows,
  *     Y = [(X V) diag(s)] U^T,   i.e. Y^T = U (diag(s) (V^T X^T)),
  *
  * with the factors of a rank-k approximation A_k = U diag(s) V^T of an
- * m x n matrix, applied to b queries at once.  The k x b intermediate
- * V^T X^T never leaves the chip.
+ * m x n matrix, applied to b queries at once.
  *
  *   U    device, m x k, row pitch lrc_packed_ld(k)
  *   S    device, k singular values s_1..s_k
@@ -119,6 +118,16 @@ LRC_API lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows,
  * all binary16 (the intermediate is rounded to binary16 as well).  Pad
  * columns of U, Vt and X are never read.  All five pointers must be 16-byte
  * aligned.  k may exceed min(m, n).  Asynchronous on `stream`.
+ *
+ * Intermediate: for LRC_F64 and LRC_F32 the b x k product (X V) diag(s)
+ * stays in shared memory.  For LRC_F16 and LRC_F16_O16 the reduction over n
+ * is split over all multiprocessors, so its partial sums and the scaled
+ * intermediate (binary16, a hi/lo pair for LRC_F16) pass through a device
+ * workspace owned by the library: one buffer per (device, stream),
+ * allocated on first use and reallocated -- after synchronizing `stream` --
+ * when a larger problem arrives, freed by lrc_shutdown().  Calls on
+ * different streams use different buffers.  Binary16 ranks: up to 320 for
+ * LRC_F16 and 512 for LRC_F16_O16, else LRC_ERR_UNSUPPORTED.
  */
 LRC_API lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X, void* Y,
                      int64_t m, int64_t n, int64_t k, int64_t b, lrc_fmt fmt,

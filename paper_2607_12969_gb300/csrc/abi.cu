@@ -279,6 +279,7 @@ lrc_status lrc_selftest_wait_timeout(int64_t limit_ns, lrc_stream_t stream) {
 
 lrc_status lrc_shutdown(void) {
     release_scratch();
+    release_workspaces();
     return LRC_OK;
 }
 

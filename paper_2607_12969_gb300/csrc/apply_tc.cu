@@ -1,34 +1,42 @@
-// apply_tc.cu -- fused low-rank apply on the 5th-generation tensor cores,
-// binary16 storage with binary32 accumulation (Sec. 4.4, Eq. gpu_matrix_apply:
+// apply_tc.cu -- low-rank apply on the 5th-generation tensor cores, binary16
+// storage with binary32 accumulation (Sec. 4.4, Eq. gpu_matrix_apply:
 // Y = [(X V) diag(s)] U^T; Sec. 3.4: FP16 products accumulate in FP32).
 //
-// One CTA owns BM = 128 query rows (the MMA M) and a contiguous range of
-// N2-wide tiles of Y's columns.  Warp roles:
-//   warp 0      TMA producer: streams X / V^T boxes (phase 1) and U boxes
-//               (phase 2) through a ring of shared-memory slots;
-//   warp 1      tensor-memory owner and MMA issuer (one thread);
-//   warps 2..5  epilogue (one TMEM lane = one query row per thread).
-// Phase 1 accumulates W = X V (128 x k', FP32) in tensor memory.  For FP32
-// output the reduction over n is split into chunks of kChunkBlocks x 64
-// elements accumulated in two ping-pong tensor-memory buffers; the epilogue
-// adds each chunk's partial sums with IEEE binary32 additions into a running
-// sum.  (The tensor core's own accumulation error grows with the number of
-// accumulation steps; chunking bounds it by the chunk length.)  The running
-// sum lives in the shared-memory region that later holds W's hi/lo halves,
-// laid out so that every thread only ever touches the bytes of its own row.
-// The epilogue scales W by diag(s) in FP32 and writes it to shared memory
-// as binary16 -- for the FP32-output variant as a hi/lo pair
-// (hi = fp16(w), lo = fp16(w - hi)) so that the second product keeps about
-// 22 significand bits; the FP16-output variant rounds W once to binary16,
-// the method-precision workspace of Sec. 3.4.  W never reaches global memory.
-// Phase 2 computes Y tiles = W U^T with two tensor-memory accumulators in
-// flight, so the epilogue drains one tile (TMEM -> registers -> swizzled
-// shared memory -> TMA store) while the next is being multiplied; each
-// epilogue warp stages and stores its own 32 rows, without barriers across
-// the four warps.
+// Three launches on the caller's stream:
+//  1. apply_w1_kernel -- W = X V in FP32 partials.  For every 128-row tile of
+//     X and every column group of W (at most 160 ranks for FP32 output, so that a
+//     running sum fits in shared memory) the reduction over n is a row of
+//     64-wide k-blocks.  The rows are laid end to end and cut into equal
+//     contiguous ranges, one per CTA of a persistent grid: every SM gets the
+//     same share of the product whatever b is (one row tile or hundreds).
+//     A CTA's range crosses a few rows; each piece (segment) accumulates in
+//     tensor memory -- for FP32 output in chunks of at most kChunkBlocks
+//     k-blocks whose results the epilogue adds with IEEE binary32 additions
+//     (the tensor core's own accumulation error grows with the number of
+//     accumulation steps) -- and is written to the workspace as an FP32
+//     partial.  Column groups are the slower index of the rows, so the CTAs
+//     working on the two groups of one row tile run side by side and the
+//     second read of an X tile hits L2.
+//  2. apply_w2_kernel -- every W entry adds its tile's partials in a fixed
+//     order (deterministic), is scaled by diag(s) in FP32 and written as
+//     binary16: a hi/lo pair (hi = fp16(w), lo = fp16(w - hi)) for FP32
+//     output, which keeps about 22 significand bits through the second
+//     product, or one rounding for FP16 output (the method-precision
+//     workspace of Sec. 3.4).  The layout is the shared-memory image of the
+//     second product's A operand, so it is loaded with one bulk copy.
+//  3. apply_y_kernel -- Y tiles = W U^T.  A persistent grid takes equal
+//     contiguous ranges of (row tile, column tile) pairs; W of the current
+//     row tile sits in shared memory, U streams through a TMA ring, and two
+//     tensor-memory accumulators let the epilogue drain one tile (TMEM ->
+//     registers -> swizzled shared memory -> TMA store, each epilogue warp
+//     storing its own 32 rows) while the next is multiplied.
+// Warp roles of kernels 1 and 3: warp 0 TMA producer, warp 1 tensor-memory
+// owner and MMA issuer (one thread), warps 2..5 epilogue (one TMEM lane = one
+// row per thread).  W is b x k' values, a few percent of the traffic.
 #include <cudaTypedefs.h>
 
 #include <mutex>
+#include <utility>
 
 #include "common.cuh"
 #include "tc.cuh"
@@ -45,296 +53,551 @@ constexpr int BM = 128;
 constexpr int BK = 64;                       // FP16 elements per 128-byte swizzled row
 constexpr int kThreads = 192;
 constexpr uint32_t kXBytes = BM * BK * 2;    // one X box
-constexpr int kChunkBlocks = 8;              // 64-wide k-blocks per accumulation chunk (FP32 output)
+constexpr int kChunkBlocks = 8;              // k-blocks per accumulation chunk (FP32 output)
+constexpr int kPfBlocks = 4;                 // k-blocks per L2 prefetch box (512-byte rows)
+constexpr int kStageBlocks = 2;              // k-blocks per phase-1 ring stage
 
-struct Args {
-    int64_t m, b;
-    int k, kp;                 // rank and rank rounded up to 16
-    int n2;                    // phase-2 tile width (MMA N)
-    int nkb;                   // phase-1 k-blocks, ceil(n / 64)
-    int kc2;                   // phase-2 k-chunks, ceil(kp / 64)
-    int mtiles;                // ceil(m / n2)
-    int mt_per_cta;
-    int chunk_blocks;          // k-blocks per phase-1 accumulation chunk
-    int nchunk;                // ceil(nkb / chunk_blocks)
-    int acc1_bufs;             // 2 = ping-pong, 1 = single phase-1 accumulator
+__device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
+    return reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
+}
+
+// Byte offset of W[r][col] (r < 128) in the canonical no-swizzle K-major
+// operand image: 8-row x 16-byte core matrices, K-direction stride 2048 B,
+// row-group stride 128 B.
+__host__ __device__ __forceinline__ uint32_t w_image_off(uint32_t r, uint32_t col) {
+    return (col >> 3) * 2048u + (r >> 3) * 128u + (r & 7u) * 16u + (col & 7u) * 2u;
+}
+
+// ================================================================ phase 1
+struct W1Args {
+    int64_t b;
+    int64_t btiles;
+    int64_t nkb;              // k-blocks per row, ceil(n / 64)
+    int64_t Q;                // rows x nkb
+    int G;                    // column groups; row = group * btiles + row tile
+    int kgp;                  // group width (ranks, multiple of 16); group g starts at g * kgp
+    int kp;                   // the last group ends at kp
+    int chunk_blocks;
     int stages;
     uint32_t slot_bytes;
-    uint32_t v_bytes;          // kp rows x 128 bytes
-    uint32_t u_bytes;          // n2 rows x 128 bytes
-    int v_boxes, v_box_rows;
+    uint32_t sum_off, bar_off;
     uint32_t tmem_cols;
-    uint32_t w_off, wlo_off, ystage_off, s_off, bar_off;   // shared-memory carve-up
-    int out16;
-    int tma_store;
-    const __half* S;
-    void* Y;
+    float* P;                 // partials: [segment id][kgp columns][128 rows]
 };
 
-struct Bars {
-    uint64_t* full;
-    uint64_t* empty;
-    uint64_t* acc1_full;    // [2]
-    uint64_t* acc1_empty;   // [2]
-    uint64_t* w_ready;
-    uint64_t* acc2_full;    // [2]
-    uint64_t* acc2_empty;   // [2]
-    uint64_t* mma_done;
-    uint32_t* tmem_slot;
-    int* abort;
-};
-
-__device__ __forceinline__ Bars carve_bars(unsigned char* smem, const Args& a) {
-    Bars B;
-    uint64_t* p = reinterpret_cast<uint64_t*>(smem + a.bar_off);
-    B.full = p;
-    B.empty = p + a.stages;
-    B.acc1_full = p + 2 * a.stages;
-    B.acc1_empty = B.acc1_full + 2;
-    B.w_ready = B.acc1_empty + 2;
-    B.acc2_full = B.w_ready + 1;
-    B.acc2_empty = B.acc2_full + 2;
-    B.mma_done = B.acc2_empty + 2;
-    B.tmem_slot = reinterpret_cast<uint32_t*>(B.mma_done + 1);
-    B.abort = reinterpret_cast<int*>(B.tmem_slot + 1);
-    return B;
+// Next accumulation chunk of the k-block range [qbeg, qend): a chunk lies in
+// one row, starts a new chunk every `cb` k-blocks from the start of its
+// segment (the part of the row inside the range) and ends with the segment.
+__device__ __forceinline__ bool next_chunk(int64_t& q, int64_t qbeg, int64_t qend, int64_t nkb, int64_t cb,
+                                           int64_t& q0, int64_t& q1, int64_t& row, bool& first, bool& last) {
+    if (q >= qend) return false;
+    row = q / nkb;
+    const int64_t re = (row + 1) * nkb;
+    const int64_t seg_end = re < qend ? re : qend;
+    q0 = q;
+    q1 = (q + cb < seg_end) ? q + cb : seg_end;
+    first = (q == qbeg) || (q == row * nkb);
+    last = (q1 == seg_end);
+    q = q1;
+    return true;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-apply_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_v,
-                    const __grid_constant__ CUtensorMap tm_u, const __grid_constant__ CUtensorMap tm_y,
-                    const Args a) {
+apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_v,
+                const __grid_constant__ CUtensorMap tm_xp, const __grid_constant__ CUtensorMap tm_vp, const W1Args a) {
     extern __shared__ unsigned char smem_raw[];
-    unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                                           ~static_cast<uintptr_t>(1023));
-    const Bars B = carve_bars(smem, a);
-    float* s_f = reinterpret_cast<float*>(smem + a.s_off);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t row0 = (int64_t)blockIdx.x * BM;
-    const int mt_begin = blockIdx.y * a.mt_per_cta;
-    const int mt_end = min(mt_begin + a.mt_per_cta, a.mtiles);
-    volatile int* abort = B.abort;
+    unsigned char* smem = align1024(smem_raw);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + a.bar_off);
+    uint64_t* empty = full + a.stages;
+    uint64_t* acc_full = empty + a.stages;     // [2]
+    uint64_t* acc_empty = acc_full + 2;        // [2]
+    uint64_t* mma_done = acc_empty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+    volatile int* abort = reinterpret_cast<int*>(tmem_slot + 1);
     unsigned int* err = &g_err_apply_tc;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t qbeg = a.Q * blockIdx.x / gridDim.x;
+    const int64_t qend = a.Q * (blockIdx.x + 1) / gridDim.x;
+    pdl_trigger();                 // the reduction kernel may be scheduled now; it waits for this grid
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < a.stages; ++i) {
-            mbar_init(&B.full[i], 1);
-            mbar_init(&B.empty[i], 1);
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
         }
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&B.acc1_full[i], 1);
-            mbar_init(&B.acc1_empty[i], 128);
+            mbar_init(&acc_full[i], 1);
+            mbar_init(&acc_empty[i], 128);
         }
-        mbar_init(B.w_ready, 128);
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(&B.acc2_full[i], 1);
-            mbar_init(&B.acc2_empty[i], 128);
-        }
-        mbar_init(B.mma_done, 1);
-        *B.abort = 0;
+        mbar_init(mma_done, 1);
+        *abort = 0;
         fence_barrier_init();
         tma_prefetch_desc(&tm_x);
         tma_prefetch_desc(&tm_v);
-        tma_prefetch_desc(&tm_u);
-        tma_prefetch_desc(&tm_y);
+        tma_prefetch_desc(&tm_xp);
+        tma_prefetch_desc(&tm_vp);
     }
-    for (int j = threadIdx.x; j < a.kp; j += kThreads) s_f[j] = j < a.k ? __half2float(a.S[j]) : 0.0f;
-    if (warp == 1) tmem_alloc(B.tmem_slot, a.tmem_cols);
+    if (warp == 1) tmem_alloc(tmem_slot, a.tmem_cols);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tmem = *B.tmem_slot;
+    const uint32_t tmem = *tmem_slot;
 
+    // a ring stage carries kStageBlocks k-blocks of one chunk: slot layout
+    // [X k-block 0][X k-block 1][V^T k-block 0][V^T k-block 1]
+    const uint32_t vbox = (uint32_t)a.kgp * 128u;
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
             int it = 0;
             bool ok = true;
-            for (int kb = 0; kb < a.nkb && ok; ++kb, ++it) {
-                const int slot = it % a.stages;
-                if (!(ok = mbar_wait(&B.empty[slot], ((it / a.stages) & 1) ^ 1, abort, err, 1u))) break;
-                unsigned char* sp = smem + (size_t)slot * a.slot_bytes;
-                mbar_arrive_expect_tx(&B.full[slot], kXBytes + a.v_bytes);
-                tma_load_2d(sp, &tm_x, kb * BK, (int32_t)row0, &B.full[slot]);
-                for (int vb = 0; vb < a.v_boxes; ++vb)
-                    tma_load_2d(sp + kXBytes + (size_t)vb * a.v_box_rows * 128, &tm_v, kb * BK, vb * a.v_box_rows,
-                                &B.full[slot]);
-            }
-            for (int mt = mt_begin; mt < mt_end && ok; ++mt) {
-                for (int kc = 0; kc < a.kc2 && ok; ++kc, ++it) {
+            int64_t q = qbeg, q0, q1, row;
+            bool first, last;
+            while (ok && next_chunk(q, qbeg, qend, a.nkb, a.chunk_blocks, q0, q1, row, first, last)) {
+                const int grp = (int)(row / a.btiles);
+                const int64_t bt = row - (int64_t)grp * a.btiles;
+                const int64_t rbase = row * a.nkb;
+                const int64_t seg_end = rbase + a.nkb < qend ? rbase + a.nkb : qend;
+                for (int64_t qs = q0; qs < q1; qs += kStageBlocks, ++it) {
+                    const int nb = (q1 - qs >= kStageBlocks) ? kStageBlocks : (int)(q1 - qs);
+                    // L2 prefetch of X and V^T in 512-byte-wide rows (four k-blocks),
+                    // up to two groups ahead, so that the operand boxes (128-byte
+                    // rows) hit L2
+                    for (int u = 0; u < nb; ++u) {
+                        const int64_t kb = qs + u - rbase;
+                        const bool seg_first = (qs + u == qbeg) || (kb == 0);
+                        if (!seg_first && (kb & (kPfBlocks - 1)) != 0) continue;
+                        const int64_t g0 = kb / kPfBlocks;
+                        for (int64_t pg = seg_first ? g0 : g0 + 2; pg <= g0 + 2; ++pg) {
+                            const int64_t pkb = pg * kPfBlocks;
+                            if (rbase + pkb >= seg_end) break;
+                            tma_prefetch_2d(&tm_xp, (int32_t)(pkb * BK), (int32_t)(bt * BM));
+                            tma_prefetch_2d(&tm_vp, (int32_t)(pkb * BK), grp * a.kgp);
+                        }
+                    }
                     const int slot = it % a.stages;
-                    if (!(ok = mbar_wait(&B.empty[slot], ((it / a.stages) & 1) ^ 1, abort, err, 1u))) break;
-                    mbar_arrive_expect_tx(&B.full[slot], a.u_bytes);
-                    tma_load_2d(smem + (size_t)slot * a.slot_bytes, &tm_u, kc * BK, mt * a.n2, &B.full[slot]);
+                    if (!(ok = mbar_wait(&empty[slot], ((it / a.stages) & 1) ^ 1, abort, err, 1u))) break;
+                    unsigned char* sp = smem + (size_t)slot * a.slot_bytes;
+                    mbar_arrive_expect_tx(&full[slot], (uint32_t)nb * (kXBytes + vbox));
+                    for (int u = 0; u < nb; ++u) {
+                        const int32_t kx = (int32_t)((qs + u - rbase) * BK);
+                        tma_load_2d(sp + (size_t)u * kXBytes, &tm_x, kx, (int32_t)(bt * BM), &full[slot]);
+                        tma_load_2d(sp + (size_t)kStageBlocks * kXBytes + (size_t)u * vbox, &tm_v, kx, grp * a.kgp,
+                                    &full[slot]);
+                    }
                 }
             }
             if (!ok) {
                 // let copies already in flight land before the CTA can exit
-                const int first = it - a.stages > 0 ? it - a.stages : 0;
-                for (int j = first; j < it; ++j) {
+                const int first_it = it - a.stages > 0 ? it - a.stages : 0;
+                for (int j = first_it; j < it; ++j) {
                     volatile int no_abort = 0;
-                    mbar_wait(&B.full[j % a.stages], (j / a.stages) & 1, &no_abort, err, 0u, 100000000ull);
+                    mbar_wait(&full[j % a.stages], (j / a.stages) & 1, &no_abort, err, 0u, 100000000ull);
                 }
             }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
+        // Descriptors are built once per stage and stepped by plain adds (32
+        // bytes = 2 in the address field): a single issuing thread is the
+        // bottleneck, so every instruction between MMAs counts.
         if (lane == 0) {
-            int it = 0;
+            int it = 0, ci = 0;
             bool ok = true;
-            const int nchunks = a.kp > 256 ? 2 : 1;
-            for (int kb = 0; kb < a.nkb && ok; ++kb, ++it) {
-                const int c = kb / a.chunk_blocks;                 // accumulation chunk
-                const int kin = kb - c * a.chunk_blocks;           // k-block within the chunk
-                const int buf = c % a.acc1_bufs;
-                if (kin == 0) {
-                    if (!(ok = mbar_wait(&B.acc1_empty[buf], ((c / a.acc1_bufs) & 1) ^ 1, abort, err, 2u))) break;
-                    tc_fence_after();
-                }
-                const int slot = it % a.stages;
-                if (!(ok = mbar_wait(&B.full[slot], (it / a.stages) & 1, abort, err, 2u))) break;
+            int64_t q = qbeg, q0, q1, row;
+            bool first, last;
+            while (ok && next_chunk(q, qbeg, qend, a.nkb, a.chunk_blocks, q0, q1, row, first, last)) {
+                const int buf = ci & 1;
+                if (!(ok = mbar_wait(&acc_empty[buf], ((ci >> 1) & 1) ^ 1, abort, err, 2u))) break;
                 tc_fence_after();
-                const uint32_t xa = smem_u32(smem + (size_t)slot * a.slot_bytes);
-                const uint32_t va = xa + kXBytes;
-                const uint32_t dacc = tmem + buf * a.kp;
+                const int grp = (int)(row / a.btiles);
+                const int kgw = min(a.kgp, a.kp - grp * a.kgp);
+                const uint32_t idesc = idesc_f16_f32(BM, (uint32_t)kgw);
+                const uint32_t dacc = tmem + (uint32_t)(buf * a.kgp);
+                uint32_t accf = 0;
+                for (int64_t qs = q0; qs < q1; qs += kStageBlocks, ++it) {
+                    const int nb = (q1 - qs >= kStageBlocks) ? kStageBlocks : (int)(q1 - qs);
+                    const int slot = it % a.stages;
+                    if (!(ok = mbar_wait(&full[slot], (it / a.stages) & 1, abort, err, 2u))) break;
+                    tc_fence_after();
+                    const uint32_t base = smem_u32(smem + (size_t)slot * a.slot_bytes);
+                    const uint64_t dx = desc_sw128(base);
+                    const uint64_t dv = desc_sw128(base + (uint32_t)kStageBlocks * kXBytes);
+                    for (int u = 0; u < nb; ++u) {
+                        const uint64_t dxu = dx + (uint64_t)u * (kXBytes >> 4);
+                        const uint64_t dvu = dv + (uint64_t)u * (vbox >> 4);
 #pragma unroll
-                for (int kk = 0; kk < BK / 16; ++kk) {
-                    const uint64_t adesc = desc_sw128(xa + kk * 32);
-                    for (int q = 0; q < nchunks; ++q) {
-                        const int r0 = q * 256;
-                        const int nn = (q == 0) ? (a.kp > 256 ? 256 : a.kp) : a.kp - 256;
-                        mma_f16(dacc + r0, adesc, desc_sw128(va + r0 * 128 + kk * 32), idesc_f16_f32(BM, nn),
-                                (kin | kk) != 0);
+                        for (int kk = 0; kk < BK / 16; ++kk) {
+                            mma_f16(dacc, dxu + 2 * kk, dvu + 2 * kk, idesc, accf);
+                            accf = 1u;
+                        }
+                    }
+                    mma_commit(&empty[slot]);
+                }
+                if (ok) mma_commit(&acc_full[buf]);
+                ++ci;
+            }
+            // every MMA issued by this thread has finished before TMEM is released
+            mma_commit(mma_done);
+            volatile int no_abort = 0;
+            mbar_wait(mma_done, 0, &no_abort, err, 2u, 100000000ull);
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int g = warp & 3;
+        const int r = g * 32 + lane;
+        const uint32_t lane_base = (uint32_t)(g * 32) << 16;
+        float* sum = reinterpret_cast<float*>(smem + a.sum_off);     // [column][128 rows]
+        int ci = 0;
+        int64_t q = qbeg, q0, q1, row;
+        bool first, last;
+        while (next_chunk(q, qbeg, qend, a.nkb, a.chunk_blocks, q0, q1, row, first, last)) {
+            const int buf = ci & 1;
+            if (!group_wait(&acc_full[buf], (ci >> 1) & 1, abort, err, 4u, 1, 128)) break;
+            tc_fence_after();
+            const int grp = (int)(row / a.btiles);
+            const int64_t bt = row - (int64_t)grp * a.btiles;
+            const int kgw = min(a.kgp, a.kp - grp * a.kgp);
+            const bool valid = bt * BM + r < a.b;
+            float* prow = a.P + ((size_t)(blockIdx.x + row) * a.kgp) * BM + r;
+            // every condition is decided once per 32 columns: the stores below
+            // are straight-line code (a branch per element costs far more than
+            // the store itself)
+            for (int c0 = 0; c0 < kgw; c0 += 32) {
+                uint32_t v[32];
+                tmem_ld32(tmem + lane_base + (uint32_t)(buf * a.kgp + c0), v);
+                tmem_ld_wait();
+                const int nj = (c0 + 32 <= kgw) ? 32 : 16;     // group widths are multiples of 16
+                float* sp = sum + c0 * BM + r;
+                if (!first) {
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) v[j] = __float_as_uint(__fadd_rn(sp[j * BM], __uint_as_float(v[j])));
+                    if (nj == 32) {
+#pragma unroll
+                        for (int j = 16; j < 32; ++j)
+                            v[j] = __float_as_uint(__fadd_rn(sp[j * BM], __uint_as_float(v[j])));
                     }
                 }
-                mma_commit(&B.empty[slot]);
-                if (kin == a.chunk_blocks - 1 || kb == a.nkb - 1) mma_commit(&B.acc1_full[buf]);
+                if (!last) {
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) sp[j * BM] = __uint_as_float(v[j]);
+                    if (nj == 32) {
+#pragma unroll
+                        for (int j = 16; j < 32; ++j) sp[j * BM] = __uint_as_float(v[j]);
+                    }
+                } else if (valid) {
+                    float* pp = prow + (size_t)c0 * BM;
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) pp[(size_t)j * BM] = __uint_as_float(v[j]);
+                    if (nj == 32) {
+#pragma unroll
+                        for (int j = 16; j < 32; ++j) pp[(size_t)j * BM] = __uint_as_float(v[j]);
+                    }
+                }
             }
-            if (ok) ok = mbar_wait(B.w_ready, 0, abort, err, 2u);
-            tc_fence_after();
-            const uint32_t whi = smem_u32(smem + a.w_off);
-            const uint32_t wlo = smem_u32(smem + a.wlo_off);
-            const uint32_t idesc2 = idesc_f16_f32(BM, a.n2);
-            for (int mt = mt_begin, t = 0; mt < mt_end && ok; ++mt, ++t) {
-                const int ab = t & 1;
-                if (!(ok = mbar_wait(&B.acc2_empty[ab], ((t >> 1) & 1) ^ 1, abort, err, 2u))) break;
-                tc_fence_after();
-                const uint32_t dcol = tmem + ab * a.n2;
-                for (int kc = 0; kc < a.kc2 && ok; ++kc, ++it) {
+            tc_fence_before();
+            mbar_arrive(&acc_empty[buf]);
+            ++ci;
+        }
+    }
+    // single-lane roles rejoin their warps first: the CTA barrier is an aligned one
+    __syncwarp();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem, a.tmem_cols);
+    }
+}
+
+// ================================================================ reduction
+struct W2Args {
+    int64_t b, btiles, nkb, Q;
+    int P1;                   // phase-1 grid size
+    int G, kgp, kp, k, planes;
+    uint32_t tile_bytes;      // one plane of one row tile: 128 x kp x 2
+    const float* P;
+    const __half* S;
+    unsigned char* W;         // [row tile][plane][tile_bytes]
+};
+
+// CTA of the phase-1 grid whose range [floor(c Q / P1), floor((c+1) Q / P1))
+// holds k-block q.
+__device__ __forceinline__ int64_t cta_of(int64_t q, int64_t Q, int64_t P1) { return ((q + 1) * P1 + Q - 1) / Q - 1; }
+
+// Writes the eight entries of W (row r, columns col0..col0+7) of row tile bt
+// into the operand image(s).
+__device__ __forceinline__ void put_w8(const W2Args& a, int64_t bt, int r, int col0, const float (&w)[8]) {
+    uint32_t hi[4], lo[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const __half h0 = __float2half_rn(w[2 * j]), h1 = __float2half_rn(w[2 * j + 1]);
+        hi[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+        lo[j] = pack_half2(w[2 * j] - __half2float(h0), w[2 * j + 1] - __half2float(h1));
+    }
+    unsigned char* base = a.W + (size_t)bt * a.planes * a.tile_bytes + w_image_off((uint32_t)r, (uint32_t)col0);
+    *reinterpret_cast<uint4*>(base) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+    if (a.planes == 2) *reinterpret_cast<uint4*>(base + a.tile_bytes) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+}
+
+// One thread per (row tile, 8 columns, row): the partials of the entry are
+// added in CTA order, kBatch partials' loads in flight at a time.
+__global__ void __launch_bounds__(256)
+apply_w2_kernel(const W2Args a) {
+    pdl_trigger();
+    pdl_wait();                    // partials of the phase-1 grid
+    const int cg8 = a.kp / 8;
+    const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= a.btiles * cg8 * BM) return;
+    const int r = (int)(e % BM);
+    const int64_t t = e / BM;
+    const int cg = (int)(t % cg8);
+    const int64_t bt = t / cg8;
+    const int col0 = cg * 8;
+    const int grp = col0 / a.kgp;               // group widths are multiples of 16
+    const int j0 = col0 - grp * a.kgp;
+    float w[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) w[i] = 0.0f;
+    if (bt * BM + r < a.b) {
+        const int64_t ur = (int64_t)grp * a.btiles + bt;
+        const int64_t cf = cta_of(ur * a.nkb, a.Q, a.P1);
+        const int64_t cl = cta_of(ur * a.nkb + a.nkb - 1, a.Q, a.P1);
+        constexpr int kBatch = 8;
+        const size_t pstride = (size_t)a.kgp * BM;
+        const float* p0 = a.P + ((size_t)(cf + ur) * a.kgp + j0) * BM + r;
+        const int64_t np = cl - cf + 1;
+        for (int64_t c0 = 0; c0 < np; c0 += kBatch) {
+            float t8[kBatch][8];
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u)
+                if (c0 + u < np) {
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) t8[u][i] = __ldg(p0 + (size_t)(c0 + u) * pstride + (size_t)i * BM);
+                }
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u)
+                if (c0 + u < np) {
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) w[i] = (c0 + u == 0) ? t8[u][i] : __fadd_rn(w[i], t8[u][i]);
+                }
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) w[i] = __fmul_rn(w[i], col0 + i < a.k ? __half2float(a.S[col0 + i]) : 0.0f);
+    }
+    put_w8(a, bt, r, col0, w);
+}
+
+// One warp per (row tile, 8 columns, row), for rows with many partials (small
+// b): lane l adds partials l, l + 32, ... in order, then the 32 lane sums are
+// combined by a fixed butterfly -- the same order on every run.
+__global__ void __launch_bounds__(256)
+apply_w2_warp_kernel(const W2Args a) {
+    pdl_trigger();
+    pdl_wait();                    // partials of the phase-1 grid
+    const int cg8 = a.kp / 8;
+    const int lane = threadIdx.x & 31;
+    const int64_t e = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (e >= a.btiles * cg8 * BM) return;
+    const int r = (int)(e % BM);
+    const int64_t t = e / BM;
+    const int cg = (int)(t % cg8);
+    const int64_t bt = t / cg8;
+    const int col0 = cg * 8;
+    const int grp = col0 / a.kgp;
+    const int j0 = col0 - grp * a.kgp;
+    float w[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) w[i] = 0.0f;
+    if (bt * BM + r < a.b) {
+        const int64_t ur = (int64_t)grp * a.btiles + bt;
+        const int64_t cf = cta_of(ur * a.nkb, a.Q, a.P1);
+        const int64_t cl = cta_of(ur * a.nkb + a.nkb - 1, a.Q, a.P1);
+        const size_t pstride = (size_t)a.kgp * BM;
+        const float* p0 = a.P + ((size_t)(cf + ur) * a.kgp + j0) * BM + r;
+        for (int64_t c = lane; c <= cl - cf; c += 32) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) w[i] = __fadd_rn(w[i], __ldg(p0 + (size_t)c * pstride + (size_t)i * BM));
+        }
+#pragma unroll
+        for (int off = 16; off >= 1; off >>= 1) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) w[i] = __fadd_rn(w[i], __shfl_xor_sync(0xffffffffu, w[i], off));
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) w[i] = __fmul_rn(w[i], col0 + i < a.k ? __half2float(a.S[col0 + i]) : 0.0f);
+    }
+    if (lane == 0) put_w8(a, bt, r, col0, w);
+}
+
+// ================================================================ phase 2
+struct YArgs {
+    int64_t m, b, T;
+    int kp, n2, kc2, mtiles, planes, stages;
+    uint32_t u_bytes, slot_bytes, tile_bytes;
+    uint32_t w_off, ystage_off, bar_off, tmem_cols;
+    int out16, tma_store;
+    const unsigned char* W;
+    void* Y;
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__ CUtensorMap tm_y, const YArgs a) {
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* smem = align1024(smem_raw);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + a.bar_off);
+    uint64_t* empty = full + a.stages;
+    uint64_t* w_full = empty + a.stages;
+    uint64_t* w_empty = w_full + 1;
+    uint64_t* acc_full = w_empty + 1;          // [2]
+    uint64_t* acc_empty = acc_full + 2;        // [2]
+    uint64_t* mma_done = acc_empty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+    volatile int* abort = reinterpret_cast<int*>(tmem_slot + 1);
+    unsigned int* err = &g_err_apply_tc;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t tbeg = a.T * blockIdx.x / gridDim.x;
+    const int64_t tend = a.T * (blockIdx.x + 1) / gridDim.x;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < a.stages; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        mbar_init(w_full, 1);
+        mbar_init(w_empty, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&acc_full[i], 1);
+            mbar_init(&acc_empty[i], 128);
+        }
+        mbar_init(mma_done, 1);
+        *abort = 0;
+        fence_barrier_init();
+        tma_prefetch_desc(&tm_u);
+        tma_prefetch_desc(&tm_y);
+    }
+    if (warp == 1) tmem_alloc(tmem_slot, a.tmem_cols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    pdl_wait();                    // W images of the reduction kernel (the prologue above overlapped it)
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            int it = 0, wl = 0;
+            int64_t cur_bt = -1;
+            bool ok = true;
+            for (int64_t t = tbeg; t < tend && ok; ++t) {
+                const int64_t bt = t / a.mtiles;
+                const int mt = (int)(t - bt * a.mtiles);
+                if (bt != cur_bt) {
+                    // W of the new row tile, once the MMAs on the previous one are done
+                    if (!(ok = mbar_wait(w_empty, (wl & 1) ^ 1, abort, err, 1u))) break;
+                    mbar_arrive_expect_tx(w_full, (uint32_t)a.planes * a.tile_bytes);
+                    for (int p = 0; p < a.planes; ++p)
+                        bulk_load(smem + a.w_off + (size_t)p * a.tile_bytes,
+                                  a.W + ((size_t)bt * a.planes + p) * a.tile_bytes, a.tile_bytes, w_full);
+                    ++wl;
+                    cur_bt = bt;
+                }
+                for (int kc = 0; kc < a.kc2; ++kc, ++it) {
                     const int slot = it % a.stages;
-                    if (!(ok = mbar_wait(&B.full[slot], (it / a.stages) & 1, abort, err, 2u))) break;
+                    if (!(ok = mbar_wait(&empty[slot], ((it / a.stages) & 1) ^ 1, abort, err, 1u))) break;
+                    mbar_arrive_expect_tx(&full[slot], a.u_bytes);
+                    tma_load_2d(smem + (size_t)slot * a.slot_bytes, &tm_u, kc * BK, (int32_t)(mt * a.n2),
+                                &full[slot]);
+                }
+            }
+            if (!ok) {
+                volatile int no_abort = 0;
+                const int first = it - a.stages > 0 ? it - a.stages : 0;
+                for (int j = first; j < it; ++j)
+                    mbar_wait(&full[j % a.stages], (j / a.stages) & 1, &no_abort, err, 0u, 100000000ull);
+                if (wl > 0) mbar_wait(w_full, (wl - 1) & 1, &no_abort, err, 0u, 100000000ull);
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            int it = 0, wl = 0, tl = 0;
+            int64_t cur_bt = -1;
+            bool ok = true;
+            const uint32_t whi = smem_u32(smem + a.w_off);
+            const uint64_t whd = smem_desc(whi, 2048, 128, 0);
+            const uint64_t wld = smem_desc(whi + a.tile_bytes, 2048, 128, 0);
+            const uint32_t idesc2 = idesc_f16_f32(BM, (uint32_t)a.n2);
+            for (int64_t t = tbeg; t < tend && ok; ++t, ++tl) {
+                const int64_t bt = t / a.mtiles;
+                if (bt != cur_bt) {
+                    if (wl > 0) mma_commit(w_empty);        // the previous W is free once these MMAs finish
+                    if (!(ok = mbar_wait(w_full, wl & 1, abort, err, 2u))) break;
                     tc_fence_after();
-                    const uint32_t ua = smem_u32(smem + (size_t)slot * a.slot_bytes);
+                    ++wl;
+                    cur_bt = bt;
+                }
+                const int ab = tl & 1;
+                if (!(ok = mbar_wait(&acc_empty[ab], ((tl >> 1) & 1) ^ 1, abort, err, 2u))) break;
+                tc_fence_after();
+                const uint32_t dcol = tmem + (uint32_t)(ab * a.n2);
+                for (int kc = 0; kc < a.kc2; ++kc, ++it) {
+                    const int slot = it % a.stages;
+                    if (!(ok = mbar_wait(&full[slot], (it / a.stages) & 1, abort, err, 2u))) break;
+                    tc_fence_after();
+                    const uint64_t ud = desc_sw128(smem_u32(smem + (size_t)slot * a.slot_bytes));
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk) {
                         const int ks = kc * (BK / 16) + kk;
                         if (ks * 16 >= a.kp) break;
-                        const uint64_t bdesc = desc_sw128(ua + kk * 32);
                         // W in the canonical layout: K-direction core matrices 2048 B apart,
-                        // M-direction core matrices 128 B apart
-                        mma_f16(dcol, smem_desc(whi + ks * 4096, 2048, 128, 0), bdesc, idesc2, (kc | kk) != 0);
-                        if (!a.out16)
-                            mma_f16(dcol, smem_desc(wlo + ks * 4096, 2048, 128, 0), bdesc, idesc2, 1u);
+                        // so 16 ranks = 4096 B = 256 in the address field
+                        mma_f16(dcol, whd + (uint64_t)ks * 256u, ud + 2 * kk, idesc2, (kc | kk) != 0);
+                        if (a.planes == 2) mma_f16(dcol, wld + (uint64_t)ks * 256u, ud + 2 * kk, idesc2, 1u);
                     }
-                    mma_commit(&B.empty[slot]);
+                    mma_commit(&empty[slot]);
                 }
-                if (ok) mma_commit(&B.acc2_full[ab]);
+                if (ok) mma_commit(&acc_full[ab]);
             }
-            // every MMA issued by this thread has finished before TMEM is released
-            mma_commit(B.mma_done);
+            mma_commit(mma_done);
             volatile int no_abort = 0;
-            mbar_wait(B.mma_done, 0, &no_abort, err, 2u, 100000000ull);
+            mbar_wait(mma_done, 0, &no_abort, err, 2u, 100000000ull);
         }
     } else {
         // ------------------------------------------------------------ epilogue
-        const int g = warp & 3;                 // TMEM lane quarter of this warp
-        const int r = g * 32 + lane;            // tile row of this thread
+        const int g = warp & 3;
+        const int r = g * 32 + lane;
         const uint32_t lane_base = (uint32_t)(g * 32) << 16;
-        bool ok = true;
-        unsigned char* whi = smem + a.w_off;
-        unsigned char* wlo = smem + a.wlo_off;
-        for (int c = 0; c < a.nchunk && ok; ++c) {
-            const int buf = c % a.acc1_bufs;
-            if (!(ok = group_wait(&B.acc1_full[buf], (c / a.acc1_bufs) & 1, abort, err, 4u, 1, 128))) break;
-            tc_fence_after();
-            const bool first = (c == 0), last = (c == a.nchunk - 1);
-            for (int c0 = 0; c0 < a.kp; c0 += 32) {
-                uint32_t v[32];
-                tmem_ld32(tmem + lane_base + buf * a.kp + c0, v);
-                tmem_ld_wait();
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const int col = c0 + q * 8;
-                    if (col >= a.kp) continue;
-                    // bytes of row r, columns col..col+7, in the core-matrix layout of W
-                    const uint32_t off = (uint32_t)(col >> 3) * 2048u + (uint32_t)(r >> 3) * 128u +
-                                         (uint32_t)(r & 7) * 16u;
-                    float w[8];
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) w[j] = __uint_as_float(v[q * 8 + j]);
-                    if (!first) {   // running sum: w[0..3] at the hi position, w[4..7] at the lo position
-                        const float4 r0 = *reinterpret_cast<const float4*>(whi + off);
-                        const float4 r1 = *reinterpret_cast<const float4*>(wlo + off);
-                        w[0] = __fadd_rn(r0.x, w[0]);
-                        w[1] = __fadd_rn(r0.y, w[1]);
-                        w[2] = __fadd_rn(r0.z, w[2]);
-                        w[3] = __fadd_rn(r0.w, w[3]);
-                        w[4] = __fadd_rn(r1.x, w[4]);
-                        w[5] = __fadd_rn(r1.y, w[5]);
-                        w[6] = __fadd_rn(r1.z, w[6]);
-                        w[7] = __fadd_rn(r1.w, w[7]);
-                    }
-                    if (!last) {
-                        *reinterpret_cast<float4*>(whi + off) = make_float4(w[0], w[1], w[2], w[3]);
-                        *reinterpret_cast<float4*>(wlo + off) = make_float4(w[4], w[5], w[6], w[7]);
-                        continue;
-                    }
-                    uint32_t hi[4], lo[4];
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const float w0 = w[2 * j] * s_f[col + 2 * j];
-                        const float w1 = w[2 * j + 1] * s_f[col + 2 * j + 1];
-                        const __half h0 = __float2half_rn(w0), h1 = __float2half_rn(w1);
-                        hi[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
-                        lo[j] = pack_half2(w0 - __half2float(h0), w1 - __half2float(h1));
-                    }
-                    *reinterpret_cast<uint4*>(whi + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-                    if (!a.out16) *reinterpret_cast<uint4*>(wlo + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-                }
-            }
-            tc_fence_before();
-            mbar_arrive(&B.acc1_empty[buf]);
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        mbar_arrive(B.w_ready);
-
         const int ecols = a.out16 ? 64 : 32;       // columns per 128-byte staging row
-        int chunk = 0;
-        for (int mt = mt_begin, t = 0; mt < mt_end && ok; ++mt, ++t) {
-            const int ab = t & 1;
-            if (!(ok = group_wait(&B.acc2_full[ab], (t >> 1) & 1, abort, err, 4u, 1, 128))) break;
+        unsigned char* wstage = smem + a.ystage_off + (size_t)g * (2 * 32 * 128);
+        int chunk = 0, tl = 0;
+        for (int64_t t = tbeg; t < tend; ++t, ++tl) {
+            const int64_t bt = t / a.mtiles;
+            const int mt = (int)(t - bt * a.mtiles);
+            const int64_t row0 = bt * BM;
+            const int ab = tl & 1;
+            if (!group_wait(&acc_full[ab], (tl >> 1) & 1, abort, err, 4u, 1, 128)) break;
             tc_fence_after();
             for (int cc = 0; cc < a.n2; cc += ecols, ++chunk) {
                 uint32_t v[64];
-                tmem_ld32(tmem + lane_base + ab * a.n2 + cc, *reinterpret_cast<uint32_t(*)[32]>(&v[0]));
-                if (a.out16)
-                    tmem_ld32(tmem + lane_base + ab * a.n2 + cc + 32, *reinterpret_cast<uint32_t(*)[32]>(&v[32]));
+                const uint32_t tcol = tmem + lane_base + (uint32_t)(ab * a.n2 + cc);
+                tmem_ld32(tcol, *reinterpret_cast<uint32_t(*)[32]>(&v[0]));
+                if (a.out16) tmem_ld32(tcol + 32, *reinterpret_cast<uint32_t(*)[32]>(&v[32]));
                 tmem_ld_wait();
-                uint32_t packed[32];
-                if (a.out16) {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        packed[j] = pack_half2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) packed[j] = v[j];
-                }
                 const int64_t col0 = (int64_t)mt * a.n2 + cc;
                 if (a.tma_store) {
-                    // this warp's 32 rows: own staging pair, own TMA store, no
-                    // barrier across the four epilogue warps
-                    unsigned char* sb = smem + a.ystage_off + (size_t)g * (2 * 32 * 128) + (chunk & 1) * (32 * 128);
+                    uint32_t packed[32];
+                    if (a.out16) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            packed[j] = pack_half2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) packed[j] = v[j];
+                    }
+                    // this warp's 32 rows: own staging pair, own TMA store
+                    unsigned char* sb = wstage + (size_t)(chunk & 1) * (32 * 128);
                     if (chunk >= 2) {
                         if (lane == 0) bulk_wait_read<1>();
                         __syncwarp();
@@ -347,9 +610,10 @@ apply_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_const
                     }
                     fence_proxy_async_smem();
                     __syncwarp();
-                    if (lane == 0 && col0 < a.m) {
-                        tma_store_2d(&tm_y, (int32_t)col0, (int32_t)(row0 + g * 32), sb);
-                        bulk_commit();
+                    if (lane == 0) {
+                        if (col0 < a.m && row0 + g * 32 < a.b)
+                            tma_store_2d(&tm_y, (int32_t)col0, (int32_t)(row0 + g * 32), sb);
+                        bulk_commit();      // one group per chunk, even empty: the staging reuse counts on it
                     }
                 } else {
                     const int64_t grow = row0 + r;
@@ -367,10 +631,12 @@ apply_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_const
                 }
             }
             tc_fence_before();
-            mbar_arrive(&B.acc2_empty[ab]);
+            mbar_arrive(&acc_empty[ab]);
         }
         if (lane == 0 && a.tma_store) bulk_wait<0>();
     }
+    // single-lane roles rejoin their warps first: the CTA barrier is an aligned one
+    __syncwarp();
     tc_fence_before();
     __syncthreads();
     if (warp == 1) {
@@ -400,16 +666,17 @@ lrc_status get_encoder() {
     return LRC_OK;
 }
 
-// 2-D map over a row-major [rows x cols] array with a row pitch of `pitch_bytes`.
-lrc_status make_map(CUtensorMap* map, CUtensorMapDataType dt, int esize, const void* base, int64_t cols,
-                    int64_t rows, int64_t pitch_bytes, uint32_t box_cols, uint32_t box_rows, const char* what) {
+// 2-D map over a row-major [rows x cols] array with a row pitch of `pitch_bytes`
+// (128-byte swizzled boxes unless stated).
+lrc_status make_map(CUtensorMap* map, CUtensorMapDataType dt, const void* base, int64_t cols, int64_t rows,
+                    int64_t pitch_bytes, uint32_t box_cols, uint32_t box_rows, const char* what,
+                    CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
     cuuint64_t strides[1] = {(cuuint64_t)pitch_bytes};
     cuuint32_t box[2] = {box_cols, box_rows};
     cuuint32_t estr[2] = {1, 1};
-    (void)esize;
     CUresult r = g_encode(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) {
         set_error("cuTensorMapEncodeTiled failed for %s (CUresult %d)", what, (int)r);
@@ -424,119 +691,196 @@ uint32_t pow2_cols(uint32_t c) {
     return p;
 }
 
+constexpr size_t kSmemMax = 227 * 1024;
+
+// Launch with programmatic stream serialization: the kernel may begin before
+// the previous kernel of the stream has finished and synchronizes with it
+// through pdl_wait().
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args&&... args) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
 }  // namespace
 
 lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y, int64_t m,
                             int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s) {
     lrc_status st = get_encoder();
     if (st != LRC_OK) return st;
-    Args a{};
-    a.m = m;
-    a.b = b;
-    a.k = (int)k;
-    a.kp = (int)((k + 15) / 16 * 16);
-    if (a.kp > 512) {
+    const int kp = (int)((k + 15) / 16 * 16);
+    if (kp > 512) {
         set_error("binary16 apply supports rank up to 512 (got %lld)", (long long)k);
         return LRC_ERR_UNSUPPORTED;
     }
-    a.out16 = out16 ? 1 : 0;
-    a.nkb = (int)((n + BK - 1) / BK);
-    a.kc2 = (a.kp + BK - 1) / BK;
-    a.v_boxes = a.kp > 256 ? 2 : 1;
-    a.v_box_rows = a.kp / a.v_boxes;
-    a.v_bytes = (uint32_t)a.kp * 128;
-    const int e_out = out16 ? 2 : 4;
-    a.tma_store = ((m * e_out) % 16 == 0) ? 1 : 0;
-    a.S = static_cast<const __half*>(S);
-    a.Y = Y;
+    const int sms = sm_count();
+    const int64_t btiles = (b + BM - 1) / BM;
+    const int planes = out16 ? 1 : 2;
+    const uint32_t tile_bytes = (uint32_t)BM * (uint32_t)kp * 2u;
 
-    // shared memory plan: widest phase-2 tile and deepest ring that fit
-    const uint32_t w_bytes = (uint32_t)BM * a.kp * 2;
-    size_t smem = 0;
-    bool chosen = false;
-    for (int n2 : {256, 128}) {
-        for (int stages = 4; stages >= 1 && !chosen; --stages) {
-            if (n2 == 256 && stages < 2) break;      // prefer a 2-deep ring with narrower tiles
-            const uint32_t u_bytes = (uint32_t)n2 * 128;
-            uint32_t slot = kXBytes + a.v_bytes > u_bytes ? kXBytes + a.v_bytes : u_bytes;
-            slot = (slot + 1023) / 1024 * 1024;
-            uint32_t off = (uint32_t)stages * slot;
-            const uint32_t w_off = off;
-            off += w_bytes;
-            const uint32_t wlo_off = out16 ? w_off : off;
-            if (!out16) off += w_bytes;
-            off = (off + 1023) / 1024 * 1024;
-            const uint32_t ystage_off = off;
-            off += 2 * 16384;
-            const uint32_t s_off = off;
-            off += (uint32_t)a.kp * 4;
-            off = (off + 7) / 8 * 8;
-            const uint32_t bar_off = off;
-            off += (uint32_t)(2 * stages + 10) * 8 + 16;
-            const size_t total = (size_t)off + 1024;    // base alignment slack
-            if (total > 227 * 1024) continue;
-            a.n2 = n2;
-            a.u_bytes = u_bytes;
-            a.slot_bytes = slot;
-            a.stages = stages;
-            a.w_off = w_off;
-            a.wlo_off = wlo_off;
-            a.ystage_off = ystage_off;
-            a.s_off = s_off;
-            a.bar_off = bar_off;
-            smem = total;
-            chosen = true;
+    // ---- phase-1 plan: column groups, ring depth, running sum
+    W1Args a1{};
+    a1.b = b;
+    a1.btiles = btiles;
+    a1.nkb = (n + BK - 1) / BK;
+    const int kg_max = out16 ? 256 : 160;
+    a1.G = (kp + kg_max - 1) / kg_max;
+    a1.kgp = ((kp + a1.G - 1) / a1.G + 15) / 16 * 16;
+    a1.kp = kp;
+    a1.Q = btiles * a1.G * a1.nkb;
+    a1.chunk_blocks = out16 ? (int)(a1.nkb < 0x7fffffff ? a1.nkb : 0x7fffffff) : kChunkBlocks;
+    const bool use_sum = a1.chunk_blocks < a1.nkb;
+    a1.slot_bytes = (uint32_t)round_up((size_t)kStageBlocks * (kXBytes + (size_t)a1.kgp * 128), 1024);
+    const uint32_t sum_bytes = use_sum ? (uint32_t)BM * a1.kgp * 4 : 0;
+    size_t smem1 = 0;
+    for (int stages = 6; stages >= 2; --stages) {
+        size_t off = (size_t)stages * a1.slot_bytes;
+        const size_t sum_off = off;
+        off += sum_bytes;
+        off = round_up(off, 8);
+        const size_t bar_off = off;
+        off += (size_t)(2 * stages + 5) * 8 + 16;
+        if (off + 1024 <= kSmemMax) {
+            a1.stages = stages;
+            a1.sum_off = (uint32_t)sum_off;
+            a1.bar_off = (uint32_t)bar_off;
+            smem1 = off + 1024;
+            break;
         }
-        if (chosen) break;
     }
-    if (!chosen) {
+    if (!smem1) {
         set_error("binary16 apply: rank %lld does not fit in shared memory", (long long)k);
         return LRC_ERR_UNSUPPORTED;
     }
-    // chunked phase-1 accumulation for FP32 output; one chunk for FP16 output
-    a.chunk_blocks = out16 ? a.nkb : kChunkBlocks;
-    a.nchunk = (a.nkb + a.chunk_blocks - 1) / a.chunk_blocks;
-    a.acc1_bufs = (a.nchunk > 1 && 2 * a.kp <= 512) ? 2 : 1;
-    const uint32_t acc1_cols = (uint32_t)(a.acc1_bufs * a.kp);
-    a.tmem_cols = pow2_cols(acc1_cols > (uint32_t)(2 * a.n2) ? acc1_cols : (uint32_t)(2 * a.n2));
-    a.mtiles = (int)((m + a.n2 - 1) / a.n2);
+    // two accumulators at columns 0 and kgp; the epilogue reads 32 columns at a time
+    a1.tmem_cols = pow2_cols((uint32_t)a1.kgp + (uint32_t)round_up((size_t)a1.kgp, 32));
+    const int64_t P1 = a1.Q < sms ? a1.Q : sms;
 
-    const int64_t btiles = (b + BM - 1) / BM;
-    if (btiles > 0x7fffffff) {
-        set_error("binary16 apply: batch too large");
+    // ---- phase-2 plan: tile width, ring depth
+    YArgs a3{};
+    a3.m = m;
+    a3.b = b;
+    a3.kp = kp;
+    a3.kc2 = (kp + BK - 1) / BK;
+    a3.planes = planes;
+    a3.tile_bytes = tile_bytes;
+    a3.out16 = out16 ? 1 : 0;
+    const int e_out = out16 ? 2 : 4;
+    a3.tma_store = ((m * e_out) % 16 == 0) ? 1 : 0;
+    a3.Y = Y;
+    size_t smem3 = 0;
+    for (int n2 : {256, 128}) {
+        if (n2 == 256 && btiles * ((m + 255) / 256) < 2 * (int64_t)sms) continue;   // too few tiles
+        for (int stages = 4; stages >= 2 && !smem3; --stages) {
+            if (n2 == 256 && stages < 3) break;      // prefer a deeper ring with narrower tiles
+            const uint32_t u_bytes = (uint32_t)n2 * 128;
+            size_t off = (size_t)stages * u_bytes;
+            const size_t w_off = off;
+            off += (size_t)planes * tile_bytes;
+            off = round_up(off, 1024);
+            const size_t ystage_off = off;
+            off += 4 * 2 * 32 * 128;
+            const size_t bar_off = off;
+            off += (size_t)(2 * stages + 7) * 8 + 16;
+            if (off + 1024 > kSmemMax) continue;
+            a3.n2 = n2;
+            a3.stages = stages;
+            a3.u_bytes = u_bytes;
+            a3.slot_bytes = u_bytes;
+            a3.w_off = (uint32_t)w_off;
+            a3.ystage_off = (uint32_t)ystage_off;
+            a3.bar_off = (uint32_t)bar_off;
+            smem3 = off + 1024;
+        }
+        if (smem3) break;
+    }
+    if (!smem3) {
+        set_error("binary16 apply: rank %lld does not fit in shared memory", (long long)k);
         return LRC_ERR_UNSUPPORTED;
     }
-    const int sms = sm_count();
-    int64_t splits = btiles >= sms ? 1 : sms / btiles;
-    if (splits < 1) splits = 1;
-    if (splits > a.mtiles) splits = a.mtiles;
-    a.mt_per_cta = (int)((a.mtiles + splits - 1) / splits);
-    const int gy = (a.mtiles + a.mt_per_cta - 1) / a.mt_per_cta;
-    if (gy > 65535) {
-        set_error("binary16 apply: too many column tiles");
-        return LRC_ERR_UNSUPPORTED;
-    }
+    a3.mtiles = (int)((m + a3.n2 - 1) / a3.n2);
+    a3.T = btiles * a3.mtiles;
+    a3.tmem_cols = pow2_cols(2u * (uint32_t)a3.n2);
+    const int64_t P3 = a3.T < sms ? a3.T : sms;
+
+    // ---- workspace: W images, then the phase-1 partials
+    const size_t w_bytes_total = round_up((size_t)btiles * planes * tile_bytes, 256);
+    const size_t p_bytes = (size_t)(btiles * a1.G + P1) * a1.kgp * BM * sizeof(float);
+    void* ws = nullptr;
+    if ((st = stream_workspace(s, w_bytes_total + p_bytes, &ws)) != LRC_OK) return st;
+    unsigned char* Wimg = static_cast<unsigned char*>(ws);
+    a1.P = reinterpret_cast<float*>(Wimg + w_bytes_total);
+    a3.W = Wimg;
 
     const int64_t ldn = lrc_packed_ld(n), ldk = lrc_packed_ld(k);
-    CUtensorMap tx, tv, tu, ty;
-    if ((st = make_map(&tx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, X, n, b, ldn * 2, BK, BM, "X")) != LRC_OK) return st;
-    if ((st = make_map(&tv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, Vt, n, k, ldn * 2, BK, (uint32_t)a.v_box_rows, "Vt")) !=
-        LRC_OK)
+    CUtensorMap tx, tv, tu, ty, txp, tvp;
+    if ((st = make_map(&tx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, X, n, b, ldn * 2, BK, BM, "X")) != LRC_OK) return st;
+    if ((st = make_map(&tv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, Vt, n, k, ldn * 2, BK, (uint32_t)a1.kgp, "Vt")) != LRC_OK)
         return st;
-    if ((st = make_map(&tu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, U, k, m, ldk * 2, BK, (uint32_t)a.n2, "U")) != LRC_OK)
+    if ((st = make_map(&txp, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, X, n, b, ldn * 2, kPfBlocks * BK, BM, "X prefetch",
+                       CU_TENSOR_MAP_SWIZZLE_NONE)) != LRC_OK)
         return st;
-    if (a.tma_store) {
-        if ((st = make_map(&ty, out16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, e_out, Y, m,
-                           b, m * e_out, out16 ? 64 : 32, 32, "Y")) != LRC_OK)
+    if ((st = make_map(&tvp, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, Vt, n, k, ldn * 2, kPfBlocks * BK, (uint32_t)a1.kgp,
+                       "Vt prefetch", CU_TENSOR_MAP_SWIZZLE_NONE)) != LRC_OK)
+        return st;
+    if ((st = make_map(&tu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, U, k, m, ldk * 2, BK, (uint32_t)a3.n2, "U")) != LRC_OK)
+        return st;
+    if (a3.tma_store) {
+        if ((st = make_map(&ty, out16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, Y, m, b,
+                           m * e_out, out16 ? 64 : 32, 32, "Y")) != LRC_OK)
             return st;
     } else {
         ty = tu;   // unused by the kernel
     }
-    cudaError_t e = cudaFuncSetAttribute(apply_f16_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return cuda_fail(e, "apply_f16_tc_kernel smem attribute");
-    dim3 grid((unsigned)btiles, (unsigned)gy);
-    apply_f16_tc_kernel<<<grid, kThreads, smem, s>>>(tx, tv, tu, ty, a);
-    return after_launch("apply_f16_tc_kernel");
+
+    cudaError_t e = cudaFuncSetAttribute(apply_w1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
+    if (e != cudaSuccess) return cuda_fail(e, "apply_w1_kernel smem attribute");
+    apply_w1_kernel<<<(unsigned)P1, kThreads, smem1, s>>>(tx, tv, txp, tvp, a1);
+    if ((st = after_launch("apply_w1_kernel")) != LRC_OK) return st;
+
+    W2Args a2{};
+    a2.b = b;
+    a2.btiles = btiles;
+    a2.nkb = a1.nkb;
+    a2.Q = a1.Q;
+    a2.P1 = (int)P1;
+    a2.G = a1.G;
+    a2.kgp = a1.kgp;
+    a2.kp = kp;
+    a2.k = (int)k;
+    a2.planes = planes;
+    a2.tile_bytes = tile_bytes;
+    a2.P = a1.P;
+    a2.S = static_cast<const __half*>(S);
+    a2.W = Wimg;
+    const int64_t n2items = btiles * (kp / 8) * BM;
+    const int64_t max_parts = (a1.nkb * P1 + a1.Q - 1) / a1.Q + 1;     // CTAs sharing one row, at most
+    if (max_parts >= 16) {
+        e = launch_pdl(apply_w2_warp_kernel, dim3((unsigned)((n2items * 32 + 255) / 256)), dim3(256), 0, s, a2);
+        if (e != cudaSuccess) return cuda_fail(e, "apply_w2_warp_kernel launch");
+        if ((st = after_launch("apply_w2_warp_kernel")) != LRC_OK) return st;
+    } else {
+        e = launch_pdl(apply_w2_kernel, dim3((unsigned)((n2items + 255) / 256)), dim3(256), 0, s, a2);
+        if (e != cudaSuccess) return cuda_fail(e, "apply_w2_kernel launch");
+        if ((st = after_launch("apply_w2_kernel")) != LRC_OK) return st;
+    }
+
+    e = cudaFuncSetAttribute(apply_y_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem3);
+    if (e != cudaSuccess) return cuda_fail(e, "apply_y_kernel smem attribute");
+    e = launch_pdl(apply_y_kernel, dim3((unsigned)P3), dim3(kThreads), smem3, s, tu, ty, a3);
+    if (e != cudaSuccess) return cuda_fail(e, "apply_y_kernel launch");
+    return after_launch("apply_y_kernel");
 }
 
 namespace {

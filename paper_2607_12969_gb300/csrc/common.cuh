@@ -80,6 +80,9 @@ lrc_status launch_wait_timeout_probe(int64_t limit_ns, cudaStream_t s);
 lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
                         double* diff_out, double* normA_out, cudaStream_t s);
 void release_scratch();
+// Per-(device, stream) workspace, grown on demand; freed by release_workspaces().
+lrc_status stream_workspace(cudaStream_t s, size_t bytes, void** out);
+void release_workspaces();
 lrc_status run_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
                                 double* diff_out, double* normA_out, cudaStream_t s);
 int64_t fro_diff_noalloc_max_count();

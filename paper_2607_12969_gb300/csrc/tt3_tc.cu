@@ -17,8 +17,9 @@
 // D1 lives in the first columns of the unit's own D2 accumulator, so two
 // units are in flight within 2 x slice <= 512 TMEM columns.  Warp roles:
 //   0..3 epilogue, 4..7 converters, 8 MMA issuer (one thread), 9..12 loaders
-//   (G_1 tile, G_2(i_2)^T per unit, G_3^T once; 4-byte loads batched eight
-//   deep so that many are in flight; operand padding is zeroed once).
+//   (G_1 tile, G_2(i_2)^T per unit through an asynchronous-copy ring).  G_3^T
+//   and the zero operand padding are written once by all threads before the
+//   roles split.
 // Intermediates never reach global memory.
 #include <cudaTypedefs.h>
 
@@ -58,7 +59,7 @@ struct T3Args {
 };
 
 struct Bars {
-    uint64_t *a1_full, *a1_empty, *b2_ready;
+    uint64_t *a1_full, *a1_empty;
     uint64_t *b1_full, *b1_empty;      // [2]
     uint64_t *d1_full;                 // [2]
     uint64_t *a2_full, *a2_empty;      // [2]
@@ -73,7 +74,6 @@ __device__ __forceinline__ Bars carve(unsigned char* smem, const T3Args& a) {
     Bars B;
     B.a1_full = p + 0;
     B.a1_empty = p + 1;
-    B.b2_ready = p + 2;
     B.b1_full = p + 3;
     B.b1_empty = p + 5;
     B.d1_full = p + 7;
@@ -171,6 +171,52 @@ __device__ __forceinline__ void b1_direct(const T3Args& a, int64_t i, int lt, un
     }
 }
 
+// Shared prologue, all threads: zero A1 and both B1 buffers (their padding
+// rows and columns stay zero), then write G_3^T (n_3 rows, r2p ranks,
+// K-major) into B2.  A thread takes a 2 x 2 block -- ranks k, k+1 of
+// outputs c, c+1 -- as two 4-byte loads along n_3 and writes it as two 4-byte
+// words, one per B2 row; eight blocks per thread are in flight.
+__device__ __forceinline__ void build_g3t(const T3Args& a, unsigned char* smem) {
+    const int nt = blockDim.x;
+    uint4* z = reinterpret_cast<uint4*>(smem + a.off_a1);
+    const uint32_t zbytes = a.off_b2 - a.off_a1;
+    for (uint32_t e = threadIdx.x; e < zbytes / 16; e += nt) z[e] = make_uint4(0, 0, 0, 0);
+    unsigned char* b2 = smem + a.off_b2;
+    const int cpairs = a.nd / 2;                              // n_3 is a multiple of 16
+    const int total = cpairs * (a.r2p / 2);
+    const bool words = (reinterpret_cast<uintptr_t>(a.G3) & 3u) == 0;
+    for (int e0 = threadIdx.x; e0 < total; e0 += nt * kBatch) {
+        uint32_t w0[kBatch], w1[kBatch];
+#pragma unroll
+        for (int t = 0; t < kBatch; ++t) {
+            const int e = e0 + t * nt;
+            const int k = 2 * (e / cpairs), c = 2 * (e % cpairs);
+            w0[t] = 0;
+            w1[t] = 0;
+            if (e < total) {
+                const __half* p0 = a.G3 + (int64_t)k * a.nd + c;
+                if (k < a.r2)
+                    w0[t] = words ? __ldg(reinterpret_cast<const unsigned int*>(p0))
+                                  : (uint32_t)__half_as_ushort(p0[0]) | ((uint32_t)__half_as_ushort(p0[1]) << 16);
+                if (k + 1 < a.r2) {
+                    const __half* p1 = p0 + a.nd;
+                    w1[t] = words ? __ldg(reinterpret_cast<const unsigned int*>(p1))
+                                  : (uint32_t)__half_as_ushort(p1[0]) | ((uint32_t)__half_as_ushort(p1[1]) << 16);
+                }
+            }
+        }
+#pragma unroll
+        for (int t = 0; t < kBatch; ++t) {
+            const int e = e0 + t * nt;
+            if (e < total) {
+                const int k = 2 * (e / cpairs), c = 2 * (e % cpairs);
+                *reinterpret_cast<uint32_t*>(b2 + canon_off(c, k, a.nd)) = (w0[t] & 0xffffu) | (w1[t] << 16);
+                *reinterpret_cast<uint32_t*>(b2 + canon_off(c + 1, k, a.nd)) = (w0[t] >> 16) | (w1[t] & 0xffff0000u);
+            }
+        }
+    }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
 tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
     extern __shared__ unsigned char smem_raw[];
@@ -188,7 +234,6 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
     if (threadIdx.x == 0) {
         mbar_init(B.a1_full, 1);
         mbar_init(B.a1_empty, 1);
-        mbar_init(B.b2_ready, 1);
         for (int q = 0; q < 2; ++q) {
             mbar_init(&B.b1_full[q], 1);
             mbar_init(&B.b1_empty[q], 1);
@@ -203,6 +248,22 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
         fence_barrier_init();
     }
     if (warp == 8) tmem_alloc(B.tmem_slot, a.tmem_cols);
+    uint32_t* raw = reinterpret_cast<uint32_t*>(smem + a.off_raw);
+    const uint32_t raw_words = a.raw_bytes / 4;
+    if (warp >= 9 && a.g2_words) {
+        // start the first kRaw - 1 G_2 slices before the shared prologue
+        for (int64_t p = 0; p < kRaw - 1; ++p) {
+            if (p < nunits) {
+                int64_t qp, ip;
+                int hp;
+                unit_coords(a, ubeg + p, qp, ip, hp);
+                raw_issue(a, ip, warp - 9, lane, raw + (uint32_t)(p % kRaw) * raw_words);
+            }
+            cp_async_commit();
+        }
+    }
+    build_g3t(a, smem);          // every thread: operand padding and G_3^T
+    fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -212,37 +273,8 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
         // ------------------------------------------------------------ loaders
         const int lt = threadIdx.x - 288;                      // 0..127
         const bool leader = (lt == 0);
-        {   // zero the operand buffers once (padding rows / columns stay zero),
-            // then G_3^T: n_3 rows x r2p
-            uint4* z = reinterpret_cast<uint4*>(smem + a.off_a1);
-            const uint32_t zbytes = a.off_b2 - a.off_a1;      // A1, B1 x 2 (A2 is written whole)
-            for (uint32_t e = lt; e < zbytes / 16; e += kLoadThreads) z[e] = make_uint4(0, 0, 0, 0);
-            unsigned char* b2 = smem + a.off_b2;
-            for (int e = lt; e < a.nd * a.r2p; e += kLoadThreads) {
-                const int row = e / a.r2p, k = e % a.r2p;
-                const __half v = k < a.r2 ? a.G3[(int64_t)k * a.nd + row] : __float2half_rn(0.0f);
-                *reinterpret_cast<__half*>(b2 + canon_off(row, k, a.nd)) = v;
-            }
-            fence_proxy_async_smem();
-            named_bar_sync(3, kLoadThreads);
-            if (leader) mbar_arrive(B.b2_ready);
-        }
         int64_t prev_qt = -1;
         int builds = 0;
-        uint32_t* raw = reinterpret_cast<uint32_t*>(smem + a.off_raw);
-        const uint32_t raw_words = a.raw_bytes / 4;
-        // keep kRaw - 1 slices in flight ahead of the unit being prepared
-        if (a.g2_words) {
-            for (int64_t p = 0; p < kRaw - 1; ++p) {
-                if (p < nunits) {
-                    int64_t qp, ip;
-                    int hp;
-                    unit_coords(a, ubeg + p, qp, ip, hp);
-                    raw_issue(a, ip, lt >> 5, lane, raw + (uint32_t)(p % kRaw) * raw_words);
-                }
-                cp_async_commit();
-            }
-        }
         for (int64_t j = 0; j < nunits; ++j) {
             int64_t qt, i;
             int h;
@@ -317,7 +349,7 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
     } else if (warp == 8) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            bool ok = mbar_wait(B.b2_ready, 0, abort, err, 2u);
+            bool ok = true;
             const uint32_t idesc1 = idesc_f16_f32(BM, (uint32_t)a.r2p);
             const uint32_t idesc2 = idesc_f16_f32(BM, (uint32_t)a.n2h);
             const uint32_t a1s = smem_u32(smem + a.off_a1);
@@ -339,9 +371,12 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
                 tc_fence_after();
                 const uint32_t b1s = smem_u32(smem + a.off_b1 + (size_t)buf * a.b1_bytes);
                 const uint32_t lbo1 = (uint32_t)a.r2p * 16u;
+                // descriptors stepped by adds: 16 ranks = 4096 B of A, 2 x lbo1 B of B
+                const uint64_t ad = smem_desc(a1s, 2048, 128, 0), bd = smem_desc(b1s, lbo1, 128, 0);
+                const uint64_t bstep = (uint64_t)(2u * lbo1) >> 4;
                 for (int ks = 0; ks < a.r1p / 16; ++ks)
-                    mma_f16(tmem + (uint32_t)buf * a.n2h, smem_desc(a1s + ks * 4096, 2048, 128, 0),
-                            smem_desc(b1s + ks * 2 * lbo1, lbo1, 128, 0), idesc1, ks > 0);
+                    mma_f16(tmem + (uint32_t)buf * a.n2h, ad + (uint64_t)ks * 256u, bd + (uint64_t)ks * bstep, idesc1,
+                            ks > 0);
                 mma_commit(&B.b1_empty[buf]);
                 mma_commit(&B.d1_full[buf]);
                 // last unit of this i_1 tile: G_1 tile may be replaced once these MMAs finish
@@ -366,13 +401,13 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
                 const uint32_t alo = ahi + a.a2_bytes;
                 const uint32_t lbo2 = (uint32_t)a.nd * 16u;
                 const uint32_t bslice = b2s + (uint32_t)h * (uint32_t)a.n2h * 16u;   // rows h*n2h..
+                const uint64_t bd = smem_desc(bslice, lbo2, 128, 0);
+                const uint64_t hd = smem_desc(ahi, 2048, 128, 0), ld = smem_desc(alo, 2048, 128, 0);
+                const uint64_t bstep = (uint64_t)(2u * lbo2) >> 4;
                 for (int ks = 0; ks < a.r2p / 16; ++ks) {
-                    const uint64_t bdesc = smem_desc(bslice + ks * 2 * lbo2, lbo2, 128, 0);
-                    mma_f16(tmem + (uint32_t)buf * a.n2h, smem_desc(ahi + ks * 4096, 2048, 128, 0), bdesc, idesc2,
-                            ks > 0);
-                    if (!a.out16)
-                        mma_f16(tmem + (uint32_t)buf * a.n2h, smem_desc(alo + ks * 4096, 2048, 128, 0), bdesc,
-                                idesc2, 1u);
+                    const uint64_t bdesc = bd + (uint64_t)ks * bstep;
+                    mma_f16(tmem + (uint32_t)buf * a.n2h, hd + (uint64_t)ks * 256u, bdesc, idesc2, ks > 0);
+                    if (!a.out16) mma_f16(tmem + (uint32_t)buf * a.n2h, ld + (uint64_t)ks * 256u, bdesc, idesc2, 1u);
                 }
                 mma_commit(&B.a2_empty[buf]);
                 mma_commit(&B.d2_full[buf]);
@@ -480,6 +515,8 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
         if (lane == 0) bulk_wait<0>();
         (void)r;
     }
+    // single-lane roles rejoin their warps first: the CTA barrier is an aligned one
+    __syncwarp();
     tc_fence_before();
     __syncthreads();
     if (warp == 8) {

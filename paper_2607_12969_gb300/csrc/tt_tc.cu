@@ -240,6 +240,8 @@ tt_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const TTArgs a) {
             const uint32_t bsm = smem_u32(smem + a.off_b);
             const uint32_t idesc = idesc_f16_f32(BM, (uint32_t)a.nd);
             const uint32_t lbo_b = (uint32_t)a.nd * 16u;
+            const uint64_t bd = smem_desc(bsm, lbo_b, 128, 0);
+            const uint64_t bstep = (uint64_t)(2u * lbo_b) >> 4;
             for (int64_t j = 0; j < my_tiles && ok; ++j) {
                 const int buf = (int)(j & 1);
                 const uint32_t par = (uint32_t)((j >> 1) & 1);
@@ -249,10 +251,12 @@ tt_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const TTArgs a) {
                 const uint32_t ahi = smem_u32(smem + a.off_a + (size_t)buf * 2 * a.a_bytes);
                 const uint32_t alo = ahi + a.a_bytes;
                 const uint32_t dcol = tmem + (uint32_t)buf * (uint32_t)a.nd;
+                // descriptors stepped by adds (16 ranks = 4096 B of A, 2 x lbo_b B of B)
+                const uint64_t hd = smem_desc(ahi, 2048, 128, 0), ld = smem_desc(alo, 2048, 128, 0);
                 for (int ks = 0; ks < a.rp / 16; ++ks) {
-                    const uint64_t bdesc = smem_desc(bsm + ks * 2 * lbo_b, lbo_b, 128, 0);
-                    mma_f16(dcol, smem_desc(ahi + ks * 4096, 2048, 128, 0), bdesc, idesc, ks > 0);
-                    if (!a.out16) mma_f16(dcol, smem_desc(alo + ks * 4096, 2048, 128, 0), bdesc, idesc, 1u);
+                    const uint64_t bdesc = bd + (uint64_t)ks * bstep;
+                    mma_f16(dcol, hd + (uint64_t)ks * 256u, bdesc, idesc, ks > 0);
+                    if (!a.out16) mma_f16(dcol, ld + (uint64_t)ks * 256u, bdesc, idesc, 1u);
                 }
                 mma_commit(&B.a_empty[buf]);
                 mma_commit(&B.acc_full[buf]);
@@ -316,6 +320,8 @@ tt_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const TTArgs a) {
         }
         if (issuer) bulk_wait<0>();
     }
+    // single-lane roles rejoin their warps first: the CTA barrier is an aligned one
+    __syncwarp();
     tc_fence_before();
     __syncthreads();
     if (warp == 8) {

@@ -1,0 +1,69 @@
+// workspace.cu -- device workspace of the split-phase apply: one buffer per
+// (device, stream), allocated on first use and grown when a larger problem
+// arrives.  Growing waits for the stream (work already queued may still use
+// the old buffer) before the old buffer is freed.  Calls on different
+// streams get different buffers, so they may run concurrently; calls on one
+// stream are ordered by the stream.  lrc_shutdown() frees every buffer.
+#include <map>
+#include <mutex>
+#include <utility>
+
+#include "common.cuh"
+
+namespace lrc {
+
+namespace {
+
+struct Buf {
+    void* ptr = nullptr;
+    size_t bytes = 0;
+};
+
+std::mutex g_ws_mu;
+std::map<std::pair<int, cudaStream_t>, Buf> g_ws;
+
+}  // namespace
+
+lrc_status stream_workspace(cudaStream_t s, size_t bytes, void** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    std::lock_guard<std::mutex> lock(g_ws_mu);
+    Buf& b = g_ws[std::make_pair(dev, s)];
+    if (b.bytes < bytes) {
+        if (b.ptr) {
+            e = cudaStreamSynchronize(s);
+            if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize (workspace growth)");
+            cudaFree(b.ptr);
+            b.ptr = nullptr;
+            b.bytes = 0;
+        }
+        const size_t want = (bytes + ((size_t)1 << 20) - 1) & ~(((size_t)1 << 20) - 1);   // whole MiB
+        e = cudaMalloc(&b.ptr, want);
+        if (e != cudaSuccess) {
+            b.ptr = nullptr;
+            cudaGetLastError();
+            set_error("workspace allocation of %zu bytes failed: %s", want, cudaGetErrorString(e));
+            return LRC_ERR_NOMEM;
+        }
+        b.bytes = want;
+    }
+    *out = b.ptr;
+    return LRC_OK;
+}
+
+void release_workspaces() {
+    std::lock_guard<std::mutex> lock(g_ws_mu);
+    int prev = -1;
+    cudaGetDevice(&prev);
+    for (auto& kv : g_ws) {
+        if (kv.second.ptr) {
+            cudaSetDevice(kv.first.first);
+            cudaFree(kv.second.ptr);
+        }
+    }
+    g_ws.clear();
+    if (prev >= 0) cudaSetDevice(prev);
+}
+
+}  // namespace lrc
