@@ -176,7 +176,7 @@ apply_cc_kernel(const T* __restrict__ U, const T* __restrict__ S, const T* __res
 // slab is fetched into registers while the current one is multiplied.
 // ---------------------------------------------------------------------------
 namespace f32k {
-constexpr int BM = 32, BN = 64, BK1 = 32, BK2 = 16, TM = 4, TN = 4, TX = 16, TY = 8, NT = 128;
+constexpr int BM = 32, BN = 64, BK1 = 32, BK2 = 16, TM = 4, TN = 4, TX = 16, NT = 128;
 constexpr int LDA = BM + 4, LDB = BN + 4;     // 16-byte aligned rows
 }
 
@@ -398,14 +398,20 @@ lrc_status launch_apply_cc(const T* U, const T* S, const T* Vt, const T* X, T* Y
 
 }  // namespace
 
+// Batches below these sizes leave the fused kernels' row tiles too few to
+// fill the GPU; they take the split path of apply_split.cu (ranks up to 1024).
+constexpr int64_t kSplitMaxBatchF64 = 2048, kSplitMaxBatchF32 = 256, kSplitMaxRank = 1024;
+
 lrc_status launch_apply_f64(const double* U, const double* S, const double* Vt, const double* X,
                             double* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s) {
+    if (b <= kSplitMaxBatchF64 && k <= kSplitMaxRank) return launch_apply_split_f64(U, S, Vt, X, Y, m, n, k, b, s);
     return launch_apply_cc<double>(U, S, Vt, X, Y, m, n, k, b, s, "apply_cc_kernel<f64>");
 }
 
 lrc_status launch_apply_f32(const float* U, const float* S, const float* Vt, const float* X,
                             float* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s) {
     using namespace f32k;
+    if (b <= kSplitMaxBatchF32 && k <= kSplitMaxRank) return launch_apply_split_f32(U, S, Vt, X, Y, m, n, k, b, s);
     const char* name = "apply_f32_kernel";
     if (k > 4096) {
         set_error("%s: rank %lld above the supported 4096", name, (long long)k);

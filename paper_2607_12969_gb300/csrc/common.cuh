@@ -54,6 +54,11 @@ lrc_status launch_apply_f64(const double* U, const double* S, const double* Vt, 
                             double* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
 lrc_status launch_apply_f32(const float* U, const float* S, const float* Vt, const float* X,
                             float* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
+// small-batch split path of the CUDA-core apply (apply_split.cu)
+lrc_status launch_apply_split_f64(const double* U, const double* S, const double* Vt, const double* X, double* Y,
+                                  int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
+lrc_status launch_apply_split_f32(const float* U, const float* S, const float* Vt, const float* X, float* Y,
+                                  int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
 lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y,
                             int64_t m, int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s);
 
