@@ -260,8 +260,9 @@ lrc_status lrc_device_status(lrc_stream_t stream) {
     const uint32_t a = take_apply_tc_error();
     const uint32_t t1 = take_tt_tc_error();
     const uint32_t t3 = take_tt3_tc_error();
-    const uint32_t t = t1 | t3;
-    if (a == 0xffffffffu || t1 == 0xffffffffu || t3 == 0xffffffffu) {
+    const uint32_t tn = take_ttn_tc_error();
+    const uint32_t t = t1 | t3 | tn;
+    if (a == 0xffffffffu || t1 == 0xffffffffu || t3 == 0xffffffffu || tn == 0xffffffffu) {
         set_error("could not read the device error words");
         return LRC_ERR_CUDA;
     }

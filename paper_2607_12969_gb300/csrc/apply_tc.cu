@@ -36,7 +36,6 @@
 #include <cudaTypedefs.h>
 
 #include <mutex>
-#include <utility>
 
 #include "common.cuh"
 #include "tc.cuh"
@@ -693,23 +692,6 @@ uint32_t pow2_cols(uint32_t c) {
 
 constexpr size_t kSmemMax = 227 * 1024;
 
-// Launch with programmatic stream serialization: the kernel may begin before
-// the previous kernel of the stream has finished and synchronizes with it
-// through pdl_wait().
-template <typename... KArgs, typename... Args>
-cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args&&... args) {
-    cudaLaunchConfig_t cfg{};
-    cfg.gridDim = grid;
-    cfg.blockDim = block;
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
-}
 
 size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 

@@ -4,6 +4,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "lrc.h"
 
 namespace lrc {
@@ -19,6 +21,24 @@ lrc_status after_launch(const char* what);
 
 // Multiprocessor count of the current device (cached per device).
 int sm_count();
+
+// Launch with programmatic stream serialization: the kernel may begin before
+// the previous kernel of the stream has finished and synchronizes with it
+// through pdl_wait().
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args&&... args) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -80,6 +100,10 @@ uint32_t take_tt3_tc_error();
 // 3-way binary16 TT on the tensor cores; *handled = false when the shape is
 // outside the kernel (nothing launched).
 lrc_status launch_tt3_f16_tc(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled);
+// binary16 TT with narrow last two modes on the tensor cores (tt_narrow_tc.cu);
+// *handled = false when the shape is outside the kernel (nothing launched).
+lrc_status launch_ttn_f16_tc(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled);
+uint32_t take_ttn_tc_error();
 lrc_status launch_wait_timeout_probe(int64_t limit_ns, cudaStream_t s);
 
 lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,

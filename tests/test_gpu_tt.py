@@ -56,6 +56,40 @@ def test_random_cores_vs_oracle(lrc, cuda, fmt, dims, r, kind):
     assert err <= TOL[fmt], (fmt, err)
 
 
+# narrow last two modes (the binary16 path batches all i_{d-1} in one product):
+# d = 3, 4, 5; ragged prefix count; rank padding in both products; a
+# non-square last pair
+NARROW = [
+    ((3, 16, 16), (1, 3, 16, 1)),
+    ((4, 5, 16, 16), (1, 3, 7, 16, 1)),
+    ((2, 3, 4, 16, 16), (1, 2, 6, 20, 16, 1)),
+    ((5, 8, 32), (1, 4, 8, 1)),
+    ((257, 16, 16), (1, 9, 12, 1)),
+    ((70, 4, 64), (1, 33, 16, 1)),
+]
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("dims,ranks", NARROW)
+def test_narrow_last_modes_vs_oracle(lrc, cuda, fmt, dims, ranks):
+    cores = W.make_tt(dims, ranks, "gauss_geo", 23)
+    got, rc = run_tt(lrc, cuda, cores, fmt)
+    want = oracle.tt_full(rc).reshape(-1)
+    err = rel_fro(got, want)
+    assert err <= TOL[fmt], (fmt, err)
+
+
+@pytest.mark.parametrize("fmt", ["f16"])
+@pytest.mark.parametrize("dims,ranks", NARROW)
+def test_narrow_last_modes_integer_exact(lrc, cuda, fmt, dims, ranks):
+    # small integers: every product and partial sum is exact, and the hi/lo
+    # split represents every intermediate exactly
+    cores = [W.integer_valued((ranks[l], dims[l], ranks[l + 1]), 70 + l, -1, 1) for l in range(len(dims))]
+    got, rc = run_tt(lrc, cuda, cores, fmt)
+    want = oracle.tt_full(rc).reshape(-1)
+    assert np.array_equal(got, want)
+
+
 @pytest.mark.parametrize("fmt", FMTS)
 @pytest.mark.parametrize("name", ["tt3", "tt6", "tt_hsi"])
 def test_workloads_sampled_entries(lrc, cuda, fmt, name):
