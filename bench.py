@@ -138,9 +138,7 @@ class Step:
         self.cfg = cfg
         q1, sig, q2 = W.matrix_bases(cfg)
         self.sigma = sig
-        X = W.queries(cfg)
-        if seed_offset:
-            X = X + 0.0  # every rank evaluates the same seeded batch shape
+        X = W.queries(cfg, replica=seed_offset)   # every rank: its own batch of the same shape
         self.host = {"Q1": np.ascontiguousarray(q1), "Q2t": np.ascontiguousarray(q2.T), "s": sig[:cfg.k_max].copy(),
                      "X": X}
         ttc = W.TT_CONFIGS["tt3"]

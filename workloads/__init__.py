@@ -156,9 +156,11 @@ def matrix_factors(cfg: MatrixConfig, fmt: str) -> Factors:
     return truncate(q1, sig, q2, cfg.ranks[fmt])
 
 
-def queries(cfg: MatrixConfig, b: int | None = None) -> np.ndarray:
-    """Seeded N(0,1) query batch X, b x n, one query per row."""
-    rng = np.random.default_rng(1000 * cfg.cfg + 3)
+def queries(cfg: MatrixConfig, b: int | None = None, replica: int = 0) -> np.ndarray:
+    """Seeded N(0,1) query batch X, b x n, one query per row.  `replica` r > 0
+    draws an independent batch of the same shape (one per GPU when the
+    benchmark runs replicas: weak scaling)."""
+    rng = np.random.default_rng(1000 * cfg.cfg + 3 + 100000 * replica)
     bb = cfg.b if b is None else b
     return rng.standard_normal((bb, cfg.n))
 
