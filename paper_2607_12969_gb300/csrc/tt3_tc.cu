@@ -14,12 +14,16 @@
 //   store    D2 -> registers -> 128-byte-swizzled staging -> 3-D TMA stores
 //            of out[i_1 tile, i_2, slice] (rows n_2 n_3 elements apart), each
 //            epilogue warp storing its own 32 rows.
-// D1 lives in the first columns of the unit's own D2 accumulator, so two
-// units are in flight within 2 x slice <= 512 TMEM columns.  Warp roles:
-//   0..3 epilogue, 4..7 converters, 8 MMA issuer (one thread), 9..12 loaders
-//   (G_1 tile, G_2(i_2)^T per unit through an asynchronous-copy ring).  G_3^T
-//   and the zero operand padding are written once by all threads before the
-//   roles split.
+// TMEM holds two D2 accumulators (slice columns each) and one or two D1
+// buffers after them; the converters release D1 as soon as it is in their
+// registers, so stage 1 of the next unit overlaps this unit's conversion and
+// stage 2.  Warp roles:
+//   0..3 epilogue, 4..7 converters, 8 MMA issuer (one thread), 9 loader (one
+//   thread).  A small image kernel first writes every operand the tensor
+//   cores read from the cores -- the G_1 rows of each i_1 tile, G_2(i_2)^T
+//   for every i_2, G_3^T -- in its shared-memory layout; the loader moves
+//   them with bulk copies (the main kernel is launched dependent on the
+//   image kernel and overlaps its set-up with it).
 // Intermediates never reach global memory.
 #include <cudaTypedefs.h>
 
@@ -37,10 +41,7 @@ namespace {
 using namespace tc;
 
 constexpr int BM = 128;
-constexpr int kThreads = 416;
-constexpr int kLoadThreads = 128;
-constexpr int kBatch = 8;                  // words per loader thread per round (synchronous paths)
-constexpr int kRaw = 4;                    // raw G_2 slices in flight (asynchronous copies)
+constexpr int kThreads = 320;
 
 struct T3Args {
     int64_t n1, n2;
@@ -48,23 +49,27 @@ struct T3Args {
     int n2h, sn;                   // n_3 slice per unit, number of slices
     int64_t units;                 // (i_1 tile, i_2, n_3 slice) units
     int cw, out16;
+    int nd1;                       // D1 buffers (TMEM columns 2 n2h .. 2 n2h + nd1 r2p)
     uint32_t tmem_cols;
     uint32_t off_a1, off_b1, off_a2, off_b2, off_stage, off_bar;
-    uint32_t b1_bytes, a2_bytes;
-    uint32_t off_raw, raw_bytes;   // ring of kRaw raw G_2(i_2) slices
+    uint32_t a1_bytes, b1_bytes, a2_bytes, b2_bytes;
     const __half* G1;
     const __half* G2;
     const __half* G3;
-    int g1_words, g2_words;        // rows of G_1 / G_2 loadable as 4-byte words
+    // operand images written by the image kernel (canonical K-major layouts)
+    const unsigned char* a1img;    // [i_1 tile][128 x r1p]   rows of G_1
+    const unsigned char* b1img;    // [i_2][r2p x r1p]        G_2(i_2)^T
+    const unsigned char* b2img;    // [n_3 x r2p]             G_3^T
 };
 
 struct Bars {
     uint64_t *a1_full, *a1_empty;
     uint64_t *b1_full, *b1_empty;      // [2]
-    uint64_t *d1_full;                 // [2]
+    uint64_t *d1_full, *d1_empty;      // [2]
     uint64_t *a2_full, *a2_empty;      // [2]
     uint64_t *d2_full, *acc_empty;     // [2]
     uint64_t *mma_done;
+    uint64_t *b2_full;
     uint32_t* tmem_slot;
     int* abort;
 };
@@ -82,7 +87,9 @@ __device__ __forceinline__ Bars carve(unsigned char* smem, const T3Args& a) {
     B.d2_full = p + 13;
     B.acc_empty = p + 15;
     B.mma_done = p + 17;
-    B.tmem_slot = reinterpret_cast<uint32_t*>(p + 18);
+    B.b2_full = p + 18;
+    B.d1_empty = p + 19;
+    B.tmem_slot = reinterpret_cast<uint32_t*>(p + 21);
     B.abort = reinterpret_cast<int*>(B.tmem_slot + 1);
     return B;
 }
@@ -102,118 +109,64 @@ __device__ __forceinline__ void unit_coords(const T3Args& a, int64_t u, int64_t&
     h = (int)(rest - i * a.sn);
 }
 
-__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-
-// Issues the asynchronous copy of G_2(i_2) (r_1 rows of r_2 ranks, 4-byte
-// words) into a raw slot laid out [a][b-pair], row pitch r_2/2 words.  Each
-// loader warp copies whole rows (lane = word; r_2 <= 64, so one pass).
-__device__ __forceinline__ void raw_issue(const T3Args& a, int64_t i, int lwarp, int lane, uint32_t* raw) {
-    const int wpr = a.r2 / 2;                           // r_2 is even on this path
-    if (lane < wpr) {
-        for (int k = lwarp; k < a.r1; k += kLoadThreads / 32)
-            cp_async4(raw + k * wpr + lane, a.G2 + ((int64_t)k * a.n2 + i) * a.r2 + 2 * lane);
-    }
-}
-
-// G_2(i_2)^T into B1 (row b, column a) from a raw slot, shared to shared:
-// a thread takes ranks a, a+1 and b, b+1 (two raw words) and writes them as
-// two 4-byte words, one per row b and b+1 of the K-major layout.
-__device__ __forceinline__ void raw_transpose(const T3Args& a, int lwarp, int lane, const uint32_t* raw,
-                                              unsigned char* b1) {
-    const int wpr = a.r2 / 2;
-    if (lane < wpr) {
-        for (int k = 2 * lwarp; k < a.r1; k += 2 * (kLoadThreads / 32)) {
-            const uint32_t w0 = raw[k * wpr + lane];                          // a = k:   (b, b+1)
-            const uint32_t w1 = (k + 1 < a.r1) ? raw[(k + 1) * wpr + lane] : 0u;  // a = k+1: (b, b+1)
-            const uint32_t rb0 = (w0 & 0xffffu) | (w1 << 16);                 // row b:   (a, a+1)
-            const uint32_t rb1 = (w0 >> 16) | (w1 & 0xffff0000u);             // row b+1: (a, a+1)
-            *reinterpret_cast<uint32_t*>(b1 + canon_off(2 * lane, k, a.r2p)) = rb0;
-            *reinterpret_cast<uint32_t*>(b1 + canon_off(2 * lane + 1, k, a.r2p)) = rb1;
-        }
-    }
-}
-
-// Synchronous path (odd rank or misaligned core): G_2(i_2)^T straight from
-// global memory, eight loads in flight per thread.
-__device__ __forceinline__ void b1_direct(const T3Args& a, int64_t i, int lt, unsigned char* b1) {
-    const int wpr = (a.r2 + 1) / 2;
-    const int total = a.r1 * wpr;
-    for (int e0 = lt; e0 < total; e0 += kLoadThreads * kBatch) {
-        uint32_t w[kBatch];
+// Operand images: the rows of G_1 of every 128-row i_1 tile, G_2(i_2)^T for
+// every i_2 (row b, column a = G_2[a, i_2, b]) and G_3^T (row c, column
+// b = G_3[b, c]), each in the canonical K-major layout with zero padding, so
+// the main kernel moves each with one bulk copy.  A thread writes one
+// 16-byte chunk (one row, eight consecutive ranks); neighbouring threads take
+// neighbouring rows, so the reads of the cores stay coalesced.
+__global__ void __launch_bounds__(256)
+tt3_img_kernel(const __grid_constant__ T3Args a, unsigned char* a1img, unsigned char* b1img, unsigned char* b2img) {
+    const int64_t qtiles = (a.n1 + BM - 1) / BM;
+    const int g1 = a.r1p / 8, g2 = a.r2p / 8;
+    const int64_t na1 = qtiles * g1 * BM;                 // (tile, k-group, row)
+    const int64_t nb1 = a.n2 * g1 * a.r2p;                // (i_2, k-group, row b)
+    const int64_t nb2 = (int64_t)g2 * a.nd;               // (k-group, row c)
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < na1 + nb1 + nb2;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        __half v[8];
+        unsigned char* dst;
+        if (e < na1) {
+            const int row = (int)(e % BM);
+            const int64_t t2 = e / BM;
+            const int kg = (int)(t2 % g1);
+            const int64_t t = t2 / g1;
+            const int64_t q = t * BM + row;
 #pragma unroll
-        for (int t = 0; t < kBatch; ++t) {
-            const int e = e0 + t * kLoadThreads;
-            w[t] = 0;
-            if (e < total) {
-                const int k = e / wpr, bw = e % wpr;
-                const __half* src = a.G2 + ((int64_t)k * a.n2 + i) * a.r2 + 2 * bw;
-                const uint32_t lo16 = __half_as_ushort(src[0]);
-                const uint32_t hi16 = (2 * bw + 1 < a.r2) ? __half_as_ushort(src[1]) : 0u;
-                w[t] = lo16 | (hi16 << 16);
+            for (int u = 0; u < 8; ++u) {
+                const int k = kg * 8 + u;
+                v[u] = (q < a.n1 && k < a.r1) ? a.G1[q * a.r1 + k] : __float2half_rn(0.0f);
             }
-        }
+            dst = a1img + t * a.a1_bytes + canon_off((uint32_t)row, (uint32_t)(kg * 8), BM);
+        } else if (e < na1 + nb1) {
+            const int64_t e1 = e - na1;
+            const int bb = (int)(e1 % a.r2p);
+            const int64_t t2 = e1 / a.r2p;
+            const int kg = (int)(t2 % g1);
+            const int64_t i = t2 / g1;
 #pragma unroll
-        for (int t = 0; t < kBatch; ++t) {
-            const int e = e0 + t * kLoadThreads;
-            if (e < total) {
-                const int k = e / wpr, bw = e % wpr;
-                *reinterpret_cast<unsigned short*>(b1 + canon_off(2 * bw, k, a.r2p)) = (unsigned short)(w[t] & 0xffffu);
-                if (2 * bw + 1 < a.r2)
-                    *reinterpret_cast<unsigned short*>(b1 + canon_off(2 * bw + 1, k, a.r2p)) =
-                        (unsigned short)(w[t] >> 16);
+            for (int u = 0; u < 8; ++u) {
+                const int k = kg * 8 + u;
+                v[u] = (bb < a.r2 && k < a.r1) ? a.G2[((int64_t)k * a.n2 + i) * a.r2 + bb] : __float2half_rn(0.0f);
             }
-        }
-    }
-}
-
-// Shared prologue, all threads: zero A1 and both B1 buffers (their padding
-// rows and columns stay zero), then write G_3^T (n_3 rows, r2p ranks,
-// K-major) into B2.  A thread takes a 2 x 2 block -- ranks k, k+1 of
-// outputs c, c+1 -- as two 4-byte loads along n_3 and writes it as two 4-byte
-// words, one per B2 row; eight blocks per thread are in flight.
-__device__ __forceinline__ void build_g3t(const T3Args& a, unsigned char* smem) {
-    const int nt = blockDim.x;
-    uint4* z = reinterpret_cast<uint4*>(smem + a.off_a1);
-    const uint32_t zbytes = a.off_b2 - a.off_a1;
-    for (uint32_t e = threadIdx.x; e < zbytes / 16; e += nt) z[e] = make_uint4(0, 0, 0, 0);
-    unsigned char* b2 = smem + a.off_b2;
-    const int cpairs = a.nd / 2;                              // n_3 is a multiple of 16
-    const int total = cpairs * (a.r2p / 2);
-    const bool words = (reinterpret_cast<uintptr_t>(a.G3) & 3u) == 0;
-    for (int e0 = threadIdx.x; e0 < total; e0 += nt * kBatch) {
-        uint32_t w0[kBatch], w1[kBatch];
+            dst = b1img + i * a.b1_bytes + canon_off((uint32_t)bb, (uint32_t)(kg * 8), (uint32_t)a.r2p);
+        } else {
+            const int64_t e2 = e - na1 - nb1;
+            const int c = (int)(e2 % a.nd);
+            const int kg = (int)(e2 / a.nd);
 #pragma unroll
-        for (int t = 0; t < kBatch; ++t) {
-            const int e = e0 + t * nt;
-            const int k = 2 * (e / cpairs), c = 2 * (e % cpairs);
-            w0[t] = 0;
-            w1[t] = 0;
-            if (e < total) {
-                const __half* p0 = a.G3 + (int64_t)k * a.nd + c;
-                if (k < a.r2)
-                    w0[t] = words ? __ldg(reinterpret_cast<const unsigned int*>(p0))
-                                  : (uint32_t)__half_as_ushort(p0[0]) | ((uint32_t)__half_as_ushort(p0[1]) << 16);
-                if (k + 1 < a.r2) {
-                    const __half* p1 = p0 + a.nd;
-                    w1[t] = words ? __ldg(reinterpret_cast<const unsigned int*>(p1))
-                                  : (uint32_t)__half_as_ushort(p1[0]) | ((uint32_t)__half_as_ushort(p1[1]) << 16);
-                }
+            for (int u = 0; u < 8; ++u) {
+                const int k = kg * 8 + u;
+                v[u] = k < a.r2 ? a.G3[(int64_t)k * a.nd + c] : __float2half_rn(0.0f);
             }
+            dst = b2img + canon_off((uint32_t)c, (uint32_t)(kg * 8), (uint32_t)a.nd);
         }
-#pragma unroll
-        for (int t = 0; t < kBatch; ++t) {
-            const int e = e0 + t * nt;
-            if (e < total) {
-                const int k = 2 * (e / cpairs), c = 2 * (e % cpairs);
-                *reinterpret_cast<uint32_t*>(b2 + canon_off(c, k, a.nd)) = (w0[t] & 0xffffu) | (w1[t] << 16);
-                *reinterpret_cast<uint32_t*>(b2 + canon_off(c + 1, k, a.nd)) = (w0[t] >> 16) | (w1[t] & 0xffff0000u);
-            }
-        }
+        uint4 w;
+        w.x = (uint32_t)__half_as_ushort(v[0]) | ((uint32_t)__half_as_ushort(v[1]) << 16);
+        w.y = (uint32_t)__half_as_ushort(v[2]) | ((uint32_t)__half_as_ushort(v[3]) << 16);
+        w.z = (uint32_t)__half_as_ushort(v[4]) | ((uint32_t)__half_as_ushort(v[5]) << 16);
+        w.w = (uint32_t)__half_as_ushort(v[6]) | ((uint32_t)__half_as_ushort(v[7]) << 16);
+        *reinterpret_cast<uint4*>(dst) = w;
     }
 }
 
@@ -244,112 +197,56 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
             mbar_init(&B.acc_empty[q], 128);
         }
         mbar_init(B.mma_done, 1);
+        mbar_init(B.b2_full, 1);
+        for (int q = 0; q < 2; ++q) mbar_init(&B.d1_empty[q], 128);
         *B.abort = 0;
         fence_barrier_init();
     }
     if (warp == 8) tmem_alloc(B.tmem_slot, a.tmem_cols);
-    uint32_t* raw = reinterpret_cast<uint32_t*>(smem + a.off_raw);
-    const uint32_t raw_words = a.raw_bytes / 4;
-    if (warp >= 9 && a.g2_words) {
-        // start the first kRaw - 1 G_2 slices before the shared prologue
-        for (int64_t p = 0; p < kRaw - 1; ++p) {
-            if (p < nunits) {
-                int64_t qp, ip;
-                int hp;
-                unit_coords(a, ubeg + p, qp, ip, hp);
-                raw_issue(a, ip, warp - 9, lane, raw + (uint32_t)(p % kRaw) * raw_words);
-            }
-            cp_async_commit();
-        }
-    }
-    build_g3t(a, smem);          // every thread: operand padding and G_3^T
-    fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *B.tmem_slot;
 
-    if (warp >= 9) {
-        // ------------------------------------------------------------ loaders
-        const int lt = threadIdx.x - 288;                      // 0..127
-        const bool leader = (lt == 0);
-        int64_t prev_qt = -1;
-        int builds = 0;
-        for (int64_t j = 0; j < nunits; ++j) {
-            int64_t qt, i;
-            int h;
-            unit_coords(a, ubeg + j, qt, i, h);
-            if (qt != prev_qt) {
-                if (builds > 0 &&
-                    !group_wait(B.a1_empty, (uint32_t)((builds - 1) & 1), abort, err, 1u, 3, kLoadThreads))
-                    break;
-                // G_1 rows of this i_1 tile: 128 x r_1 (words of two ranks)
-                unsigned char* a1 = smem + a.off_a1;
-                const int wpr = (a.r1 + 1) / 2;                 // words per row
-                const int total = BM * wpr;
-                for (int e0 = lt; e0 < total; e0 += kLoadThreads * kBatch) {
-                    uint32_t w[kBatch];
-#pragma unroll
-                    for (int t = 0; t < kBatch; ++t) {
-                        const int e = e0 + t * kLoadThreads;
-                        const int row = e / wpr, kw = e % wpr;
-                        const int64_t q = qt * BM + row;
-                        w[t] = 0;
-                        if (e < total && q < a.n1) {
-                            const __half* src = a.G1 + q * a.r1 + 2 * kw;
-                            if (a.g1_words) w[t] = __ldg(reinterpret_cast<const unsigned int*>(src));
-                            else {
-                                const uint32_t lo16 = __half_as_ushort(src[0]);
-                                const uint32_t hi16 = (2 * kw + 1 < a.r1) ? __half_as_ushort(src[1]) : 0u;
-                                w[t] = lo16 | (hi16 << 16);
-                            }
-                        }
-                    }
-#pragma unroll
-                    for (int t = 0; t < kBatch; ++t) {
-                        const int e = e0 + t * kLoadThreads;
-                        if (e < total) {
-                            const int row = e / wpr, kw = e % wpr;
-                            // ranks 2kw and 2kw+1 are adjacent in a row of the K-major layout
-                            *reinterpret_cast<uint32_t*>(a1 + canon_off(row, 2 * kw, BM)) = w[t];
-                        }
-                    }
+    if (warp == 9) {
+        // ------------------------------------------------------------ loader
+        // one thread: bulk copies of the operand images (G_3^T once, the G_1
+        // tile per i_1 tile, G_2(i_2)^T per unit through two slots)
+        if (lane == 0) {
+            pdl_wait();                // the image kernel's writes are complete and visible
+            mbar_arrive_expect_tx(B.b2_full, a.b2_bytes);
+            bulk_load(smem + a.off_b2, a.b2img, a.b2_bytes, B.b2_full);
+            int64_t prev_qt = -1;
+            int builds = 0;
+            int64_t j = 0;
+            for (; j < nunits; ++j) {
+                int64_t qt, i;
+                int h;
+                unit_coords(a, ubeg + j, qt, i, h);
+                if (qt != prev_qt) {
+                    if (builds > 0 && !mbar_wait(B.a1_empty, (uint32_t)((builds - 1) & 1), abort, err, 1u)) break;
+                    mbar_arrive_expect_tx(B.a1_full, a.a1_bytes);
+                    bulk_load(smem + a.off_a1, a.a1img + (size_t)qt * a.a1_bytes, a.a1_bytes, B.a1_full);
+                    prev_qt = qt;
+                    ++builds;
                 }
-                fence_proxy_async_smem();
-                named_bar_sync(3, kLoadThreads);
-                if (leader) mbar_arrive(B.a1_full);
-                prev_qt = qt;
-                ++builds;
+                const int slot = (int)(j & 1);
+                if (!mbar_wait(&B.b1_empty[slot], (uint32_t)((j >> 1) & 1) ^ 1u, abort, err, 1u)) break;
+                mbar_arrive_expect_tx(&B.b1_full[slot], a.b1_bytes);
+                bulk_load(smem + a.off_b1 + (size_t)slot * a.b1_bytes, a.b1img + (size_t)i * a.b1_bytes, a.b1_bytes,
+                          &B.b1_full[slot]);
             }
-            const int slot = (int)(j & 1);
-            if (a.g2_words) {
-                {   // issue unit j + kRaw - 1, then wait for unit j's slice (in-order groups)
-                    const int64_t p = j + kRaw - 1;
-                    if (p < nunits) {
-                        int64_t qp, ip;
-                        int hp;
-                        unit_coords(a, ubeg + p, qp, ip, hp);
-                        raw_issue(a, ip, lt >> 5, lane, raw + (uint32_t)(p % kRaw) * raw_words);
-                    }
-                    cp_async_commit();
-                    cp_async_wait<kRaw - 1>();
-                }
-                named_bar_sync(3, kLoadThreads);             // every thread's part of slice j has landed
-            }
-            if (!group_wait(&B.b1_empty[slot], (uint32_t)((j >> 1) & 1) ^ 1u, abort, err, 1u, 3, kLoadThreads)) break;
-            // G_2(i_2)^T: row b (r_2), column a (r_1): element G_2[a, i_2, b]
-            unsigned char* b1 = smem + a.off_b1 + (size_t)slot * a.b1_bytes;
-            if (a.g2_words) raw_transpose(a, lt >> 5, lane, raw + (uint32_t)(j % kRaw) * raw_words, b1);
-            else b1_direct(a, i, lt, b1);
-            fence_proxy_async_smem();
-            named_bar_sync(3, kLoadThreads);
-            if (leader) mbar_arrive(&B.b1_full[slot]);
+            // copies in flight land before the CTA can exit
+            volatile int no_abort = 0;
+            mbar_wait(B.b2_full, 0, &no_abort, err, 0u, 100000000ull);
+            if (builds > 0) mbar_wait(B.a1_full, (uint32_t)((builds - 1) & 1), &no_abort, err, 0u, 100000000ull);
+            for (int64_t q = (j - 2 > 0 ? j - 2 : 0); q < j && q < nunits; ++q)
+                mbar_wait(&B.b1_full[q & 1], (uint32_t)((q >> 1) & 1), &no_abort, err, 0u, 100000000ull);
         }
-        cp_async_wait<0>();                                // no copy in flight when the CTA exits
     } else if (warp == 8) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            bool ok = true;
+            bool ok = mbar_wait(B.b2_full, 0, abort, err, 2u);
             const uint32_t idesc1 = idesc_f16_f32(BM, (uint32_t)a.r2p);
             const uint32_t idesc2 = idesc_f16_f32(BM, (uint32_t)a.n2h);
             const uint32_t a1s = smem_u32(smem + a.off_a1);
@@ -366,7 +263,11 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
                     cur_qt = qt;
                     ++qcount;
                 }
-                if (!mbar_wait(&B.acc_empty[buf], (uint32_t)((j >> 1) & 1) ^ 1u, abort, err, 2u)) return false;
+                // D1 has its own columns: it waits only for the converters of unit j - nd1
+                const int db = (int)(j % a.nd1);
+                if (j >= a.nd1 &&
+                    !mbar_wait(&B.d1_empty[db], (uint32_t)(((j / a.nd1) - 1) & 1), abort, err, 2u))
+                    return false;
                 if (!mbar_wait(&B.b1_full[buf], (uint32_t)((j >> 1) & 1), abort, err, 2u)) return false;
                 tc_fence_after();
                 const uint32_t b1s = smem_u32(smem + a.off_b1 + (size_t)buf * a.b1_bytes);
@@ -374,11 +275,11 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
                 // descriptors stepped by adds: 16 ranks = 4096 B of A, 2 x lbo1 B of B
                 const uint64_t ad = smem_desc(a1s, 2048, 128, 0), bd = smem_desc(b1s, lbo1, 128, 0);
                 const uint64_t bstep = (uint64_t)(2u * lbo1) >> 4;
+                const uint32_t d1col = tmem + 2u * (uint32_t)a.n2h + (uint32_t)(db * a.r2p);
                 for (int ks = 0; ks < a.r1p / 16; ++ks)
-                    mma_f16(tmem + (uint32_t)buf * a.n2h, ad + (uint64_t)ks * 256u, bd + (uint64_t)ks * bstep, idesc1,
-                            ks > 0);
+                    mma_f16(d1col, ad + (uint64_t)ks * 256u, bd + (uint64_t)ks * bstep, idesc1, ks > 0);
                 mma_commit(&B.b1_empty[buf]);
-                mma_commit(&B.d1_full[buf]);
+                mma_commit(&B.d1_full[db]);
                 // last unit of this i_1 tile: G_1 tile may be replaced once these MMAs finish
                 bool last = (j + 1 == nunits);
                 if (!last) {
@@ -396,6 +297,7 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
                 unit_coords(a, ubeg + j, qt, i, h);
                 const int buf = (int)(j & 1);
                 if (!mbar_wait(&B.a2_full[buf], (uint32_t)((j >> 1) & 1), abort, err, 2u)) return false;
+                if (!mbar_wait(&B.acc_empty[buf], (uint32_t)((j >> 1) & 1) ^ 1u, abort, err, 2u)) return false;
                 tc_fence_after();
                 const uint32_t ahi = smem_u32(smem + a.off_a2 + (size_t)buf * 2 * a.a2_bytes);
                 const uint32_t alo = ahi + a.a2_bytes;
@@ -413,12 +315,15 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
                 mma_commit(&B.d2_full[buf]);
                 return true;
             };
-            // stage 2 of unit j goes before stage 1 of unit j+1: stage 1 needs the
-            // TMEM buffer the epilogue is still draining, stage 2 does not
-            if (ok && nunits > 0) ok = stage1(0);
+            // stage 1 runs nd1 units ahead of stage 2: with one D1 buffer the next
+            // stage 1 goes as soon as the converters have read D1 (before this
+            // unit's stage 2), with two it follows this unit's stage 2
+            for (int64_t u = 0; u < a.nd1 && u < nunits && ok; ++u) ok = stage1(u);
             for (int64_t j = 0; j < nunits && ok; ++j) {
+                const int64_t u = j + a.nd1;
+                if (a.nd1 == 1 && u < nunits && !(ok = stage1(u))) break;
                 if (!(ok = stage2(j))) break;
-                if (j + 1 < nunits) ok = stage1(j + 1);
+                if (a.nd1 == 2 && u < nunits) ok = stage1(u);
             }
             mma_commit(B.mma_done);
             volatile int no_abort = 0;
@@ -431,13 +336,16 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
         const uint32_t lane_base = (uint32_t)(g * 32) << 16;
         for (int64_t j = 0; j < nunits; ++j) {
             const int buf = (int)(j & 1);
-            if (!group_wait(&B.d1_full[buf], (uint32_t)((j >> 1) & 1), abort, err, 4u, 2, 128)) break;
+            const int db = (int)(j % a.nd1);
+            if (!group_wait(&B.d1_full[db], (uint32_t)((j / a.nd1) & 1), abort, err, 4u, 2, 128)) break;
             tc_fence_after();
             uint32_t v[64];
-            const uint32_t tcol = tmem + lane_base + (uint32_t)buf * a.n2h;
+            const uint32_t tcol = tmem + lane_base + 2u * (uint32_t)a.n2h + (uint32_t)(db * a.r2p);
             tmem_ld32(tcol, *reinterpret_cast<uint32_t(*)[32]>(&v[0]));
             if (a.r2p > 32) tmem_ld32(tcol + 32, *reinterpret_cast<uint32_t(*)[32]>(&v[32]));
             tmem_ld_wait();
+            tc_fence_before();
+            mbar_arrive(&B.d1_empty[db]);          // D1 is in registers: the next stage 1 may overwrite it
             if (!group_wait(&B.a2_empty[buf], (uint32_t)((j >> 1) & 1) ^ 1u, abort, err, 4u, 2, 128)) break;
             unsigned char* ahi = smem + a.off_a2 + (size_t)buf * 2 * a.a2_bytes;
             unsigned char* alo = ahi + a.a2_bytes;
@@ -573,39 +481,38 @@ bool tt3_f16_tc_plan(const TTShape& sh, bool out16, T3Args* out_args, size_t* sm
     a.n2h = a.nd / a.sn;
     if (a.n2h < a.r2p) return false;
     a.units = qtiles * a.n2 * a.sn;
-    a.tmem_cols = pow2_cols(2u * (uint32_t)a.n2h);
+    // TMEM: two D2 accumulators of n2h columns, then nd1 D1 buffers of r2p
+    // columns (two when they fit, so stage 1 runs a unit ahead)
+    a.nd1 = (2 * a.n2h + 2 * a.r2p <= 512) ? 2 : 1;
+    const uint32_t need = 2u * (uint32_t)a.n2h + (uint32_t)(a.nd1 * a.r2p);
+    const uint32_t d1_read_end = 2u * (uint32_t)a.n2h + (uint32_t)((a.nd1 - 1) * a.r2p) + (a.r2p > 32 ? 64u : 32u);
+    a.tmem_cols = pow2_cols(need > d1_read_end ? need : d1_read_end);
     const uint32_t chunks = (uint32_t)((a.n2h + a.cw - 1) / a.cw * a.cw);
-    if ((uint32_t)a.n2h + chunks > a.tmem_cols || a.tmem_cols > 512) return false;
+    if ((uint32_t)a.n2h + chunks > 2u * (uint32_t)a.n2h + (uint32_t)a.r2p || a.tmem_cols > 512) return false;
+    a.a1_bytes = (uint32_t)BM * a.r1p * 2;
     a.b1_bytes = (uint32_t)a.r2p * a.r1p * 2;
     a.a2_bytes = (uint32_t)BM * a.r2p * 2;
+    a.b2_bytes = (uint32_t)a.nd * a.r2p * 2;
     uint32_t off = 0;
     a.off_a1 = off;
-    off += (uint32_t)BM * a.r1p * 2;
+    off += a.a1_bytes;
     a.off_b1 = off;
     off += 2 * a.b1_bytes;
     a.off_a2 = off;
     off += 4 * a.a2_bytes;
     a.off_b2 = off;
-    off += (uint32_t)a.nd * a.r2p * 2;
-    off = (off + 15) / 16 * 16;
-    a.raw_bytes = (uint32_t)a.r1 * (uint32_t)((a.r2 + 1) / 2) * 4u;
-    a.raw_bytes = (a.raw_bytes + 15) / 16 * 16;
-    a.off_raw = off;
-    off += kRaw * a.raw_bytes;
+    off += a.b2_bytes;
     off = (off + 1023) / 1024 * 1024;
     a.off_stage = off;
     off += 2 * BM * 128;
     off = (off + 7) / 8 * 8;
     a.off_bar = off;
-    off += 18 * 8 + 16;
+    off += 21 * 8 + 16;
     const size_t smem = (size_t)off + 1024;
     if (smem > 227 * 1024) return false;
     a.G1 = static_cast<const __half*>(sh.cores[0]);
     a.G2 = static_cast<const __half*>(sh.cores[1]);
     a.G3 = static_cast<const __half*>(sh.cores[2]);
-    // 4-byte loads need an even rank and a 4-byte aligned core
-    a.g1_words = ((a.r1 & 1) == 0 && (reinterpret_cast<uintptr_t>(a.G1) & 3u) == 0) ? 1 : 0;
-    a.g2_words = ((a.r2 & 1) == 0 && (reinterpret_cast<uintptr_t>(a.G2) & 3u) == 0) ? 1 : 0;
     *out_args = a;
     *smem_out = smem;
     *grid_out = a.units < sms ? a.units : sms;
@@ -646,9 +553,27 @@ lrc_status launch_tt3_f16_tc(const TTShape& sh, bool out16, void* out, cudaStrea
         set_error("cuTensorMapEncodeTiled failed for the 3-way TT output (CUresult %d)", (int)cr);
         return LRC_ERR_CUDA;
     }
+    // operand images in the stream workspace
+    const int64_t qtiles = (a.n1 + BM - 1) / BM;
+    auto r256 = [](size_t v) { return (v + 255) / 256 * 256; };
+    const size_t a1_total = r256((size_t)qtiles * a.a1_bytes), b1_total = r256((size_t)a.n2 * a.b1_bytes);
+    void* ws = nullptr;
+    lrc_status st = stream_workspace(s, a1_total + b1_total + a.b2_bytes, &ws);
+    if (st != LRC_OK) return st;
+    unsigned char* wb = static_cast<unsigned char*>(ws);
+    a.a1img = wb;
+    a.b1img = wb + a1_total;
+    a.b2img = wb + a1_total + b1_total;
+    const int64_t nel = (qtiles * BM * a.r1p + a.n2 * a.r2p * a.r1p + (int64_t)a.nd * a.r2p) / 8;   // 16-byte chunks
+    const int64_t iblocks = (nel + 255) / 256;
+    const int sms = sm_count();
+    tt3_img_kernel<<<(unsigned)(iblocks < 8 * sms ? iblocks : 8 * sms), 256, 0, s>>>(a, wb, wb + a1_total,
+                                                                                     wb + a1_total + b1_total);
+    if ((st = after_launch("tt3_img_kernel")) != LRC_OK) return st;
     cudaError_t e = cudaFuncSetAttribute(tt3_f16_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "tt3_f16_tc_kernel smem attribute");
-    tt3_f16_tc_kernel<<<(unsigned)grid, kThreads, smem, s>>>(tm, a);
+    e = launch_pdl(tt3_f16_tc_kernel, dim3((unsigned)grid), dim3(kThreads), smem, s, tm, a);
+    if (e != cudaSuccess) return cuda_fail(e, "tt3_f16_tc_kernel launch");
     return after_launch("tt3_f16_tc_kernel");
 }
 
