@@ -105,6 +105,23 @@ def work_tt(dims, ranks, fmt):
     return {"bytes": cores * E[fmt] + N * E_OUT[fmt], "flops": flops, "alu": ALU[fmt]}
 
 
+def work_eta_lowrank(m, n, k, fmt):
+    """Fused eta: the two symmetric 2k x 2k Gram matrices over m and n rows."""
+    return {"bytes": (m + n + 1) * k * (8 + E[fmt]), "flops": 2 * (m + n) * k * (2 * k + 1), "alu": "f64"}
+
+
+def work_eta_tt(dims, ranks, fmt):
+    """Fused eta_TT: Gram of [dG_1, Gh_1], per interior core the product
+    M C (zero block not counted) and the symmetric C^T X, Gram of [G_d; dG_d]."""
+    d = len(dims)
+    flops = 2 * dims[0] * ranks[1] * (2 * ranks[1] + 1) + 2 * dims[-1] * ranks[d - 1] * (2 * ranks[d - 1] + 1)
+    for l in range(1, d - 1):
+        ra, n, rb = ranks[l], dims[l], ranks[l + 1]
+        flops += 12 * ra * ra * n * rb + 7 * ra * n * rb * rb
+    cores = sum(ranks[l] * dims[l] * ranks[l + 1] for l in range(d))
+    return {"bytes": cores * (8 + E[fmt]), "flops": flops, "alu": "f64"}
+
+
 def work_fro(count, fa, fb):
     return {"bytes": count * (E[fa] + E[fb]), "flops": 0, "alu": None}
 
@@ -517,6 +534,21 @@ def run_case(args):
         out = torch.empty(int(np.prod(cfg.dims)), dtype=lrc.output_dtype(fmt), device=dev)
         call = lambda: lrc.tt_reconstruct(cores, cfg.dims, ranks, fmt, out)  # noqa: E731
         work = work_tt(cfg.dims, ranks, fmt)
+    elif args.case == "eta_matrix":
+        m, n, k = args.m, args.n, args.k
+        f = W.random_factors(m, n, k, seed=7)
+        mk = lambda a, ft: lrc.round_matrix(torch.from_numpy(a if a.ndim == 2 else a[None, :]).to(dev), ft)  # noqa: E731
+        f64 = [mk(a, "f64") for a in (f.U, f.s, f.Vt)]
+        low = [mk(a, fmt) for a in (f.U, f.s, f.Vt)]
+        call = lambda: lrc.lrc_lowrank_eta(*f64, *low, fmt, m, n, k)  # noqa: E731
+        work = work_eta_lowrank(m, n, k, fmt)
+    elif args.case == "eta_tt":
+        cfg = W.TT_CONFIGS[args.tt]
+        c64 = [torch.from_numpy(c).to(dev).contiguous() for c in W.tt_cores(cfg, base)]
+        low = [c.to(lrc.storage_dtype(fmt)).contiguous() for c in c64]
+        ranks = cfg.ranks[base]
+        call = lambda: lrc.lrc_tt_eta(c64, low, cfg.dims, ranks, fmt)  # noqa: E731
+        work = work_eta_tt(cfg.dims, ranks, fmt)
     elif args.case == "fro":
         a = torch.randn(args.count, dtype=torch.float64, device=dev)
         b2 = torch.randn(args.count, dtype=torch.float64, device=dev)
@@ -560,7 +592,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", choices=["apply", "tt", "fro", "round"], default=None,
+    ap.add_argument("--case", choices=["apply", "tt", "fro", "round", "eta_matrix", "eta_tt"], default=None,
                     help="time one call type instead of the step (profiling captures)")
     ap.add_argument("--fmt", default="f16")
     ap.add_argument("--m", type=int, default=16384)

@@ -22,8 +22,9 @@
  *    lrc_last_error() gives a message for the last failure of the calling
  *    thread.
  *  - Sizes are int64_t; products of sizes must not overflow int64.
- *  - The library never traps, never allocates on the apply / TT / rounding
- *    paths, and has no CPU fallback: it needs an sm_103a GPU.
+ *  - The library never traps and has no CPU fallback: it needs an sm_103a
+ *    GPU.  Device scratch is allocated only where an entry point says so
+ *    (library workspaces, allocated on first use and reused).
  */
 #ifndef LRC_H
 #define LRC_H
@@ -200,6 +201,65 @@ LRC_API lrc_status lrc_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fm
 LRC_API lrc_status lrc_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb,
                                         int64_t count, double* diff_out, double* normA_out,
                                         lrc_stream_t stream);
+
+/*
+ * lrc_lowrank_eta -- eta = ||U diag(s) V^T - Uh diag(sh) Vh^T||_F, the
+ * perturbation of Thm 4.1 (remark after it: the three factors are rounded
+ * individually), without forming either m x n matrix.
+ *
+ *   U, S, Vt     device, the binary64 rank-k factors in the layout of
+ *                lrc_apply: U m x k with row pitch lrc_packed_ld(k), S k
+ *                values, Vt = V^T k x n with row pitch lrc_packed_ld(n)
+ *   Uh, Sh, Vht  device, the stored factors in format `fmt`, same layout
+ *                (what lrc_round_factors writes)
+ *   eta_out      host: eta
+ *   norm_out     host, may be NULL: ||U diag(s) V^T||_F
+ *
+ * With the rounding errors dU = U - Uh, dV = V - Vh, ds = s - sh (exact in
+ * binary64) the difference is exactly [dU, Uh] M [dV, Vh]^T with
+ * M = [[S, S], [S, dS]] (diagonal blocks), so eta^2 = tr(M^T Gu M Gv) with
+ * the 2k x 2k Gram matrices Gu = [dU, Uh]^T [dU, Uh], Gv = [dV, Vh]^T
+ * [dV, Vh].  Every term carries the rounding errors explicitly, so nothing
+ * of the size of ||A|| cancels: the result is accurate relative to eta,
+ * where the dense route (lrc_apply with X = I, lrc_fro_diff) is accurate
+ * relative to ||A||.  Work: about 2 (m + n) k (2k + 1) binary64 flops.
+ * All arithmetic binary64; deterministic on a device.  k <= 4096.  Pointers
+ * 16-byte aligned.  Scratch: the stream's library workspace (see
+ * lrc_apply), 16 (m + n) k bytes plus O(k^2).  SYNCHRONISES `stream`.
+ */
+LRC_API lrc_status lrc_lowrank_eta(const double* U, const double* S, const double* Vt,
+                                   const void* Uh, const void* Sh, const void* Vht, lrc_fmt fmt,
+                                   int64_t m, int64_t n, int64_t k, double* eta_out,
+                                   double* norm_out, lrc_stream_t stream);
+
+/*
+ * lrc_tt_eta -- eta_TT = ||T(G_1..G_d) - T(Gh_1..Gh_d)||_F, the perturbation
+ * of Thm 6.1 (Sec. 6.1: rounded cores compared in FP64), without forming
+ * either tensor.
+ *
+ *   cores      HOST array of d DEVICE pointers to the binary64 cores, layout
+ *              of tt_reconstruct (core l: ranks[l] x dims[l] x ranks[l+1])
+ *   cores_hat  HOST array of d DEVICE pointers to the stored cores in format
+ *              `fmt`, same shapes
+ *   dims, ranks, d  as in tt_reconstruct
+ *   eta_out    host: eta_TT
+ *   norm_out   host, may be NULL: ||T(G)||_F
+ *
+ * With D_l = Z_l - Zh_l the difference of the partial products of Eq.
+ * gpu_tt_reconstruction, [D_l, Zh_l] = [D_{l-1}, Zh_{l-1}] C_l(i_l) with the
+ * block core C_l(i) = [[G_l(i), 0], [G_l(i) - Gh_l(i), Gh_l(i)]], and
+ * T - Th = [D_{d-1}, Zh_{d-1}] [G_d; G_d - Gh_d].  The 2 r_l x 2 r_l Gram
+ * matrix of [D_l, Zh_l] over all prefixes is carried from core to core
+ * (M_l = sum_i C_l(i)^T M_{l-1} C_l(i)) and contracted with the last core.
+ * Work: about sum over interior cores of 8 r_{l-1} n_l r_l (2 r_{l-1} +
+ * r_l) binary64 flops.  Deterministic on a device.  Cores aligned to their
+ * element size.  Scratch: the stream's workspace, two buffers of
+ * 4 r_{l-1} n_l r_l binary64 for the largest interior core plus O(r^2).
+ * SYNCHRONISES `stream`.
+ */
+LRC_API lrc_status lrc_tt_eta(const double* const* cores, const void* const* cores_hat,
+                              const int64_t* dims, const int64_t* ranks, int d, lrc_fmt fmt,
+                              double* eta_out, double* norm_out, lrc_stream_t stream);
 
 /* Thm 4.1 Eq. matrix_condition and Thm 6.1 Eq. tt_condition:
  * returns 1 if e_aug + eta <= e_base (certified non-increase), else 0. */

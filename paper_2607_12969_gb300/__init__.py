@@ -58,6 +58,10 @@ def load() -> ctypes.CDLL:
     L.lrc_fro_diff.restype = i32
     L.lrc_fro_diff_noalloc.argtypes = [vp, i32, vp, i32, i64, vp, vp, vp]
     L.lrc_fro_diff_noalloc.restype = i32
+    L.lrc_lowrank_eta.argtypes = [vp, vp, vp, vp, vp, vp, i32, i64, i64, i64, vp, vp, vp]
+    L.lrc_lowrank_eta.restype = i32
+    L.lrc_tt_eta.argtypes = [vp, vp, vp, vp, i32, i32, vp, vp, vp]
+    L.lrc_tt_eta.restype = i32
     L.lrc_certified.argtypes = [dbl, dbl, dbl]
     L.lrc_certified.restype = i32
     L.lrc_tail_error.argtypes = [vp, i64, i64]
@@ -168,6 +172,38 @@ def lrc_fro_diff_noalloc(A, fa, B, fb, count: int, stream=None) -> Tuple[float, 
     _check(load().lrc_fro_diff_noalloc(_ptr(A), _fmt(fa), _ptr(B), _fmt(fb) if B is not None else 0, count,
                                        ctypes.addressof(diff), ctypes.addressof(norm), _stream(stream)))
     return diff.value, norm.value
+
+
+def lrc_lowrank_eta(U, S, Vt, Uh, Sh, Vht, fmt, m: int, n: int, k: int, stream=None,
+                    want_norm: bool = True) -> Tuple[float, float]:
+    """Returns (eta, ||U diag(s) V^T||_F) for binary64 factors U, S, Vt and the
+    stored factors Uh, Sh, Vht of format fmt (layouts of lrc_apply).  With
+    want_norm=False the norm is not returned (NaN in its place)."""
+    eta = ctypes.c_double(0.0)
+    norm = ctypes.c_double(float("nan"))
+    _check(load().lrc_lowrank_eta(_ptr(U), _ptr(S), _ptr(Vt), _ptr(Uh), _ptr(Sh), _ptr(Vht), _fmt(fmt),
+                                  m, n, k, ctypes.addressof(eta),
+                                  ctypes.addressof(norm) if want_norm else None, _stream(stream)))
+    return eta.value, norm.value
+
+
+def lrc_tt_eta(cores: Sequence, cores_hat: Sequence, dims: Sequence[int], ranks: Sequence[int], fmt,
+               stream=None, want_norm: bool = True) -> Tuple[float, float]:
+    """Returns (eta_TT, ||T||_F) for binary64 cores and stored cores of format fmt."""
+    d = len(cores)
+    if len(cores_hat) != d:
+        raise ValueError("cores and cores_hat differ in length")
+    p64 = (ctypes.c_void_p * d)(*[c.data_ptr() for c in cores])
+    ph = (ctypes.c_void_p * d)(*[c.data_ptr() for c in cores_hat])
+    dd = (ctypes.c_int64 * d)(*[int(x) for x in dims])
+    rr = (ctypes.c_int64 * (d + 1))(*[int(x) for x in ranks])
+    eta = ctypes.c_double(0.0)
+    norm = ctypes.c_double(float("nan"))
+    _check(load().lrc_tt_eta(ctypes.cast(p64, ctypes.c_void_p), ctypes.cast(ph, ctypes.c_void_p),
+                             ctypes.cast(dd, ctypes.c_void_p), ctypes.cast(rr, ctypes.c_void_p), d, _fmt(fmt),
+                             ctypes.addressof(eta), ctypes.addressof(norm) if want_norm else None,
+                             _stream(stream)))
+    return eta.value, norm.value
 
 
 def lrc_certified(e_base: float, e_aug: float, eta: float) -> bool:

@@ -61,6 +61,36 @@ static lrc_status misaligned(const char* name) {
     return LRC_ERR_ALIGNMENT;
 }
 
+// Validates a TT shape (Sec. 5.1: ranks r_0 = r_d = 1, core l of size
+// r_{l-1} x n_l x r_l) and fills *sh; `es` is the element size of the cores.
+static lrc_status tt_shape(const void* const* cores, const int64_t* dims, const int64_t* ranks, int d,
+                           int64_t es, const char* what, TTShape* sh) {
+    if (!cores || !dims || !ranks) return invalid("null pointer");
+    if (d < 2 || d > 16) return invalid("d must be in [2, 16] (d=%d)", d);
+    if (ranks[0] != 1 || ranks[d] != 1) return invalid("ranks[0] and ranks[d] must be 1");
+    sh->d = d;
+    int64_t numel = 1;
+    for (int l = 0; l < d; ++l) {
+        if (dims[l] <= 0) return invalid("dims[%d] = %lld must be positive", l, (long long)dims[l]);
+        if (ranks[l] <= 0 || ranks[l] > 4096) return invalid("ranks[%d] out of range", l);
+        if (!cores[l]) return invalid("%s[%d] is null", what, l);
+        if ((reinterpret_cast<uintptr_t>(cores[l]) % (uintptr_t)es) != 0) {
+            set_error("%s[%d] is not aligned to its element size", what, l);
+            return LRC_ERR_ALIGNMENT;
+        }
+        int64_t c;
+        if (!mul_ok(ranks[l], dims[l], &c) || !mul_ok(c, ranks[l + 1], &c) || !mul_ok(c, 8, &c))
+            return invalid("core %d size overflow", l);
+        if (!mul_ok(numel, dims[l], &numel)) return invalid("tensor size overflow");
+        sh->dims[l] = dims[l];
+        sh->ranks[l] = ranks[l];
+        sh->cores[l] = cores[l];
+    }
+    sh->ranks[d] = 1;
+    sh->numel = numel;
+    return LRC_OK;
+}
+
 }  // namespace lrc
 
 using namespace lrc;
@@ -139,37 +169,57 @@ lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X
 lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims, const int64_t* ranks,
                           int d, lrc_fmt fmt, void* out, lrc_stream_t stream) {
     if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
-    if (!cores || !dims || !ranks || !out) return invalid("null pointer");
-    if (d < 2 || d > 16) return invalid("d must be in [2, 16] (d=%d)", d);
-    if (ranks[0] != 1 || ranks[d] != 1) return invalid("ranks[0] and ranks[d] must be 1");
+    if (!out) return invalid("null pointer");
     TTShape sh;
-    sh.d = d;
-    int64_t numel = 1;
-    const int64_t es = storage_bytes(fmt);
-    for (int l = 0; l < d; ++l) {
-        if (dims[l] <= 0) return invalid("dims[%d] = %lld must be positive", l, (long long)dims[l]);
-        if (ranks[l] <= 0 || ranks[l] > 4096) return invalid("ranks[%d] out of range", l);
-        if (!cores[l]) return invalid("cores[%d] is null", l);
-        if ((reinterpret_cast<uintptr_t>(cores[l]) % (uintptr_t)es) != 0) {
-            set_error("cores[%d] is not aligned to its element size", l);
-            return LRC_ERR_ALIGNMENT;
-        }
-        int64_t c;
-        if (!mul_ok(ranks[l], dims[l], &c) || !mul_ok(c, ranks[l + 1], &c) || !mul_ok(c, 8, &c))
-            return invalid("core %d size overflow", l);
-        if (!mul_ok(numel, dims[l], &numel)) return invalid("tensor size overflow");
-        sh.dims[l] = dims[l];
-        sh.ranks[l] = ranks[l];
-        sh.cores[l] = cores[l];
-    }
-    sh.ranks[d] = 1;
+    lrc_status st = tt_shape(cores, dims, ranks, d, storage_bytes(fmt), "cores", &sh);
+    if (st != LRC_OK) return st;
     int64_t t;
-    if (!mul_ok(numel, 8, &t)) return invalid("tensor size overflow");
-    sh.numel = numel;
+    if (!mul_ok(sh.numel, 8, &t)) return invalid("tensor size overflow");
     if (!aligned16(out)) return misaligned("out");
     cudaStream_t s = as_stream(stream);
     if (fmt == LRC_F16 || fmt == LRC_F16_O16) return launch_tt_f16(sh, fmt == LRC_F16_O16, out, s);
     return launch_tt_cc(sh, fmt, out, s);
+}
+
+lrc_status lrc_lowrank_eta(const double* U, const double* S, const double* Vt, const void* Uh, const void* Sh,
+                           const void* Vht, lrc_fmt fmt, int64_t m, int64_t n, int64_t k, double* eta_out,
+                           double* norm_out, lrc_stream_t stream) {
+    if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    if (m <= 0 || n <= 0 || k <= 0)
+        return invalid("sizes must be positive (m=%lld n=%lld k=%lld)", (long long)m, (long long)n, (long long)k);
+    if (k > 4096) return invalid("k = %lld exceeds 4096", (long long)k);
+    int64_t t;
+    const int64_t ldk = lrc_packed_ld(k), ldn = lrc_packed_ld(n);
+    if (!mul_ok(m, ldk, &t) || !mul_ok(t, 8, &t) || !mul_ok(k, ldn, &t) || !mul_ok(t, 8, &t) ||
+        !mul_ok(m + n, 2 * k, &t) || !mul_ok(t, 8, &t))
+        return invalid("size overflow");
+    if (!U || !S || !Vt || !Uh || !Sh || !Vht || !eta_out) return invalid("null pointer");
+    if (!aligned16(U)) return misaligned("U");
+    if (!aligned16(S)) return misaligned("S");
+    if (!aligned16(Vt)) return misaligned("Vt");
+    if (!aligned16(Uh)) return misaligned("Uh");
+    if (!aligned16(Sh)) return misaligned("Sh");
+    if (!aligned16(Vht)) return misaligned("Vht");
+    return run_lowrank_eta(U, S, Vt, Uh, Sh, Vht, fmt, m, n, k, eta_out, norm_out, as_stream(stream));
+}
+
+lrc_status lrc_tt_eta(const double* const* cores, const void* const* cores_hat, const int64_t* dims,
+                      const int64_t* ranks, int d, lrc_fmt fmt, double* eta_out, double* norm_out,
+                      lrc_stream_t stream) {
+    if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    if (!eta_out) return invalid("null eta_out");
+    TTShape sh, shh;
+    lrc_status st = tt_shape((const void* const*)cores, dims, ranks, d, 8, "cores", &sh);
+    if (st != LRC_OK) return st;
+    st = tt_shape(cores_hat, dims, ranks, d, storage_bytes(fmt), "cores_hat", &shh);
+    if (st != LRC_OK) return st;
+    for (int l = 0; l < d; ++l) {
+        int64_t c;
+        // block cores of an interior level: 2 r_l x n_l x 2 r_{l+1} binary64, twice
+        if (!mul_ok(4 * ranks[l] * dims[l], ranks[l + 1], &c) || !mul_ok(c, 16, &c))
+            return invalid("core %d too large for eta_TT", l);
+    }
+    return run_tt_eta(sh, shh.cores, fmt, eta_out, norm_out, as_stream(stream));
 }
 
 lrc_status lrc_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,

@@ -116,4 +116,11 @@ lrc_status run_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fm
                                 double* diff_out, double* normA_out, cudaStream_t s);
 int64_t fro_diff_noalloc_max_count();
 
+// eta of Thm 4.1 / eta_TT of Thm 6.1 from Gram blocks (eta.cu); synchronise s.
+lrc_status run_lowrank_eta(const double* U, const double* S, const double* Vt, const void* Uh, const void* Sh,
+                           const void* Vht, lrc_fmt fmt, int64_t m, int64_t n, int64_t k, double* eta_out,
+                           double* norm_out, cudaStream_t s);
+lrc_status run_tt_eta(const TTShape& sh, const void* const* hats, lrc_fmt fmt, double* eta_out, double* norm_out,
+                      cudaStream_t s);
+
 }  // namespace lrc

@@ -102,3 +102,29 @@ def test_host_helpers_agree_with_oracle(L):
         dims, base, aug = (256, 256, 256), (1, 32, 32, 1), (1, 34, 34, 1)
         assert abs(lrc.lrc_tt_storage_bytes(dims, aug, fmt) * 8 - oracle.tt_storage_bits(dims, aug, fmt)) < 1e-6
     assert lrc.lrc_matrix_storage_ratio(10, 10, 40, 41, "f16") == pytest.approx(0.25625)
+
+
+def test_eta_validation_rejects_before_launch(L):
+    """lrc_lowrank_eta / lrc_tt_eta reject bad arguments on the host."""
+    out = ctypes.c_double(0.0)
+    po = ctypes.addressof(out)
+    # null factor, zero size, bad format, misaligned pointer, k too large
+    assert L.lrc_lowrank_eta(None, 16, 16, 16, 16, 16, 2, 4, 4, 2, po, None, None) == -1
+    assert L.lrc_lowrank_eta(16, 16, 16, 16, 16, 16, 2, 0, 4, 2, po, None, None) == -1
+    assert L.lrc_lowrank_eta(16, 16, 16, 16, 16, 16, 9, 4, 4, 2, po, None, None) == -1
+    assert L.lrc_lowrank_eta(16, 16, 16, 24, 16, 16, 2, 4, 4, 2, po, None, None) == -2
+    assert L.lrc_lowrank_eta(16, 16, 16, 16, 16, 16, 2, 4, 4, 5000, po, None, None) == -1
+    assert L.lrc_lowrank_eta(16, 16, 16, 16, 16, 16, 2, 4, 4, 2, None, None, None) == -1
+    d = 3
+    c = (ctypes.c_void_p * d)(16, 16, 16)
+    ch = (ctypes.c_void_p * d)(16, 16, 16)
+    dims = (ctypes.c_int64 * d)(4, 5, 6)
+    bad = (ctypes.c_int64 * (d + 1))(2, 3, 3, 1)          # r_0 != 1
+    assert L.lrc_tt_eta(c, ch, dims, bad, d, 2, po, None, None) == -1
+    good = (ctypes.c_int64 * (d + 1))(1, 3, 3, 1)
+    assert L.lrc_tt_eta(c, ch, dims, good, 1, 2, po, None, None) == -1   # d < 2
+    assert L.lrc_tt_eta(c, ch, dims, good, d, 2, None, None, None) == -1  # null eta_out
+    nul = (ctypes.c_void_p * d)(16, None, 16)
+    assert L.lrc_tt_eta(c, nul, dims, good, d, 2, po, None, None) == -1
+    odd = (ctypes.c_void_p * d)(16, 20, 16)                 # binary64 core not 8-byte aligned
+    assert L.lrc_tt_eta(odd, ch, dims, good, d, 0, po, None, None) == -2
