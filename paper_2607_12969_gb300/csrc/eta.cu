@@ -36,11 +36,11 @@ namespace lrc {
 
 namespace {
 
-constexpr int kGT = 16;          // Gram output tile (kGT x kGT), one entry per thread
+constexpr int kGT = 16;          // largest Gram output tile (T x T, one entry per thread)
 constexpr int kGRows = 32;       // rows of the reduction per chunk
-constexpr int kGThreads = kGT * kGT;
-constexpr int kMmR = 32;         // GEMM tile rows
-constexpr int kMmC = 128;        // GEMM tile columns
+constexpr int kGThreads = 256;
+constexpr int kMaxProbs = 3;     // products per batched launch
+constexpr int kMmT = 16;         // GEMM tile: up to 16 rows x 16 columns, one entry per thread
 constexpr int kMmK = 16;         // GEMM k-chunk
 constexpr int kCombineBlocks = 304;
 
@@ -107,55 +107,62 @@ __global__ void eta_pack_cols_kernel(const double* __restrict__ X, int64_t ldx, 
     }
 }
 
-// Block cores of one interior TT level: Cb (2ra x n x 2rb) from G (ra x n x rb,
-// binary64) and Gh (stored format): rows a < ra hold [G(a,i,:), 0], rows
-// ra + a hold [G - Gh, Gh].
+// Operands of one interior TT level from G (ra x n x rb, binary64) and Gh
+// (stored format): CD (2ra x n x rb) holds G in rows a < ra and G - Gh in
+// rows ra + a (the D-columns of the block cores [[G, 0], [dG, Gh]]), CZ
+// (ra x n x rb) holds Gh in binary64 (their Z-columns; the zero block is not
+// stored).
 template <typename T>
-__global__ void eta_tt_blocks_kernel(const double* __restrict__ G, const T* __restrict__ Gh, int ra, int64_t n,
-                                     int rb, double* __restrict__ Cb) {
-    const int64_t total = (int64_t)ra * n * rb;
-    const int64_t w = 2 * (int64_t)rb;
-    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+__global__ void eta_tt_blocks_kernel(const double* __restrict__ G, const T* __restrict__ Gh, int64_t cnt,
+                                     double* __restrict__ CD, double* __restrict__ CZ) {
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < cnt;
          e += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t ai = e / rb;              // a * n + i
-        const int b = (int)(e - ai * rb);
         const double g = G[e];
         const double gh = wide(Gh[e]);
-        double* top = Cb + ai * w;
-        double* bot = Cb + (ai + (int64_t)ra * n) * w;
-        top[b] = g;
-        top[rb + b] = 0.0;
-        bot[b] = g - gh;
-        bot[rb + b] = gh;
+        CD[e] = g;
+        CD[cnt + e] = g - gh;
+        CZ[e] = gh;
     }
 }
 
 // ---- C = A^T B over a long reduction, split over CTAs --------------------
-// A: L x p (pitch lda), B: L x q (pitch ldb), binary64.  Output tiles of
-// kGT x kGT; with `sym` only tiles ta <= tb are formed (C symmetric).  The
-// units (tile pair, 32-row chunk) are ordered pair-major and cut into equal
-// contiguous ranges, one per CTA; a CTA writes one partial tile per pair it
-// touches, at slot blockIdx.x + pair (distinct for every (CTA, pair)).
-struct GramArgs {
+// Up to three products per launch.  Product j: A (L x p, pitch lda), B (L x p,
+// pitch ldb), binary64; C (p x p, pitch ldc).  Output tiles are T x T with
+// T = ceil(p / ceil(p / 16)) so that padding stays small; with `sym` only
+// tiles ta <= tb are formed (C symmetric), otherwise C2 (may be null)
+// receives C^T.  The units (product, tile pair, 32-row chunk) are laid end to
+// end and cut into equal contiguous ranges, one per CTA; a CTA writes one
+// partial tile per pair it touches at slot blockIdx.x + global pair index,
+// which is distinct for every (CTA, pair).
+struct GramProb {
     const double* A;
     const double* B;
-    int64_t lda, ldb, L;
-    int p, q, tq, sym;
-    int npairs;
-    int64_t nchunks, Q;
+    double* C;
+    double* C2;
+    int64_t lda, ldb, ldc, L;
+    int p, T, nt, sym;
+    int npairs, t0;            // tile pairs; first global pair index
+    int64_t nchunks, u0, e0;   // chunks per pair; first unit; first output entry
+};
+
+struct GramBatch {
+    GramProb pr[kMaxProbs];
+    int np;
     int G;
+    int64_t Q;                 // units of all products
+    int64_t E;                 // output entries of all products
     double* part;
 };
 
-__device__ __forceinline__ void pair_tiles(const GramArgs& g, int t, int* ta, int* tb) {
-    if (!g.sym) {
-        *ta = t / g.tq;
-        *tb = t - *ta * g.tq;
+__device__ __forceinline__ void pair_tiles(const GramProb& P, int t, int* ta, int* tb) {
+    if (!P.sym) {
+        *ta = t / P.nt;
+        *tb = t - *ta * P.nt;
         return;
     }
     int a = 0, rem = t;
-    while (rem >= g.tq - a) {
-        rem -= g.tq - a;
+    while (rem >= P.nt - a) {
+        rem -= P.nt - a;
         ++a;
     }
     *ta = a;
@@ -166,135 +173,152 @@ __host__ __device__ __forceinline__ int64_t cta_of_unit(int64_t u, int64_t Q, in
     return ((u + 1) * (int64_t)G + Q - 1) / Q - 1;
 }
 
-__global__ void __launch_bounds__(kGThreads) eta_gram_kernel(const __grid_constant__ GramArgs g) {
+__global__ void __launch_bounds__(kGThreads) eta_gram_kernel(const __grid_constant__ GramBatch g) {
     __shared__ double sA[2][kGRows][kGT];
     __shared__ double sB[2][kGRows][kGT];
     const int tid = threadIdx.x;
-    const int tx = tid % kGT, ty = tid / kGT;
-    // loader mapping: 2 elements of A and 2 of B per thread per chunk
-    const int lr = tid / kGT, lc = tid % kGT;     // rows lr and lr + 16
     const int64_t q0 = (int64_t)blockIdx.x * g.Q / g.G;
     const int64_t q1 = (int64_t)(blockIdx.x + 1) * g.Q / g.G;
     int buf = 0;
+    int j = 0;
     int64_t u = q0;
     while (u < q1) {
-        const int t = (int)(u / g.nchunks);
-        const int64_t ce = min(q1, (int64_t)(t + 1) * g.nchunks);
+        while (j + 1 < g.np && u >= g.pr[j + 1].u0) ++j;
+        const GramProb& P = g.pr[j];
+        const double* A = P.A;
+        const double* B = P.B;
+        const int64_t lda = P.lda, ldb = P.ldb, L = P.L, nch = P.nchunks;
+        const int T = P.T, p = P.p;
+        const int64_t lu = u - P.u0;
+        const int t = (int)(lu / nch);
+        const int64_t ce = min(q1, P.u0 + (int64_t)(t + 1) * nch);
         int ta, tb;
-        pair_tiles(g, t, &ta, &tb);
-        const int ca = ta * kGT + lc, cb = tb * kGT + lc;
-        const bool va = ca < g.p, vb = cb < g.q;
-        double acc = 0.0;
-        double ra0, ra1, rb0, rb1;
-        auto fetch = [&](int64_t chunk) {
-            const int64_t r0 = chunk * kGRows + lr, r1 = r0 + 16;
-            ra0 = (va && r0 < g.L) ? g.A[r0 * g.lda + ca] : 0.0;
-            ra1 = (va && r1 < g.L) ? g.A[r1 * g.lda + ca] : 0.0;
-            rb0 = (vb && r0 < g.L) ? g.B[r0 * g.ldb + cb] : 0.0;
-            rb1 = (vb && r1 < g.L) ? g.B[r1 * g.ldb + cb] : 0.0;
-        };
-        fetch(u - (int64_t)t * g.nchunks);
-        for (int64_t v = u; v < ce; ++v) {
-            sA[buf][lr][lc] = ra0;
-            sA[buf][lr + 16][lc] = ra1;
-            sB[buf][lr][lc] = rb0;
-            sB[buf][lr + 16][lc] = rb1;
-            __syncthreads();
-            if (v + 1 < ce) fetch(v + 1 - (int64_t)t * g.nchunks);
+        pair_tiles(P, t, &ta, &tb);
+        const bool compute = tid < T * T;
+        const int tx = compute ? tid % T : 0, ty = compute ? tid / T : 0;
+        // loader: elements e = tid and tid + 256 of the 32 x T chunk
+        int lr[2], lc[2];
+        bool lv[2];
 #pragma unroll
-            for (int r = 0; r < kGRows; ++r) acc = fma(sA[buf][r][ty], sB[buf][r][tx], acc);
+        for (int x = 0; x < 2; ++x) {
+            const int e = tid + kGThreads * x;
+            lv[x] = e < kGRows * T;
+            lr[x] = lv[x] ? e / T : 0;
+            lc[x] = lv[x] ? e % T : 0;
+        }
+        double acc = 0.0;
+        double ra[2], rb[2];
+        auto fetch = [&](int64_t chunk) {
+#pragma unroll
+            for (int x = 0; x < 2; ++x) {
+                const int64_t r = chunk * kGRows + lr[x];
+                const int ca = ta * T + lc[x], cb = tb * T + lc[x];
+                const bool ok = lv[x] && r < L;
+                ra[x] = (ok && ca < p) ? A[r * lda + ca] : 0.0;
+                rb[x] = (ok && cb < p) ? B[r * ldb + cb] : 0.0;
+            }
+        };
+        fetch(lu - (int64_t)t * nch);
+        for (int64_t v = u; v < ce; ++v) {
+#pragma unroll
+            for (int x = 0; x < 2; ++x) {
+                if (lv[x]) {
+                    sA[buf][lr[x]][lc[x]] = ra[x];
+                    sB[buf][lr[x]][lc[x]] = rb[x];
+                }
+            }
+            __syncthreads();
+            if (v + 1 < ce) fetch(v + 1 - P.u0 - (int64_t)t * nch);
+            if (compute) {
+#pragma unroll
+                for (int r = 0; r < kGRows; ++r) acc = fma(sA[buf][r][ty], sB[buf][r][tx], acc);
+            }
             buf ^= 1;
         }
-        g.part[((int64_t)blockIdx.x + t) * (kGT * kGT) + ty * kGT + tx] = acc;
+        if (compute) g.part[((int64_t)blockIdx.x + P.t0 + t) * (kGT * kGT) + ty * T + tx] = acc;
         u = ce;
     }
 }
 
-// C (p x q, pitch ldc) = sum of the partial tiles in CTA order; with `sym`
-// both C[i][j] and C[j][i] take the entry formed for i <= j.
-__global__ void eta_gram_reduce_kernel(const __grid_constant__ GramArgs g, double* __restrict__ C, int64_t ldc) {
+// Every output entry: the partial tiles of its pair added in CTA order.
+__global__ void eta_gram_reduce_kernel(const __grid_constant__ GramBatch g) {
     const int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-    if (e >= (int64_t)g.p * g.q) return;
-    int i = (int)(e / g.q), j = (int)(e % g.q);
-    if (g.sym && i > j) {
-        const int s = i;
-        i = j;
-        j = s;
+    if (e >= g.E) return;
+    int jp = 0;
+    while (jp + 1 < g.np && e >= g.pr[jp + 1].e0) ++jp;
+    const GramProb& P = g.pr[jp];
+    const int64_t le = e - P.e0;
+    const int i0 = (int)(le / P.p), j0 = (int)(le % P.p);
+    int i = i0, j = j0;
+    if (P.sym && i > j) {
+        i = j0;
+        j = i0;
     }
-    const int ta = i / kGT, tb = j / kGT;
-    int t;
-    if (!g.sym) {
-        t = ta * g.tq + tb;
-    } else {
-        t = ta * g.tq - ta * (ta - 1) / 2 + (tb - ta);
-    }
-    const int64_t c0 = cta_of_unit((int64_t)t * g.nchunks, g.Q, g.G);
-    const int64_t c1 = cta_of_unit((int64_t)(t + 1) * g.nchunks - 1, g.Q, g.G);
-    const int off = (i % kGT) * kGT + (j % kGT);
+    const int T = P.T;
+    const int ta = i / T, tb = j / T;
+    const int t = P.sym ? ta * P.nt - ta * (ta - 1) / 2 + (tb - ta) : ta * P.nt + tb;
+    const int64_t c0 = cta_of_unit(P.u0 + (int64_t)t * P.nchunks, g.Q, g.G);
+    const int64_t c1 = cta_of_unit(P.u0 + (int64_t)(t + 1) * P.nchunks - 1, g.Q, g.G);
+    const int off = (i % T) * T + (j % T);
+    const int64_t tg = P.t0 + t;
     double s = 0.0;
-    for (int64_t c = c0; c <= c1; ++c) s += g.part[(c + t) * (kGT * kGT) + off];
-    C[(e / g.q) * ldc + (e % g.q)] = s;
+    for (int64_t c = c0; c <= c1; ++c) s += g.part[(c + tg) * (kGT * kGT) + off];
+    P.C[(int64_t)i0 * P.ldc + j0] = s;
+    if (P.C2) P.C2[(int64_t)j0 * P.ldc + i0] = s;
 }
 
 // ---- C = A B, A p x K (small), B K x N (wide), binary64 ------------------
-__global__ void __launch_bounds__(256) eta_gemm_kernel(const double* __restrict__ A, int64_t lda,
-                                                       const double* __restrict__ B, int64_t ldb,
-                                                       double* __restrict__ C, int64_t ldc, int p, int K,
-                                                       int64_t N) {
-    __shared__ double sA[kMmK][kMmR];
-    __shared__ double sB[kMmK][kMmC];
+// Up to two products per launch; tiles of TR x 16 entries (TR = ceil(p /
+// ceil(p / 16))), one entry per thread, row tiles of one column block in
+// consecutive CTAs.
+struct MmProb {
+    const double* A;
+    const double* B;
+    double* C;
+    int64_t lda, ldb, ldc, N;
+    int p, K, TR, ntr;
+    int64_t b0;                // first CTA
+};
+
+struct MmBatch {
+    MmProb pr[2];
+    int np;
+};
+
+__global__ void __launch_bounds__(256) eta_gemm_kernel(const __grid_constant__ MmBatch g) {
+    __shared__ double sA[kMmK][kMmT];
+    __shared__ double sB[kMmK][kMmT];
+    const int jp = (g.np > 1 && (int64_t)blockIdx.x >= g.pr[1].b0) ? 1 : 0;
+    const MmProb& P = g.pr[jp];
+    const double* A = P.A;
+    const double* B = P.B;
+    const int64_t lb = (int64_t)blockIdx.x - P.b0;
+    const int row0 = (int)(lb % P.ntr) * P.TR;
+    const int64_t col0 = (lb / P.ntr) * kMmT;
     const int tid = threadIdx.x;
-    const int tx = tid % 32, ty = tid / 32;       // 32 x 8 threads, 4 x 4 outputs each
-    const int row0 = blockIdx.y * kMmR;
-    const int64_t col0 = (int64_t)blockIdx.x * kMmC;
-    double acc[4][4];
-#pragma unroll
-    for (int a = 0; a < 4; ++a)
-#pragma unroll
-        for (int b = 0; b < 4; ++b) acc[a][b] = 0.0;
+    const int ty = tid / kMmT, tx = tid % kMmT;
+    const int TR = P.TR, p = P.p, K = P.K;
+    const int64_t N = P.N;
+    double acc = 0.0;
     for (int k0 = 0; k0 < K; k0 += kMmK) {
-        // A tile: 32 rows x 16 k -> 2 per thread
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-            const int e = tid + 256 * q;
-            const int r = e / kMmK, kk = e % kMmK;
+        {
+            const int r = tid / kMmK, kk = tid % kMmK;       // A: TR rows x 16 k
             const int gr = row0 + r, gk = k0 + kk;
-            sA[kk][r] = (gr < p && gk < K) ? A[(int64_t)gr * lda + gk] : 0.0;
-        }
-        // B tile: 16 k x 128 columns -> 8 per thread
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            const int e = tid + 256 * q;
-            const int kk = e / kMmC, c = e % kMmC;
-            const int gk = k0 + kk;
+            sA[kk][r] = (r < TR && gr < p && gk < K) ? A[(int64_t)gr * P.lda + gk] : 0.0;
+            const int kb = tid / kMmT, c = tid % kMmT;       // B: 16 k x 16 columns
             const int64_t gc = col0 + c;
-            sB[kk][c] = (gk < K && gc < N) ? B[(int64_t)gk * ldb + gc] : 0.0;
+            sB[kb][c] = (k0 + kb < K && gc < N) ? B[(int64_t)(k0 + kb) * P.ldb + gc] : 0.0;
         }
         __syncthreads();
+        if (ty < TR) {
 #pragma unroll
-        for (int kk = 0; kk < kMmK; ++kk) {
-            double a[4], b[4];
-#pragma unroll
-            for (int x = 0; x < 4; ++x) a[x] = sA[kk][ty * 4 + x];
-#pragma unroll
-            for (int x = 0; x < 4; ++x) b[x] = sB[kk][tx + 32 * x];
-#pragma unroll
-            for (int x = 0; x < 4; ++x)
-#pragma unroll
-                for (int y = 0; y < 4; ++y) acc[x][y] = fma(a[x], b[y], acc[x][y]);
+            for (int kk = 0; kk < kMmK; ++kk) acc = fma(sA[kk][ty], sB[kk][tx], acc);
         }
         __syncthreads();
     }
-#pragma unroll
-    for (int x = 0; x < 4; ++x) {
-        const int gr = row0 + ty * 4 + x;
-        if (gr >= p) continue;
-#pragma unroll
-        for (int y = 0; y < 4; ++y) {
-            const int64_t gc = col0 + tx + 32 * y;
-            if (gc < N) C[(int64_t)gr * ldc + gc] = acc[x][y];
-        }
-    }
+    const int gr = row0 + ty;
+    const int64_t gc = col0 + tx;
+    if (ty < TR && gr < p && gc < N) P.C[(int64_t)gr * P.ldc + gc] = acc;
 }
 
 // ---- final contractions ------------------------------------------------------
@@ -405,43 +429,105 @@ int grid_for(int64_t work, int threads) {
     return (int)std::max<int64_t>(1, std::min<int64_t>(g, cap));
 }
 
-// Plan of one A^T B reduction; slot count written to *slots.
-GramArgs plan_gram(const double* A, int64_t lda, const double* B, int64_t ldb, int64_t L, int p, int q,
-                   bool sym, double* part) {
-    GramArgs g{};
-    g.A = A;
-    g.B = B;
-    g.lda = lda;
-    g.ldb = ldb;
-    g.L = L;
-    g.p = p;
-    g.q = q;
-    g.sym = sym ? 1 : 0;
-    const int tp = (p + kGT - 1) / kGT;
-    g.tq = (q + kGT - 1) / kGT;
-    g.npairs = sym ? tp * (tp + 1) / 2 : tp * g.tq;
-    g.nchunks = (L + kGRows - 1) / kGRows;
-    g.Q = (int64_t)g.npairs * g.nchunks;
+struct GramSpec {
+    const double* A;
+    const double* B;
+    int64_t lda, ldb, L;
+    int p;
+    bool sym;
+    double* C;
+    double* C2;
+    int64_t ldc;
+};
+
+GramBatch plan_gram(const GramSpec* sp, int np, double* part) {
+    GramBatch g{};
+    g.np = np;
+    int64_t u = 0, e = 0;
+    int t0 = 0;
+    for (int j = 0; j < np; ++j) {
+        GramProb& P = g.pr[j];
+        P.A = sp[j].A;
+        P.B = sp[j].B;
+        P.C = sp[j].C;
+        P.C2 = sp[j].C2;
+        P.lda = sp[j].lda;
+        P.ldb = sp[j].ldb;
+        P.ldc = sp[j].ldc;
+        P.L = sp[j].L;
+        P.p = sp[j].p;
+        P.sym = sp[j].sym ? 1 : 0;
+        const int nt = (P.p + kGT - 1) / kGT;
+        P.T = (P.p + nt - 1) / nt;
+        P.nt = (P.p + P.T - 1) / P.T;
+        P.npairs = P.sym ? P.nt * (P.nt + 1) / 2 : P.nt * P.nt;
+        P.nchunks = std::max<int64_t>(1, (P.L + kGRows - 1) / kGRows);
+        P.u0 = u;
+        P.t0 = t0;
+        P.e0 = e;
+        u += (int64_t)P.npairs * P.nchunks;
+        t0 += P.npairs;
+        e += (int64_t)P.p * P.p;
+    }
+    g.Q = u;
+    g.E = e;
     g.G = (int)std::max<int64_t>(1, std::min<int64_t>(g.Q, 2 * (int64_t)sm_count()));
     g.part = part;
     return g;
 }
 
-int64_t gram_slots(int64_t L, int p, int q, bool sym) {
-    const int tp = (p + kGT - 1) / kGT, tq = (q + kGT - 1) / kGT;
-    const int64_t npairs = sym ? (int64_t)tp * (tp + 1) / 2 : (int64_t)tp * tq;
-    const int64_t nchunks = (L + kGRows - 1) / kGRows;
-    const int64_t G = std::max<int64_t>(1, std::min<int64_t>(npairs * nchunks, 2 * (int64_t)sm_count()));
-    return (G + npairs - 1) * (int64_t)(kGT * kGT);
+// Partial-slot entries a batch needs (computed without a device pointer).
+int64_t gram_slots(const GramSpec* sp, int np) {
+    const GramBatch g = plan_gram(sp, np, nullptr);
+    int pairs = 0;
+    for (int j = 0; j < np; ++j) pairs += g.pr[j].npairs;
+    return ((int64_t)g.G + pairs - 1) * (kGT * kGT);
 }
 
-lrc_status run_gram(const GramArgs& g, double* C, int64_t ldc, cudaStream_t s) {
+lrc_status run_gram(const GramSpec* sp, int np, double* part, cudaStream_t s) {
+    const GramBatch g = plan_gram(sp, np, part);
     eta_gram_kernel<<<g.G, kGThreads, 0, s>>>(g);
     lrc_status st = after_launch("eta_gram_kernel");
     if (st != LRC_OK) return st;
-    const int64_t n = (int64_t)g.p * g.q;
-    eta_gram_reduce_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(g, C, ldc);
+    eta_gram_reduce_kernel<<<(unsigned)((g.E + 255) / 256), 256, 0, s>>>(g);
     return after_launch("eta_gram_reduce_kernel");
+}
+
+struct MmSpec {
+    const double* A;
+    const double* B;
+    double* C;
+    int64_t lda, ldb, ldc, N;
+    int p, K;
+};
+
+lrc_status run_gemm(const MmSpec* sp, int np, cudaStream_t s) {
+    MmBatch g{};
+    g.np = np;
+    int64_t b = 0;
+    for (int j = 0; j < np; ++j) {
+        MmProb& P = g.pr[j];
+        P.A = sp[j].A;
+        P.B = sp[j].B;
+        P.C = sp[j].C;
+        P.lda = sp[j].lda;
+        P.ldb = sp[j].ldb;
+        P.ldc = sp[j].ldc;
+        P.N = sp[j].N;
+        P.p = sp[j].p;
+        P.K = sp[j].K;
+        const int nt = (P.p + kMmT - 1) / kMmT;
+        P.TR = (P.p + nt - 1) / nt;
+        P.ntr = (P.p + P.TR - 1) / P.TR;
+        P.b0 = b;
+        b += (int64_t)P.ntr * ((P.N + kMmT - 1) / kMmT);
+    }
+    if (b > 0x7fffffffLL) {
+        set_error("eta GEMM grid too large");
+        return LRC_ERR_UNSUPPORTED;
+    }
+    eta_gemm_kernel<<<(unsigned)b, 256, 0, s>>>(g);
+    return after_launch("eta_gemm_kernel");
 }
 
 template <typename T>
@@ -459,19 +545,6 @@ lrc_status pack_cols(const double* X, int64_t ldx, const void* Xh, int64_t ldh, 
     return after_launch("eta_pack_cols_kernel");
 }
 
-template <typename T>
-lrc_status tt_blocks(const double* G, const void* Gh, int ra, int64_t n, int rb, double* Cb, cudaStream_t s) {
-    eta_tt_blocks_kernel<T><<<grid_for((int64_t)ra * n * rb, 256), 256, 0, s>>>(G, (const T*)Gh, ra, n, rb, Cb);
-    return after_launch("eta_tt_blocks_kernel");
-}
-
-lrc_status gemm(const double* A, int64_t lda, const double* B, int64_t ldb, double* C, int64_t ldc, int p, int K,
-                int64_t N, cudaStream_t s) {
-    dim3 grid((unsigned)((N + kMmC - 1) / kMmC), (unsigned)((p + kMmR - 1) / kMmR));
-    eta_gemm_kernel<<<grid, 256, 0, s>>>(A, lda, B, ldb, C, ldc, p, K, N);
-    return after_launch("eta_gemm_kernel");
-}
-
 lrc_status read_result(const double* res, double* eta_out, double* norm_out, cudaStream_t s) {
     double host[2];
     cudaError_t e = cudaMemcpyAsync(host, res, sizeof host, cudaMemcpyDeviceToHost, s);
@@ -485,6 +558,16 @@ lrc_status read_result(const double* res, double* eta_out, double* norm_out, cud
 
 size_t align_up(size_t v) { return (v + 255) & ~(size_t)255; }
 
+// Carves consecutive 256-byte aligned regions out of one workspace.
+struct Carve {
+    size_t off = 0;
+    size_t take(size_t bytes) {
+        const size_t o = off;
+        off = align_up(off + bytes);
+        return o;
+    }
+};
+
 template <typename T>
 lrc_status lowrank_eta_t(const double* U, const double* S, const double* Vt, const void* Uh, const void* Sh,
                          const void* Vht, int64_t m, int64_t n, int64_t k, double* eta_out, double* norm_out,
@@ -492,38 +575,31 @@ lrc_status lowrank_eta_t(const double* U, const double* S, const double* Vt, con
     const int kk = (int)k;
     const int w = 2 * kk;
     const int64_t ldk = lrc_packed_ld(k), ldn = lrc_packed_ld(n);
-    const int64_t slots = std::max(gram_slots(m, w, w, true), gram_slots(n, w, w, true));
-    size_t off = 0;
-    const size_t o_pu = off;
-    off = align_up(off + (size_t)m * w * 8);
-    const size_t o_pv = off;
-    off = align_up(off + (size_t)n * w * 8);
-    const size_t o_gu = off;
-    off = align_up(off + (size_t)w * w * 8);
-    const size_t o_gv = off;
-    off = align_up(off + (size_t)w * w * 8);
-    const size_t o_part = off;
-    off = align_up(off + (size_t)slots * 8);
-    const size_t o_cp = off;
-    off = align_up(off + (size_t)2 * kCombineBlocks * 8);
-    const size_t o_res = off;
-    off = align_up(off + 16);
+    GramSpec sp[2] = {{nullptr, nullptr, w, w, m, w, true, nullptr, nullptr, w},
+                      {nullptr, nullptr, w, w, n, w, true, nullptr, nullptr, w}};
+    Carve c;
+    const size_t o_pu = c.take((size_t)m * w * 8), o_pv = c.take((size_t)n * w * 8);
+    const size_t o_gu = c.take((size_t)w * w * 8), o_gv = c.take((size_t)w * w * 8);
+    const size_t o_part = c.take((size_t)gram_slots(sp, 2) * 8);
+    const size_t o_cp = c.take((size_t)2 * kCombineBlocks * 8), o_res = c.take(16);
     void* ws = nullptr;
-    lrc_status st = stream_workspace(s, off, &ws);
+    lrc_status st = stream_workspace(s, c.off, &ws);
     if (st != LRC_OK) return st;
     char* base = (char*)ws;
     double* Pu = (double*)(base + o_pu);
     double* Pv = (double*)(base + o_pv);
     double* Gu = (double*)(base + o_gu);
     double* Gv = (double*)(base + o_gv);
-    double* part = (double*)(base + o_part);
     double* cpart = (double*)(base + o_cp);
     double* res = (double*)(base + o_res);
+    sp[0].A = sp[0].B = Pu;
+    sp[0].C = Gu;
+    sp[1].A = sp[1].B = Pv;
+    sp[1].C = Gv;
 
     if ((st = pack_rows<T>(U, ldk, Uh, ldk, m, kk, 0, Pu, s)) != LRC_OK) return st;
-    if ((st = run_gram(plan_gram(Pu, w, Pu, w, m, w, w, true, part), Gu, w, s)) != LRC_OK) return st;
     if ((st = pack_cols<T>(Vt, ldn, Vht, ldn, n, kk, 0, Pv, s)) != LRC_OK) return st;
-    if ((st = run_gram(plan_gram(Pv, w, Pv, w, n, w, w, true, part), Gv, w, s)) != LRC_OK) return st;
+    if ((st = run_gram(sp, 2, (double*)(base + o_part), s)) != LRC_OK) return st;
     const int cb = std::min(kCombineBlocks, kk);
     eta_lowrank_combine_kernel<T><<<cb, 256, 0, s>>>(Gu, Gv, S, (const T*)Sh, kk, cpart);
     if ((st = after_launch("eta_lowrank_combine_kernel")) != LRC_OK) return st;
@@ -532,48 +608,52 @@ lrc_status lowrank_eta_t(const double* U, const double* S, const double* Vt, con
     return read_result(res, eta_out, norm_out, s);
 }
 
+// The three products of one interior level (D-columns: CD, X_D; Z-columns:
+// CZ, X_Z), written into the blocks of Mn (pitch 2 rb).
+void interior_gram_specs(int ra, int64_t n, int rb, const double* CD, const double* CZ, const double* XD,
+                         const double* XZ, double* Mn, GramSpec* sp) {
+    const int64_t ld = 2 * (int64_t)rb;
+    const int64_t L2 = 2 * (int64_t)ra * n, L1 = (int64_t)ra * n;
+    sp[0] = {CD, XD, rb, rb, L2, rb, true, Mn, nullptr, ld};                              // M'_DD
+    sp[1] = {CD, XZ, rb, rb, L2, rb, false, Mn + rb, Mn + (int64_t)rb * ld, ld};          // M'_DZ, M'_ZD
+    sp[2] = {CZ, XZ + L1 * rb, rb, rb, L1, rb, true, Mn + (int64_t)rb * ld + rb, nullptr, ld};   // M'_ZZ
+}
+
 template <typename T>
 lrc_status tt_eta_t(const TTShape& sh, const void* const* hats, double* eta_out, double* norm_out,
                     cudaStream_t s) {
     const int d = sh.d;
     int rmax = 1;
-    int64_t blocks_max = 0, slots = 0;
     for (int l = 0; l <= d; ++l) rmax = std::max<int>(rmax, (int)sh.ranks[l]);
-    // level 1: Gram of [dG_1, Gh_1] over n_1 rows; levels 2..d-1: block cores
-    // and M C over 2 r_{l-1} n_l rows; level d: Gram of [G_d; dG_d] columns
-    slots = std::max(slots, gram_slots(sh.dims[0], 2 * (int)sh.ranks[1], 2 * (int)sh.ranks[1], true));
-    for (int l = 1; l < d - 1; ++l) {
-        const int64_t ra = sh.ranks[l], rb = sh.ranks[l + 1], n = sh.dims[l];
-        blocks_max = std::max(blocks_max, 4 * ra * n * rb);
-        slots = std::max(slots, gram_slots(2 * ra * n, 2 * (int)rb, 2 * (int)rb, true));
+    const int r1 = (int)sh.ranks[1], rl = (int)sh.ranks[d - 1];
+    const int64_t n1 = sh.dims[0], nl = sh.dims[d - 1];
+    // workspace sizes: packed first / last core, per-level operands, slots
+    int64_t lev_max = 0, slots = 0;
+    {
+        GramSpec a = {nullptr, nullptr, 2 * r1, 2 * r1, n1, 2 * r1, true, nullptr, nullptr, 2 * r1};
+        GramSpec b = {nullptr, nullptr, 2 * rl, 2 * rl, nl, 2 * rl, true, nullptr, nullptr, 2 * rl};
+        slots = std::max(gram_slots(&a, 1), gram_slots(&b, 1));
     }
-    const int64_t rl = sh.ranks[d - 1], nl = sh.dims[d - 1];
-    slots = std::max(slots, gram_slots(nl, 2 * (int)rl, 2 * (int)rl, true));
-    const int64_t pack_max = std::max(sh.dims[0] * 2 * sh.ranks[1], nl * 2 * rl);
-    size_t off = 0;
-    const size_t o_pk = off;
-    off = align_up(off + (size_t)pack_max * 8);
-    const size_t o_cb = off;
-    off = align_up(off + (size_t)blocks_max * 8);
-    const size_t o_x = off;
-    off = align_up(off + (size_t)blocks_max * 8);
-    const size_t o_m0 = off;
-    off = align_up(off + (size_t)4 * rmax * rmax * 8);
-    const size_t o_m1 = off;
-    off = align_up(off + (size_t)4 * rmax * rmax * 8);
-    const size_t o_part = off;
-    off = align_up(off + (size_t)slots * 8);
-    const size_t o_cp = off;
-    off = align_up(off + (size_t)2 * kCombineBlocks * 8);
-    const size_t o_res = off;
-    off = align_up(off + 16);
+    for (int l = 1; l < d - 1; ++l) {
+        const int ra = (int)sh.ranks[l], rb = (int)sh.ranks[l + 1];
+        const int64_t n = sh.dims[l];
+        lev_max = std::max(lev_max, 7 * (int64_t)ra * n * rb);
+        GramSpec sp[3];
+        interior_gram_specs(ra, n, rb, nullptr, nullptr, nullptr, nullptr, nullptr, sp);
+        slots = std::max(slots, gram_slots(sp, 3));
+    }
+    const int64_t pack_max = std::max(n1 * 2 * r1, nl * 2 * rl);
+    Carve c;
+    const size_t o_pk = c.take((size_t)pack_max * 8), o_lev = c.take((size_t)lev_max * 8);
+    const size_t o_m0 = c.take((size_t)4 * rmax * rmax * 8), o_m1 = c.take((size_t)4 * rmax * rmax * 8);
+    const size_t o_part = c.take((size_t)slots * 8);
+    const size_t o_cp = c.take((size_t)2 * kCombineBlocks * 8), o_res = c.take(16);
     void* ws = nullptr;
-    lrc_status st = stream_workspace(s, off, &ws);
+    lrc_status st = stream_workspace(s, c.off, &ws);
     if (st != LRC_OK) return st;
     char* base = (char*)ws;
     double* Pk = (double*)(base + o_pk);
-    double* Cb = (double*)(base + o_cb);
-    double* Xb = (double*)(base + o_x);
+    double* lev = (double*)(base + o_lev);
     double* Mcur = (double*)(base + o_m0);
     double* Mnext = (double*)(base + o_m1);
     double* part = (double*)(base + o_part);
@@ -581,41 +661,44 @@ lrc_status tt_eta_t(const TTShape& sh, const void* const* hats, double* eta_out,
     double* res = (double*)(base + o_res);
 
     // level 1: M_1 = [dG_1, Gh_1]^T [dG_1, Gh_1]  (G_1 is n_1 x r_1)
+    if ((st = pack_rows<T>((const double*)sh.cores[0], r1, hats[0], r1, n1, r1, 0, Pk, s)) != LRC_OK) return st;
     {
-        const int r1 = (int)sh.ranks[1];
-        const int64_t n1 = sh.dims[0];
-        if ((st = pack_rows<T>((const double*)sh.cores[0], r1, hats[0], r1, n1, r1, 0, Pk, s)) != LRC_OK) return st;
-        if ((st = run_gram(plan_gram(Pk, 2 * r1, Pk, 2 * r1, n1, 2 * r1, 2 * r1, true, part), Mcur, 2 * r1, s)) !=
-            LRC_OK)
-            return st;
+        GramSpec a = {Pk, Pk, 2 * r1, 2 * r1, n1, 2 * r1, true, Mcur, nullptr, 2 * r1};
+        if ((st = run_gram(&a, 1, part, s)) != LRC_OK) return st;
     }
     // interior levels: M_l = sum_i C_l(i)^T M_{l-1} C_l(i)
     for (int l = 1; l < d - 1; ++l) {
         const int ra = (int)sh.ranks[l], rb = (int)sh.ranks[l + 1];
         const int64_t n = sh.dims[l];
-        if ((st = tt_blocks<T>((const double*)sh.cores[l], hats[l], ra, n, rb, Cb, s)) != LRC_OK) return st;
-        const int64_t N = n * 2 * rb;
-        if ((st = gemm(Mcur, 2 * ra, Cb, N, Xb, N, 2 * ra, 2 * ra, N, s)) != LRC_OK) return st;
-        const int64_t L = 2 * (int64_t)ra * n;
-        if ((st = run_gram(plan_gram(Cb, 2 * rb, Xb, 2 * rb, L, 2 * rb, 2 * rb, true, part), Mnext, 2 * rb, s)) !=
-            LRC_OK)
-            return st;
+        const int64_t cnt = (int64_t)ra * n * rb, N = n * rb;
+        double* CD = lev;
+        double* CZ = CD + 2 * cnt;
+        double* XD = CZ + cnt;
+        double* XZ = XD + 2 * cnt;
+        eta_tt_blocks_kernel<T><<<grid_for(cnt, 256), 256, 0, s>>>((const double*)sh.cores[l], (const T*)hats[l],
+                                                                    cnt, CD, CZ);
+        if ((st = after_launch("eta_tt_blocks_kernel")) != LRC_OK) return st;
+        // X_D = M [G; dG], X_Z = M[:, Z] Gh  (2ra x n rb each)
+        MmSpec mm[2] = {{Mcur, CD, XD, 2 * ra, N, N, N, 2 * ra, 2 * ra},
+                        {Mcur + ra, CZ, XZ, 2 * ra, N, N, N, 2 * ra, ra}};
+        if ((st = run_gemm(mm, 2, s)) != LRC_OK) return st;
+        GramSpec sp[3];
+        interior_gram_specs(ra, n, rb, CD, CZ, XD, XZ, Mnext, sp);
+        if ((st = run_gram(sp, 3, part, s)) != LRC_OK) return st;
         std::swap(Mcur, Mnext);
     }
     // level d: H = Gram of the columns [G_d(:, i); dG_d(:, i)] (G_d is r x n_d)
+    if ((st = pack_cols<T>((const double*)sh.cores[d - 1], nl, hats[d - 1], nl, nl, rl, 1, Pk, s)) != LRC_OK)
+        return st;
     {
-        const int r = (int)rl;
-        if ((st = pack_cols<T>((const double*)sh.cores[d - 1], nl, hats[d - 1], nl, nl, r, 1, Pk, s)) != LRC_OK)
-            return st;
-        if ((st = run_gram(plan_gram(Pk, 2 * r, Pk, 2 * r, nl, 2 * r, 2 * r, true, part), Mnext, 2 * r, s)) !=
-            LRC_OK)
-            return st;
-        const int cb = std::min(kCombineBlocks, r);
-        eta_tt_combine_kernel<<<cb, 256, 0, s>>>(Mcur, Mnext, r, cpart);
-        if ((st = after_launch("eta_tt_combine_kernel")) != LRC_OK) return st;
-        eta_finish_kernel<<<1, 32, 0, s>>>(cpart, cb, res);
-        if ((st = after_launch("eta_finish_kernel")) != LRC_OK) return st;
+        GramSpec b = {Pk, Pk, 2 * rl, 2 * rl, nl, 2 * rl, true, Mnext, nullptr, 2 * rl};
+        if ((st = run_gram(&b, 1, part, s)) != LRC_OK) return st;
     }
+    const int cb = std::min(kCombineBlocks, rl);
+    eta_tt_combine_kernel<<<cb, 256, 0, s>>>(Mcur, Mnext, rl, cpart);
+    if ((st = after_launch("eta_tt_combine_kernel")) != LRC_OK) return st;
+    eta_finish_kernel<<<1, 32, 0, s>>>(cpart, cb, res);
+    if ((st = after_launch("eta_finish_kernel")) != LRC_OK) return st;
     return read_result(res, eta_out, norm_out, s);
 }
 
