@@ -122,6 +122,16 @@ def work_eta_tt(dims, ranks, fmt):
     return {"bytes": cores * (8 + E[fmt]), "flops": flops, "alu": "f64"}
 
 
+def work_gather(dims, ranks, fmt, count):
+    """Sampled entries: one chain of vector-matrix products per entry (CUDA
+    cores: binary64 for FP64, binary32 otherwise); indices in, values out."""
+    d = len(dims)
+    per = sum(ranks[l] * ranks[l + 1] for l in range(d))
+    cores = sum(ranks[l] * dims[l] * ranks[l + 1] for l in range(d))
+    return {"bytes": count * (8 + E_OUT[fmt]) + cores * E[fmt], "flops": 2 * per * count,
+            "alu": "f64" if fmt == "f64" else "f32"}
+
+
 def work_fro(count, fa, fb):
     return {"bytes": count * (E[fa] + E[fb]), "flops": 0, "alu": None}
 
@@ -549,6 +559,15 @@ def run_case(args):
         ranks = cfg.ranks[base]
         call = lambda: lrc.lrc_tt_eta(c64, low, cfg.dims, ranks, fmt)  # noqa: E731
         work = work_eta_tt(cfg.dims, ranks, fmt)
+    elif args.case == "gather":
+        cfg = W.TT_CONFIGS[args.tt]
+        cores = [torch.from_numpy(c).to(dev).to(lrc.storage_dtype(fmt)).contiguous() for c in W.tt_cores(cfg, base)]
+        ranks = cfg.ranks[base]
+        total = int(np.prod(cfg.dims))
+        idx = torch.from_numpy(np.random.default_rng(9).integers(0, total, size=args.count)).to(dev)
+        out = torch.empty(args.count, dtype=lrc.output_dtype(fmt), device=dev)
+        call = lambda: lrc.tt_gather(cores, cfg.dims, ranks, fmt, idx, out)  # noqa: E731
+        work = work_gather(cfg.dims, ranks, fmt, args.count)
     elif args.case == "fro":
         a = torch.randn(args.count, dtype=torch.float64, device=dev)
         b2 = torch.randn(args.count, dtype=torch.float64, device=dev)
@@ -592,7 +611,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", choices=["apply", "tt", "fro", "round", "eta_matrix", "eta_tt"], default=None,
+    ap.add_argument("--case", choices=["apply", "tt", "fro", "round", "eta_matrix", "eta_tt", "gather"], default=None,
                     help="time one call type instead of the step (profiling captures)")
     ap.add_argument("--fmt", default="f16")
     ap.add_argument("--m", type=int, default=16384)

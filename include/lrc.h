@@ -156,6 +156,31 @@ LRC_API lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims,
                           int d, lrc_fmt fmt, void* out, lrc_stream_t stream);
 
 /*
+ * tt_gather -- sampled entries T(i_1..i_d) = G_1(i_1) G_2(i_2) ... G_d(i_d)
+ * of a Tensor Train (Sec. 5.1), each evaluated by its own core chain: the
+ * independent check of a dense reconstruction on sampled entries.
+ *
+ *   cores, dims, ranks, d, fmt  as in tt_reconstruct; ranks up to 256, else
+ *           LRC_ERR_UNSUPPORTED
+ *   idx     device, `count` int64 flat indices into the C-order vectorised
+ *           tensor (i_1 slowest), 8-byte aligned; an index outside
+ *           [0, prod(dims)) yields a quiet NaN in its output slot
+ *   count   number of entries, >= 0 (0: nothing is launched)
+ *   out     device, `count` values: binary64 for LRC_F64, binary32 for
+ *           LRC_F32 and LRC_F16, binary16 for LRC_F16_O16; aligned to the
+ *           element size
+ *
+ * Arithmetic: binary64 FMA for LRC_F64; binary32 FMA for LRC_F32 and for
+ * binary16 cores (products of binary16 values accumulated in binary32,
+ * Sec. 3.4); LRC_F16_O16 rounds the binary32 result to binary16 once.
+ * Entries are independent: duplicates and any order are allowed.
+ * Asynchronous on `stream`.
+ */
+LRC_API lrc_status tt_gather(const void* const* cores, const int64_t* dims, const int64_t* ranks, int d,
+                             lrc_fmt fmt, const int64_t* idx, int64_t count, void* out,
+                             lrc_stream_t stream);
+
+/*
  * lrc_fro_diff -- Frobenius norm of a difference (Sec. 5.1 "Frobenius norm";
  * eta of Thm 4.1 and eta_TT of Thm 6.1 are ||A_k' - Ahat_k'||_F and
  * ||T_R+ - That_R+||_F of the FP64 reconstructions).

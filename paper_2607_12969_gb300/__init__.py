@@ -58,6 +58,8 @@ def load() -> ctypes.CDLL:
     L.lrc_fro_diff.restype = i32
     L.lrc_fro_diff_noalloc.argtypes = [vp, i32, vp, i32, i64, vp, vp, vp]
     L.lrc_fro_diff_noalloc.restype = i32
+    L.tt_gather.argtypes = [vp, vp, vp, i32, i32, vp, i64, vp, vp]
+    L.tt_gather.restype = i32
     L.lrc_lowrank_eta.argtypes = [vp, vp, vp, vp, vp, vp, i32, i64, i64, i64, vp, vp, vp]
     L.lrc_lowrank_eta.restype = i32
     L.lrc_tt_eta.argtypes = [vp, vp, vp, vp, i32, i32, vp, vp, vp]
@@ -151,6 +153,17 @@ def tt_reconstruct(cores: Sequence, dims: Sequence[int], ranks: Sequence[int], f
     _check(load().tt_reconstruct(ctypes.cast(ptrs, ctypes.c_void_p), ctypes.cast(dd, ctypes.c_void_p),
                                  ctypes.cast(rr, ctypes.c_void_p), d, _fmt(fmt), _ptr(out),
                                  _stream(stream)))
+
+
+def tt_gather(cores: Sequence, dims: Sequence[int], ranks: Sequence[int], fmt, idx, out, stream=None):
+    """Entries of the TT at the flat indices `idx` (int64 CUDA tensor) into `out`."""
+    d = len(cores)
+    ptrs = (ctypes.c_void_p * d)(*[c.data_ptr() for c in cores])
+    dd = (ctypes.c_int64 * d)(*[int(x) for x in dims])
+    rr = (ctypes.c_int64 * (d + 1))(*[int(x) for x in ranks])
+    _check(load().tt_gather(ctypes.cast(ptrs, ctypes.c_void_p), ctypes.cast(dd, ctypes.c_void_p),
+                            ctypes.cast(rr, ctypes.c_void_p), d, _fmt(fmt), _ptr(idx), int(idx.numel()),
+                            _ptr(out), _stream(stream)))
 
 
 def lrc_fro_diff(A, fa, B, fb, count: int, stream=None, want_norm: bool = True) -> Tuple[float, float]:

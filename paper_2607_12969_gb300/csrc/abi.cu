@@ -181,6 +181,35 @@ lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims, const i
     return launch_tt_cc(sh, fmt, out, s);
 }
 
+lrc_status tt_gather(const void* const* cores, const int64_t* dims, const int64_t* ranks, int d, lrc_fmt fmt,
+                     const int64_t* idx, int64_t count, void* out, lrc_stream_t stream) {
+    if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    if (count < 0) return invalid("negative count");
+    TTShape sh;
+    lrc_status st = tt_shape(cores, dims, ranks, d, storage_bytes(fmt), "cores", &sh);
+    if (st != LRC_OK) return st;
+    for (int l = 0; l <= d; ++l)
+        if (ranks[l] > tt_gather_max_rank()) {
+            set_error("tt_gather supports ranks up to %d (ranks[%d] = %lld)", tt_gather_max_rank(), l,
+                      (long long)ranks[l]);
+            return LRC_ERR_UNSUPPORTED;
+        }
+    if (count == 0) return LRC_OK;
+    if (!idx || !out) return invalid("null pointer");
+    int64_t t;
+    if (!mul_ok(count, 8, &t)) return invalid("size overflow");
+    if ((reinterpret_cast<uintptr_t>(idx) & 7u) != 0) {
+        set_error("idx is not 8-byte aligned");
+        return LRC_ERR_ALIGNMENT;
+    }
+    const uintptr_t oa = (fmt == LRC_F16_O16) ? 2u : (fmt == LRC_F64 ? 8u : 4u);
+    if ((reinterpret_cast<uintptr_t>(out) % oa) != 0) {
+        set_error("out is not aligned to its element size");
+        return LRC_ERR_ALIGNMENT;
+    }
+    return launch_tt_gather(sh, fmt, idx, count, out, as_stream(stream));
+}
+
 lrc_status lrc_lowrank_eta(const double* U, const double* S, const double* Vt, const void* Uh, const void* Sh,
                            const void* Vht, lrc_fmt fmt, int64_t m, int64_t n, int64_t k, double* eta_out,
                            double* norm_out, lrc_stream_t stream) {

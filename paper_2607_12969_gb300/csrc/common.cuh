@@ -116,6 +116,11 @@ lrc_status run_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fm
                                 double* diff_out, double* normA_out, cudaStream_t s);
 int64_t fro_diff_noalloc_max_count();
 
+// Sampled TT entries (tt_gather.cu); ranks up to tt_gather_max_rank().
+int tt_gather_max_rank();
+lrc_status launch_tt_gather(const TTShape& sh, lrc_fmt fmt, const int64_t* idx, int64_t count, void* out,
+                            cudaStream_t s);
+
 // eta of Thm 4.1 / eta_TT of Thm 6.1 from Gram blocks (eta.cu); synchronise s.
 lrc_status run_lowrank_eta(const double* U, const double* S, const double* Vt, const void* Uh, const void* Sh,
                            const void* Vht, lrc_fmt fmt, int64_t m, int64_t n, int64_t k, double* eta_out,

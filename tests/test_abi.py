@@ -128,3 +128,17 @@ def test_eta_validation_rejects_before_launch(L):
     assert L.lrc_tt_eta(c, nul, dims, good, d, 2, po, None, None) == -1
     odd = (ctypes.c_void_p * d)(16, 20, 16)                 # binary64 core not 8-byte aligned
     assert L.lrc_tt_eta(odd, ch, dims, good, d, 0, po, None, None) == -2
+
+
+def test_gather_validation_rejects_before_launch(L):
+    d = 2
+    c = (ctypes.c_void_p * d)(16, 16)
+    dims = (ctypes.c_int64 * d)(4, 5)
+    ranks = (ctypes.c_int64 * (d + 1))(1, 3, 1)
+    assert L.tt_gather(c, dims, ranks, d, 0, 16, -1, 16, None) == -1            # negative count
+    assert L.tt_gather(c, dims, ranks, d, 0, 16, 0, 16, None) == 0              # nothing to do
+    assert L.tt_gather(c, dims, ranks, d, 0, None, 3, 16, None) == -1           # null idx
+    assert L.tt_gather(c, dims, ranks, d, 0, 12, 3, 16, None) == -2             # idx misaligned
+    assert L.tt_gather(c, dims, ranks, d, 0, 16, 3, 20, None) == -2             # out misaligned (f64)
+    big = (ctypes.c_int64 * (d + 1))(1, 300, 1)
+    assert L.tt_gather(c, dims, big, d, 0, 16, 3, 16, None) == -3               # rank above 256
