@@ -19,11 +19,12 @@
 // element per row so that the transposing stores are conflict-free too.
 //
 // binary64 (DFMA-bound: the GB300 issues about 2 DFMA per clock per SM) uses
-// this generic kernel with thin 8-row tiles and many CTAs per SM, so the work
-// spreads evenly over the SMs.  binary32 has its own kernel below
-// (apply_f32_kernel) with vectorised shared loads and prefetching; it adds
-// each slab's partial sums to the running sums separately (blocked
-// accumulation, rounding error growing like sqrt(n / BK1)).
+// this kernel with thin 8-row tiles and many CTAs per SM, so the work spreads
+// evenly over the SMs.  binary32 (FFMA-bound) runs the two products on the
+// register-tiled kernel of gemm_cc.cu instead: phase 1 split over n (partial
+// sums of at most 1024 terms, added in split order by
+// reduce_scale_f32_kernel, which also applies diag(s)), phase 2 over
+// 128 x 128 tiles of Y.  W (b x k') passes through the stream's workspace.
 #include "common.cuh"
 
 namespace lrc {
@@ -168,166 +169,6 @@ apply_cc_kernel(const T* __restrict__ U, const T* __restrict__ S, const T* __res
     }
 }
 
-// ---------------------------------------------------------------------------
-// binary32: FFMA-bound (128 FMA per clock per SM), so shared-memory traffic
-// per FMA matters.  Each thread owns a contiguous 4 x 4 register tile and
-// reads its operands as 128-bit shared loads (the A operand is the same for
-// the 16 threads of a half-warp row group, a broadcast); the next global
-// slab is fetched into registers while the current one is multiplied.
-// ---------------------------------------------------------------------------
-namespace f32k {
-constexpr int BM = 32, BN = 64, BK1 = 32, BK2 = 16, TM = 4, TN = 4, TX = 16, NT = 128;
-constexpr int LDA = BM + 4, LDB = BN + 4;     // 16-byte aligned rows
-}
-
-__device__ __forceinline__ float4 ld4(const float* p) { return *reinterpret_cast<const float4*>(p); }
-
-// Loads 8 consecutive floats of row `r` (of `rows`), columns c0..c0+7 (of
-// `cols`), zero outside.  Rows have pitch `ld` (a multiple of 16 floats).
-__device__ __forceinline__ void load8(const float* __restrict__ base, int64_t ld, int64_t r, int64_t rows,
-                                      int64_t c0, int64_t cols, float (&v)[8]) {
-    if (r < rows && c0 + 8 <= cols) {
-        const float4 a = __ldg(reinterpret_cast<const float4*>(base + r * ld + c0));
-        const float4 b = __ldg(reinterpret_cast<const float4*>(base + r * ld + c0 + 4));
-        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-        v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-    } else {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) v[j] = (r < rows && c0 + j < cols) ? __ldg(base + r * ld + c0 + j) : 0.0f;
-    }
-}
-
-// X slab (32 x 32) row xr cols xc..+7, and Vt slab rows xr and xr+32 of the
-// chunk starting at rank kc (only rows below cols_v are real).
-__device__ __forceinline__ void fetch_phase1(const float* __restrict__ X, const float* __restrict__ Vt, int64_t ldn,
-                                             int64_t row0, int64_t b, int64_t n, int k, int kc, int cols_v,
-                                             int xr, int xc, int64_t k0, float (&xv)[8], float (&v0)[8],
-                                             float (&v1)[8]) {
-    load8(X, ldn, row0 + xr, b, k0 + xc, n, xv);
-    if (xr < cols_v) {
-        load8(Vt, ldn, kc + xr, k, k0 + xc, n, v0);
-    } else {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) v0[j] = 0.0f;
-    }
-    if (xr + 32 < cols_v) {
-        load8(Vt, ldn, kc + xr + 32, k, k0 + xc, n, v1);
-    } else {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) v1[j] = 0.0f;
-    }
-}
-
-__global__ void __launch_bounds__(f32k::NT, 3)
-apply_f32_kernel(const float* __restrict__ U, const float* __restrict__ S, const float* __restrict__ Vt,
-                 const float* __restrict__ X, float* __restrict__ Y, int64_t m, int64_t n, int k, int64_t b,
-                 int64_t ldk, int64_t ldn, int kp16, int64_t ntiles, int64_t m_chunk) {
-    using namespace f32k;
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    float* Ws = reinterpret_cast<float*>(smem_raw);    // [kp16][BM]   scaled W, transposed
-    float* As = Ws + (size_t)kp16 * BM;                 // [BK1][LDA]   X slab, transposed
-    float* Bs = As + BK1 * LDA;                         // [BK1][LDB]   Vt / U slab, transposed
-    const int tid = threadIdx.x;
-    const int tx = tid % TX, ty = tid / TX;
-    const int64_t mbeg = (int64_t)blockIdx.y * m_chunk;
-    const int64_t mend = (mbeg + m_chunk < m) ? mbeg + m_chunk : m;
-    // slab-load mapping: X slab 32 x 32 -> thread loads row tid/4, columns (tid%4)*8 .. +7
-    const int xr = tid / 4, xc = (tid % 4) * 8;
-
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-        const int64_t row0 = tile * BM;
-        // ---------------- phase 1 -----------------------------------------------
-        for (int kc = 0; kc < kp16; kc += BN) {
-            const int cols_v = (kp16 - kc) < BN ? (kp16 - kc) : BN;     // rank columns in this chunk
-            float acc[TM][TN] = {};
-            float xv[8], v0[8], v1[8];
-            fetch_phase1(X, Vt, ldn, row0, b, n, k, kc, cols_v, xr, xc, 0, xv, v0, v1);
-            for (int64_t k0 = 0; k0 < n; k0 += BK1) {
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    As[(xc + j) * LDA + xr] = xv[j];
-                    Bs[(xc + j) * LDB + xr] = v0[j];
-                    Bs[(xc + j) * LDB + xr + 32] = v1[j];
-                }
-                __syncthreads();
-                if (k0 + BK1 < n) fetch_phase1(X, Vt, ldn, row0, b, n, k, kc, cols_v, xr, xc, k0 + BK1, xv, v0, v1);
-                float part[TM][TN] = {};
-#pragma unroll 8
-                for (int c = 0; c < BK1; ++c) {
-                    const float4 a = ld4(As + c * LDA + ty * TM);
-                    const float4 bb = ld4(Bs + c * LDB + tx * TN);
-                    part[0][0] = fmaf(a.x, bb.x, part[0][0]); part[0][1] = fmaf(a.x, bb.y, part[0][1]);
-                    part[0][2] = fmaf(a.x, bb.z, part[0][2]); part[0][3] = fmaf(a.x, bb.w, part[0][3]);
-                    part[1][0] = fmaf(a.y, bb.x, part[1][0]); part[1][1] = fmaf(a.y, bb.y, part[1][1]);
-                    part[1][2] = fmaf(a.y, bb.z, part[1][2]); part[1][3] = fmaf(a.y, bb.w, part[1][3]);
-                    part[2][0] = fmaf(a.z, bb.x, part[2][0]); part[2][1] = fmaf(a.z, bb.y, part[2][1]);
-                    part[2][2] = fmaf(a.z, bb.z, part[2][2]); part[2][3] = fmaf(a.z, bb.w, part[2][3]);
-                    part[3][0] = fmaf(a.w, bb.x, part[3][0]); part[3][1] = fmaf(a.w, bb.y, part[3][1]);
-                    part[3][2] = fmaf(a.w, bb.z, part[3][2]); part[3][3] = fmaf(a.w, bb.w, part[3][3]);
-                }
-#pragma unroll
-                for (int i = 0; i < TM; ++i)
-#pragma unroll
-                    for (int j = 0; j < TN; ++j) acc[i][j] += part[i][j];
-                __syncthreads();
-            }
-#pragma unroll
-            for (int j = 0; j < TN; ++j) {
-                const int cj = tx * TN + j;
-                if (cj >= cols_v) break;
-                const int gj = kc + cj;
-                const float sj = (gj < k) ? S[gj] : 0.0f;
-#pragma unroll
-                for (int i = 0; i < TM; ++i) Ws[(size_t)gj * BM + ty * TM + i] = acc[i][j] * sj;
-            }
-        }
-        __syncthreads();
-        // ---------------- phase 2 -----------------------------------------------
-        // U slab: 64 rows x 16 cols -> thread loads row tid/2, columns (tid%2)*8 .. +7
-        const int ur = tid / 2, uc = (tid % 2) * 8;
-        for (int64_t mt = mbeg; mt < mend; mt += BN) {
-            float acc[TM][TN] = {};
-            float uv[8];
-            load8(U, ldk, mt + ur, mend, uc, k, uv);
-            for (int k0 = 0; k0 < kp16; k0 += BK2) {
-#pragma unroll
-                for (int j = 0; j < 8; ++j) Bs[(uc + j) * LDB + ur] = uv[j];
-                __syncthreads();
-                if (k0 + BK2 < kp16) load8(U, ldk, mt + ur, mend, k0 + BK2 + uc, k, uv);
-#pragma unroll
-                for (int c = 0; c < BK2; ++c) {
-                    const float4 a = ld4(Ws + (size_t)(k0 + c) * BM + ty * TM);
-                    const float4 bb = ld4(Bs + c * LDB + tx * TN);
-                    acc[0][0] = fmaf(a.x, bb.x, acc[0][0]); acc[0][1] = fmaf(a.x, bb.y, acc[0][1]);
-                    acc[0][2] = fmaf(a.x, bb.z, acc[0][2]); acc[0][3] = fmaf(a.x, bb.w, acc[0][3]);
-                    acc[1][0] = fmaf(a.y, bb.x, acc[1][0]); acc[1][1] = fmaf(a.y, bb.y, acc[1][1]);
-                    acc[1][2] = fmaf(a.y, bb.z, acc[1][2]); acc[1][3] = fmaf(a.y, bb.w, acc[1][3]);
-                    acc[2][0] = fmaf(a.z, bb.x, acc[2][0]); acc[2][1] = fmaf(a.z, bb.y, acc[2][1]);
-                    acc[2][2] = fmaf(a.z, bb.z, acc[2][2]); acc[2][3] = fmaf(a.z, bb.w, acc[2][3]);
-                    acc[3][0] = fmaf(a.w, bb.x, acc[3][0]); acc[3][1] = fmaf(a.w, bb.y, acc[3][1]);
-                    acc[3][2] = fmaf(a.w, bb.z, acc[3][2]); acc[3][3] = fmaf(a.w, bb.w, acc[3][3]);
-                }
-                __syncthreads();
-            }
-#pragma unroll
-            for (int i = 0; i < TM; ++i) {
-                const int64_t gr = row0 + ty * TM + i;
-                if (gr >= b) continue;
-                const int64_t gm = mt + tx * TN;
-                float* yp = Y + gr * m + gm;
-                if (gm + TN <= mend && (m % 4) == 0) {
-                    *reinterpret_cast<float4*>(yp) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
-                } else {
-#pragma unroll
-                    for (int j = 0; j < TN; ++j)
-                        if (gm + j < mend) yp[j] = acc[i][j];
-                }
-            }
-        }
-        __syncthreads();
-    }
-}
-
 template <typename T, int TN1>
 lrc_status launch_apply_cc_n(const T* U, const T* S, const T* Vt, const T* X, T* Y, int64_t m, int64_t n,
                              int64_t k, int64_t b, int kp16, int passes, cudaStream_t s, const char* name) {
@@ -396,6 +237,38 @@ lrc_status launch_apply_cc(const T* U, const T* S, const T* Vt, const T* X, T* Y
     }
 }
 
+// W[r][c] = (sum of the splits' partial products, in split order) * s[c] for
+// c < k, zero for k <= c < ldw; one thread per four columns.
+__global__ void __launch_bounds__(256)
+reduce_scale_f32_kernel(const float* __restrict__ part, int splits, int64_t split_stride, int64_t rows, int64_t k,
+                        int64_t ldw, const float* __restrict__ S, float* __restrict__ W) {
+    const int64_t q = ldw / 4;
+    const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= rows * q) return;
+    const int64_t r = e / q, c = (e - r * q) * 4;
+    float4 acc = __ldcs(reinterpret_cast<const float4*>(part + r * ldw + c));
+    for (int z = 1; z < splits; ++z) {
+        const float4 v = __ldcs(reinterpret_cast<const float4*>(part + (int64_t)z * split_stride + r * ldw + c));
+        acc.x = __fadd_rn(acc.x, v.x);
+        acc.y = __fadd_rn(acc.y, v.y);
+        acc.z = __fadd_rn(acc.z, v.z);
+        acc.w = __fadd_rn(acc.w, v.w);
+    }
+    acc.x = c + 0 < k ? __fmul_rn(acc.x, S[c + 0]) : 0.0f;
+    acc.y = c + 1 < k ? __fmul_rn(acc.y, S[c + 1]) : 0.0f;
+    acc.z = c + 2 < k ? __fmul_rn(acc.z, S[c + 2]) : 0.0f;
+    acc.w = c + 3 < k ? __fmul_rn(acc.w, S[c + 3]) : 0.0f;
+    *reinterpret_cast<float4*>(W + r * ldw + c) = acc;
+}
+
+lrc_status launch_reduce_scale_f32(const float* part, int splits, int64_t split_stride, int64_t rows, int64_t k,
+                                   int64_t ldw, const float* S, float* W, cudaStream_t s) {
+    const int64_t items = rows * (ldw / 4);
+    reduce_scale_f32_kernel<<<(unsigned)((items + 255) / 256), 256, 0, s>>>(part, splits, split_stride, rows, k, ldw,
+                                                                           S, W);
+    return after_launch("reduce_scale_f32_kernel");
+}
+
 }  // namespace
 
 // Batches below these sizes leave the fused kernels' row tiles too few to
@@ -410,40 +283,40 @@ lrc_status launch_apply_f64(const double* U, const double* S, const double* Vt, 
 
 lrc_status launch_apply_f32(const float* U, const float* S, const float* Vt, const float* X,
                             float* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s) {
-    using namespace f32k;
     if (b <= kSplitMaxBatchF32 && k <= kSplitMaxRank) return launch_apply_split_f32(U, S, Vt, X, Y, m, n, k, b, s);
-    const char* name = "apply_f32_kernel";
-    if (k > 4096) {
-        set_error("%s: rank %lld above the supported 4096", name, (long long)k);
-        return LRC_ERR_UNSUPPORTED;
-    }
-    const int kp16 = (int)((k + 15) / 16 * 16);
-    const size_t smem = ((size_t)kp16 * BM + BK1 * LDA + BK1 * LDB) * sizeof(float);
-    if (smem > 227 * 1024) {
-        set_error("%s: rank %lld needs %zu bytes of shared memory", name, (long long)k, smem);
-        return LRC_ERR_UNSUPPORTED;
-    }
-    cudaError_t e = cudaFuncSetAttribute(apply_f32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return cuda_fail(e, name);
-    const int64_t ntiles = (b + BM - 1) / BM;
-    const int64_t m_tiles = (m + BN - 1) / BN;
+    // phase 1: partial products of W = X V over n-splits, with V = (V^T)^T read
+    // from the stored V^T rows; phase 2 after the ordered reduction and diag(s)
+    const int64_t kp16 = (k + 15) / 16 * 16;
+    const int64_t ldn = lrc_packed_ld(n), ldk = lrc_packed_ld(k);
     const int sms = sm_count();
-    int per_sm = (int)((228 * 1024) / (smem + 1024));
-    if (per_sm > 8) per_sm = 8;
-    if (per_sm < 1) per_sm = 1;
-    int64_t splits = 1;
-    if (ntiles * 2 < sms) splits = (sms + ntiles - 1) / ntiles;
-    if (splits > m_tiles) splits = m_tiles;
-    if (splits > 65535) splits = 65535;
-    const int64_t tiles_per_split = (m_tiles + splits - 1) / splits;
-    const int64_t m_chunk = tiles_per_split * BN;
-    splits = (m + m_chunk - 1) / m_chunk;
-    const int64_t slots = (int64_t)sms * per_sm;
-    int64_t gx = ntiles < slots ? ntiles : slots;
-    dim3 grid((unsigned)gx, (unsigned)splits);
-    apply_f32_kernel<<<grid, NT, smem, s>>>(U, S, Vt, X, Y, m, n, (int)k, b, lrc_packed_ld(k), lrc_packed_ld(n),
-                                            kp16, ntiles, m_chunk);
-    return after_launch(name);
+    const int ex = gemm_cc_ex(k);
+    const int64_t bn = 128 + 16 * ex;
+    const int64_t tiles1 = ((b + 127) / 128) * ((k + bn - 1) / bn);
+    const int64_t resident = (int64_t)sms * (ex ? 1 : 2);   // CTAs per SM of the two tile widths
+    // at least two waves of CTAs; at most kMaxChunk terms of n per partial sum
+    constexpr int64_t kMaxChunk = 1024;
+    int64_t splits = (2 * resident + tiles1 - 1) / tiles1;
+    const int64_t min_splits = (n + kMaxChunk - 1) / kMaxChunk;
+    if (splits < min_splits) splits = min_splits;
+    const int64_t max_splits = (n + 255) / 256;
+    if (splits > max_splits) splits = max_splits > min_splits ? max_splits : min_splits;
+    if (splits < 1) splits = 1;
+    // the product rounds each split's K range up to its 16-wide slabs
+    const int64_t kchunk = ((n + splits - 1) / splits + 15) / 16 * 16;
+    splits = (n + kchunk - 1) / kchunk;
+    int64_t part_elems, w_elems, t;
+    if (!mul_ok(b, kp16, &w_elems) || !mul_ok(w_elems, splits, &part_elems) || !mul_ok(part_elems + w_elems, 4, &t)) {
+        set_error("apply_f32: workspace size overflow");
+        return LRC_ERR_INVALID_ARG;
+    }
+    void* ws = nullptr;
+    lrc_status st = stream_workspace(s, (size_t)(part_elems + w_elems) * sizeof(float), &ws);
+    if (st != LRC_OK) return st;
+    float* part = static_cast<float*>(ws);
+    float* Wd = part + part_elems;
+    if ((st = gemm_cc_f32(X, ldn, Vt, ldn, true, part, kp16, b, k, n, (int)splits, w_elems, s)) != LRC_OK) return st;
+    if ((st = launch_reduce_scale_f32(part, (int)splits, w_elems, b, k, kp16, S, Wd, s)) != LRC_OK) return st;
+    return gemm_cc_f32(Wd, kp16, U, ldk, true, Y, m, b, m, k, 1, 0, s);
 }
 
 }  // namespace lrc

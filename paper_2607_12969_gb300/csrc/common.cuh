@@ -82,6 +82,19 @@ lrc_status launch_apply_split_f32(const float* U, const float* S, const float* V
 lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y,
                             int64_t m, int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s);
 
+// Register-tiled binary32 products on the CUDA cores (gemm_cc.cu):
+// C[M x N] = A[M x K] B with B stored K x N (b_trans = false) or N x K
+// (b_trans = true), all row-major; `splits` > 1 splits K and writes split z's
+// partial product at C + z * c_split.  gemm_cc_ex(N): the tile width the
+// launcher uses for N columns is 128 + 16 * gemm_cc_ex(N).  The kernels wait
+// for the previous kernel of the stream (programmatic dependent launch).
+int gemm_cc_ex(int64_t N);
+lrc_status gemm_cc_f32(const float* A, int64_t lda, const float* B, int64_t ldb, bool b_trans, float* C,
+                       int64_t ldc, int64_t M, int64_t N, int64_t K, int splits, int64_t c_split, cudaStream_t s);
+// binary16 operands (widened exactly), binary32 products and output; B stored K x N
+lrc_status gemm_cc_f16in(const void* A, int64_t lda, const void* B, int64_t ldb, float* C, int64_t ldc, int64_t M,
+                         int64_t N, int64_t K, cudaStream_t s);
+
 struct TTShape {
     int d;
     int64_t dims[16];
@@ -90,6 +103,10 @@ struct TTShape {
     int64_t numel;
 };
 lrc_status launch_tt_cc(const TTShape& sh, lrc_fmt fmt, void* out, cudaStream_t s);
+// binary32 TT as a chain of products meeting at one bond (tt_chain.cu)
+lrc_status launch_tt_chain_f32(const TTShape& sh, float* out, cudaStream_t s);
+// multiply count (x2) of that chain at its cheapest bond
+double tt_chain_flops(const TTShape& sh);
 lrc_status launch_tt_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s);
 
 // Device error words of the tensor-core kernels (bounded waits that gave up);

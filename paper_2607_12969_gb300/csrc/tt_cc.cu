@@ -1,4 +1,4 @@
-// tt_cc.cu -- dense TT reconstruction on the CUDA cores, binary64 and binary32
+// tt_cc.cu -- dense TT reconstruction on the CUDA cores, binary64 and binary16 cores
 // (Sec. 5.1: T(i_1..i_d) = G_1(i_1)...G_d(i_d); Sec. 7.5,
 // Eq. gpu_tt_reconstruction: B_l = Z_{l-1} K_l, Z_l = reshape(B_l)).
 //
@@ -12,9 +12,10 @@
 // the tile.  The final product uses a TM x TN register tile per thread and
 // writes contiguous output rows.
 //
-// Element types: binary64 cores with binary64 arithmetic, binary32 with
-// binary32, and binary16 cores with binary32 arithmetic and a binary32 or
-// binary16 output (the latter rounded once per entry).
+// Element types: binary64 cores with binary64 arithmetic, and binary16 cores
+// with binary32 arithmetic and a binary32 or binary16 output (the latter
+// rounded once per entry) for the shapes the tensor-core kernels do not take.
+// binary32 cores take the product chain of tt_chain.cu.
 #include <cuda_fp16.h>
 
 #include "common.cuh"
@@ -203,8 +204,6 @@ lrc_status launch_tt_cc(const TTShape& sh, lrc_fmt fmt, void* out, cudaStream_t 
     switch (fmt) {
         case LRC_F64:
             return launch_tt_cc_t<double, double, double>(sh, static_cast<double*>(out), s, "tt_cc_kernel<f64>");
-        case LRC_F32:
-            return launch_tt_cc_t<float, float, float>(sh, static_cast<float*>(out), s, "tt_cc_kernel<f32>");
         case LRC_F16:
             return launch_tt_cc_t<float, __half, float>(sh, static_cast<float*>(out), s, "tt_cc_kernel<f16,o32>");
         default:

@@ -104,3 +104,20 @@ def test_identity_queries_reconstruct_dense_f64(lrc, cuda):
     got = run_apply(lrc, cuda, f.U, f.s, f.Vt, np.eye(200), "f64")
     want = (f.Vt.T * f.s) @ f.U.T
     assert np.max(np.abs(got - want)) <= 1e-14 * np.max(np.abs(want))
+
+
+@pytest.mark.parametrize("fmt", ["f32", "f64"])
+@pytest.mark.parametrize("m,n,k,b", [
+    (257, 1100, 136, 300),     # several n-splits, one 160-wide rank tile
+    (130, 3000, 161, 517),     # rank above 160: two rank tiles, ragged everything
+    (40, 24, 5, 2100),         # n shorter than one slab
+])
+def test_large_batch_integer_exact(lrc, cuda, fmt, m, n, k, b):
+    # batches above the small-batch split path: every product and partial sum
+    # of the register-tiled products is an exact integer below 2^24
+    U = W.integer_valued((m, k), 11, -2, 2)
+    s = W.integer_valued((k,), 12, 1, 2)
+    Vt = W.integer_valued((k, n), 13, -2, 2)
+    X = W.integer_valued((b, n), 14, -2, 2)
+    got = run_apply(lrc, cuda, U, s, Vt, X, fmt)
+    assert np.array_equal(got, oracle.apply(U, s, Vt, X)), fmt
