@@ -60,13 +60,6 @@ __device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
     return reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
 }
 
-// Byte offset of W[r][col] (r < 128) in the canonical no-swizzle K-major
-// operand image: 8-row x 16-byte core matrices, K-direction stride 2048 B,
-// row-group stride 128 B.
-__host__ __device__ __forceinline__ uint32_t w_image_off(uint32_t r, uint32_t col) {
-    return (col >> 3) * 2048u + (r >> 3) * 128u + (r & 7u) * 16u + (col & 7u) * 2u;
-}
-
 // ================================================================ phase 1
 struct W1Args {
     int64_t b;
@@ -437,8 +430,14 @@ struct YArgs {
     uint32_t u_bytes, slot_bytes, tile_bytes;
     uint32_t w_off, ystage_off, bar_off, tmem_cols;
     int out16, tma_store;
+    int ydepth;               // staging buffers per epilogue warp (2 or 4): TMA stores in flight
     const unsigned char* W;
     void* Y;
+    // optional power-of-two scales of the operands, in groups of 32 rows of W
+    // and 32 rows of U: entry (i, j) of the product is multiplied by
+    // 2^-(esc_w[i / 32] + esc_u[j / 32]) (exact in binary32)
+    const int* esc_w;
+    const int* esc_u;
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -569,13 +568,23 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
         const int r = g * 32 + lane;
         const uint32_t lane_base = (uint32_t)(g * 32) << 16;
         const int ecols = a.out16 ? 64 : 32;       // columns per 128-byte staging row
-        unsigned char* wstage = smem + a.ystage_off + (size_t)g * (2 * 32 * 128);
+        unsigned char* wstage = smem + a.ystage_off + (size_t)g * (a.ydepth * 32 * 128);
         int chunk = 0, tl = 0;
         for (int64_t t = tbeg; t < tend; ++t, ++tl) {
             const int64_t bt = t / a.mtiles;
             const int mt = (int)(t - bt * a.mtiles);
             const int64_t row0 = bt * BM;
             const int ab = tl & 1;
+            const bool scaled = a.esc_w != nullptr;
+            // this warp's 32 rows are one scale group of W; lane j holds the
+            // scale of the tile's j-th group of 32 columns (read before the
+            // accumulator wait, so the loads overlap it)
+            int ew = 0, eu_lane = 0;
+            if (scaled) {
+                ew = row0 + g * 32 < a.b ? a.esc_w[(row0 >> 5) + g] : 0;
+                const int64_t cl = (int64_t)mt * a.n2 + lane * 32;
+                eu_lane = (lane < (a.n2 >> 5) && cl < a.m) ? a.esc_u[cl >> 5] : 0;
+            }
             if (!group_wait(&acc_full[ab], (tl >> 1) & 1, abort, err, 4u, 1, 128)) break;
             tc_fence_after();
             for (int cc = 0; cc < a.n2; cc += ecols, ++chunk) {
@@ -585,6 +594,20 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
                 if (a.out16) tmem_ld32(tcol + 32, *reinterpret_cast<uint32_t(*)[32]>(&v[32]));
                 tmem_ld_wait();
                 const int64_t col0 = (int64_t)mt * a.n2 + cc;
+                if (scaled) {
+                    // columns [col0, col0 + 32) and, for binary16 output, [col0 + 32, col0 + 64)
+                    // are one scale group of U each
+                    const int eu0 = __shfl_sync(0xffffffffu, eu_lane, cc >> 5);
+                    const float f0 = __int_as_float((127 - ew - eu0) << 23);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(__fmul_rn(__uint_as_float(v[j]), f0));
+                    if (a.out16) {
+                        const int eu1 = __shfl_sync(0xffffffffu, eu_lane, (cc >> 5) + 1);
+                        const float f1 = __int_as_float((127 - ew - eu1) << 23);
+#pragma unroll
+                        for (int j = 32; j < 64; ++j) v[j] = __float_as_uint(__fmul_rn(__uint_as_float(v[j]), f1));
+                    }
+                }
                 if (a.tma_store) {
                     uint32_t packed[32];
                     if (a.out16) {
@@ -596,9 +619,12 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
                         for (int j = 0; j < 32; ++j) packed[j] = v[j];
                     }
                     // this warp's 32 rows: own staging pair, own TMA store
-                    unsigned char* sb = wstage + (size_t)(chunk & 1) * (32 * 128);
-                    if (chunk >= 2) {
-                        if (lane == 0) bulk_wait_read<1>();
+                    unsigned char* sb = wstage + (size_t)(chunk & (a.ydepth - 1)) * (32 * 128);
+                    if (chunk >= a.ydepth) {
+                        if (lane == 0) {
+                            if (a.ydepth == 4) bulk_wait_read<3>();
+                            else bulk_wait_read<1>();
+                        }
                         __syncwarp();
                     }
 #pragma unroll
@@ -695,6 +721,87 @@ constexpr size_t kSmemMax = 227 * 1024;
 
 size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
+// Phase-2 plan for a b x m product with kp columns of W per plane: tile
+// width n2, ring depth, shared-memory offsets.  `balance` picks the width
+// that gives the CTAs the most even share (largest tiles per CTA x width);
+// otherwise 256-wide tiles whenever there are at least two per SM.
+lrc_status plan_y(YArgs& a3, size_t& smem3, int64_t m, int64_t b, int kp, int planes, bool out16, bool balance) {
+    const int sms = sm_count();
+    const int64_t btiles = (b + BM - 1) / BM;
+    a3.m = m;
+    a3.b = b;
+    a3.kp = kp;
+    a3.kc2 = (kp + BK - 1) / BK;
+    a3.planes = planes;
+    a3.out16 = out16 ? 1 : 0;
+    const int e_out = out16 ? 2 : 4;
+    a3.tma_store = ((m * e_out) % 16 == 0) ? 1 : 0;
+    const uint32_t tile_bytes = (uint32_t)BM * (uint32_t)kp * 2u;
+    int order[2] = {256, 128};
+    if (balance) {
+        const int64_t w256 = (btiles * ((m + 255) / 256) + sms - 1) / sms * 256;
+        const int64_t w128 = (btiles * ((m + 127) / 128) + sms - 1) / sms * 128;
+        if (w128 < w256) {
+            order[0] = 128;
+            order[1] = 256;
+        }
+    }
+    smem3 = 0;
+    for (int n2 : order) {
+        if (!balance && n2 == 256 && btiles * ((m + 255) / 256) < 2 * (int64_t)sms) continue;   // too few tiles
+        // deeper output staging first (more TMA stores in flight), then the ring
+        for (int depth = 4; depth >= 2 && !smem3; depth -= 2) {
+            for (int stages = 4; stages >= 2 && !smem3; --stages) {
+                if (n2 == 256 && stages < 3) break;      // prefer a deeper ring with narrower tiles
+                const uint32_t u_bytes = (uint32_t)n2 * 128;
+                size_t off = (size_t)stages * u_bytes;
+                const size_t w_off = off;
+                off += (size_t)planes * tile_bytes;
+                off = round_up(off, 1024);
+                const size_t ystage_off = off;
+                off += (size_t)4 * depth * 32 * 128;
+                const size_t bar_off = off;
+                off += (size_t)(2 * stages + 7) * 8 + 16;
+                if (off + 1024 > kSmemMax) continue;
+                a3.n2 = n2;
+                a3.stages = stages;
+                a3.ydepth = depth;
+                a3.u_bytes = u_bytes;
+                a3.slot_bytes = u_bytes;
+                a3.w_off = (uint32_t)w_off;
+                a3.ystage_off = (uint32_t)ystage_off;
+                a3.bar_off = (uint32_t)bar_off;
+                smem3 = off + 1024;
+            }
+        }
+        if (smem3) break;
+    }
+    if (!smem3) {
+        set_error("binary16 product: %d columns of W do not fit in shared memory", kp);
+        return LRC_ERR_UNSUPPORTED;
+    }
+    a3.mtiles = (int)((m + a3.n2 - 1) / a3.n2);
+    a3.T = btiles * a3.mtiles;
+    a3.tmem_cols = pow2_cols(2u * (uint32_t)a3.n2);
+    return LRC_OK;
+}
+
+lrc_status make_y_map(CUtensorMap* ty, const YArgs& a3, void* Y, int64_t m, int64_t b, bool out16) {
+    if (!a3.tma_store) return LRC_OK;   // unused by the kernel
+    const int e_out = out16 ? 2 : 4;
+    return make_map(ty, out16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, Y, m, b, m * e_out,
+                    out16 ? 64 : 32, 32, "Y");
+}
+
+lrc_status launch_y(const CUtensorMap& tu, const CUtensorMap& ty, const YArgs& a3, size_t smem3, int64_t P3,
+                    cudaStream_t s) {
+    cudaError_t e = cudaFuncSetAttribute(apply_y_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem3);
+    if (e != cudaSuccess) return cuda_fail(e, "apply_y_kernel smem attribute");
+    e = launch_pdl(apply_y_kernel, dim3((unsigned)P3), dim3(kThreads), smem3, s, tu, a3.tma_store ? ty : tu, a3);
+    if (e != cudaSuccess) return cuda_fail(e, "apply_y_kernel launch");
+    return after_launch("apply_y_kernel");
+}
+
 }  // namespace
 
 lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y, int64_t m,
@@ -751,49 +858,10 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
 
     // ---- phase-2 plan: tile width, ring depth
     YArgs a3{};
-    a3.m = m;
-    a3.b = b;
-    a3.kp = kp;
-    a3.kc2 = (kp + BK - 1) / BK;
-    a3.planes = planes;
-    a3.tile_bytes = tile_bytes;
-    a3.out16 = out16 ? 1 : 0;
-    const int e_out = out16 ? 2 : 4;
-    a3.tma_store = ((m * e_out) % 16 == 0) ? 1 : 0;
-    a3.Y = Y;
     size_t smem3 = 0;
-    for (int n2 : {256, 128}) {
-        if (n2 == 256 && btiles * ((m + 255) / 256) < 2 * (int64_t)sms) continue;   // too few tiles
-        for (int stages = 4; stages >= 2 && !smem3; --stages) {
-            if (n2 == 256 && stages < 3) break;      // prefer a deeper ring with narrower tiles
-            const uint32_t u_bytes = (uint32_t)n2 * 128;
-            size_t off = (size_t)stages * u_bytes;
-            const size_t w_off = off;
-            off += (size_t)planes * tile_bytes;
-            off = round_up(off, 1024);
-            const size_t ystage_off = off;
-            off += 4 * 2 * 32 * 128;
-            const size_t bar_off = off;
-            off += (size_t)(2 * stages + 7) * 8 + 16;
-            if (off + 1024 > kSmemMax) continue;
-            a3.n2 = n2;
-            a3.stages = stages;
-            a3.u_bytes = u_bytes;
-            a3.slot_bytes = u_bytes;
-            a3.w_off = (uint32_t)w_off;
-            a3.ystage_off = (uint32_t)ystage_off;
-            a3.bar_off = (uint32_t)bar_off;
-            smem3 = off + 1024;
-        }
-        if (smem3) break;
-    }
-    if (!smem3) {
-        set_error("binary16 apply: rank %lld does not fit in shared memory", (long long)k);
-        return LRC_ERR_UNSUPPORTED;
-    }
-    a3.mtiles = (int)((m + a3.n2 - 1) / a3.n2);
-    a3.T = btiles * a3.mtiles;
-    a3.tmem_cols = pow2_cols(2u * (uint32_t)a3.n2);
+    if ((st = plan_y(a3, smem3, m, b, kp, planes, out16, false)) != LRC_OK) return st;
+    a3.tile_bytes = tile_bytes;
+    a3.Y = Y;
     const int64_t P3 = a3.T < sms ? a3.T : sms;
 
     // ---- workspace: W images, then the phase-1 partials
@@ -818,13 +886,7 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
         return st;
     if ((st = make_map(&tu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, U, k, m, ldk * 2, BK, (uint32_t)a3.n2, "U")) != LRC_OK)
         return st;
-    if (a3.tma_store) {
-        if ((st = make_map(&ty, out16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, Y, m, b,
-                           m * e_out, out16 ? 64 : 32, 32, "Y")) != LRC_OK)
-            return st;
-    } else {
-        ty = tu;   // unused by the kernel
-    }
+    if ((st = make_y_map(&ty, a3, Y, m, b, out16)) != LRC_OK) return st;
 
     cudaError_t e = cudaFuncSetAttribute(apply_w1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
     if (e != cudaSuccess) return cuda_fail(e, "apply_w1_kernel smem attribute");
@@ -858,11 +920,36 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
         if ((st = after_launch("apply_w2_kernel")) != LRC_OK) return st;
     }
 
-    e = cudaFuncSetAttribute(apply_y_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem3);
-    if (e != cudaSuccess) return cuda_fail(e, "apply_y_kernel smem attribute");
-    e = launch_pdl(apply_y_kernel, dim3((unsigned)P3), dim3(kThreads), smem3, s, tu, ty, a3);
-    if (e != cudaSuccess) return cuda_fail(e, "apply_y_kernel launch");
-    return after_launch("apply_y_kernel");
+    return launch_y(tu, ty, a3, smem3, P3, s);
+}
+
+lrc_status y_product_plan(int64_t m, int64_t b, int kp, bool out16, int* n2) {
+    YArgs a{};
+    size_t smem = 0;
+    lrc_status st = plan_y(a, smem, m, b, kp, 1, out16, false);
+    if (st == LRC_OK) *n2 = a.n2;
+    return st;
+}
+
+lrc_status launch_y_product(const unsigned char* Wimg, int kp, const void* U, int64_t ldu, int64_t m, int64_t b,
+                            bool out16, void* Y, const int* esc_w, const int* esc_u, cudaStream_t s) {
+    lrc_status st = get_encoder();
+    if (st != LRC_OK) return st;
+    YArgs a3{};
+    size_t smem3 = 0;
+    if ((st = plan_y(a3, smem3, m, b, kp, 1, out16, false)) != LRC_OK) return st;
+    a3.tile_bytes = (uint32_t)BM * (uint32_t)kp * 2u;
+    a3.W = Wimg;
+    a3.Y = Y;
+    a3.esc_w = esc_w;
+    a3.esc_u = esc_u;
+    CUtensorMap tu, ty;
+    if ((st = make_map(&tu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, U, kp, m, ldu * 2, BK, (uint32_t)a3.n2, "U")) != LRC_OK)
+        return st;
+    if ((st = make_y_map(&ty, a3, Y, m, b, out16)) != LRC_OK) return st;
+    const int sms = sm_count();
+    const int64_t P3 = a3.T < sms ? a3.T : sms;
+    return launch_y(tu, ty, a3, smem3, P3, s);
 }
 
 namespace {

@@ -91,9 +91,17 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
 int gemm_cc_ex(int64_t N);
 lrc_status gemm_cc_f32(const float* A, int64_t lda, const float* B, int64_t ldb, bool b_trans, float* C,
                        int64_t ldc, int64_t M, int64_t N, int64_t K, int splits, int64_t c_split, cudaStream_t s);
-// binary16 operands (widened exactly), binary32 products and output; B stored K x N
-lrc_status gemm_cc_f16in(const void* A, int64_t lda, const void* B, int64_t ldb, float* C, int64_t ldc, int64_t M,
-                         int64_t N, int64_t K, cudaStream_t s);
+
+// The second product of the binary16 apply for other callers (apply_tc.cu):
+// Y[b x m] = W U^T on the tensor cores, binary32 accumulation, binary32 or
+// binary16 output.  W is given as 128-row tile images (canonical K-major
+// layout, tc::w_image_off, 128 x kp binary16 each), U as m rows of kp
+// binary16 with row pitch ldu elements.  esc_w / esc_u (nullable together)
+// scale entry (i, j) by 2^-(esc_w[i / 32] + esc_u[j / 32]), each in
+// [-60, 60]; y_product_plan checks that the product fits the kernel.
+lrc_status y_product_plan(int64_t m, int64_t b, int kp, bool out16, int* n2);
+lrc_status launch_y_product(const unsigned char* Wimg, int kp, const void* U, int64_t ldu, int64_t m, int64_t b,
+                            bool out16, void* Y, const int* esc_w, const int* esc_u, cudaStream_t s);
 
 struct TTShape {
     int d;
@@ -108,6 +116,11 @@ lrc_status launch_tt_chain_f32(const TTShape& sh, float* out, cudaStream_t s);
 // multiply count (x2) of that chain at its cheapest bond
 double tt_chain_flops(const TTShape& sh);
 lrc_status launch_tt_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s);
+// binary16 TT as a product chain with the output product on the tensor cores
+// (tt_split.cu); *handled = false when the shape is outside it (nothing launched)
+lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled);
+// bond at which the product chain of tt_chain.cu meets
+int tt_chain_bond(const TTShape& sh);
 
 // Device error words of the tensor-core kernels (bounded waits that gave up);
 // read and cleared by lrc_device_status().  0xffffffff = could not be read.

@@ -12,13 +12,10 @@
 // and its stores are 256-byte row segments.
 // K advances in slabs of 16: the next slab is fetched into registers while
 // the current one is multiplied (two shared-memory buffers, one barrier per
-// slab).  binary16 operands are widened to binary32 when staged; products
-// and sums are binary32 FMAs (no TF32: Sec. 3.4).
+// slab).  Products and sums are binary32 FMAs (no TF32: Sec. 3.4).
 //
 // A split over K (blockIdx.y) writes one partial product per split at
 // C + split * c_split; the caller adds them in a fixed order.
-#include <cuda_fp16.h>
-
 #include "common.cuh"
 #include "tc.cuh"
 
@@ -29,14 +26,7 @@ constexpr int BM = 128, BK = 16, NT = 256;
 constexpr int LDA = BM + 4;          // A slab pitch in floats (rows stay 16-byte aligned)
 
 __device__ __forceinline__ float4 ld4(const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); }
-__device__ __forceinline__ float4 ld4(const __half* p) {
-    const uint2 u = __ldg(reinterpret_cast<const uint2*>(p));
-    const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&u.x));
-    const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&u.y));
-    return make_float4(a.x, a.y, b.x, b.y);
-}
 __device__ __forceinline__ float ld1(const float* p) { return __ldg(p); }
-__device__ __forceinline__ float ld1(const __half* p) { return __half2float(__ldg(p)); }
 
 // Four consecutive elements (r, c..c+3) of a row-major [R x C] array; zero
 // outside.  `vec`: rows are aligned for a vector load.
@@ -55,10 +45,10 @@ __device__ __forceinline__ void st4(float* p, const float* v) {
     __stcs(reinterpret_cast<float4*>(p), make_float4(v[0], v[1], v[2], v[3]));
 }
 
-template <typename TIn, typename TOut>
+template <typename TA, typename TB, typename TOut>
 struct GemmArgs {
-    const TIn* A;
-    const TIn* B;
+    const TA* A;
+    const TB* B;
     TOut* C;
     int64_t lda, ldb, ldc;
     int64_t M, N, K;
@@ -193,9 +183,9 @@ __device__ __forceinline__ void rank1_update(const float* __restrict__ Ab, const
 
 // Two CTAs per SM for 128-wide tiles (128 registers a thread); the 144-wide
 // tile needs more and runs one CTA per SM.
-template <typename TIn, typename TOut, bool BT, int EX>
+template <typename TA, typename TB, typename TOut, bool BT, int EX>
 __global__ void __launch_bounds__(NT, EX == 0 ? 2 : 1)
-gemm_cc_kernel(const GemmArgs<TIn, TOut> a) {
+gemm_cc_kernel(const GemmArgs<TA, TB, TOut> a) {
     constexpr int BN = 128 + 16 * EX;
     constexpr int LDB = BN + 4;
     __shared__ __align__(16) float As[2][BK * LDA];
@@ -210,9 +200,9 @@ gemm_cc_kernel(const GemmArgs<TIn, TOut> a) {
     const int64_t kend = (kbeg + a.kchunk < a.K) ? kbeg + a.kchunk : a.K;
     TOut* C = a.C + (int64_t)blockIdx.y * a.c_split;
 
-    RowSlab<TIn, BM> sa;
-    ColSlab<TIn, BN> sbn;    // NN: 16 x BN slabs of the K x N array
-    RowSlab<TIn, BN> sbt;    // NT: BN rows of the N x K array
+    RowSlab<TA, BM> sa;
+    ColSlab<TB, BN> sbn;     // NN: 16 x BN slabs of the K x N array
+    RowSlab<TB, BN> sbt;     // NT: BN rows of the N x K array
     tc::pdl_wait();          // operands written by the previous kernel of the stream
     sa.init(a.A, a.lda, a.M, m0, kbeg);
     if (BT) sbt.init(a.B, a.ldb, a.N, n0, kbeg);
@@ -297,11 +287,11 @@ bool vec_ok(const T* p, int64_t ld) {
     return (reinterpret_cast<uintptr_t>(p) % quad) == 0 && (ld % 4) == 0;
 }
 
-template <typename TIn, typename TOut, bool BT, int EX>
-lrc_status launch_t(const TIn* A, int64_t lda, const TIn* B, int64_t ldb, TOut* C, int64_t ldc, int64_t M,
+template <typename TA, typename TB, typename TOut, bool BT, int EX>
+lrc_status launch_t(const TA* A, int64_t lda, const TB* B, int64_t ldb, TOut* C, int64_t ldc, int64_t M,
                     int64_t N, int64_t K, int splits, int64_t c_split, cudaStream_t s, const char* name) {
     constexpr int BN = 128 + 16 * EX;
-    GemmArgs<TIn, TOut> a{};
+    GemmArgs<TA, TB, TOut> a{};
     a.A = A;
     a.B = B;
     a.C = C;
@@ -325,7 +315,7 @@ lrc_status launch_t(const TIn* A, int64_t lda, const TIn* B, int64_t ldb, TOut* 
         return LRC_ERR_UNSUPPORTED;
     }
     if (tiles == 0) return LRC_OK;
-    cudaError_t e = launch_pdl(gemm_cc_kernel<TIn, TOut, BT, EX>, dim3((unsigned)tiles, (unsigned)splits), dim3(NT), 0,
+    cudaError_t e = launch_pdl(gemm_cc_kernel<TA, TB, TOut, BT, EX>, dim3((unsigned)tiles, (unsigned)splits), dim3(NT), 0,
                                s, a);
     if (e != cudaSuccess) return cuda_fail(e, name);
     return after_launch(name);
@@ -345,22 +335,16 @@ lrc_status gemm_cc_f32(const float* A, int64_t lda, const float* B, int64_t ldb,
     const int ex = gemm_cc_ex(N);
     if (b_trans) {
         if (ex)
-            return launch_t<float, float, true, 1>(A, lda, B, ldb, C, ldc, M, N, K, splits, c_split, s,
-                                                   "gemm_cc_kernel<f32,NT,144>");
-        return launch_t<float, float, true, 0>(A, lda, B, ldb, C, ldc, M, N, K, splits, c_split, s,
-                                               "gemm_cc_kernel<f32,NT,128>");
+            return launch_t<float, float, float, true, 1>(A, lda, B, ldb, C, ldc, M, N, K, splits, c_split, s,
+                                                          "gemm_cc_kernel<f32,NT,144>");
+        return launch_t<float, float, float, true, 0>(A, lda, B, ldb, C, ldc, M, N, K, splits, c_split, s,
+                                                      "gemm_cc_kernel<f32,NT,128>");
     }
     if (ex)
-        return launch_t<float, float, false, 1>(A, lda, B, ldb, C, ldc, M, N, K, splits, c_split, s,
-                                                "gemm_cc_kernel<f32,NN,144>");
-    return launch_t<float, float, false, 0>(A, lda, B, ldb, C, ldc, M, N, K, splits, c_split, s,
-                                            "gemm_cc_kernel<f32,NN,128>");
-}
-
-lrc_status gemm_cc_f16in(const void* A, int64_t lda, const void* B, int64_t ldb, float* C, int64_t ldc, int64_t M,
-                         int64_t N, int64_t K, cudaStream_t s) {
-    return launch_t<__half, float, false, 0>(static_cast<const __half*>(A), lda, static_cast<const __half*>(B), ldb,
-                                             C, ldc, M, N, K, 1, 0, s, "gemm_cc_kernel<f16,NN,128>");
+        return launch_t<float, float, float, false, 1>(A, lda, B, ldb, C, ldc, M, N, K, splits, c_split, s,
+                                                       "gemm_cc_kernel<f32,NN,144>");
+    return launch_t<float, float, float, false, 0>(A, lda, B, ldb, C, ldc, M, N, K, splits, c_split, s,
+                                                   "gemm_cc_kernel<f32,NN,128>");
 }
 
 }  // namespace lrc

@@ -19,6 +19,13 @@ namespace tc {
 
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s: far above any single launch
 
+// Byte offset of W[r][col] (r < 128) in the canonical no-swizzle K-major
+// operand image of a 128-row tile: 8-row x 16-byte core matrices, K-direction
+// stride 2048 B, row-group stride 128 B.
+__host__ __device__ __forceinline__ uint32_t w_image_off(uint32_t r, uint32_t col) {
+    return (col >> 3) * 2048u + (r >> 3) * 128u + (r & 7u) * 16u + (col & 7u) * 2u;
+}
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

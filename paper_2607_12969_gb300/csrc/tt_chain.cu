@@ -59,6 +59,8 @@ size_t round256(size_t bytes) { return (bytes + 255) / 256 * 256; }
 
 double tt_chain_flops(const TTShape& sh) { return plan_chain(sh).flops; }
 
+int tt_chain_bond(const TTShape& sh) { return plan_chain(sh).c; }
+
 lrc_status launch_tt_chain_f32(const TTShape& sh, float* out, cudaStream_t s) {
     const int d = sh.d;
     const int c = plan_chain(sh).c;

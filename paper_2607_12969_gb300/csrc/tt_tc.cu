@@ -474,6 +474,8 @@ lrc_status launch_tt_f16(const TTShape& sh, bool out16, void* out, cudaStream_t 
     bool handled = false;
     lrc_status st = launch_tt3_f16_tc(sh, out16, out, s, &handled);
     if (handled) return st;
+    st = launch_tt_split_f16(sh, out16, out, s, &handled);
+    if (handled) return st;
     st = launch_ttn_f16_tc(sh, out16, out, s, &handled);
     if (handled) return st;
     if (tt_f16_tc_supported(sh, out16)) return launch_tt_f16_tc(sh, out16, out, s);
