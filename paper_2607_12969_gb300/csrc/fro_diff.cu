@@ -95,9 +95,62 @@ __device__ __forceinline__ void block_sum2(double& a, double& b, double* sh) {
     }
 }
 
+// ---------------------------------------------------------------------------
+// Squares summed in binary32 pairs.  The GB300 issues about two binary64
+// instructions per clock per SM, while streaming two binary64 arrays at HBM
+// speed delivers about 1.35 element pairs per clock per SM: with a binary64
+// subtraction and a binary64 FMA per element the reduction is bound by the
+// FP64 pipe, not by memory.  For two binary64 arrays only the subtraction
+// d = a - b stays binary64.  d is cut, with integer operations on its bits,
+// into hi (its sign, exponent and leading 24 significand bits) and lo (the
+// next 23 bits; the last 6 are dropped, a relative change of at most 2^-47),
+// and d^2 = hi^2 + (2 hi lo + lo^2) is formed with an exact two-product
+// (hi^2 = p + e, e = fma(hi, hi, -p)) and added to a binary32 pair sum with
+// two-sum.  Every 16 groups the pair sum is added to a binary64 accumulator.
+// Elements with |d| outside [2^-60, 2^60) (where hi^2 or a sum of them could
+// leave the binary32 range) are squared in binary64 instead.
+// ---------------------------------------------------------------------------
+struct Pair {
+    float hi = 0.0f, lo = 0.0f;
+};
+
+// hi, lo of d; false when d is out of the binary32 path's range (d = 0 is in range)
+__device__ __forceinline__ bool split_hi_lo(double d, float& hi, float& lo) {
+    const unsigned long long b = (unsigned long long)__double_as_longlong(d);
+    const int e = (int)((b >> 52) & 0x7ffu);
+    if (e < 1023 - 60 || e >= 1023 + 60) {
+        hi = lo = 0.0f;
+        return (b << 1) == 0ull;
+    }
+    const unsigned int sign = (unsigned int)(b >> 32) & 0x80000000u;
+    hi = __int_as_float((int)(sign | ((unsigned int)(e - 1023 + 127) << 23) | (unsigned int)((b >> 29) & 0x7fffffu)));
+    // bits 28..6 of the significand, as an exact binary32 integer, times +-2^(E - 46)
+    const unsigned int m = (unsigned int)((b >> 6) & 0x7fffffu);
+    const float mf = __int_as_float((int)(0x4B000000u | m)) - 8388608.0f;
+    const float scale = __int_as_float((int)(sign | ((unsigned int)(e - 1023 - 46 + 127) << 23)));
+    lo = mf * scale;
+    return true;
+}
+
+// s += hi^2 + 2 hi lo + lo^2
+__device__ __forceinline__ void add_square(Pair& s, float hi, float lo) {
+    const float p = hi * hi;
+    const float e = fmaf(hi, hi, -p);                 // hi^2 - p, exact
+    const float t = fmaf(2.0f * hi, lo, fmaf(lo, lo, e));
+    const float sh = s.hi + p;                        // two-sum of s.hi and p
+    const float bp = sh - s.hi;
+    const float err = (s.hi - (sh - bp)) + (p - bp);
+    s.hi = sh;
+    s.lo += err + t;
+}
+
+__device__ __forceinline__ void flush(Pair& s, double& acc) {
+    acc += (double)s.hi + (double)s.lo;
+    s.hi = s.lo = 0.0f;
+}
+
 // FB = -1: B absent (treated as zero).  NORM = false skips the ||A||
-// accumulation (the reduction is bound by FP64 issue on this GPU, so the
-// extra FMA per element costs time when nobody reads the norm).
+// accumulation.
 template <int FA, int FB, bool NORM>
 __global__ void __launch_bounds__(kThreads)
 fro_partial_kernel(const void* __restrict__ A, const void* __restrict__ B, int64_t count,
@@ -106,15 +159,44 @@ fro_partial_kernel(const void* __restrict__ A, const void* __restrict__ B, int64
     double sd = 0.0, sa = 0.0;
     const int64_t groups = count / kGroup;
     const int64_t stride = (int64_t)gridDim.x * kThreads;
-    for (int64_t g = (int64_t)blockIdx.x * kThreads + threadIdx.x; g < groups; g += stride) {
-        double a[kGroup], b[kGroup];
-        load8<FA>(A, g, a);
-        if (FB >= 0) load8<FB>(B, g, b);
+    if constexpr (FA == 0 && FB <= 0) {
+        // binary64 inputs: binary32-pair squares (see above)
+        Pair pd, pa;
+        int n = 0;
+        for (int64_t g = (int64_t)blockIdx.x * kThreads + threadIdx.x; g < groups; g += stride) {
+            double a[kGroup], b[kGroup];
+            load8<FA>(A, g, a);
+            if (FB == 0) load8<0>(B, g, b);
 #pragma unroll
-        for (int j = 0; j < kGroup; ++j) {
-            const double d = (FB >= 0) ? a[j] - b[j] : a[j];
-            sd = fma(d, d, sd);
-            if (NORM) sa = fma(a[j], a[j], sa);
+            for (int j = 0; j < kGroup; ++j) {
+                const double d = (FB == 0) ? a[j] - b[j] : a[j];
+                float hi, lo;
+                if (split_hi_lo(d, hi, lo)) add_square(pd, hi, lo);
+                else sd = fma(d, d, sd);
+                if (NORM) {
+                    if (split_hi_lo(a[j], hi, lo)) add_square(pa, hi, lo);
+                    else sa = fma(a[j], a[j], sa);
+                }
+            }
+            if (++n == 16) {
+                flush(pd, sd);
+                if (NORM) flush(pa, sa);
+                n = 0;
+            }
+        }
+        flush(pd, sd);
+        if (NORM) flush(pa, sa);
+    } else {
+        for (int64_t g = (int64_t)blockIdx.x * kThreads + threadIdx.x; g < groups; g += stride) {
+            double a[kGroup], b[kGroup];
+            load8<FA>(A, g, a);
+            if (FB >= 0) load8<FB>(B, g, b);
+#pragma unroll
+            for (int j = 0; j < kGroup; ++j) {
+                const double d = (FB >= 0) ? a[j] - b[j] : a[j];
+                sd = fma(d, d, sd);
+                if (NORM) sa = fma(a[j], a[j], sa);
+            }
         }
     }
     if (blockIdx.x == 0) {  // ragged tail, fixed owner

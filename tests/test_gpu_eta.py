@@ -34,6 +34,23 @@ def test_fro_diff_mixed_formats(lrc, cuda, fa, fb):
     assert abs(d - wd) <= 1e-12 * wd and abs(na - wna) <= 1e-12 * wna
 
 
+@pytest.mark.parametrize("lo,hi", [(-63, 63), (-62, -58), (58, 62), (-1074, -1000)])
+def test_fro_diff_f64_magnitude_ranges(lrc, cuda, lo, hi):
+    """Values and differences whose binary exponents straddle the limits of
+    the binary32-pair squaring (|d| in [2^-60, 2^60)), binary64 subnormals,
+    zeros and both signs: the sum of squares stays within 1e-12 relative."""
+    rng = np.random.default_rng(lo + 2000)
+    count = 400_003
+    e = rng.integers(lo, hi + 1, size=count)
+    a = np.ldexp(rng.uniform(0.5, 1.0, size=count), e) * rng.choice([-1.0, 1.0], size=count)
+    b = a - np.ldexp(rng.uniform(0.5, 1.0, size=count), e - rng.integers(0, 3, size=count))
+    a[::97] = 0.0
+    b[::89] = a[::89]
+    d, na = lrc.lrc_fro_diff(to_dev(a, cuda), "f64", to_dev(b, cuda), "f64", count)
+    wd, wna = oracle.fro_diff(a, b)
+    assert abs(d - wd) <= 1e-12 * wd and abs(na - wna) <= 1e-12 * wna
+
+
 def test_fro_diff_null_b_and_determinism(lrc, cuda):
     a = to_dev(W.gaussian((5_000_001,), 9), cuda)
     r1 = lrc.lrc_fro_diff(a, "f64", None, "f64", a.numel())
