@@ -273,7 +273,7 @@ lrc_status launch_reduce_scale_f32(const float* part, int splits, int64_t split_
 
 // Batches below these sizes leave the fused kernels' row tiles too few to
 // fill the GPU; they take the split path of apply_split.cu (ranks up to 1024).
-constexpr int64_t kSplitMaxBatchF64 = 2048, kSplitMaxBatchF32 = 256, kSplitMaxRank = 1024;
+constexpr int64_t kSplitMaxBatchF64 = 2048, kSplitMaxBatchF32 = 32, kSplitMaxRank = 1024;
 
 lrc_status launch_apply_f64(const double* U, const double* S, const double* Vt, const double* X,
                             double* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s) {

@@ -98,27 +98,78 @@ round_pack_kernel(const double* __restrict__ src, int64_t cols, int64_t ld_src,
     }
 }
 
-// FMT as above; dst is binary64.
+// Exact binary32 -> binary64 from the bit fields: normal numbers and zeros
+// take integer operations only (the exponent rebias and significand shift of
+// the IEEE 754 formats); subnormals, infinities and NaNs take the conversion
+// instruction.
+__device__ __forceinline__ double widen_f32(float f) {
+    const uint32_t u = __float_as_uint(f);
+    const uint32_t e = (u >> 23) & 0xffu;
+    const unsigned long long sign = (unsigned long long)(u & 0x80000000u) << 32;
+    if (e != 0u && e != 0xffu)
+        return __longlong_as_double((long long)(sign | ((unsigned long long)(e + 896u) << 52) |
+                                                ((unsigned long long)(u & 0x7fffffu) << 29)));
+    if ((u & 0x7fffffffu) == 0u) return __longlong_as_double((long long)sign);
+    return (double)f;
+}
+
+// FMT as above; dst is binary64.  Each thread widens a group of 8 elements of
+// one row: one 16-byte (binary16) or two (binary32) loads, four 16-byte stores
+// when the row pitches allow it.
 template <int FMT>
 __global__ void __launch_bounds__(kThreads)
 widen_kernel(const void* __restrict__ src, int64_t cols, int64_t ld_src, double* __restrict__ dst,
-             int64_t ld_dst, int64_t groups_per_row, int64_t total_groups) {
+             int64_t ld_dst, int64_t groups_per_row, int64_t total_groups, bool vec_src, bool vec_dst) {
     const int64_t stride = (int64_t)gridDim.x * kThreads;
     for (int64_t g = (int64_t)blockIdx.x * kThreads + threadIdx.x; g < total_groups; g += stride) {
         const int64_t r = g / groups_per_row;
         const int64_t c0 = (g - r * groups_per_row) * kGroup;
-        double* drow = dst + r * ld_dst;
+        double v[kGroup];
+        if (vec_src && c0 + kGroup <= cols) {
+            if (FMT == 2) {
+                const uint4 q = __ldcs(reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(src) + r * ld_src + c0));
+                const uint32_t w[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
-        for (int j = 0; j < kGroup; ++j) {
-            const int64_t c = c0 + j;
-            if (c >= ld_dst) break;
-            double v = 0.0;
-            if (c < cols) {
-                if (FMT == 2) v = widen_f16(static_cast<const uint16_t*>(src)[r * ld_src + c]);
-                else if (FMT == 1) v = (double)static_cast<const float*>(src)[r * ld_src + c];
-                else v = static_cast<const double*>(src)[r * ld_src + c];
+                for (int j = 0; j < 4; ++j) {
+                    const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w[j]));
+                    v[2 * j] = widen_f32(f.x);
+                    v[2 * j + 1] = widen_f32(f.y);
+                }
+            } else if (FMT == 1) {
+                const float4* p = reinterpret_cast<const float4*>(static_cast<const float*>(src) + r * ld_src + c0);
+                const float4 a = __ldcs(p), b = __ldcs(p + 1);
+                v[0] = widen_f32(a.x); v[1] = widen_f32(a.y); v[2] = widen_f32(a.z); v[3] = widen_f32(a.w);
+                v[4] = widen_f32(b.x); v[5] = widen_f32(b.y); v[6] = widen_f32(b.z); v[7] = widen_f32(b.w);
+            } else {
+                const double2* p = reinterpret_cast<const double2*>(static_cast<const double*>(src) + r * ld_src + c0);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const double2 t = __ldcs(p + j);
+                    v[2 * j] = t.x;
+                    v[2 * j + 1] = t.y;
+                }
             }
-            drow[c] = v;
+        } else {
+#pragma unroll
+            for (int j = 0; j < kGroup; ++j) {
+                const int64_t c = c0 + j;
+                double x = 0.0;
+                if (c < cols) {
+                    if (FMT == 2) x = widen_f16(static_cast<const uint16_t*>(src)[r * ld_src + c]);
+                    else if (FMT == 1) x = (double)static_cast<const float*>(src)[r * ld_src + c];
+                    else x = static_cast<const double*>(src)[r * ld_src + c];
+                }
+                v[j] = x;
+            }
+        }
+        double* drow = dst + r * ld_dst;
+        if (vec_dst && c0 + kGroup <= ld_dst) {
+#pragma unroll
+            for (int j = 0; j < kGroup; j += 2)
+                __stcs(reinterpret_cast<double2*>(drow + c0 + j), make_double2(v[j], v[j + 1]));
+        } else {
+            for (int j = 0; j < kGroup; ++j)
+                if (c0 + j < ld_dst) drow[c0 + j] = v[j];
         }
     }
 }
@@ -159,15 +210,19 @@ lrc_status launch_widen(const void* src, lrc_fmt fmt, int64_t rows, int64_t cols
     const int64_t gpr = (ld_dst + kGroup - 1) / kGroup;
     const int64_t total = rows * gpr;
     const int grid = grid_for(total);
+    const int64_t e = storage_bytes(fmt);
+    // 16-byte vectors: row starts (base and pitch) on 16-byte boundaries
+    const bool vec_src = (reinterpret_cast<uintptr_t>(src) % 16 == 0) && ((ld_src * e) % 16 == 0);
+    const bool vec_dst = (reinterpret_cast<uintptr_t>(dst) % 16 == 0) && (ld_dst % 2 == 0);
     switch (fmt) {
         case LRC_F64:
-            widen_kernel<0><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total);
+            widen_kernel<0><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total, vec_src, vec_dst);
             break;
         case LRC_F32:
-            widen_kernel<1><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total);
+            widen_kernel<1><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total, vec_src, vec_dst);
             break;
         default:
-            widen_kernel<2><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total);
+            widen_kernel<2><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total, vec_src, vec_dst);
             break;
     }
     return after_launch("widen_kernel");

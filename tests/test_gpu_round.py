@@ -80,3 +80,31 @@ def test_large_factor_set_bit_exact(lrc, cuda):
             torch.cuda.synchronize()
             got = bits(p, fmt)[:, :a.shape[1]]
             assert np.array_equal(got, oracle.round_bits(a, fmt))
+
+
+@pytest.mark.parametrize("fmt", ["f32", "f16"])
+def test_widen_special_values_exact(lrc, cuda, fmt):
+    """Widening is exact for every class of value: signed zeros, subnormals,
+    the largest finite values, infinities, NaN, and random normal numbers."""
+    dt = np.float32 if fmt == "f32" else np.float16
+    fi = np.finfo(dt)
+    rng = np.random.default_rng(11)
+    specials = np.array([0.0, -0.0, fi.tiny, -fi.tiny, fi.smallest_subnormal, -fi.smallest_subnormal,
+                         float(fi.max), -float(fi.max), np.inf, -np.inf, np.nan, 1.0, -2.5], dtype=np.float64)
+    normals = rng.standard_normal(300) * np.exp2(rng.integers(-10, 10, 300))
+    subnormals = rng.uniform(-1, 1, 200) * float(fi.tiny)
+    vals = np.concatenate([specials, normals, subnormals]).astype(dt)
+    rows, cols = 8, 73                       # 513 values + padding, ragged rows
+    src = np.zeros(rows * cols, dtype=dt)
+    src[:vals.size] = vals
+    src = src.reshape(rows, cols)
+    ld = lrc.lrc_packed_ld(cols)
+    p = torch.zeros((rows, ld), dtype=lrc.storage_dtype(fmt), device=cuda)
+    p[:, :cols] = torch.from_numpy(src).to(cuda)
+    w = lrc.widen_matrix(p, fmt, cols)
+    torch.cuda.synchronize()
+    got = w.cpu().numpy()[:, :cols]
+    want = src.astype(np.float64)
+    nan = np.isnan(want)
+    assert np.array_equal(np.isnan(got), nan)
+    assert np.array_equal(got[~nan].view(np.uint64), want[~nan].view(np.uint64))
