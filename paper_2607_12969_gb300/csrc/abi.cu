@@ -152,6 +152,8 @@ lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X
     if (!aligned16(X)) return misaligned("X");
     if (!aligned16(Y)) return misaligned("Y");
     cudaStream_t s = as_stream(stream);
+    if (b <= apply_skinny_max_batch(fmt) && k <= 1024)
+        return launch_apply_skinny(U, S, Vt, X, Y, m, n, k, b, fmt, s);
     switch (fmt) {
         case LRC_F64:
             return launch_apply_f64((const double*)U, (const double*)S, (const double*)Vt,

@@ -81,6 +81,11 @@ lrc_status launch_apply_split_f32(const float* U, const float* S, const float* V
                                   int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
 lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y,
                             int64_t m, int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s);
+// batches of at most apply_skinny_max_batch(fmt) queries, ranks up to 1024,
+// every format (apply_skinny.cu)
+int64_t apply_skinny_max_batch(lrc_fmt fmt);
+lrc_status launch_apply_skinny(const void* U, const void* S, const void* Vt, const void* X, void* Y, int64_t m,
+                               int64_t n, int64_t k, int64_t b, lrc_fmt fmt, cudaStream_t s);
 
 // Register-tiled binary32 products on the CUDA cores (gemm_cc.cu):
 // C[M x N] = A[M x K] B with B stored K x N (b_trans = false) or N x K

@@ -121,3 +121,21 @@ def test_large_batch_integer_exact(lrc, cuda, fmt, m, n, k, b):
     X = W.integer_valued((b, n), 14, -2, 2)
     got = run_apply(lrc, cuda, U, s, Vt, X, fmt)
     assert np.array_equal(got, oracle.apply(U, s, Vt, X)), fmt
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("m,n,k,b", [
+    (333, 1031, 37, 5),        # ragged n (not a whole number of 16-byte vectors), b between the kernel's widths
+    (64, 7, 3, 16),            # n shorter than one vector row, largest batch of the small-batch kernels
+    (1000, 5000, 272, 16),     # several n-chunks with a ragged last chunk
+    (4097, 2049, 1024, 2),     # largest rank of the small-batch kernels
+    (517, 3001, 100, 4),       # largest batch of the small-batch kernels for FP64 and FP16
+    (257, 129, 19, 1),         # single query, ragged everything
+])
+def test_small_batch_kernels_vs_oracle(lrc, cuda, fmt, m, n, k, b):
+    f = W.random_factors(m, n, k, seed=m + 3 * n + k)
+    X = W.gaussian((b, n), b + 11)
+    got = run_apply(lrc, cuda, f.U, f.s, f.Vt, X, fmt)
+    want = oracle.apply(*oracle_inputs(f.U, f.s, f.Vt, X, fmt))
+    err = rel_fro(got, want)
+    assert err <= TOL[fmt], (fmt, err)
