@@ -181,6 +181,7 @@ lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims, const i
     cudaStream_t s = as_stream(stream);
     if (fmt == LRC_F16 || fmt == LRC_F16_O16) return launch_tt_f16(sh, fmt == LRC_F16_O16, out, s);
     if (fmt == LRC_F32) return launch_tt_chain_f32(sh, static_cast<float*>(out), s);
+    if (tt_chain_saves(sh)) return launch_tt_chain_f64(sh, static_cast<double*>(out), s);
     return launch_tt_cc(sh, fmt, out, s);
 }
 

@@ -94,6 +94,9 @@ lrc_status launch_apply_skinny(const void* U, const void* S, const void* Vt, con
 // launcher uses for N columns is 128 + 16 * gemm_cc_ex(N).  The kernels wait
 // for the previous kernel of the stream (programmatic dependent launch).
 int gemm_cc_ex(int64_t N);
+// binary64 C[M x N] = A[M x K] B[K x N], all row-major (DFMA-bound tiles)
+lrc_status gemm_cc_f64(const double* A, int64_t lda, const double* B, int64_t ldb, double* C, int64_t ldc,
+                       int64_t M, int64_t N, int64_t K, cudaStream_t s);
 lrc_status gemm_cc_f32(const float* A, int64_t lda, const float* B, int64_t ldb, bool b_trans, float* C,
                        int64_t ldc, int64_t M, int64_t N, int64_t K, int splits, int64_t c_split, cudaStream_t s);
 
@@ -116,8 +119,12 @@ struct TTShape {
     int64_t numel;
 };
 lrc_status launch_tt_cc(const TTShape& sh, lrc_fmt fmt, void* out, cudaStream_t s);
-// binary32 TT as a chain of products meeting at one bond (tt_chain.cu)
+// binary32 / binary64 TT as a chain of products meeting at one bond
+// (tt_chain.cu); binary64 takes it where it saves at least a fifth of the
+// left-to-right chain's multiplies (tt_chain_saves)
 lrc_status launch_tt_chain_f32(const TTShape& sh, float* out, cudaStream_t s);
+lrc_status launch_tt_chain_f64(const TTShape& sh, double* out, cudaStream_t s);
+bool tt_chain_saves(const TTShape& sh);
 // multiply count (x2) of that chain at its cheapest bond
 double tt_chain_flops(const TTShape& sh);
 lrc_status launch_tt_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s);

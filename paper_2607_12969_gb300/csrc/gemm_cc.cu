@@ -321,6 +321,88 @@ lrc_status launch_t(const TA* A, int64_t lda, const TB* B, int64_t ldb, TOut* C,
     return after_launch(name);
 }
 
+// ---------------------------------------------------------------------------
+// binary64: C = A B (both row-major, B stored K x N), bound by the DFMA rate
+// (about 2 per clock per SM on this GPU), so a plain tile is enough: 64 x 64
+// tiles, 256 threads, each thread 4 rows x 4 columns strided by 16 (a warp's
+// shared reads are two broadcast rows of A and 16 consecutive doubles of B),
+// K in 16-wide slabs through two shared-memory buffers with the next slab
+// prefetched in registers.
+// ---------------------------------------------------------------------------
+constexpr int BM64 = 64, BN64 = 64, BK64 = 16;
+
+__global__ void __launch_bounds__(NT)
+gemm_f64_kernel(const double* __restrict__ A, int64_t lda, const double* __restrict__ B, int64_t ldb,
+                double* __restrict__ C, int64_t ldc, int64_t M, int64_t N, int64_t K, int64_t ntn) {
+    __shared__ double As[2][BK64][BM64 + 1];
+    __shared__ double Bs[2][BK64][BN64 + 1];
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+    const int64_t mt = blockIdx.x / ntn, nt = blockIdx.x - mt * ntn;
+    const int64_t m0 = mt * BM64, n0 = nt * BN64;
+    tc::pdl_wait();
+    double ra[4], rb[4];
+    // A slab: element e = tid + 256 q -> row e / 16, k e % 16; B slab: row e / 64, column e % 64
+#define LRC_F64_LOAD(k0)                                                                   \
+    _Pragma("unroll") for (int q = 0; q < 4; ++q) {                                         \
+        const int e = tid + NT * q;                                                        \
+        const int64_t ar = m0 + (e >> 4), ak = (k0) + (e & 15);                            \
+        ra[q] = (ar < M && ak < K) ? __ldg(A + ar * lda + ak) : 0.0;                       \
+        const int64_t bk = (k0) + (e >> 6), bc = n0 + (e & 63);                            \
+        rb[q] = (bk < K && bc < N) ? __ldg(B + bk * ldb + bc) : 0.0;                       \
+    }
+#define LRC_F64_STORE(buf)                                                                 \
+    _Pragma("unroll") for (int q = 0; q < 4; ++q) {                                         \
+        const int e = tid + NT * q;                                                        \
+        As[buf][e & 15][e >> 4] = ra[q];                                                   \
+        Bs[buf][e >> 6][e & 63] = rb[q];                                                   \
+    }
+    double acc[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0.0;
+    const int64_t nslabs = (K + BK64 - 1) / BK64;
+    if (nslabs > 0) {
+        LRC_F64_LOAD(0)
+        LRC_F64_STORE(0)
+        __syncthreads();
+    }
+    for (int64_t s = 0; s < nslabs; ++s) {
+        const int buf = (int)(s & 1);
+        const bool more = s + 1 < nslabs;
+        if (more) { LRC_F64_LOAD((s + 1) * BK64) }
+        // the last slab multiplies only its real columns
+        const int kn = (K - s * BK64) < BK64 ? (int)(K - s * BK64) : BK64;
+#pragma unroll 4
+        for (int kk = 0; kk < kn; ++kk) {
+            double a[4], b[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) a[i] = As[buf][kk][ty + 16 * i];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) b[j] = Bs[buf][kk][tx + 16 * j];
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fma(a[i], b[j], acc[i][j]);
+        }
+        if (more) { LRC_F64_STORE(buf ^ 1) }
+        __syncthreads();
+    }
+#undef LRC_F64_LOAD
+#undef LRC_F64_STORE
+    tc::pdl_trigger();
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int64_t r = m0 + ty + 16 * i;
+        if (r >= M) continue;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int64_t c = n0 + tx + 16 * j;
+            if (c < N) C[r * ldc + c] = acc[i][j];
+        }
+    }
+}
+
 }  // namespace
 
 // Extra 16-column groups per tile for N columns: 128 + 16 ex wide tiles,
@@ -345,6 +427,21 @@ lrc_status gemm_cc_f32(const float* A, int64_t lda, const float* B, int64_t ldb,
                                                        "gemm_cc_kernel<f32,NN,144>");
     return launch_t<float, float, float, false, 0>(A, lda, B, ldb, C, ldc, M, N, K, splits, c_split, s,
                                                    "gemm_cc_kernel<f32,NN,128>");
+}
+
+lrc_status gemm_cc_f64(const double* A, int64_t lda, const double* B, int64_t ldb, double* C, int64_t ldc,
+                       int64_t M, int64_t N, int64_t K, cudaStream_t s) {
+    const int64_t ntn = (N + BN64 - 1) / BN64;
+    const int64_t tiles = ((M + BM64 - 1) / BM64) * ntn;
+    if (tiles > 0x7fffffff) {
+        set_error("gemm_f64_kernel: product too large (%lld tiles)", (long long)tiles);
+        return LRC_ERR_UNSUPPORTED;
+    }
+    if (tiles == 0) return LRC_OK;
+    cudaError_t e = launch_pdl(gemm_f64_kernel, dim3((unsigned)tiles), dim3(NT), 0, s, A, lda, B, ldb, C, ldc, M, N,
+                               K, ntn);
+    if (e != cudaSuccess) return cuda_fail(e, "gemm_f64_kernel launch");
+    return after_launch("gemm_f64_kernel");
 }
 
 }  // namespace lrc

@@ -12,9 +12,9 @@
 // tensor with ranks (1,16,26,26,26,16,1) the chain meets at the middle bond:
 // 0.88 GFLOP, against 1.50 GFLOP for the left-to-right chain.
 //
-// Every product runs on the register-tiled binary32 kernel of gemm_cc.cu;
-// intermediates live in the stream's workspace (two buffers per side,
-// alternating).
+// Every product runs on the product kernels of gemm_cc.cu (register-tiled
+// binary32, DFMA-bound binary64); intermediates live in the stream's
+// workspace (two buffers per side, alternating).
 #include <math.h>
 
 #include "common.cuh"
@@ -61,10 +61,22 @@ double tt_chain_flops(const TTShape& sh) { return plan_chain(sh).flops; }
 
 int tt_chain_bond(const TTShape& sh) { return plan_chain(sh).c; }
 
-lrc_status launch_tt_chain_f32(const TTShape& sh, float* out, cudaStream_t s) {
+namespace {
+
+lrc_status product(const float* A, int64_t lda, const float* B, int64_t ldb, float* C, int64_t ldc, int64_t M,
+                   int64_t N, int64_t K, cudaStream_t s) {
+    return gemm_cc_f32(A, lda, B, ldb, false, C, ldc, M, N, K, 1, 0, s);
+}
+lrc_status product(const double* A, int64_t lda, const double* B, int64_t ldb, double* C, int64_t ldc, int64_t M,
+                   int64_t N, int64_t K, cudaStream_t s) {
+    return gemm_cc_f64(A, lda, B, ldb, C, ldc, M, N, K, s);
+}
+
+template <typename T>
+lrc_status launch_chain(const TTShape& sh, T* out, cudaStream_t s) {
     const int d = sh.d;
     const int c = plan_chain(sh).c;
-    const float* const* G = reinterpret_cast<const float* const*>(sh.cores);
+    const T* const* G = reinterpret_cast<const T* const*>(sh.cores);
     // P[j]: rows of Z(j); Q[j]: columns of S(j) (0-based core index j)
     int64_t P[17] = {0}, Q[17] = {0};
     P[1] = sh.dims[0];
@@ -73,11 +85,11 @@ lrc_status launch_tt_chain_f32(const TTShape& sh, float* out, cudaStream_t s) {
     for (int j = d - 2; j >= c; --j) Q[j] = sh.dims[j] * Q[j + 1];
     size_t lsz[2] = {0, 0}, rsz[2] = {0, 0};
     for (int j = 2; j <= c; ++j) {
-        const size_t b = round256((size_t)P[j] * (size_t)sh.ranks[j] * sizeof(float));
+        const size_t b = round256((size_t)P[j] * (size_t)sh.ranks[j] * sizeof(T));
         if (b > lsz[j & 1]) lsz[j & 1] = b;
     }
     for (int j = c; j <= d - 2; ++j) {
-        const size_t b = round256((size_t)sh.ranks[j] * (size_t)Q[j] * sizeof(float));
+        const size_t b = round256((size_t)sh.ranks[j] * (size_t)Q[j] * sizeof(T));
         if (b > rsz[j & 1]) rsz[j & 1] = b;
     }
     unsigned char* ws = nullptr;
@@ -88,27 +100,35 @@ lrc_status launch_tt_chain_f32(const TTShape& sh, float* out, cudaStream_t s) {
         if (st != LRC_OK) return st;
         ws = static_cast<unsigned char*>(p);
     }
-    float* L[2] = {reinterpret_cast<float*>(ws), reinterpret_cast<float*>(ws + lsz[0])};
-    float* R[2] = {reinterpret_cast<float*>(ws + lsz[0] + lsz[1]),
-                   reinterpret_cast<float*>(ws + lsz[0] + lsz[1] + rsz[0])};
+    T* L[2] = {reinterpret_cast<T*>(ws), reinterpret_cast<T*>(ws + lsz[0])};
+    T* R[2] = {reinterpret_cast<T*>(ws + lsz[0] + lsz[1]), reinterpret_cast<T*>(ws + lsz[0] + lsz[1] + rsz[0])};
     lrc_status st = LRC_OK;
-    const float* Z = G[0];   // Z(1) = G_1: n_1 x r_1
+    const T* Z = G[0];   // Z(1) = G_1: n_1 x r_1
     for (int j = 1; j <= c - 1; ++j) {
         const int64_t w = sh.dims[j] * sh.ranks[j + 1];
-        float* dst = L[(j + 1) & 1];
-        if ((st = gemm_cc_f32(Z, sh.ranks[j], G[j], w, false, dst, w, P[j], w, sh.ranks[j], 1, 0, s)) != LRC_OK)
-            return st;
+        T* dst = L[(j + 1) & 1];
+        if ((st = product(Z, sh.ranks[j], G[j], w, dst, w, P[j], w, sh.ranks[j], s)) != LRC_OK) return st;
         Z = dst;
     }
-    const float* S = G[d - 1];   // S(d) = G_d: r_{d-1} x n_d
+    const T* S = G[d - 1];   // S(d) = G_d: r_{d-1} x n_d
     for (int j = d - 2; j >= c; --j) {
-        float* dst = R[j & 1];
-        if ((st = gemm_cc_f32(G[j], sh.ranks[j + 1], S, Q[j + 1], false, dst, Q[j + 1], sh.ranks[j] * sh.dims[j],
-                              Q[j + 1], sh.ranks[j + 1], 1, 0, s)) != LRC_OK)
+        T* dst = R[j & 1];
+        if ((st = product(G[j], sh.ranks[j + 1], S, Q[j + 1], dst, Q[j + 1], sh.ranks[j] * sh.dims[j], Q[j + 1],
+                          sh.ranks[j + 1], s)) != LRC_OK)
             return st;
         S = dst;
     }
-    return gemm_cc_f32(Z, sh.ranks[c], S, Q[c], false, out, Q[c], P[c], Q[c], sh.ranks[c], 1, 0, s);
+    return product(Z, sh.ranks[c], S, Q[c], out, Q[c], P[c], Q[c], sh.ranks[c], s);
 }
+
+}  // namespace
+
+lrc_status launch_tt_chain_f32(const TTShape& sh, float* out, cudaStream_t s) { return launch_chain<float>(sh, out, s); }
+
+lrc_status launch_tt_chain_f64(const TTShape& sh, double* out, cudaStream_t s) {
+    return launch_chain<double>(sh, out, s);
+}
+
+bool tt_chain_saves(const TTShape& sh) { return plan_chain(sh).flops <= 0.8 * chain_flops(sh, sh.d - 1); }
 
 }  // namespace lrc
