@@ -131,6 +131,10 @@ lrc_status launch_tt_f16(const TTShape& sh, bool out16, void* out, cudaStream_t 
 // binary16 TT as a product chain with the output product on the tensor cores
 // (tt_split.cu); *handled = false when the shape is outside it (nothing launched)
 lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled);
+// binary32 TT whose chain has several small products at its ends: one side
+// launch forms Z and S, one product forms the tensor (tt_split.cu);
+// *handled = false when the shape is outside it
+lrc_status launch_tt_side_f32(const TTShape& sh, float* out, cudaStream_t s, bool* handled);
 // bond at which the product chain of tt_chain.cu meets
 int tt_chain_bond(const TTShape& sh);
 

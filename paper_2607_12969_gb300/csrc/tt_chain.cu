@@ -123,7 +123,12 @@ lrc_status launch_chain(const TTShape& sh, T* out, cudaStream_t s) {
 
 }  // namespace
 
-lrc_status launch_tt_chain_f32(const TTShape& sh, float* out, cudaStream_t s) { return launch_chain<float>(sh, out, s); }
+lrc_status launch_tt_chain_f32(const TTShape& sh, float* out, cudaStream_t s) {
+    bool handled = false;
+    const lrc_status st = launch_tt_side_f32(sh, out, s, &handled);
+    if (handled) return st;
+    return launch_chain<float>(sh, out, s);
+}
 
 lrc_status launch_tt_chain_f64(const TTShape& sh, double* out, cudaStream_t s) {
     return launch_chain<double>(sh, out, s);

@@ -82,22 +82,25 @@ struct SideArgs {
     int ranks[17];
     int64_t D[16];            // D[l] = n_{l+1} ... n_{c-1}: prefix p passes through row p / D[l] of Z_{l+1}
     int64_t Qs[17];           // Qs[l] = n_l ... n_{d-1}: suffix counts of the right side
-    const __half* cores[16];
+    const void* cores[16];    // binary16 (image mode) or binary32 cores
     Parts pw, pu;
     int scale_w, scale_u;
     unsigned char* Wimg;      // ceil(P / 128) images of 128 x kp
     __half* Uimg;             // Q rows of kp
+    float* Zout;              // binary32 mode: Z (P x r) and S (r x Q), row-major
+    float* Sout;
     int* esc_w;               // [ceil(P / kUnit)]
     int* esc_u;               // [ceil(Q / kUnit)]
 };
 
 __device__ __forceinline__ float core_at(const __half* g, int64_t i) { return __half2float(__ldg(g + i)); }
+__device__ __forceinline__ float core_at(const float* g, int64_t i) { return __ldg(g + i); }
 
 // Copies count core elements to shared memory, dst[didx(e)] = G[sidx(e)],
 // eight loads in flight per thread before their stores (a loop that stores to
 // shared memory between global loads would wait out each load in turn).
-template <typename SI, typename DI>
-__device__ __forceinline__ void copy_core(const __half* __restrict__ g, int64_t count, SI sidx, DI didx, float* dst) {
+template <typename TC, typename SI, typename DI>
+__device__ __forceinline__ void copy_core(const TC* __restrict__ g, int64_t count, SI sidx, DI didx, float* dst) {
     for (int64_t e0 = 0; e0 < count; e0 += 8 * (int64_t)blockDim.x) {
         float v[8];
 #pragma unroll
@@ -116,11 +119,13 @@ __device__ __forceinline__ void copy_core(const __half* __restrict__ g, int64_t 
 // Core l widened to binary32 in shared memory (every interior core of a
 // shape this path takes fits; gs is 16-byte aligned); the barriers retire
 // the previous level and publish the core.
+template <typename TC>
 __device__ __forceinline__ const float* stage_core(const SideArgs& a, int l, float* gs) {
+    constexpr int EV = 16 / (int)sizeof(TC);
     const int64_t n = (int64_t)a.ranks[l] * a.dims[l] * a.ranks[l + 1];
-    const __half* g = a.cores[l];
+    const TC* g = static_cast<const TC*>(a.cores[l]);
     __syncthreads();
-    const int64_t nv = ((reinterpret_cast<uintptr_t>(g) & 15u) == 0) ? n / 8 : 0;   // 16-byte vectors
+    const int64_t nv = ((reinterpret_cast<uintptr_t>(g) & 15u) == 0) ? n / EV : 0;   // 16-byte vectors
     for (int64_t v0 = 0; v0 < nv; v0 += 4 * (int64_t)blockDim.x) {
         uint4 w[4];
 #pragma unroll
@@ -132,15 +137,19 @@ __device__ __forceinline__ const float* stage_core(const SideArgs& a, int l, flo
         for (int u = 0; u < 4; ++u) {
             const int64_t i = v0 + u * (int64_t)blockDim.x + threadIdx.x;
             if (i < nv) {
-                const __half2* h = reinterpret_cast<const __half2*>(&w[u]);
-                const float2 f0 = __half22float2(h[0]), f1 = __half22float2(h[1]);
-                const float2 f2 = __half22float2(h[2]), f3 = __half22float2(h[3]);
-                reinterpret_cast<float4*>(gs + i * 8)[0] = make_float4(f0.x, f0.y, f1.x, f1.y);
-                reinterpret_cast<float4*>(gs + i * 8)[1] = make_float4(f2.x, f2.y, f3.x, f3.y);
+                if constexpr (sizeof(TC) == 2) {
+                    const __half2* h = reinterpret_cast<const __half2*>(&w[u]);
+                    const float2 f0 = __half22float2(h[0]), f1 = __half22float2(h[1]);
+                    const float2 f2 = __half22float2(h[2]), f3 = __half22float2(h[3]);
+                    reinterpret_cast<float4*>(gs + i * 8)[0] = make_float4(f0.x, f0.y, f1.x, f1.y);
+                    reinterpret_cast<float4*>(gs + i * 8)[1] = make_float4(f2.x, f2.y, f3.x, f3.y);
+                } else {
+                    reinterpret_cast<uint4*>(gs + i * 4)[0] = w[u];
+                }
             }
         }
     }
-    const int64_t done = nv * 8;
+    const int64_t done = nv * EV;
     copy_core(g, n - done, [=](int64_t e) { return done + e; }, [=](int64_t e) { return done + e; }, gs);
     __syncthreads();
     return gs;
@@ -149,13 +158,14 @@ __device__ __forceinline__ const float* stage_core(const SideArgs& a, int l, flo
 // Rows [p0, pend) of Z = G_1...G_c (binary32, buffer rows of pitch ldb);
 // returns the buffer that holds them.  Level l keeps only the rows of
 // Z_{l+1} the tile's prefixes pass through: a contiguous range.
+template <typename TC>
 __device__ float* left_rows(const SideArgs& a, int64_t p0, int64_t pend, float* buf0, float* buf1, float* gs) {
     float* cur = buf0;
     int64_t lo = p0 / a.D[0];
     {
         const int r1 = a.ranks[1], ldb = a.ldb;
         const int cnt = (int)((pend - 1) / a.D[0] - lo + 1);
-        copy_core(a.cores[0], (int64_t)cnt * r1, [=](int64_t e) { return lo * r1 + e; },
+        copy_core(static_cast<const TC*>(a.cores[0]), (int64_t)cnt * r1, [=](int64_t e) { return lo * r1 + e; },
                   [=](int64_t e) { return (e / r1) * ldb + e % r1; }, cur);
     }
     __syncthreads();
@@ -165,7 +175,7 @@ __device__ float* left_rows(const SideArgs& a, int64_t p0, int64_t pend, float* 
         const int64_t nlo = p0 / a.D[l];
         const int cnt = (int)((pend - 1) / a.D[l] - nlo + 1);
         float* nxt = (cur == buf0) ? buf1 : buf0;
-        const float* G = stage_core(a, l, gs);
+        const float* G = stage_core<TC>(a, l, gs);
         for (int e = threadIdx.x; e < cnt * r1; e += blockDim.x) {
             const int q = e / r1, b = e - q * r1;
             const int64_t gq = nlo + q, parent = gq / nl;
@@ -190,6 +200,7 @@ __device__ float* left_rows(const SideArgs& a, int64_t p0, int64_t pend, float* 
 // whose suffix count Qs[l] is at most kUnit computes every suffix (row =
 // suffix); otherwise it computes the suffixes t mod Qs[l] of the unit's
 // columns (row = t - q0).
+template <typename TC>
 __device__ float* right_cols(const SideArgs& a, int64_t q0, int64_t qend, float* buf0, float* buf1, float* gs,
                             bool* direct) {
     float* cur = buf0;
@@ -200,7 +211,7 @@ __device__ float* right_cols(const SideArgs& a, int64_t q0, int64_t qend, float*
         const bool all = a.Qs[last] <= kUnit;
         const int cnt = all ? (int)nl : (int)(qend - q0);
         const int ldb = a.ldb;
-        copy_core(a.cores[last], (int64_t)cnt * rl,
+        copy_core(static_cast<const TC*>(a.cores[last]), (int64_t)cnt * rl,
                   [=](int64_t e) {
                       const int64_t k = e / cnt, col = e - k * cnt;
                       return k * nl + (all ? col : (q0 + col) % nl);
@@ -214,7 +225,7 @@ __device__ float* right_cols(const SideArgs& a, int64_t q0, int64_t qend, float*
         const bool all = a.Qs[l] <= kUnit, all_next = qn <= kUnit;
         const int cnt = all ? (int)a.Qs[l] : (int)(qend - q0);
         float* nxt = (cur == buf0) ? buf1 : buf0;
-        const float* G = stage_core(a, l, gs);
+        const float* G = stage_core<TC>(a, l, gs);
         // columns fastest across threads: a warp reads one core row (broadcast)
         // and rows of the column buffer an odd pitch apart (no bank conflicts)
         for (int e = threadIdx.x; e < cnt * r0; e += blockDim.x) {
@@ -235,8 +246,10 @@ __device__ float* right_cols(const SideArgs& a, int64_t q0, int64_t qend, float*
 }
 
 // One CTA per kUnit rows of Z (blockIdx < wunits) or kUnit columns of S:
-// forms them, scales them by one power of two (computed operands), and
-// writes their binary16 parts into the operand images.
+// forms them and, in image mode (IMG), scales them by one power of two
+// (computed operands) and writes their binary16 parts into the operand
+// images; otherwise writes them as binary32 Z and S.
+template <typename TC, bool IMG>
 __global__ void __launch_bounds__(256)
 tt_side_kernel(const SideArgs a) {
     extern __shared__ float sbuf[];
@@ -251,7 +264,13 @@ tt_side_kernel(const SideArgs a) {
         const int64_t t = blockIdx.x;
         const int64_t p0 = t * kUnit, pend = (p0 + kUnit < a.P) ? p0 + kUnit : a.P;
         const int nrow = (int)(pend - p0);
-        const float* z = left_rows(a, p0, pend, buf0, buf1, gs);
+        const float* z = left_rows<TC>(a, p0, pend, buf0, buf1, gs);
+        if constexpr (!IMG) {
+            tc::pdl_trigger();
+            for (int e = threadIdx.x; e < nrow * a.r; e += blockDim.x)
+                a.Zout[p0 * a.r + e] = z[(e / a.r) * a.ldb + e % a.r];
+            return;
+        }
         float mx = 0.0f;
         for (int e = threadIdx.x; e < nrow * a.r; e += blockDim.x)
             mx = fmaxf(mx, fabsf(z[(e / a.r) * a.ldb + e % a.r]));
@@ -281,8 +300,17 @@ tt_side_kernel(const SideArgs a) {
         const int64_t q0 = t * kUnit, qend = (q0 + kUnit < a.Q) ? q0 + kUnit : a.Q;
         const int nq = (int)(qend - q0);
         bool direct = false;
-        const float* sc = right_cols(a, q0, qend, buf0, buf1, gs, &direct);
+        const float* sc = right_cols<TC>(a, q0, qend, buf0, buf1, gs, &direct);
         const int64_t base = direct ? q0 : 0;      // buffer row of column q0
+        if constexpr (!IMG) {
+            tc::pdl_trigger();
+            // S[k][q0 + q], columns fastest: 128-byte runs per row of S
+            for (int e = threadIdx.x; e < nq * a.r; e += blockDim.x) {
+                const int k = e / nq, q = e - k * nq;
+                a.Sout[(int64_t)k * a.Q + q0 + q] = sc[(base + q) * a.ldb + k];
+            }
+            return;
+        }
         float mx = 0.0f;
         for (int e = threadIdx.x; e < nq * a.r; e += blockDim.x)
             mx = fmaxf(mx, fabsf(sc[(base + e / a.r) * a.ldb + e % a.r]));
@@ -311,6 +339,49 @@ tt_side_kernel(const SideArgs a) {
 
 size_t r256(size_t v) { return (v + 255) / 256 * 256; }
 
+// SideArgs fields common to both modes; returns the largest rank.
+int fill_side(const TTShape& sh, int c, SideArgs& a) {
+    const int d = sh.d;
+    a.d = d;
+    a.c = c;
+    a.r = (int)sh.ranks[c];
+    a.rp = (a.r + 15) / 16 * 16;
+    int rmax = 1;
+    for (int l = 0; l < d; ++l) {
+        a.dims[l] = sh.dims[l];
+        a.ranks[l] = (int)sh.ranks[l];
+        a.cores[l] = sh.cores[l];
+        if (sh.ranks[l] > rmax) rmax = (int)sh.ranks[l];
+    }
+    a.ranks[d] = 1;
+    a.P = 1;
+    for (int l = 0; l < c; ++l) a.P *= sh.dims[l];
+    a.Q = 1;
+    for (int l = c; l < d; ++l) a.Q *= sh.dims[l];
+    for (int l = 0; l < c; ++l) {
+        int64_t v = 1;
+        for (int j = l + 1; j < c; ++j) v *= sh.dims[j];
+        a.D[l] = v;
+    }
+    a.Qs[d] = 1;
+    for (int l = d - 1; l >= 0; --l) a.Qs[l] = a.Qs[l + 1] * sh.dims[l];
+    a.ldb = rmax | 1;
+    a.buf_rows = kUnit + 1;
+    a.wunits = (a.P + kUnit - 1) / kUnit;
+    return rmax;
+}
+
+// Shared memory of the side kernel: two level buffers and the largest
+// interior core (staged in binary32).
+size_t side_smem(const TTShape& sh, const SideArgs& a) {
+    int64_t core_max = 0;
+    for (int l = 1; l <= sh.d - 2; ++l) {
+        const int64_t n = sh.ranks[l] * sh.dims[l] * sh.ranks[l + 1];
+        if (n > core_max) core_max = n;
+    }
+    return (((size_t)2 * a.buf_rows * a.ldb + 3) / 4 * 4 + (size_t)core_max) * sizeof(float);
+}
+
 }  // namespace
 
 lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled) {
@@ -337,47 +408,16 @@ lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStr
     }
     const int kp = pw.n * rp;
     SideArgs a{};
-    a.d = d;
-    a.c = c;
-    a.r = r;
-    a.rp = rp;
-    int rmax = 1;
-    for (int l = 0; l < d; ++l) {
-        a.dims[l] = sh.dims[l];
-        a.ranks[l] = (int)sh.ranks[l];
-        a.cores[l] = static_cast<const __half*>(sh.cores[l]);
-        if (sh.ranks[l] > rmax) rmax = (int)sh.ranks[l];
-    }
-    a.ranks[d] = 1;
-    a.P = 1;
-    for (int l = 0; l < c; ++l) a.P *= sh.dims[l];
-    a.Q = 1;
-    for (int l = c; l < d; ++l) a.Q *= sh.dims[l];
-    for (int l = 0; l < c; ++l) {
-        int64_t v = 1;
-        for (int j = l + 1; j < c; ++j) v *= sh.dims[j];
-        a.D[l] = v;
-    }
-    a.Qs[d] = 1;
-    for (int l = d - 1; l >= 0; --l) a.Qs[l] = a.Qs[l + 1] * sh.dims[l];
-    a.ldb = rmax | 1;
+    const int rmax = fill_side(sh, c, a);
     int n2 = 0;
     if (kp > kMaxParts * 64 || rmax > 64 || y_product_plan(a.Q, a.P, kp, out16, &n2) != LRC_OK) return LRC_OK;
-    a.buf_rows = kUnit + 1;
-    // the interior cores the two sides multiply by are staged in shared memory
-    int64_t core_max = 0;
-    for (int l = 1; l <= d - 2; ++l) {
-        const int64_t n = sh.ranks[l] * sh.dims[l] * sh.ranks[l + 1];
-        if (n > core_max) core_max = n;
-    }
-    const size_t smem = (((size_t)2 * a.buf_rows * a.ldb + 3) / 4 * 4 + (size_t)core_max) * sizeof(float);
+    const size_t smem = side_smem(sh, a);
     if (smem > 200 * 1024) return LRC_OK;
     *handled = true;
     a.pw = pw;
     a.pu = pu;
     a.scale_w = z_core ? 0 : 1;
     a.scale_u = s_core ? 0 : 1;
-    a.wunits = (a.P + kUnit - 1) / kUnit;
     const int64_t uunits = (a.Q + kUnit - 1) / kUnit;
     const int64_t btiles = (a.P + BM - 1) / BM;
     const size_t w_bytes = r256((size_t)btiles * BM * kp * 2), u_bytes = r256((size_t)a.Q * kp * 2);
@@ -390,12 +430,44 @@ lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStr
     a.Uimg = reinterpret_cast<__half*>(ws + w_bytes);
     a.esc_w = reinterpret_cast<int*>(ws + w_bytes + u_bytes);
     a.esc_u = a.esc_w + a.wunits;
-    cudaError_t e = cudaFuncSetAttribute(tt_side_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = cudaFuncSetAttribute(tt_side_kernel<__half, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "tt_side_kernel smem attribute");
-    e = launch_pdl(tt_side_kernel, dim3((unsigned)(a.wunits + uunits)), dim3(256), smem, s, a);
+    e = launch_pdl(tt_side_kernel<__half, true>, dim3((unsigned)(a.wunits + uunits)), dim3(256), smem, s, a);
     if (e != cudaSuccess) return cuda_fail(e, "tt_side_kernel launch");
     if ((st = after_launch("tt_side_kernel")) != LRC_OK) return st;
     return launch_y_product(a.Wimg, kp, a.Uimg, kp, a.Q, a.P, out16, out, a.esc_w, a.esc_u, s);
+}
+
+lrc_status launch_tt_side_f32(const TTShape& sh, float* out, cudaStream_t s, bool* handled) {
+    *handled = false;
+    const int d = sh.d;
+    if (d > 16) return LRC_OK;
+    const int c = tt_chain_bond(sh);
+    if ((c - 1) + (d - 1 - c) < 2) return LRC_OK;    // at most one chain product per side: nothing to fuse
+    SideArgs a{};
+    const int rmax = fill_side(sh, c, a);
+    int64_t zq;
+    if (rmax > 64 || !mul_ok(a.P, a.r, &zq) || zq > ((int64_t)1 << 22) || !mul_ok(a.Q, a.r, &zq) ||
+        zq > ((int64_t)1 << 22))
+        return LRC_OK;                                 // sides too large for one pass of per-unit chains
+    const size_t smem = side_smem(sh, a);
+    if (smem > 200 * 1024) return LRC_OK;
+    *handled = true;
+    const int64_t uunits = (a.Q + kUnit - 1) / kUnit;
+    const size_t z_bytes = r256((size_t)a.P * a.r * sizeof(float)), s_bytes = r256((size_t)a.r * a.Q * sizeof(float));
+    void* wsp = nullptr;
+    lrc_status st = stream_workspace(s, z_bytes + s_bytes, &wsp);
+    if (st != LRC_OK) return st;
+    a.Zout = static_cast<float*>(wsp);
+    a.Sout = reinterpret_cast<float*>(static_cast<unsigned char*>(wsp) + z_bytes);
+    cudaError_t e = cudaFuncSetAttribute(tt_side_kernel<float, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "tt_side_kernel smem attribute");
+    e = launch_pdl(tt_side_kernel<float, false>, dim3((unsigned)(a.wunits + uunits)), dim3(256), smem, s, a);
+    if (e != cudaSuccess) return cuda_fail(e, "tt_side_kernel launch");
+    if ((st = after_launch("tt_side_kernel")) != LRC_OK) return st;
+    return gemm_cc_f32(a.Zout, a.r, a.Sout, a.Q, false, out, a.Q, a.P, a.Q, a.r, 1, 0, s);
 }
 
 }  // namespace lrc
