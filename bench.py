@@ -243,7 +243,10 @@ class Step:
         else:
             fn()
 
-    def run(self, record=False):
+    def run(self, record=False, on_outputs=None):
+        """One pass of the path.  on_outputs, if given, is called once the
+        apply and TT outputs are enqueued (the eta and certificate work that
+        follows reads none of them)."""
         self.record = record
         lrc, cfg = self.lrc, self.cfg
         m, n, b = cfg.m, cfg.n, cfg.b
@@ -277,6 +280,8 @@ class Step:
             ranks = tt.ranks[base]
             self.timed(f"tt_{fmt}", work_tt(tt.dims, ranks, fmt), lambda: lrc.tt_reconstruct(
                 cores, tt.dims, ranks, fmt, self.tt_out[fmt]))
+        if on_outputs is not None:
+            on_outputs()
         # a6: eta for the matrix (FP64 dense products of unrounded and widened factors)
         for fmt in ("f32", "f16"):
             F = self.fac[fmt]
@@ -703,6 +708,19 @@ def main():
     outs = {f: torch.empty(F["Y"].shape, dtype=F["Y"].dtype, pin_memory=True) for f, F in step.fac.items()}
     outs_tt = {f: torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for f, t in step.tt_out.items()}
 
+    copy_stream = torch.cuda.Stream()
+
+    def read_back():
+        # the outputs come back on a copy stream while the eta work runs
+        ready = torch.cuda.Event()
+        ready.record()
+        copy_stream.wait_event(ready)
+        with torch.cuda.stream(copy_stream):
+            for f, F in step.fac.items():
+                outs[f].copy_(F["Y"], non_blocking=True)
+            for f, t in step.tt_out.items():
+                outs_tt[f].copy_(t, non_blocking=True)
+
     def e2e_once():
         step.d_Q1.copy_(pinned["Q1"], non_blocking=True)
         step.d_Q2t.copy_(pinned["Q2t"], non_blocking=True)
@@ -711,12 +729,9 @@ def main():
         for f in pinned_tt:
             for d, h in zip(step.tt_dev[f], pinned_tt[f]):
                 d.copy_(h, non_blocking=True)
-        step.run(record=False)
-        for f, F in step.fac.items():
-            outs[f].copy_(F["Y"], non_blocking=True)
-        for f, t in step.tt_out.items():
-            outs_tt[f].copy_(t, non_blocking=True)
+        step.run(record=False, on_outputs=read_back)
         torch.cuda.current_stream().synchronize()
+        copy_stream.synchronize()
 
     e2e_once()
     barrier(world)
