@@ -81,6 +81,13 @@ ALU = {"f64": "f64", "f32": "f32", "f16": "f16", "f16_o16": "f16"}
 # algorithmic work of each call (bytes moved at least once, useful flops)
 # ---------------------------------------------------------------------------
 
+# DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from
+# one ncu capture of the call type's kernel as it stands; an entry is removed
+# when its kernel changes.  apply_f64_dense: profiles/
+# apply_cc_kernel_f64_m16384_n8192_b8192_k144.md.
+MEASURED_TRAFFIC = {"apply_f64_dense": 604_804_096 + 1_014_732_288}
+
+
 def work_round(rows, cols, ld, fmt):
     return {"bytes": rows * cols * 8 + rows * ld * E[fmt], "flops": 0, "alu": None}
 
@@ -776,7 +783,7 @@ def main():
             "config": {"workload": WORKLOAD, "l2": "inputs larger than L2 (no flush needed)",
                        "parallelism": f"replicas x{world} (independent batches, no collective)"},
             "roofline": {"kernel": dname, "bound": dp["bound"], "achieved": ach, "peak": peak, "unit": unit_r,
-                         "frac": ach / peak, "traffic": None,
+                         "frac": ach / peak, "traffic": MEASURED_TRAFFIC.get(dname),
                          "peak_source": ("measured" if dp["bound"] == "hbm" or dp["alu"] == "f16" else "derived")
                          + f" ({PEAKS['source']} file)"},
             "kernels": kernels,
