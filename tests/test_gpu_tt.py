@@ -104,3 +104,23 @@ def test_workloads_sampled_entries(lrc, cuda, fmt, name):
     err = rel_fro(got[idx], want)
     assert err <= TOL[fmt], (name, fmt, err)
     assert np.isfinite(got).all()
+
+
+# Interior cores too large for the small-core product-chain path's shared
+# memory: these shapes take the narrow-mode tensor-core kernel (last two
+# modes 16 x 16) and the d >= 4 wide-mode kernel (last mode 64).
+LARGE_CORES = [
+    ((8, 128, 16, 16), (1, 8, 64, 16, 1)),
+    ((8, 128, 8, 64), (1, 8, 64, 32, 1)),
+]
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("dims,ranks", LARGE_CORES)
+def test_large_interior_cores_vs_oracle(lrc, cuda, fmt, dims, ranks):
+    cores = W.make_tt(dims, ranks, "gauss_geo", 31)
+    got, rc = run_tt(lrc, cuda, cores, fmt)
+    want = oracle.tt_full(rc).reshape(-1)
+    err = rel_fro(got, want)
+    assert err <= TOL[fmt], (fmt, err)
+    assert np.isfinite(got).all()
