@@ -51,6 +51,12 @@ using namespace tc;
 constexpr int BM = 128;
 constexpr int BK = 64;                       // FP16 elements per 128-byte swizzled row
 constexpr int kThreads = 192;
+// the second product: warp 0 producer, warp 1 MMA, warps 2..9 epilogue -- two
+// warps per tensor-memory lane quarter, taking alternate column chunks (the
+// epilogue is bound by the latency of each chunk's load / stage / fence /
+// store sequence, not by bandwidth)
+constexpr int kEpiWarpsY = 8;
+constexpr int kThreadsY = 64 + 32 * kEpiWarpsY;
 constexpr uint32_t kXBytes = BM * BK * 2;    // one X box
 constexpr int kChunkBlocks = 8;              // k-blocks per accumulation chunk (FP32 output)
 constexpr int kPfBlocks = 4;                 // k-blocks per L2 prefetch box (512-byte rows)
@@ -430,7 +436,7 @@ struct YArgs {
     uint32_t u_bytes, slot_bytes, tile_bytes;
     uint32_t w_off, ystage_off, bar_off, tmem_cols;
     int out16, tma_store;
-    int ydepth;               // staging buffers per epilogue warp (2 or 4): TMA stores in flight
+    int ydepth;               // staging buffers per epilogue warp (1 or 2): TMA stores in flight
     const unsigned char* W;
     void* Y;
     // optional power-of-two scales of the operands, in groups of 32 rows of W
@@ -440,7 +446,7 @@ struct YArgs {
     const int* esc_u;
 };
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreadsY, 1)
 apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__ CUtensorMap tm_y, const YArgs a) {
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = align1024(smem_raw);
@@ -467,7 +473,7 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
         mbar_init(w_empty, 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(&acc_full[i], 1);
-            mbar_init(&acc_empty[i], 128);
+            mbar_init(&acc_empty[i], 32 * kEpiWarpsY);
         }
         mbar_init(mma_done, 1);
         *abort = 0;
@@ -568,7 +574,12 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
         const int r = g * 32 + lane;
         const uint32_t lane_base = (uint32_t)(g * 32) << 16;
         const int ecols = a.out16 ? 64 : 32;       // columns per 128-byte staging row
-        unsigned char* wstage = smem + a.ystage_off + (size_t)g * (a.ydepth * 32 * 128);
+        const int half = (warp - 2) >> 2;          // which of the two warps of this lane quarter
+        // the four warps of a half stage one column chunk of all 128 rows (one
+        // 32-row slice each, lane quarter g at g * 4 KB) and one of them stores it
+        // with a single 128-row TMA box
+        const bool issuer = (g == 0) && (lane == 0);
+        unsigned char* hstage = smem + a.ystage_off + (size_t)half * a.ydepth * (128 * 128);
         int chunk = 0, tl = 0;
         for (int64_t t = tbeg; t < tend; ++t, ++tl) {
             const int64_t bt = t / a.mtiles;
@@ -585,9 +596,9 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
                 const int64_t cl = (int64_t)mt * a.n2 + lane * 32;
                 eu_lane = (lane < (a.n2 >> 5) && cl < a.m) ? a.esc_u[cl >> 5] : 0;
             }
-            if (!group_wait(&acc_full[ab], (tl >> 1) & 1, abort, err, 4u, 1, 128)) break;
+            if (!group_wait(&acc_full[ab], (tl >> 1) & 1, abort, err, 4u, 1, 32 * kEpiWarpsY)) break;
             tc_fence_after();
-            for (int cc = 0; cc < a.n2; cc += ecols, ++chunk) {
+            for (int cc = half * ecols; cc < a.n2; cc += 2 * ecols, ++chunk) {
                 uint32_t v[64];
                 const uint32_t tcol = tmem + lane_base + (uint32_t)(ab * a.n2 + cc);
                 tmem_ld32(tcol, *reinterpret_cast<uint32_t(*)[32]>(&v[0]));
@@ -618,15 +629,13 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
 #pragma unroll
                         for (int j = 0; j < 32; ++j) packed[j] = v[j];
                     }
-                    // this warp's 32 rows: own staging pair, own TMA store
-                    unsigned char* sb = wstage + (size_t)(chunk & (a.ydepth - 1)) * (32 * 128);
-                    if (chunk >= a.ydepth) {
-                        if (lane == 0) {
-                            if (a.ydepth == 4) bulk_wait_read<3>();
-                            else bulk_wait_read<1>();
-                        }
-                        __syncwarp();
+                    unsigned char* box = hstage + (size_t)(chunk & (a.ydepth - 1)) * (128 * 128);
+                    unsigned char* sb = box + (size_t)g * (32 * 128);
+                    if (chunk >= a.ydepth && issuer) {
+                        if (a.ydepth == 2) bulk_wait_read<1>();
+                        else bulk_wait_read<0>();
                     }
+                    named_bar_sync(2 + half, 128);      // the buffer's previous store has read it
 #pragma unroll
                     for (int j = 0; j < 8; ++j) {
                         const uint32_t off = (uint32_t)lane * 128u + (uint32_t)((j ^ (lane & 7)) * 16);
@@ -634,10 +643,9 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
                             make_uint4(packed[4 * j], packed[4 * j + 1], packed[4 * j + 2], packed[4 * j + 3]);
                     }
                     fence_proxy_async_smem();
-                    __syncwarp();
-                    if (lane == 0) {
-                        if (col0 < a.m && row0 + g * 32 < a.b)
-                            tma_store_2d(&tm_y, (int32_t)col0, (int32_t)(row0 + g * 32), sb);
+                    named_bar_sync(2 + half, 128);      // all four slices are written
+                    if (issuer) {
+                        if (col0 < a.m) tma_store_2d(&tm_y, (int32_t)col0, (int32_t)row0, box);
                         bulk_commit();      // one group per chunk, even empty: the staging reuse counts on it
                     }
                 } else {
@@ -749,8 +757,8 @@ lrc_status plan_y(YArgs& a3, size_t& smem3, int64_t m, int64_t b, int kp, int pl
     smem3 = 0;
     for (int n2 : order) {
         if (!balance && n2 == 256 && btiles * ((m + 255) / 256) < 2 * (int64_t)sms) continue;   // too few tiles
-        // deeper output staging first (more TMA stores in flight), then the ring
-        for (int depth = 4; depth >= 2 && !smem3; depth -= 2) {
+        // two staging buffers per epilogue warp if they fit, else one; then the ring
+        for (int depth = 2; depth >= 1 && !smem3; --depth) {
             for (int stages = 4; stages >= 2 && !smem3; --stages) {
                 if (n2 == 256 && stages < 3) break;      // prefer a deeper ring with narrower tiles
                 const uint32_t u_bytes = (uint32_t)n2 * 128;
@@ -759,7 +767,7 @@ lrc_status plan_y(YArgs& a3, size_t& smem3, int64_t m, int64_t b, int kp, int pl
                 off += (size_t)planes * tile_bytes;
                 off = round_up(off, 1024);
                 const size_t ystage_off = off;
-                off += (size_t)4 * depth * 32 * 128;
+                off += (size_t)kEpiWarpsY * depth * 32 * 128;
                 const size_t bar_off = off;
                 off += (size_t)(2 * stages + 7) * 8 + 16;
                 if (off + 1024 > kSmemMax) continue;
@@ -790,14 +798,14 @@ lrc_status make_y_map(CUtensorMap* ty, const YArgs& a3, void* Y, int64_t m, int6
     if (!a3.tma_store) return LRC_OK;   // unused by the kernel
     const int e_out = out16 ? 2 : 4;
     return make_map(ty, out16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, Y, m, b, m * e_out,
-                    out16 ? 64 : 32, 32, "Y");
+                    out16 ? 64 : 32, BM, "Y");
 }
 
 lrc_status launch_y(const CUtensorMap& tu, const CUtensorMap& ty, const YArgs& a3, size_t smem3, int64_t P3,
                     cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(apply_y_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem3);
     if (e != cudaSuccess) return cuda_fail(e, "apply_y_kernel smem attribute");
-    e = launch_pdl(apply_y_kernel, dim3((unsigned)P3), dim3(kThreads), smem3, s, tu, a3.tma_store ? ty : tu, a3);
+    e = launch_pdl(apply_y_kernel, dim3((unsigned)P3), dim3(kThreadsY), smem3, s, tu, a3.tma_store ? ty : tu, a3);
     if (e != cudaSuccess) return cuda_fail(e, "apply_y_kernel launch");
     return after_launch("apply_y_kernel");
 }
