@@ -152,7 +152,7 @@ lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X
     if (!aligned16(X)) return misaligned("X");
     if (!aligned16(Y)) return misaligned("Y");
     cudaStream_t s = as_stream(stream);
-    if (b <= apply_skinny_max_batch(fmt) && k <= 1024)
+    if (apply_skinny_takes(fmt, b, k))
         return launch_apply_skinny(U, S, Vt, X, Y, m, n, k, b, fmt, s);
     switch (fmt) {
         case LRC_F64:
@@ -344,13 +344,15 @@ lrc_status lrc_device_status(lrc_stream_t stream) {
     const uint32_t t1 = take_tt_tc_error();
     const uint32_t t3 = take_tt3_tc_error();
     const uint32_t tn = take_ttn_tc_error();
+    const uint32_t sk = take_skinny_error();
     const uint32_t t = t1 | t3 | tn;
-    if (a == 0xffffffffu || t1 == 0xffffffffu || t3 == 0xffffffffu || tn == 0xffffffffu) {
+    if (a == 0xffffffffu || t1 == 0xffffffffu || t3 == 0xffffffffu || tn == 0xffffffffu || sk == 0xffffffffu) {
         set_error("could not read the device error words");
         return LRC_ERR_CUDA;
     }
-    if (a | t) {
-        set_error("a bounded device wait gave up (apply code 0x%x, TT code 0x%x)", a, t);
+    if (a | t | sk) {
+        set_error("a bounded device wait gave up (apply code 0x%x, TT code 0x%x, small-batch apply code 0x%x)", a,
+                  t, sk);
         return LRC_ERR_TIMEOUT;
     }
     return LRC_OK;

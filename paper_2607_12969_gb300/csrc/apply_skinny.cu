@@ -3,21 +3,25 @@
 // Y = [(X V) diag(s)] U^T).
 //
 // With a handful of queries the apply streams the two factors once and does
-// b multiply-adds per factor element: two matrix-vector streams that must
-// keep every SM's loads in flight.  Three launches on the caller's stream:
-//   skinny_w1_kernel  grid (n-chunk, group of 32 rows of V^T): the chunk of X
-//                     (at most 16 rows) is staged in shared memory; each warp
-//                     takes 4 rows of V^T and streams them with 16-byte loads
-//                     (four in flight per lane), each lane keeping the b
-//                     partial dot products of every row, which a fixed
-//                     butterfly then adds across the warp.  One partial W per
-//                     chunk.
-//   skinny_w2_kernel  W = (sum of the chunks' partials, in chunk order) diag(s);
-//                     for binary16 output W is rounded to binary16 (the
+// b multiply-adds per factor element: two matrix-vector streams whose speed
+// is set by how many bytes each SM has in flight.  Every operand tile is
+// therefore one set of TMA copies issued at the start of its CTA (2-D boxes,
+// zero-filled outside the arrays, so the arithmetic needs no bounds tests).
+// Three launches on the caller's stream:
+//   skinny_w1_kernel  grid (n-chunk, block of 32 rows of V^T): the chunk of X
+//                     (at most 16 rows) and of the 32 rows of V^T land in
+//                     shared memory; each warp takes 4 rows of V^T, each lane
+//                     keeps the b partial dot products of every row over its
+//                     16-byte columns, a recursive halving adds them across
+//                     the warp.  One partial W per chunk.  The CTAs also bring U
+//                     into L2 for the last kernel.
+//   skinny_w2_kernel  W = (sum of the chunks' partials) diag(s), a warp per
+//                     entry; for binary16 output W is rounded to binary16 (the
 //                     method-precision workspace of Sec. 3.4).
-//   skinny_y_kernel   W (b x k) in shared memory; each warp takes 4 rows of U,
-//                     streams them the same way and keeps the results of its
-//                     rows so that Y's rows are written as contiguous runs.
+//   skinny_y_kernel   a CTA per 64 rows of U (32 for binary64): the rows are
+//                     requested before the wait for the previous kernel, W
+//                     (b x k) follows as one bulk copy; groups of 8 lanes
+//                     take 4 rows (2) each, a lane every 8th column.
 // Arithmetic: binary64 FMAs for binary64, binary32 FMAs otherwise (binary16
 // factors widened exactly; Sec. 3.4: FP16 products accumulate in FP32).  The
 // summation order is fixed: results are reproducible on a device.
@@ -27,22 +31,30 @@
 #include "tc.cuh"
 
 namespace lrc {
+
+__device__ unsigned int g_err_skinny;
+
 namespace {
 
 constexpr int kWarps = 8;
 constexpr int kThreadsS = 32 * kWarps;
-constexpr int kRows = 4;                      // factor rows per warp and pass
+constexpr int kRows = 4;                      // factor rows per warp
+constexpr int kBlockRows = kWarps * kRows;    // factor rows per CTA
+constexpr int kBox = 256;                     // columns per TMA box of the first product
+constexpr size_t kSmemW1 = 100 * 1024;        // shared-memory budget of a first-product CTA
+constexpr size_t kSmemMaxS = 220 * 1024;      // largest dynamic shared memory a CTA asks for
+constexpr uint64_t kPrefetchMaxBytes = 64ull << 20;   // U prefetched into L2 up to this size
 
 template <typename TS>
 struct EVof {
     static constexpr int v = 16 / (int)sizeof(TS);     // elements per 16-byte vector
 };
 
-// 16 bytes of storage at p (16-byte aligned) as arithmetic values.
+// 16 bytes of storage at p (16-byte aligned, shared memory) as arithmetic values.
 template <typename T, typename TS>
 __device__ __forceinline__ void load_vec(const TS* p, T (&v)[EVof<TS>::v]) {
     if constexpr (sizeof(TS) == 2) {
-        const uint4 q = __ldg(reinterpret_cast<const uint4*>(p));
+        const uint4 q = *reinterpret_cast<const uint4*>(p);
         const uint32_t w[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -51,10 +63,10 @@ __device__ __forceinline__ void load_vec(const TS* p, T (&v)[EVof<TS>::v]) {
             v[2 * i + 1] = f.y;
         }
     } else if constexpr (sizeof(TS) == 4) {
-        const float4 q = __ldg(reinterpret_cast<const float4*>(p));
+        const float4 q = *reinterpret_cast<const float4*>(p);
         v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
     } else {
-        const double2 q = __ldg(reinterpret_cast<const double2*>(p));
+        const double2 q = *reinterpret_cast<const double2*>(p);
         v[0] = q.x; v[1] = q.y;
     }
 }
@@ -73,233 +85,359 @@ __device__ __forceinline__ T warp_sum(T v) {
     return v;
 }
 
+// Sums each of the N values v[] over the aligned groups of G lanes (G a
+// power of two <= 32) by recursive halving: at the step with lane offset o
+// (G/2, G/4, ...) a lane keeps one half of its values -- the upper half when
+// lane & o -- and adds the partner's copy of that half.  After
+// min(log2 G, log2 N) steps a butterfly over the remaining offsets finishes:
+// lane L then holds, in v[0 .. max(N/G, 1) - 1], the group totals of the
+// values halving_index<N, G>(L) + t.  Fixed order: the same result on every
+// run.  About N shuffles instead of N log2 G.
+template <int N, int G>
+__device__ __forceinline__ constexpr int halving_steps() {
+    int s = 0;
+    while ((1 << s) < G && (2 << s) <= N) ++s;
+    return s;
+}
+template <int N, int G>
+__device__ __forceinline__ int halving_index(int lane) {
+    int base = 0;
+#pragma unroll
+    for (int s = 0; s < halving_steps<N, G>(); ++s)
+        if (lane & ((G / 2) >> s)) base += N >> (s + 1);
+    return base;
+}
+template <int N, int G>
+__device__ __forceinline__ bool halving_writer(int lane) {
+    return (lane & ((G >> halving_steps<N, G>()) - 1)) == 0;
+}
+template <typename T, int N, int G>
+__device__ __forceinline__ void halving_sum(T (&v)[N], int lane) {
+    static_assert((N & (N - 1)) == 0 && (G & (G - 1)) == 0 && G <= 32, "powers of two");
+#pragma unroll
+    for (int s = 0; s < halving_steps<N, G>(); ++s) {
+        const int o = (G / 2) >> s, h = N >> (s + 1);
+        const bool up = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < h; ++i) {
+            const T send = up ? v[i] : v[i + h];
+            const T keep = up ? v[i + h] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+#pragma unroll
+    for (int o = (G / 2) >> halving_steps<N, G>(); o > 0; o >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
+}
+
 __device__ __forceinline__ void store_out(double* p, double v) { *p = v; }
 __device__ __forceinline__ void store_out(float* p, float v) { *p = v; }
 __device__ __forceinline__ void store_out(__half* p, float v) { *p = __float2half_rn(v); }
 
+__device__ __forceinline__ unsigned char* align128(unsigned char* p) {
+    return reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 127) & ~static_cast<uintptr_t>(127));
+}
+
+// Waits for copy group q of the CTA's nq (all threads).  On a timeout thread
+// 0 waits a little longer for every group still in flight before the CTA may
+// exit.
+__device__ __forceinline__ bool wait_tiles(uint64_t* bar, int q, int nq, volatile int* abort, unsigned int code) {
+    if (tc::mbar_wait(&bar[q], 0, abort, &g_err_skinny, code)) return true;
+    if (threadIdx.x == 0) {
+        volatile int no_abort = 0;
+        for (int i = 0; i < nq; ++i) tc::mbar_wait(&bar[i], 0, &no_abort, &g_err_skinny, code, 100000000ull);
+    }
+    return false;
+}
+
+// EV consecutive entries of W in shared memory (16-byte aligned when T is
+// the storage type, 32-byte aligned when binary16 storage is widened to
+// binary32) as 16-byte loads.
+template <typename T, int EV>
+__device__ __forceinline__ void load_w(const T* p, T (&v)[EV]) {
+    if constexpr (sizeof(T) == 8) {
+        static_assert(EV % 2 == 0, "binary64 vectors hold two entries");
+#pragma unroll
+        for (int e = 0; e < EV; e += 2) {
+            const double2 q = *reinterpret_cast<const double2*>(p + e);
+            v[e] = q.x; v[e + 1] = q.y;
+        }
+    } else {
+        static_assert(EV % 4 == 0, "binary32 vectors hold four entries");
+#pragma unroll
+        for (int e = 0; e < EV; e += 4) {
+            const float4 q = *reinterpret_cast<const float4*>(p + e);
+            v[e] = q.x; v[e + 1] = q.y; v[e + 2] = q.z; v[e + 3] = q.w;
+        }
+    }
+}
+
+// 1-D bulk copy global -> shared (both 16-byte aligned, size a multiple of 16).
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(tc::smem_u32(dst)), "l"(src), "r"(bytes), "r"(tc::smem_u32(bar))
+                 : "memory");
+}
+
 // ---------------------------------------------------------------- phase 1
+// Shared memory: [X boxes: nbox x B x kBox][V^T boxes: nbox x 32 x kBox]
+// [a barrier per box pair][abort flag]; column i of the chunk is box i / kBox,
+// offset i % kBox.  The boxes are multiplied in order as they land.
 template <typename TS, typename T, int B>
-__global__ void __launch_bounds__(kThreadsS)
-skinny_w1_kernel(const TS* __restrict__ X, const TS* __restrict__ Vt, int64_t n, int64_t ldn, int k, int b,
-                 int64_t L, T* __restrict__ Wp) {
+__global__ void __launch_bounds__(kThreadsS, 2)
+skinny_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_v, int k, int b,
+                 int L, T* __restrict__ Wp, const void* upf, uint64_t upf_bytes) {
     constexpr int EV = EVof<TS>::v;
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    T* xs = reinterpret_cast<T*>(smem_raw);      // [B][L], zero past the batch and the chunk
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* smem = align128(smem_raw);
+    const int nbox = L / kBox;
+    TS* xs = reinterpret_cast<TS*>(smem);
+    TS* vs = xs + (size_t)nbox * B * kBox;
+    uint64_t* bar = reinterpret_cast<uint64_t*>(vs + (size_t)nbox * kBlockRows * kBox);
+    volatile int* abort = reinterpret_cast<volatile int*>(bar + nbox);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t chunk = blockIdx.x;
-    const int64_t i0 = chunk * L;
-    const int64_t len = (n - i0) < L ? (n - i0) : L;
-    // stage X: 16-byte vectors, four loads in flight per thread before their stores
-    {
-        const int64_t nv = (int64_t)B * (L / EV);
-        for (int64_t v0 = threadIdx.x; v0 < nv; v0 += 4 * kThreadsS) {
-            T val[4][EV];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int64_t v = v0 + (int64_t)u * kThreadsS;
-                const int64_t c = v / (L / EV), i = (v - c * (L / EV)) * EV;
-                if (v < nv && c < b && i + EV <= len) {
-                    load_vec<T, TS>(X + c * ldn + i0 + i, val[u]);
-                } else {
-#pragma unroll
-                    for (int e = 0; e < EV; ++e)
-                        val[u][e] = (v < nv && c < b && i + e < len) ? to_t<T>(X[c * ldn + i0 + i + e]) : T(0);
-                }
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int64_t v = v0 + (int64_t)u * kThreadsS;
-                if (v < nv) {
-                    const int64_t c = v / (L / EV), i = (v - c * (L / EV)) * EV;
-#pragma unroll
-                    for (int e = 0; e < EV; ++e) xs[c * L + i + e] = val[u][e];
-                }
-            }
+    const int32_t i0 = (int32_t)(chunk * L);
+    const int jb = (int)blockIdx.y * kBlockRows;
+    if (threadIdx.x == 0) {
+        for (int q = 0; q < nbox; ++q) tc::mbar_init(&bar[q], 1);
+        *abort = 0;
+        tc::fence_barrier_init();
+        for (int q = 0; q < nbox; ++q) {
+            tc::mbar_arrive_expect_tx(&bar[q], (uint32_t)((B + kBlockRows) * kBox * (int)sizeof(TS)));
+            tc::tma_load_2d(vs + (size_t)q * kBlockRows * kBox, &tm_v, i0 + q * kBox, jb, &bar[q]);
+            tc::tma_load_2d(xs + (size_t)q * B * kBox, &tm_x, i0 + q * kBox, 0, &bar[q]);
         }
+        // U, read by the last kernel, comes into L2 alongside this kernel's stream
+        if (upf) tc::bulk_prefetch_share(upf, upf_bytes, blockIdx.y * gridDim.x + blockIdx.x, gridDim.x * gridDim.y);
     }
     __syncthreads();
-    const int j0 = (blockIdx.y * kWarps + warp) * kRows;
-    T acc[kRows][B];
+    const int jl = warp * kRows;                 // first local row of the warp
+    T acc[kRows * B];                            // acc[r * B + c]: row jl + r, query c
 #pragma unroll
-    for (int r = 0; r < kRows; ++r)
+    for (int i = 0; i < kRows * B; ++i) acc[i] = T(0);
+    for (int q = 0; q < nbox; ++q) {
+        if (!wait_tiles(bar, q, nbox, abort, 1u)) return;
+        const TS* vq = vs + ((size_t)q * kBlockRows + jl) * kBox;
+        const TS* xq = xs + (size_t)q * B * kBox;
+        for (int o = lane * EV; o < kBox; o += 32 * EV) {
+            T vv[kRows][EV];
 #pragma unroll
-        for (int c = 0; c < B; ++c) acc[r][c] = T(0);
-    const int64_t nvec = len / EV;
-    for (int64_t v = lane; v < nvec; v += 32) {
-        T vv[kRows][EV];
+            for (int r = 0; r < kRows; ++r) load_vec<T, TS>(vq + (size_t)r * kBox + o, vv[r]);
 #pragma unroll
-        for (int r = 0; r < kRows; ++r) {
-            if (j0 + r < k) load_vec<T, TS>(Vt + (int64_t)(j0 + r) * ldn + i0 + v * EV, vv[r]);
-            else {
+            for (int c = 0; c < B; ++c) {
+                T xv[EV];
+                load_vec<T, TS>(xq + (size_t)c * kBox + o, xv);
 #pragma unroll
-                for (int e = 0; e < EV; ++e) vv[r][e] = T(0);
+                for (int r = 0; r < kRows; ++r)
+#pragma unroll
+                    for (int e = 0; e < EV; ++e) acc[r * B + c] = fma(xv[e], vv[r][e], acc[r * B + c]);
             }
-        }
-#pragma unroll
-        for (int c = 0; c < B; ++c) {
-            T xv[EV];
-#pragma unroll
-            for (int e = 0; e < EV; ++e) xv[e] = xs[c * L + v * EV + e];
-#pragma unroll
-            for (int r = 0; r < kRows; ++r)
-#pragma unroll
-                for (int e = 0; e < EV; ++e) acc[r][c] = fma(xv[e], vv[r][e], acc[r][c]);
-        }
-    }
-    // ragged end of the chunk: single elements
-    for (int64_t i = nvec * EV + lane; i < len; i += 32) {
-#pragma unroll
-        for (int r = 0; r < kRows; ++r) {
-            const T x = (j0 + r < k) ? to_t<T>(Vt[(int64_t)(j0 + r) * ldn + i0 + i]) : T(0);
-#pragma unroll
-            for (int c = 0; c < B; ++c) acc[r][c] = fma(xs[c * L + i], x, acc[r][c]);
         }
     }
     tc::pdl_trigger();
+    constexpr int N = kRows * B;
+    halving_sum<T, N, 32>(acc, lane);
+    if (halving_writer<N, 32>(lane)) {
+        const int base = halving_index<N, 32>(lane);
 #pragma unroll
-    for (int r = 0; r < kRows; ++r) {
-#pragma unroll
-        for (int c = 0; c < B; ++c) {
-            const T sum = warp_sum(acc[r][c]);
-            if (lane == c && c < b && j0 + r < k) Wp[(chunk * b + c) * k + j0 + r] = sum;
+        for (int t = 0; t < (N >= 32 ? N / 32 : 1); ++t) {
+            const int idx = base + t, r = idx / B, c = idx - r * B;
+            const int j = jb + jl + r;
+            if (c < b && j < k) Wp[(chunk * b + c) * k + j] = acc[t];
         }
     }
 }
 
 // ---------------------------------------------------------------- phase 1b
+// A warp per entry of W ([b][kv], zero in the columns k..kv-1): lane l adds
+// chunks l, l + 32, ... in order, a fixed butterfly adds the lane sums (the
+// same order on every run).
 template <typename TS, typename T>
 __global__ void __launch_bounds__(256)
-skinny_w2_kernel(const T* __restrict__ Wp, int nchunks, int b, int k, const TS* __restrict__ S, int round16,
+skinny_w2_kernel(const T* __restrict__ Wp, int nchunks, int b, int k, int kv, const TS* __restrict__ S, int round16,
                  T* __restrict__ W) {
     tc::pdl_wait();                  // partials of the phase-1 grid
     tc::pdl_trigger();
-    const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (e >= (int64_t)b * k) return;
-    const int j = (int)(e % k);
-    T acc = Wp[e];
-    for (int ch = 1; ch < nchunks; ++ch) acc += Wp[(int64_t)ch * b * k + e];
-    acc *= to_t<T>(S[j]);
-    if (round16) acc = (T)__half2float(__float2half_rn((float)acc));
-    W[e] = acc;
+    const int lane = threadIdx.x & 31;
+    const int64_t e = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (e >= (int64_t)b * kv) return;
+    const int c = (int)(e / kv), j = (int)(e - (int64_t)c * kv);
+    T acc = T(0);
+    if (j < k) {
+        const int64_t bk = (int64_t)b * k;
+        for (int ch = lane; ch < nchunks; ch += 32) acc += Wp[(int64_t)ch * bk + (int64_t)c * k + j];
+        acc = warp_sum(acc);
+        acc *= to_t<T>(S[j]);
+        if (round16) acc = (T)__half2float(__float2half_rn((float)acc));
+    }
+    if (lane == 0) W[e] = acc;
 }
 
 // ---------------------------------------------------------------- phase 2
-template <typename TS, typename T, typename TOut, int B>
-__global__ void __launch_bounds__(kThreadsS)
-skinny_y_kernel(const T* __restrict__ W, const TS* __restrict__ U, int64_t m, int k, int64_t ldk, int b,
-                TOut* __restrict__ Y) {
+// A CTA of kYWarps warps owns 16 RPG rows of U: each warp's four groups of 8
+// lanes take RPG rows each, and a lane covers every 8th 16-byte column of
+// its rows (a short reduction: the rank is only a few hundred).  Shared
+// memory: [U: nkb boxes of 16 RPG rows x kbw][W: B x kv][barrier of U]
+// [barrier of W][abort flag]; column j of U is box j / kbw, offset j % kbw;
+// kv = nkb * kbw.
+constexpr int kYWarps = 4;
+constexpr int kYGroup = 8;
+template <typename TS, typename T, typename TOut, int B, int RPG>
+__global__ void __launch_bounds__(32 * kYWarps)
+skinny_y_kernel(const __grid_constant__ CUtensorMap tm_u, const T* __restrict__ W, int64_t m, int b, int nkb,
+                int kbw, TOut* __restrict__ Y) {
     constexpr int EV = EVof<TS>::v;
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    T* ws = reinterpret_cast<T*>(smem_raw);      // [B][kv], zero past the batch and the rank
-    const int kv = (k + EV - 1) / EV * EV;
+    constexpr int RC = kYWarps * (32 / kYGroup) * RPG;     // rows of the CTA
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* smem = align128(smem_raw);
+    const int kv = nkb * kbw;
+    TS* us = reinterpret_cast<TS*>(smem);
+    T* ws = reinterpret_cast<T*>(us + (size_t)nkb * RC * kbw);
+    uint64_t* bar = reinterpret_cast<uint64_t*>(ws + (size_t)B * kv);
+    volatile int* abort = reinterpret_cast<volatile int*>(bar + 2);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    tc::pdl_wait();                  // W of the reduction kernel
-    for (int e = threadIdx.x; e < B * kv; e += kThreadsS) {
-        const int c = e / kv, j = e - c * kv;
-        ws[e] = (c < b && j < k) ? W[c * k + j] : T(0);
+    const int64_t rb = (int64_t)blockIdx.x * RC;
+    const uint32_t w_bytes = (uint32_t)((size_t)b * kv * sizeof(T));
+    if (threadIdx.x == 0) {
+        tc::mbar_init(&bar[0], 1);
+        tc::mbar_init(&bar[1], 1);
+        *abort = 0;
+        tc::fence_barrier_init();
+        tc::mbar_arrive_expect_tx(&bar[0], (uint32_t)(nkb * RC * kbw * (int)sizeof(TS)));
+        for (int q = 0; q < nkb; ++q)
+            tc::tma_load_2d(us + (size_t)q * RC * kbw, &tm_u, q * kbw, (int32_t)rb, &bar[0]);
+        tc::pdl_wait();              // W of the reduction kernel
+        tc::mbar_arrive_expect_tx(&bar[1], w_bytes);
+        bulk_load(ws, W, w_bytes, &bar[1]);
     }
+    // rows b..B-1 of W are zero
+    for (int e = b * kv + threadIdx.x; e < B * kv; e += 32 * kYWarps) ws[e] = T(0);
     __syncthreads();
-    const int64_t r0 = ((int64_t)blockIdx.x * kWarps + warp) * kRows;
-    T acc[kRows][B];
+    if (!wait_tiles(bar, 1, 2, abort, 2u)) return;
+    if (!wait_tiles(bar, 0, 2, abort, 2u)) return;
+    const int sl = lane & (kYGroup - 1);
+    const int rl = (warp * (32 / kYGroup) + (lane / kYGroup)) * RPG;
+    constexpr int N = RPG * B;
+    T acc[N];                                    // acc[r * B + c]: row rl + r, query c
 #pragma unroll
-    for (int r = 0; r < kRows; ++r)
+    for (int i = 0; i < N; ++i) acc[i] = T(0);
+    for (int v = sl; v < kv / EV; v += kYGroup) {
+        const int j = v * EV, q = j / kbw, o = j - q * kbw;
+        T uu[RPG][EV];
 #pragma unroll
-        for (int c = 0; c < B; ++c) acc[r][c] = T(0);
-    const int nvk = kv / EV;
-    for (int v = lane; v < nvk; v += 32) {
-        T uu[kRows][EV];
-#pragma unroll
-        for (int r = 0; r < kRows; ++r) {
-            if (r0 + r < m) {
-                load_vec<T, TS>(U + (r0 + r) * ldk + v * EV, uu[r]);
-#pragma unroll
-                for (int e = 0; e < EV; ++e)
-                    if (v * EV + e >= k) uu[r][e] = T(0);    // pad columns of U are not read as numbers
-            } else {
-#pragma unroll
-                for (int e = 0; e < EV; ++e) uu[r][e] = T(0);
-            }
-        }
+        for (int r = 0; r < RPG; ++r) load_vec<T, TS>(us + ((size_t)q * RC + rl + r) * kbw + o, uu[r]);
 #pragma unroll
         for (int c = 0; c < B; ++c) {
             T wv[EV];
+            load_w(ws + (size_t)c * kv + j, wv);
 #pragma unroll
-            for (int e = 0; e < EV; ++e) wv[e] = ws[c * kv + v * EV + e];
+            for (int r = 0; r < RPG; ++r)
 #pragma unroll
-            for (int r = 0; r < kRows; ++r)
-#pragma unroll
-                for (int e = 0; e < EV; ++e) acc[r][c] = fma(wv[e], uu[r][e], acc[r][c]);
+                for (int e = 0; e < EV; ++e) acc[r * B + c] = fma(wv[e], uu[r][e], acc[r * B + c]);
         }
     }
-    // output q = c * kRows + r (Y[c][r0 + r]) is kept by lane q % 32 in out[q / 32]
-    constexpr int NOUT = (B * kRows + 31) / 32;
-    T out[NOUT];
+    halving_sum<T, N, kYGroup>(acc, lane);
+    const int64_t r0 = rb + rl;
+    if (halving_writer<N, kYGroup>(lane)) {
+        const int base = halving_index<N, kYGroup>(lane);
 #pragma unroll
-    for (int q = 0; q < NOUT; ++q) out[q] = T(0);
-#pragma unroll
-    for (int r = 0; r < kRows; ++r)
-#pragma unroll
-        for (int c = 0; c < B; ++c) {
-            const T sum = warp_sum(acc[r][c]);
-            const int q = c * kRows + r;
-            if (lane == (q & 31)) out[q >> 5] = sum;
+        for (int t = 0; t < (N >= kYGroup ? N / kYGroup : 1); ++t) {
+            const int idx = base + t, r = idx / B, c = idx - r * B;
+            if (c < b && r0 + r < m) store_out(Y + (int64_t)c * m + r0 + r, acc[t]);
         }
-#pragma unroll
-    for (int q = 0; q < NOUT; ++q) {
-        const int idx = q * 32 + lane;
-        const int c = idx / kRows, r = idx % kRows;
-        if (c < b && c < B && r0 + r < m) store_out(Y + (int64_t)c * m + r0 + r, out[q]);
     }
+}
+
+template <typename TS>
+constexpr int y_rpg() { return sizeof(TS) == 8 ? 2 : 4; }
+
+template <typename TS>
+CUtensorMapDataType map_type() {
+    if constexpr (sizeof(TS) == 2) return CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+    else if constexpr (sizeof(TS) == 4) return CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+    else return CU_TENSOR_MAP_DATA_TYPE_FLOAT64;
+}
+
+// Launch plan of one size: chunk length of the first product, boxes of the
+// second, shared memory of both.
+struct SkinnyPlan {
+    int64_t L, nchunks, jblocks, nkb, kbw, kv, yblocks;
+    size_t smem1, smem3;
+};
+
+SkinnyPlan plan_skinny(int64_t m, int64_t n, int64_t k, int B, int64_t e, int64_t et) {
+    SkinnyPlan p{};
+    const int64_t ev = 16 / e;
+    // chunk length: a multiple of kBox with the CTA's tiles within the
+    // shared-memory budget (two CTAs per SM), and enough chunks for two CTAs
+    // per SM
+    p.jblocks = (k + kBlockRows - 1) / kBlockRows;
+    int64_t L = (int64_t)(kSmemW1 / (size_t)((B + kBlockRows) * e)) / kBox * kBox;
+    if (L < kBox) L = kBox;
+    const int64_t want = (2 * (int64_t)sm_count() + p.jblocks - 1) / p.jblocks;
+    int64_t Lw = (n + want - 1) / want;
+    Lw = (Lw + kBox - 1) / kBox * kBox;
+    if (Lw < L) L = Lw;
+    p.L = L;
+    p.nchunks = (n + L - 1) / L;
+    // second product: U in nkb boxes of kbw columns (kbw a multiple of the
+    // 16-byte vector, at most 256)
+    p.nkb = (k + 255) / 256;
+    p.kbw = ((k + p.nkb - 1) / p.nkb + ev - 1) / ev * ev;
+    p.kv = p.nkb * p.kbw;
+    p.smem1 = (size_t)(L / kBox) * (B + kBlockRows) * kBox * e + 8 * (size_t)(L / kBox + 1) + 128;
+    // second product: CTAs of 16 RPG rows of U
+    const int64_t rc = (int64_t)kYWarps * (32 / kYGroup) * (e == 8 ? 2 : 4);
+    p.yblocks = (m + rc - 1) / rc;
+    p.smem3 = (size_t)p.nkb * rc * p.kbw * e + (size_t)B * p.kv * et + 24 + 128;
+    return p;
 }
 
 template <typename TS, typename T, typename TOut, int B>
 lrc_status launch_skinny_b(const TS* U, const TS* S, const TS* Vt, const TS* X, TOut* Y, int64_t m, int64_t n,
                            int64_t k, int64_t b, bool round16, cudaStream_t s) {
-    constexpr int EV = EVof<TS>::v;
-    const int sms = sm_count();
     const int64_t ldn = lrc_packed_ld(n), ldk = lrc_packed_ld(k);
-    // chunk length: a multiple of 256 elements with the staged X within 48 KB,
-    // and enough chunks for two waves of CTAs
-    const int64_t jblocks = (k + kWarps * kRows - 1) / (kWarps * kRows);
-    int64_t L = (48 * 1024) / ((int64_t)B * (int64_t)sizeof(T)) / 256 * 256;
-    if (L > 4096) L = 4096;
-    const int64_t want = (2 * (int64_t)sms + jblocks - 1) / jblocks;
-    int64_t Lw = (n + want - 1) / want;
-    Lw = (Lw + 255) / 256 * 256;
-    if (Lw < L) L = Lw;
-    if (L < 256) L = 256;
-    const int64_t nchunks = (n + L - 1) / L;
+    const int64_t e = (int64_t)sizeof(TS);
+    const SkinnyPlan p = plan_skinny(m, n, k, B, e, (int64_t)sizeof(T));
     int64_t t;
-    if (!mul_ok(nchunks * b, k, &t) || nchunks > 65535 || jblocks > 65535) {
-        set_error("small-batch apply: problem too large");
+    if (!mul_ok(p.nchunks * b, k, &t) || p.nchunks > 65535 || p.jblocks > 65535 || n > INT32_MAX ||
+        m > INT32_MAX || p.smem1 > kSmemMaxS || p.smem3 > kSmemMaxS) {
+        set_error("small-batch apply: problem outside the kernel");
         return LRC_ERR_UNSUPPORTED;
     }
-    const size_t part_bytes = ((size_t)nchunks * b * k * sizeof(T) + 255) / 256 * 256;
-    const size_t w_bytes = (size_t)b * k * sizeof(T);
+    const size_t part_bytes = ((size_t)p.nchunks * b * k * sizeof(T) + 255) / 256 * 256;
+    const size_t w_bytes = (size_t)b * p.kv * sizeof(T);
     void* ws = nullptr;
     lrc_status st = stream_workspace(s, part_bytes + w_bytes, &ws);
     if (st != LRC_OK) return st;
     T* Wp = static_cast<T*>(ws);
     T* Wd = reinterpret_cast<T*>(static_cast<unsigned char*>(ws) + part_bytes);
-    const size_t smem1 = (size_t)B * L * sizeof(T);
-    skinny_w1_kernel<TS, T, B><<<dim3((unsigned)nchunks, (unsigned)jblocks), kThreadsS, smem1, s>>>(
-        X, Vt, n, ldn, (int)k, (int)b, L, Wp);
+
+    CUtensorMap tx, tv, tu;
+    if ((st = encode_map_2d(&tx, map_type<TS>(), X, n, b, ldn * e, kBox, B, false, "X")) != LRC_OK) return st;
+    if ((st = encode_map_2d(&tv, map_type<TS>(), Vt, n, k, ldn * e, kBox, kBlockRows, false, "Vt")) != LRC_OK)
+        return st;
+    constexpr int kRowsY = kYWarps * (32 / kYGroup) * y_rpg<TS>();
+    if ((st = encode_map_2d(&tu, map_type<TS>(), U, k, m, ldk * e, (uint32_t)p.kbw, kRowsY, false, "U")) != LRC_OK)
+        return st;
+
+    cudaError_t ce = cudaFuncSetAttribute(skinny_w1_kernel<TS, T, B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)p.smem1);
+    if (ce != cudaSuccess) return cuda_fail(ce, "skinny_w1_kernel smem attribute");
+    const uint64_t u_bytes = ((uint64_t)(m - 1) * (uint64_t)ldk + (uint64_t)k) * (uint64_t)e;
+    skinny_w1_kernel<TS, T, B><<<dim3((unsigned)p.nchunks, (unsigned)p.jblocks), kThreadsS, p.smem1, s>>>(
+        tx, tv, (int)k, (int)b, (int)p.L, Wp, u_bytes <= kPrefetchMaxBytes ? (const void*)U : nullptr, u_bytes);
     if ((st = after_launch("skinny_w1_kernel")) != LRC_OK) return st;
-    cudaError_t e = launch_pdl(skinny_w2_kernel<TS, T>, dim3((unsigned)((b * k + 255) / 256)), dim3(256), 0, s,
-                               (const T*)Wp, (int)nchunks, (int)b, (int)k, S, round16 ? 1 : 0, Wd);
-    if (e != cudaSuccess) return cuda_fail(e, "skinny_w2_kernel launch");
+    ce = launch_pdl(skinny_w2_kernel<TS, T>, dim3((unsigned)((b * p.kv * 32 + 255) / 256)), dim3(256), 0, s,
+                    (const T*)Wp, (int)p.nchunks, (int)b, (int)k, (int)p.kv, S, round16 ? 1 : 0, Wd);
+    if (ce != cudaSuccess) return cuda_fail(ce, "skinny_w2_kernel launch");
     if ((st = after_launch("skinny_w2_kernel")) != LRC_OK) return st;
-    const int kv = (int)((k + EV - 1) / EV * EV);
-    const size_t smem3 = (size_t)B * kv * sizeof(T);
-    if (smem3 > 48 * 1024) {
-        e = cudaFuncSetAttribute(skinny_y_kernel<TS, T, TOut, B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)smem3);
-        if (e != cudaSuccess) return cuda_fail(e, "skinny_y_kernel smem attribute");
-    }
-    const int64_t yblocks = (m + kWarps * kRows - 1) / (kWarps * kRows);
-    e = launch_pdl(skinny_y_kernel<TS, T, TOut, B>, dim3((unsigned)yblocks), dim3(kThreadsS), smem3, s,
-                   (const T*)Wd, U, m, (int)k, ldk, (int)b, Y);
-    if (e != cudaSuccess) return cuda_fail(e, "skinny_y_kernel launch");
+    auto ykernel = skinny_y_kernel<TS, T, TOut, B, y_rpg<TS>()>;
+    ce = cudaFuncSetAttribute(ykernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem3);
+    if (ce != cudaSuccess) return cuda_fail(ce, "skinny_y_kernel smem attribute");
+    ce = launch_pdl(ykernel, dim3((unsigned)p.yblocks), dim3(32 * kYWarps), p.smem3, s, tu, (const T*)Wd, m, (int)b,
+                    (int)p.nkb, (int)p.kbw, Y);
+    if (ce != cudaSuccess) return cuda_fail(ce, "skinny_y_kernel launch");
     return after_launch("skinny_y_kernel");
 }
 
@@ -308,19 +446,29 @@ lrc_status launch_skinny_t(const TS* U, const TS* S, const TS* Vt, const TS* X, 
                            int64_t k, int64_t b, bool round16, cudaStream_t s) {
     if (b <= 1) return launch_skinny_b<TS, T, TOut, 1>(U, S, Vt, X, Y, m, n, k, b, round16, s);
     if (b <= 4) return launch_skinny_b<TS, T, TOut, 4>(U, S, Vt, X, Y, m, n, k, b, round16, s);
-    return launch_skinny_b<TS, T, TOut, 16>(U, S, Vt, X, Y, m, n, k, b, round16, s);
+    if constexpr (sizeof(TS) == 4) return launch_skinny_b<TS, T, TOut, 16>(U, S, Vt, X, Y, m, n, k, b, round16, s);
+    set_error("small-batch apply: b = %lld above the kernel's batch", (long long)b);
+    return LRC_ERR_UNSUPPORTED;
 }
+
+int64_t max_batch(lrc_fmt fmt) { return fmt == LRC_F32 ? 16 : 4; }
 
 }  // namespace
 
-// Largest batch this path takes per format: up to 16 queries for binary32;
-// binary64 (DFMA-bound from a few queries on) and binary16 (whose tensor-core
-// path is faster from 16 queries on) up to 4.
-int64_t apply_skinny_max_batch(lrc_fmt fmt) { return fmt == LRC_F32 ? 16 : 4; }
+// Batches this path takes: up to 16 queries for binary32; binary64
+// (DFMA-bound from a few queries on) and binary16 (whose tensor-core path is
+// faster from 16 queries on) up to 4; ranks whose tiles fit in shared memory.
+bool apply_skinny_takes(lrc_fmt fmt, int64_t b, int64_t k) {
+    if (b < 1 || b > max_batch(fmt) || k < 1 || k > 1024) return false;
+    const int B = b <= 1 ? 1 : (b <= 4 ? 4 : 16);
+    const int64_t e = storage_bytes(fmt);
+    const SkinnyPlan p = plan_skinny(1, 1, k, B, e, fmt == LRC_F64 ? 8 : 4);
+    return p.smem1 <= kSmemMaxS && p.smem3 <= kSmemMaxS;
+}
 
 lrc_status launch_apply_skinny(const void* U, const void* S, const void* Vt, const void* X, void* Y, int64_t m,
                                int64_t n, int64_t k, int64_t b, lrc_fmt fmt, cudaStream_t s) {
-    if (b < 1 || b > apply_skinny_max_batch(fmt) || k > 1024) {
+    if (!apply_skinny_takes(fmt, b, k)) {
         set_error("small-batch apply: b = %lld, k = %lld outside the kernel", (long long)b, (long long)k);
         return LRC_ERR_UNSUPPORTED;
     }
@@ -338,6 +486,16 @@ lrc_status launch_apply_skinny(const void* U, const void* S, const void* Vt, con
             return launch_skinny_t<__half, float, __half>((const __half*)U, (const __half*)S, (const __half*)Vt,
                                                          (const __half*)X, (__half*)Y, m, n, k, b, true, s);
     }
+}
+
+uint32_t take_skinny_error() {
+    unsigned int v = 0;
+    if (cudaMemcpyFromSymbol(&v, g_err_skinny, sizeof v) != cudaSuccess) return 0xffffffffu;
+    if (v) {
+        const unsigned int z = 0;
+        cudaMemcpyToSymbol(g_err_skinny, &z, sizeof z);
+    }
+    return v;
 }
 
 }  // namespace lrc

@@ -61,6 +61,8 @@ constexpr uint32_t kXBytes = BM * BK * 2;    // one X box
 constexpr int kChunkBlocks = 8;              // k-blocks per accumulation chunk (FP32 output)
 constexpr int kPfBlocks = 4;                 // k-blocks per L2 prefetch box (512-byte rows)
 constexpr int kStageBlocks = 2;              // k-blocks per phase-1 ring stage
+constexpr int64_t kPrefetchMaxBatch = 1024;  // U prefetched into L2 by phase 1 up to this batch
+constexpr uint64_t kPrefetchMaxBytes = 48ull << 20;
 
 __device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
     return reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -81,6 +83,8 @@ struct W1Args {
     uint32_t sum_off, bar_off;
     uint32_t tmem_cols;
     float* P;                 // partials: [segment id][kgp columns][128 rows]
+    const void* upf;          // optional: buffer (U) that the CTAs prefetch into L2 for the next product
+    uint64_t upf_bytes;
 };
 
 // Next accumulation chunk of the k-block range [qbeg, qend): a chunk lies in
@@ -151,6 +155,7 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
             bool ok = true;
             int64_t q = qbeg, q0, q1, row;
             bool first, last;
+            if (a.upf) bulk_prefetch_share(a.upf, a.upf_bytes, blockIdx.x, gridDim.x);
             while (ok && next_chunk(q, qbeg, qend, a.nkb, a.chunk_blocks, q0, q1, row, first, last)) {
                 const int grp = (int)(row / a.btiles);
                 const int64_t bt = row - (int64_t)grp * a.btiles;
@@ -387,46 +392,78 @@ apply_w2_kernel(const W2Args a) {
     put_w8(a, bt, r, col0, w);
 }
 
-// One warp per (row tile, 8 columns, row), for rows with many partials (small
-// b): lane l adds partials l, l + 32, ... in order, then the 32 lane sums are
-// combined by a fixed butterfly -- the same order on every run.
-__global__ void __launch_bounds__(256)
-apply_w2_warp_kernel(const W2Args a) {
+// For rows with many partials (small b): a CTA per (row tile, block of 32
+// rows, 8 columns) with 16 warps.  Lane = row (coalesced loads of the
+// partials' row runs), warp w adds partials w, w + 16, ... in order, several
+// partials' loads in flight at a time; warp 0 then adds the 16 warp sums in
+// warp order -- the same order on every run.
+constexpr int kW2Slices = 16;
+__global__ void __launch_bounds__(32 * kW2Slices)
+apply_w2_slice_kernel(const W2Args a) {
+    __shared__ float red[kW2Slices][8][33];
     pdl_trigger();
     pdl_wait();                    // partials of the phase-1 grid
     const int cg8 = a.kp / 8;
-    const int lane = threadIdx.x & 31;
-    const int64_t e = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    if (e >= a.btiles * cg8 * BM) return;
-    const int r = (int)(e % BM);
-    const int64_t t = e / BM;
-    const int cg = (int)(t % cg8);
-    const int64_t bt = t / cg8;
-    const int col0 = cg * 8;
-    const int grp = col0 / a.kgp;
-    const int j0 = col0 - grp * a.kgp;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t cg = blockIdx.x % cg8;
+    const int64_t t = blockIdx.x / cg8;
+    const int rb = (int)(t & 3);
+    const int64_t bt = t >> 2;
+    const int col0 = (int)cg * 8;
+    const int r = rb * 32 + lane;
+    const bool any = bt * BM + rb * 32 < a.b;
     float w[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) w[i] = 0.0f;
-    if (bt * BM + r < a.b) {
+    if (any) {
+        const int grp = col0 / a.kgp;               // group widths are multiples of 16
+        const int j0 = col0 - grp * a.kgp;
         const int64_t ur = (int64_t)grp * a.btiles + bt;
         const int64_t cf = cta_of(ur * a.nkb, a.Q, a.P1);
         const int64_t cl = cta_of(ur * a.nkb + a.nkb - 1, a.Q, a.P1);
+        const int64_t np = cl - cf + 1;
         const size_t pstride = (size_t)a.kgp * BM;
         const float* p0 = a.P + ((size_t)(cf + ur) * a.kgp + j0) * BM + r;
-        for (int64_t c = lane; c <= cl - cf; c += 32) {
+        if (bt * BM + r < a.b) {
+            constexpr int kBatch = 4;
+            for (int64_t c0 = warp; c0 < np; c0 += kW2Slices * kBatch) {
+                float t8[kBatch][8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) w[i] = __fadd_rn(w[i], __ldg(p0 + (size_t)c * pstride + (size_t)i * BM));
+                for (int u = 0; u < kBatch; ++u) {
+                    const int64_t c = c0 + (int64_t)u * kW2Slices;
+                    if (c < np) {
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) t8[u][i] = __ldg(p0 + (size_t)c * pstride + (size_t)i * BM);
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < kBatch; ++u) {
+                    if (c0 + (int64_t)u * kW2Slices < np) {
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) w[i] = __fadd_rn(w[i], t8[u][i]);
+                    }
+                }
+            }
         }
 #pragma unroll
-        for (int off = 16; off >= 1; off >>= 1) {
+        for (int i = 0; i < 8; ++i) red[warp][i][lane] = w[i];
+        __syncthreads();
+        if (warp != 0) return;
 #pragma unroll
-            for (int i = 0; i < 8; ++i) w[i] = __fadd_rn(w[i], __shfl_xor_sync(0xffffffffu, w[i], off));
+        for (int i = 0; i < 8; ++i) {
+            float v = red[0][i][lane];
+#pragma unroll
+            for (int q = 1; q < kW2Slices; ++q) v = __fadd_rn(v, red[q][i][lane]);
+            w[i] = __fmul_rn(v, col0 + i < a.k ? __half2float(a.S[col0 + i]) : 0.0f);
         }
+        if (bt * BM + r >= a.b) {
 #pragma unroll
-        for (int i = 0; i < 8; ++i) w[i] = __fmul_rn(w[i], col0 + i < a.k ? __half2float(a.S[col0 + i]) : 0.0f);
+            for (int i = 0; i < 8; ++i) w[i] = 0.0f;
+        }
+    } else if (warp != 0) {
+        return;
     }
-    if (lane == 0) put_w8(a, bt, r, col0, w);
+    put_w8(a, bt, r, col0, w);
 }
 
 // ================================================================ phase 2
@@ -882,6 +919,13 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
     a3.W = Wimg;
 
     const int64_t ldn = lrc_packed_ld(n), ldk = lrc_packed_ld(k);
+    // small batches: the second product reads U a few times only, so phase 1
+    // brings it into L2 alongside its own stream
+    const uint64_t u_bytes = ((uint64_t)(m - 1) * (uint64_t)ldk + (uint64_t)k) * 2u;
+    if (b <= kPrefetchMaxBatch && u_bytes <= kPrefetchMaxBytes) {
+        a1.upf = U;
+        a1.upf_bytes = u_bytes;
+    }
     CUtensorMap tx, tv, tu, ty, txp, tvp;
     if ((st = make_map(&tx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, X, n, b, ldn * 2, BK, BM, "X")) != LRC_OK) return st;
     if ((st = make_map(&tv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, Vt, n, k, ldn * 2, BK, (uint32_t)a1.kgp, "Vt")) != LRC_OK)
@@ -919,9 +963,10 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
     const int64_t n2items = btiles * (kp / 8) * BM;
     const int64_t max_parts = (a1.nkb * P1 + a1.Q - 1) / a1.Q + 1;     // CTAs sharing one row, at most
     if (max_parts >= 16) {
-        e = launch_pdl(apply_w2_warp_kernel, dim3((unsigned)((n2items * 32 + 255) / 256)), dim3(256), 0, s, a2);
-        if (e != cudaSuccess) return cuda_fail(e, "apply_w2_warp_kernel launch");
-        if ((st = after_launch("apply_w2_warp_kernel")) != LRC_OK) return st;
+        e = launch_pdl(apply_w2_slice_kernel, dim3((unsigned)(btiles * 4 * (kp / 8))), dim3(32 * kW2Slices), 0, s,
+                       a2);
+        if (e != cudaSuccess) return cuda_fail(e, "apply_w2_slice_kernel launch");
+        if ((st = after_launch("apply_w2_slice_kernel")) != LRC_OK) return st;
     } else {
         e = launch_pdl(apply_w2_kernel, dim3((unsigned)((n2items + 255) / 256)), dim3(256), 0, s, a2);
         if (e != cudaSuccess) return cuda_fail(e, "apply_w2_kernel launch");
@@ -929,6 +974,15 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
     }
 
     return launch_y(tu, ty, a3, smem3, P3, s);
+}
+
+lrc_status encode_map_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, int64_t cols, int64_t rows,
+                         int64_t pitch_bytes, uint32_t box_cols, uint32_t box_rows, bool swizzle128,
+                         const char* what) {
+    lrc_status st = get_encoder();
+    if (st != LRC_OK) return st;
+    return make_map(map, dt, base, cols, rows, pitch_bytes, box_cols, box_rows, what,
+                    swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
 lrc_status y_product_plan(int64_t m, int64_t b, int kp, bool out16, int* n2) {

@@ -1,6 +1,7 @@
 // common.cuh -- internal helpers shared by the translation units of liblrc.so.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -81,9 +82,9 @@ lrc_status launch_apply_split_f32(const float* U, const float* S, const float* V
                                   int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
 lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y,
                             int64_t m, int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s);
-// batches of at most apply_skinny_max_batch(fmt) queries, ranks up to 1024,
-// every format (apply_skinny.cu)
-int64_t apply_skinny_max_batch(lrc_fmt fmt);
+// small batches (at most 16 queries for binary32, 4 otherwise), ranks up to
+// 1024 whose tiles fit in shared memory, every format (apply_skinny.cu)
+bool apply_skinny_takes(lrc_fmt fmt, int64_t b, int64_t k);
 lrc_status launch_apply_skinny(const void* U, const void* S, const void* Vt, const void* X, void* Y, int64_t m,
                                int64_t n, int64_t k, int64_t b, lrc_fmt fmt, cudaStream_t s);
 
@@ -138,6 +139,13 @@ lrc_status launch_tt_side_f32(const TTShape& sh, float* out, cudaStream_t s, boo
 // bond at which the product chain of tt_chain.cu meets
 int tt_chain_bond(const TTShape& sh);
 
+// 2-D TMA map over a row-major [rows x cols] array with a row pitch of
+// `pitch_bytes`: boxes of box_cols x box_rows elements, 128-byte swizzle or
+// none, elements outside the array read as zero.
+lrc_status encode_map_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, int64_t cols, int64_t rows,
+                         int64_t pitch_bytes, uint32_t box_cols, uint32_t box_rows, bool swizzle128,
+                         const char* what);
+
 // Device error words of the tensor-core kernels (bounded waits that gave up);
 // read and cleared by lrc_device_status().  0xffffffff = could not be read.
 uint32_t take_apply_tc_error();
@@ -150,6 +158,7 @@ lrc_status launch_tt3_f16_tc(const TTShape& sh, bool out16, void* out, cudaStrea
 // *handled = false when the shape is outside the kernel (nothing launched).
 lrc_status launch_ttn_f16_tc(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled);
 uint32_t take_ttn_tc_error();
+uint32_t take_skinny_error();
 lrc_status launch_wait_timeout_probe(int64_t limit_ns, cudaStream_t s);
 
 lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
