@@ -80,7 +80,8 @@ struct W1Args {
     int chunk_blocks;
     int stages;
     uint32_t slot_bytes;
-    uint32_t sum_off, bar_off;
+    uint32_t bar_off;
+    uint32_t sum_col;         // tensor-memory column of the running sum (FP32 output)
     uint32_t tmem_cols;
     float* P;                 // partials: [segment id][kgp columns][128 rows]
     const void* upf;          // optional: buffer (U) that the CTAs prefetch into L2 for the next product
@@ -165,8 +166,13 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
                     const int nb = (q1 - qs >= kStageBlocks) ? kStageBlocks : (int)(q1 - qs);
                     // L2 prefetch of X and V^T in 512-byte-wide rows (four k-blocks),
                     // up to two groups ahead, so that the operand boxes (128-byte
-                    // rows) hit L2
-                    for (int u = 0; u < nb; ++u) {
+                    // rows) hit L2.  Only first touches are prefetched: X by the
+                    // CTAs of column group 0 (those of the other groups read the
+                    // same tile side by side), V^T on the first row tile (it stays
+                    // in L2 for the others) -- a prefetch of a resident line still
+                    // costs an L2 transaction, and L2 is this kernel's busiest unit.
+                    const bool pf_x = grp == 0, pf_v = bt == 0;
+                    for (int u = 0; u < nb && (pf_x || pf_v); ++u) {
                         const int64_t kb = qs + u - rbase;
                         const bool seg_first = (qs + u == qbeg) || (kb == 0);
                         if (!seg_first && (kb & (kPfBlocks - 1)) != 0) continue;
@@ -174,8 +180,8 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
                         for (int64_t pg = seg_first ? g0 : g0 + 2; pg <= g0 + 2; ++pg) {
                             const int64_t pkb = pg * kPfBlocks;
                             if (rbase + pkb >= seg_end) break;
-                            tma_prefetch_2d(&tm_xp, (int32_t)(pkb * BK), (int32_t)(bt * BM));
-                            tma_prefetch_2d(&tm_vp, (int32_t)(pkb * BK), grp * a.kgp);
+                            if (pf_x) tma_prefetch_2d(&tm_xp, (int32_t)(pkb * BK), (int32_t)(bt * BM));
+                            if (pf_v) tma_prefetch_2d(&tm_vp, (int32_t)(pkb * BK), grp * a.kgp);
                         }
                     }
                     const int slot = it % a.stages;
@@ -250,7 +256,6 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
         const int g = warp & 3;
         const int r = g * 32 + lane;
         const uint32_t lane_base = (uint32_t)(g * 32) << 16;
-        float* sum = reinterpret_cast<float*>(smem + a.sum_off);     // [column][128 rows]
         int ci = 0;
         int64_t q = qbeg, q0, q1, row;
         bool first, last;
@@ -269,25 +274,23 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
             for (int c0 = 0; c0 < kgw; c0 += 32) {
                 uint32_t v[32];
                 tmem_ld32(tmem + lane_base + (uint32_t)(buf * a.kgp + c0), v);
-                tmem_ld_wait();
                 const int nj = (c0 + 32 <= kgw) ? 32 : 16;     // group widths are multiples of 16
-                float* sp = sum + c0 * BM + r;
+                // running sum of the segment's chunks: 32 tensor-memory columns per
+                // 32 accumulator columns (the region is a whole number of 32-column
+                // pieces, so the pieces past the group width are scratch)
+                const uint32_t sp = tmem + lane_base + a.sum_col + (uint32_t)c0;
                 if (!first) {
+                    uint32_t sv[32];
+                    tmem_ld32(sp, sv);
+                    tmem_ld_wait();
 #pragma unroll
-                    for (int j = 0; j < 16; ++j) v[j] = __float_as_uint(__fadd_rn(sp[j * BM], __uint_as_float(v[j])));
-                    if (nj == 32) {
-#pragma unroll
-                        for (int j = 16; j < 32; ++j)
-                            v[j] = __float_as_uint(__fadd_rn(sp[j * BM], __uint_as_float(v[j])));
-                    }
+                    for (int j = 0; j < 32; ++j)
+                        v[j] = __float_as_uint(__fadd_rn(__uint_as_float(sv[j]), __uint_as_float(v[j])));
+                } else {
+                    tmem_ld_wait();
                 }
                 if (!last) {
-#pragma unroll
-                    for (int j = 0; j < 16; ++j) sp[j * BM] = __uint_as_float(v[j]);
-                    if (nj == 32) {
-#pragma unroll
-                        for (int j = 16; j < 32; ++j) sp[j * BM] = __uint_as_float(v[j]);
-                    }
+                    tmem_st32(sp, v);
                 } else if (valid) {
                     float* pp = prow + (size_t)c0 * BM;
 #pragma unroll
@@ -298,6 +301,7 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
                     }
                 }
             }
+            tmem_st_wait();
             tc_fence_before();
             mbar_arrive(&acc_empty[buf]);
             ++ci;
@@ -876,18 +880,14 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
     a1.chunk_blocks = out16 ? (int)(a1.nkb < 0x7fffffff ? a1.nkb : 0x7fffffff) : kChunkBlocks;
     const bool use_sum = a1.chunk_blocks < a1.nkb;
     a1.slot_bytes = (uint32_t)round_up((size_t)kStageBlocks * (kXBytes + (size_t)a1.kgp * 128), 1024);
-    const uint32_t sum_bytes = use_sum ? (uint32_t)BM * a1.kgp * 4 : 0;
     size_t smem1 = 0;
     for (int stages = 6; stages >= 2; --stages) {
         size_t off = (size_t)stages * a1.slot_bytes;
-        const size_t sum_off = off;
-        off += sum_bytes;
         off = round_up(off, 8);
         const size_t bar_off = off;
         off += (size_t)(2 * stages + 5) * 8 + 16;
         if (off + 1024 <= kSmemMax) {
             a1.stages = stages;
-            a1.sum_off = (uint32_t)sum_off;
             a1.bar_off = (uint32_t)bar_off;
             smem1 = off + 1024;
             break;
@@ -897,8 +897,15 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
         set_error("binary16 apply: rank %lld does not fit in shared memory", (long long)k);
         return LRC_ERR_UNSUPPORTED;
     }
-    // two accumulators at columns 0 and kgp; the epilogue reads 32 columns at a time
-    a1.tmem_cols = pow2_cols((uint32_t)a1.kgp + (uint32_t)round_up((size_t)a1.kgp, 32));
+    // two accumulators at columns 0 and kgp; the epilogue reads 32 columns at a
+    // time; the running sum of FP32 output follows in whole 32-column pieces
+    const uint32_t acc_cols = (uint32_t)a1.kgp + (uint32_t)round_up((size_t)a1.kgp, 32);
+    a1.sum_col = (uint32_t)round_up(acc_cols, 32);
+    a1.tmem_cols = pow2_cols(use_sum ? a1.sum_col + (uint32_t)round_up((size_t)a1.kgp, 32) : acc_cols);
+    if (a1.tmem_cols > 512) {
+        set_error("binary16 apply: rank %lld does not fit in tensor memory", (long long)k);
+        return LRC_ERR_UNSUPPORTED;
+    }
     const int64_t P1 = a1.Q < sms ? a1.Q : sms;
 
     // ---- phase-2 plan: tile width, ring depth
