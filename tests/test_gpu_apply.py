@@ -139,3 +139,25 @@ def test_small_batch_kernels_vs_oracle(lrc, cuda, fmt, m, n, k, b):
     want = oracle.apply(*oracle_inputs(f.U, f.s, f.Vt, X, fmt))
     err = rel_fro(got, want)
     assert err <= TOL[fmt], (fmt, err)
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("b", [1, 4, 16, 200, 3000])
+def test_apply_bitwise_reproducible(lrc, cuda, fmt, b):
+    """Every batch regime (small-batch streams, split products, the
+    tensor-core path with its sliced partial reduction, stream-K partials)
+    adds in a fixed order: two calls on the same inputs agree bit for bit,
+    with other work queued on the stream in between."""
+    m, n, k = 700, 2100, 72
+    f = W.random_factors(m, n, k, seed=b + 41)
+    X = W.gaussian((b, n), b + 42)
+    Ud, Sd, Vd, Xd = (packed(lrc, a, fmt, cuda) for a in (f.U, f.s, f.Vt, X))
+    outs = []
+    for _ in range(2):
+        Y = torch.full((b, m), float("nan"), dtype=lrc.output_dtype(fmt), device=cuda)
+        lrc.lrc_apply(Ud, Sd, Vd, Xd, Y, m, n, k, b, fmt)
+        torch.empty(1 << 22, device=cuda).uniform_()       # unrelated work between the calls
+        outs.append(Y.clone())
+    assert lrc.lrc_device_status() == 0
+    assert torch.equal(outs[0].view(torch.int8), outs[1].view(torch.int8)), (fmt, b)
+    assert not torch.isnan(outs[0].double()).any()

@@ -124,3 +124,18 @@ def test_large_interior_cores_vs_oracle(lrc, cuda, fmt, dims, ranks):
     err = rel_fro(got, want)
     assert err <= TOL[fmt], (fmt, err)
     assert np.isfinite(got).all()
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("dims,ranks", [
+    ((64, 48, 80), (1, 12, 9, 1)),           # 3-way, wide last mode
+    ((8, 8, 8, 8, 8), (1, 6, 7, 7, 6, 1)),   # narrow modes, chain meeting in the middle
+])
+def test_tt_bitwise_reproducible(lrc, cuda, fmt, dims, ranks):
+    """Two reconstructions of the same cores agree bit for bit."""
+    cores = [W.gaussian((ranks[l], dims[l], ranks[l + 1]), 90 + l) for l in range(len(dims))]
+    a, _ = run_tt(lrc, cuda, cores, fmt)
+    torch.empty(1 << 22, device=cuda).uniform_()
+    b, _ = run_tt(lrc, cuda, cores, fmt)
+    assert np.array_equal(a.view(np.uint64), b.view(np.uint64)), fmt
+    assert np.isfinite(a).all()
