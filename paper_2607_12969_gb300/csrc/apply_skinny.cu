@@ -38,8 +38,7 @@ namespace {
 
 constexpr int kWarps = 8;
 constexpr int kThreadsS = 32 * kWarps;
-constexpr int kRows = 4;                      // factor rows per warp
-constexpr int kBlockRows = kWarps * kRows;    // factor rows per CTA
+constexpr int kRows = 4;                      // factor rows per warp (first product: 2 for 16 binary64 queries)
 constexpr int kBox = 256;                     // columns per TMA box of the first product
 constexpr size_t kSmemW1 = 100 * 1024;        // shared-memory budget of a first-product CTA
 constexpr size_t kSmemMaxS = 220 * 1024;      // largest dynamic shared memory a CTA asks for
@@ -179,63 +178,65 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
 }
 
 // ---------------------------------------------------------------- phase 1
-// Shared memory: [X boxes: nbox x B x kBox][V^T boxes: nbox x 32 x kBox]
+// Shared memory: [X boxes: nbox x B x kBox][V^T boxes: nbox x 8 RW x kBox]
 // [a barrier per box pair][abort flag]; column i of the chunk is box i / kBox,
-// offset i % kBox.  The boxes are multiplied in order as they land.
-template <typename TS, typename T, int B>
+// offset i % kBox.  The boxes are multiplied in order as they land.  RW rows
+// of V^T per warp.
+template <typename TS, typename T, int B, int RW>
 __global__ void __launch_bounds__(kThreadsS, 2)
 skinny_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_v, int k, int b,
                  int L, T* __restrict__ Wp, const void* upf, uint64_t upf_bytes) {
     constexpr int EV = EVof<TS>::v;
+    constexpr int BR = kWarps * RW;              // rows of V^T per CTA
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = align128(smem_raw);
     const int nbox = L / kBox;
     TS* xs = reinterpret_cast<TS*>(smem);
     TS* vs = xs + (size_t)nbox * B * kBox;
-    uint64_t* bar = reinterpret_cast<uint64_t*>(vs + (size_t)nbox * kBlockRows * kBox);
+    uint64_t* bar = reinterpret_cast<uint64_t*>(vs + (size_t)nbox * BR * kBox);
     volatile int* abort = reinterpret_cast<volatile int*>(bar + nbox);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t chunk = blockIdx.x;
     const int32_t i0 = (int32_t)(chunk * L);
-    const int jb = (int)blockIdx.y * kBlockRows;
+    const int jb = (int)blockIdx.y * BR;
     if (threadIdx.x == 0) {
         for (int q = 0; q < nbox; ++q) tc::mbar_init(&bar[q], 1);
         *abort = 0;
         tc::fence_barrier_init();
         for (int q = 0; q < nbox; ++q) {
-            tc::mbar_arrive_expect_tx(&bar[q], (uint32_t)((B + kBlockRows) * kBox * (int)sizeof(TS)));
-            tc::tma_load_2d(vs + (size_t)q * kBlockRows * kBox, &tm_v, i0 + q * kBox, jb, &bar[q]);
+            tc::mbar_arrive_expect_tx(&bar[q], (uint32_t)((B + BR) * kBox * (int)sizeof(TS)));
+            tc::tma_load_2d(vs + (size_t)q * BR * kBox, &tm_v, i0 + q * kBox, jb, &bar[q]);
             tc::tma_load_2d(xs + (size_t)q * B * kBox, &tm_x, i0 + q * kBox, 0, &bar[q]);
         }
         // U, read by the last kernel, comes into L2 alongside this kernel's stream
         if (upf) tc::bulk_prefetch_share(upf, upf_bytes, blockIdx.y * gridDim.x + blockIdx.x, gridDim.x * gridDim.y);
     }
     __syncthreads();
-    const int jl = warp * kRows;                 // first local row of the warp
-    T acc[kRows * B];                            // acc[r * B + c]: row jl + r, query c
+    const int jl = warp * RW;                 // first local row of the warp
+    T acc[RW * B];                            // acc[r * B + c]: row jl + r, query c
 #pragma unroll
-    for (int i = 0; i < kRows * B; ++i) acc[i] = T(0);
+    for (int i = 0; i < RW * B; ++i) acc[i] = T(0);
     for (int q = 0; q < nbox; ++q) {
         if (!wait_tiles(bar, q, nbox, abort, 1u)) return;
-        const TS* vq = vs + ((size_t)q * kBlockRows + jl) * kBox;
+        const TS* vq = vs + ((size_t)q * BR + jl) * kBox;
         const TS* xq = xs + (size_t)q * B * kBox;
         for (int o = lane * EV; o < kBox; o += 32 * EV) {
-            T vv[kRows][EV];
+            T vv[RW][EV];
 #pragma unroll
-            for (int r = 0; r < kRows; ++r) load_vec<T, TS>(vq + (size_t)r * kBox + o, vv[r]);
+            for (int r = 0; r < RW; ++r) load_vec<T, TS>(vq + (size_t)r * kBox + o, vv[r]);
 #pragma unroll
             for (int c = 0; c < B; ++c) {
                 T xv[EV];
                 load_vec<T, TS>(xq + (size_t)c * kBox + o, xv);
 #pragma unroll
-                for (int r = 0; r < kRows; ++r)
+                for (int r = 0; r < RW; ++r)
 #pragma unroll
                     for (int e = 0; e < EV; ++e) acc[r * B + c] = fma(xv[e], vv[r][e], acc[r * B + c]);
             }
         }
     }
     tc::pdl_trigger();
-    constexpr int N = kRows * B;
+    constexpr int N = RW * B;
     halving_sum<T, N, 32>(acc, lane);
     if (halving_writer<N, 32>(lane)) {
         const int base = halving_index<N, 32>(lane);
@@ -351,6 +352,10 @@ skinny_y_kernel(const __grid_constant__ CUtensorMap tm_u, const T* __restrict__ 
 template <typename TS>
 constexpr int y_rpg() { return sizeof(TS) == 8 ? 2 : 4; }
 
+// rows of V^T per warp in the first product: 4, or 2 for 16 binary64 queries
+// (64 binary64 accumulators a thread would spill)
+constexpr int w1_rows(int B, int64_t e) { return (B == 16 && e == 8) ? 2 : kRows; }
+
 template <typename TS>
 CUtensorMapDataType map_type() {
     if constexpr (sizeof(TS) == 2) return CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
@@ -366,13 +371,14 @@ struct SkinnyPlan {
 };
 
 SkinnyPlan plan_skinny(int64_t m, int64_t n, int64_t k, int B, int64_t e, int64_t et) {
+    const int64_t br = kWarps * (int64_t)w1_rows(B, e);
     SkinnyPlan p{};
     const int64_t ev = 16 / e;
     // chunk length: a multiple of kBox with the CTA's tiles within the
     // shared-memory budget (two CTAs per SM), and enough chunks for two CTAs
     // per SM
-    p.jblocks = (k + kBlockRows - 1) / kBlockRows;
-    int64_t L = (int64_t)(kSmemW1 / (size_t)((B + kBlockRows) * e)) / kBox * kBox;
+    p.jblocks = (k + br - 1) / br;
+    int64_t L = (int64_t)(kSmemW1 / (size_t)((B + br) * e)) / kBox * kBox;
     if (L < kBox) L = kBox;
     const int64_t want = (2 * (int64_t)sm_count() + p.jblocks - 1) / p.jblocks;
     int64_t Lw = (n + want - 1) / want;
@@ -385,7 +391,7 @@ SkinnyPlan plan_skinny(int64_t m, int64_t n, int64_t k, int B, int64_t e, int64_
     p.nkb = (k + 255) / 256;
     p.kbw = ((k + p.nkb - 1) / p.nkb + ev - 1) / ev * ev;
     p.kv = p.nkb * p.kbw;
-    p.smem1 = (size_t)(L / kBox) * (B + kBlockRows) * kBox * e + 8 * (size_t)(L / kBox + 1) + 128;
+    p.smem1 = (size_t)(L / kBox) * (B + br) * kBox * e + 8 * (size_t)(L / kBox + 1) + 128;
     // second product: CTAs of 16 RPG rows of U
     const int64_t rc = (int64_t)kYWarps * (32 / kYGroup) * (e == 8 ? 2 : 4);
     p.yblocks = (m + rc - 1) / rc;
@@ -415,17 +421,18 @@ lrc_status launch_skinny_b(const TS* U, const TS* S, const TS* Vt, const TS* X, 
 
     CUtensorMap tx, tv, tu;
     if ((st = encode_map_2d(&tx, map_type<TS>(), X, n, b, ldn * e, kBox, B, false, "X")) != LRC_OK) return st;
-    if ((st = encode_map_2d(&tv, map_type<TS>(), Vt, n, k, ldn * e, kBox, kBlockRows, false, "Vt")) != LRC_OK)
+    constexpr int RW = w1_rows(B, (int64_t)sizeof(TS));
+    if ((st = encode_map_2d(&tv, map_type<TS>(), Vt, n, k, ldn * e, kBox, kWarps * RW, false, "Vt")) != LRC_OK)
         return st;
     constexpr int kRowsY = kYWarps * (32 / kYGroup) * y_rpg<TS>();
     if ((st = encode_map_2d(&tu, map_type<TS>(), U, k, m, ldk * e, (uint32_t)p.kbw, kRowsY, false, "U")) != LRC_OK)
         return st;
 
-    cudaError_t ce = cudaFuncSetAttribute(skinny_w1_kernel<TS, T, B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)p.smem1);
+    cudaError_t ce = cudaFuncSetAttribute(skinny_w1_kernel<TS, T, B, RW>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem1);
     if (ce != cudaSuccess) return cuda_fail(ce, "skinny_w1_kernel smem attribute");
     const uint64_t u_bytes = ((uint64_t)(m - 1) * (uint64_t)ldk + (uint64_t)k) * (uint64_t)e;
-    skinny_w1_kernel<TS, T, B><<<dim3((unsigned)p.nchunks, (unsigned)p.jblocks), kThreadsS, p.smem1, s>>>(
+    skinny_w1_kernel<TS, T, B, RW><<<dim3((unsigned)p.nchunks, (unsigned)p.jblocks), kThreadsS, p.smem1, s>>>(
         tx, tv, (int)k, (int)b, (int)p.L, Wp, u_bytes <= kPrefetchMaxBytes ? (const void*)U : nullptr, u_bytes);
     if ((st = after_launch("skinny_w1_kernel")) != LRC_OK) return st;
     ce = launch_pdl(skinny_w2_kernel<TS, T>, dim3((unsigned)((b * p.kv * 32 + 255) / 256)), dim3(256), 0, s,
@@ -446,21 +453,23 @@ lrc_status launch_skinny_t(const TS* U, const TS* S, const TS* Vt, const TS* X, 
                            int64_t k, int64_t b, bool round16, cudaStream_t s) {
     if (b <= 1) return launch_skinny_b<TS, T, TOut, 1>(U, S, Vt, X, Y, m, n, k, b, round16, s);
     if (b <= 4) return launch_skinny_b<TS, T, TOut, 4>(U, S, Vt, X, Y, m, n, k, b, round16, s);
-    if constexpr (sizeof(TS) == 4) return launch_skinny_b<TS, T, TOut, 16>(U, S, Vt, X, Y, m, n, k, b, round16, s);
+    if constexpr (sizeof(TS) != 2)
+        if (b <= 8) return launch_skinny_b<TS, T, TOut, 8>(U, S, Vt, X, Y, m, n, k, b, round16, s);
+    if constexpr (sizeof(TS) != 2) return launch_skinny_b<TS, T, TOut, 16>(U, S, Vt, X, Y, m, n, k, b, round16, s);
     set_error("small-batch apply: b = %lld above the kernel's batch", (long long)b);
     return LRC_ERR_UNSUPPORTED;
 }
 
-int64_t max_batch(lrc_fmt fmt) { return fmt == LRC_F32 ? 16 : 4; }
+int64_t max_batch(lrc_fmt fmt) { return fmt == LRC_F16 || fmt == LRC_F16_O16 ? 4 : 16; }
 
 }  // namespace
 
-// Batches this path takes: up to 16 queries for binary32; binary64
-// (DFMA-bound from a few queries on) and binary16 (whose tensor-core path is
-// faster from 16 queries on) up to 4; ranks whose tiles fit in shared memory.
+// Batches this path takes: up to 16 queries for binary32 and binary64, up
+// to 4 for binary16 (whose tensor-core path is faster from 16 queries on);
+// ranks whose tiles fit in shared memory.
 bool apply_skinny_takes(lrc_fmt fmt, int64_t b, int64_t k) {
     if (b < 1 || b > max_batch(fmt) || k < 1 || k > 1024) return false;
-    const int B = b <= 1 ? 1 : (b <= 4 ? 4 : 16);
+    const int B = b <= 1 ? 1 : (b <= 4 ? 4 : (b <= 8 ? 8 : 16));
     const int64_t e = storage_bytes(fmt);
     const SkinnyPlan p = plan_skinny(1, 1, k, B, e, fmt == LRC_F64 ? 8 : 4);
     return p.smem1 <= kSmemMaxS && p.smem3 <= kSmemMaxS;

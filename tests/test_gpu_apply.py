@@ -129,7 +129,9 @@ def test_large_batch_integer_exact(lrc, cuda, fmt, m, n, k, b):
     (64, 7, 3, 16),            # n shorter than one vector row, largest batch of the small-batch kernels
     (1000, 5000, 272, 16),     # several n-chunks with a ragged last chunk
     (4097, 2049, 1024, 2),     # largest rank of the small-batch kernels
-    (517, 3001, 100, 4),       # largest batch of the small-batch kernels for FP64 and FP16
+    (517, 3001, 100, 4),       # largest batch of the small-batch kernels for FP16
+    (600, 2500, 200, 12),      # 16-query kernels (two rows of V^T per warp for FP64)
+    (301, 777, 45, 8),         # 8-query kernels
     (257, 129, 19, 1),         # single query, ragged everything
 ])
 def test_small_batch_kernels_vs_oracle(lrc, cuda, fmt, m, n, k, b):
