@@ -72,9 +72,13 @@ def load_peaks():
 
 
 PEAKS = load_peaks()
-E = {"f64": 8, "f32": 4, "f16": 2, "f16_o16": 2}
-E_OUT = {"f64": 8, "f32": 4, "f16": 4, "f16_o16": 2}
-ALU = {"f64": "f64", "f32": "f32", "f16": "f16", "f16_o16": "f16"}
+E = {"f64": 8, "f32": 4, "f16": 2, "f16_o16": 2, "f32tc": 4}
+E_OUT = {"f64": 8, "f32": 4, "f16": 4, "f16_o16": 2, "f32tc": 4}
+ALU = {"f64": "f64", "f32": "f32", "f16": "f16", "f16_o16": "f16", "f32tc": None}
+# LRC_F32_TC: binary32 storage; the output product on the tensor cores as
+# three binary16 products (hi/lo split), the rest on the CUDA cores.  Its
+# arithmetic bound is the sum of the two engines' times (alu_time).
+F32TC_PASSES = 3
 
 
 # ---------------------------------------------------------------------------
@@ -97,8 +101,11 @@ def work_widen(rows, cols, ld, fmt):
 
 
 def work_apply(m, n, k, b, fmt):
-    return {"bytes": (m + n + 1) * k * E[fmt] + b * n * E[fmt] + b * m * E_OUT[fmt],
-            "flops": 2 * (m + n) * k * b + k * b, "alu": ALU[fmt]}
+    w = {"bytes": (m + n + 1) * k * E[fmt] + b * n * E[fmt] + b * m * E_OUT[fmt],
+         "flops": 2 * (m + n) * k * b + k * b, "alu": ALU[fmt]}
+    if fmt == "f32tc":
+        w["alu_time"] = 2 * n * k * b / PEAKS["f32"] + F32TC_PASSES * 2 * m * k * b / PEAKS["f16"]
+    return w
 
 
 def tt_chain_flops(dims, ranks):
@@ -126,7 +133,13 @@ def tt_chain_flops(dims, ranks):
 def work_tt(dims, ranks, fmt):
     cores = sum(ranks[l] * dims[l] * ranks[l + 1] for l in range(len(dims)))
     N = int(np.prod(dims))
-    return {"bytes": cores * E[fmt] + N * E_OUT[fmt], "flops": tt_chain_flops(dims, ranks), "alu": ALU[fmt]}
+    w = {"bytes": cores * E[fmt] + N * E_OUT[fmt], "flops": tt_chain_flops(dims, ranks), "alu": ALU[fmt]}
+    if fmt == "f32tc":
+        # the output product (2 N r_c at the chain's bond) on the tensor cores,
+        # the side products on the CUDA cores
+        out = min(2 * N * ranks[c] for c in range(1, len(dims)))
+        w["alu_time"] = (w["flops"] - out) / PEAKS["f32"] + F32TC_PASSES * out / PEAKS["f16"]
+    return w
 
 
 def work_eta_lowrank(m, n, k, fmt):
@@ -164,6 +177,8 @@ def roofline_time(w):
     t = w["bytes"] / PEAKS["hbm"]
     if w["alu"]:
         t = max(t, w["flops"] / PEAKS[w["alu"]])
+    if "alu_time" in w:
+        t = max(t, w["alu_time"])
     return t
 
 
@@ -556,7 +571,7 @@ def run_case(args):
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     fmt = args.fmt
-    base = "f16" if fmt.startswith("f16") else fmt
+    base = "f16" if fmt.startswith("f16") else ("f32" if fmt == "f32tc" else fmt)
     if args.case == "apply":
         m, n, b, k = args.m, args.n, args.b, args.k
         f = W.random_factors(m, n, k, seed=7)

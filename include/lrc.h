@@ -47,8 +47,14 @@ typedef enum {
     LRC_F64 = 0,      /* binary64 storage, binary64 arithmetic, binary64 output             */
     LRC_F32 = 1,      /* binary32 storage, binary32 FMA arithmetic, binary32 output         */
     LRC_F16 = 2,      /* binary16 storage, binary32 accumulation, binary32 output           */
-    LRC_F16_O16 = 3   /* binary16 storage, binary32 accumulation, binary16 workspaces and
+    LRC_F16_O16 = 3,  /* binary16 storage, binary32 accumulation, binary16 workspaces and
                          output: the method-precision FP16 path of Sec. 3.4                 */
+    LRC_F32_TC = 4    /* binary32 storage and output; the output product of lrc_apply and
+                         tt_reconstruct on the tensor cores: each binary32 operand is scaled
+                         by a power of two per 32 rows and split into binary16 parts
+                         hi + lo, and Z S ~ Z_hi S_hi + Z_lo S_hi + Z_hi S_lo accumulates in
+                         binary32 (about 22 significand bits per operand).  A variant of
+                         LRC_F32; every other call treats it as LRC_F32                      */
 } lrc_fmt;
 
 typedef enum {
@@ -130,6 +136,8 @@ LRC_API lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows,
  * different streams use different buffers.  Binary16 ranks: up to 320 for
  * LRC_F16 and 512 for LRC_F16_O16, else LRC_ERR_UNSUPPORTED.
  */
+/* LRC_F32_TC: as LRC_F32, with the second product (W U^T) on the tensor
+ * cores when b > 32 and k <= 192; otherwise the LRC_F32 kernels. */
 LRC_API lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X, void* Y,
                      int64_t m, int64_t n, int64_t k, int64_t b, lrc_fmt fmt,
                      lrc_stream_t stream);
@@ -152,6 +160,9 @@ LRC_API lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const
  * out.  Cores must be aligned to their element size, out to 16 bytes.
  * Intermediate products Z_l stay on chip.  Asynchronous on `stream`.
  */
+/* LRC_F32_TC: binary32 cores and output; the chain's output product on the
+ * tensor cores when the chain's sides fit its one-pass side kernel
+ * (bond rank <= 64), otherwise the LRC_F32 kernels. */
 LRC_API lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims, const int64_t* ranks,
                           int d, lrc_fmt fmt, void* out, lrc_stream_t stream);
 

@@ -19,8 +19,8 @@ from typing import Optional, Sequence, Tuple
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "liblrc.so")
 
-F64, F32, F16, F16_O16 = 0, 1, 2, 3
-FORMATS = {"f64": F64, "f32": F32, "f16": F16, "f16_o16": F16_O16}
+F64, F32, F16, F16_O16, F32_TC = 0, 1, 2, 3, 4
+FORMATS = {"f64": F64, "f32": F32, "f16": F16, "f16_o16": F16_O16, "f32tc": F32_TC}
 STATUS = {0: "ok", -1: "invalid argument", -2: "misaligned pointer", -3: "unsupported",
           -4: "CUDA error", -5: "out of memory", -6: "device wait timed out"}
 
@@ -94,13 +94,15 @@ def _fmt(fmt) -> int:
 def storage_dtype(fmt):
     import torch
     f = _fmt(fmt)
-    return {F64: torch.float64, F32: torch.float32, F16: torch.float16, F16_O16: torch.float16}[f]
+    return {F64: torch.float64, F32: torch.float32, F16: torch.float16, F16_O16: torch.float16,
+            F32_TC: torch.float32}[f]
 
 
 def output_dtype(fmt):
     import torch
     f = _fmt(fmt)
-    return {F64: torch.float64, F32: torch.float32, F16: torch.float32, F16_O16: torch.float16}[f]
+    return {F64: torch.float64, F32: torch.float32, F16: torch.float32, F16_O16: torch.float16,
+            F32_TC: torch.float32}[f]
 
 
 def _check(status: int) -> None:

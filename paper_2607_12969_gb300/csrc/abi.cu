@@ -105,6 +105,7 @@ int64_t lrc_packed_ld(int64_t cols) {
 lrc_status lrc_round_factors(const double* src, int64_t rows, int64_t cols, int64_t ld_src,
                              void* dst, int64_t ld_dst, lrc_fmt fmt, lrc_stream_t stream) {
     if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    fmt = plain_fmt(fmt);
     if (rows < 0 || cols < 0) return invalid("negative size (rows=%lld cols=%lld)", (long long)rows, (long long)cols);
     if (ld_src < cols || ld_dst < cols) return invalid("leading dimension below cols");
     if (rows == 0 || cols == 0) return LRC_OK;
@@ -120,6 +121,7 @@ lrc_status lrc_round_factors(const double* src, int64_t rows, int64_t cols, int6
 lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows, int64_t cols,
                              int64_t ld_src, double* dst, int64_t ld_dst, lrc_stream_t stream) {
     if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    fmt = plain_fmt(fmt);
     if (rows < 0 || cols < 0) return invalid("negative size");
     if (ld_src < cols || ld_dst < cols) return invalid("leading dimension below cols");
     if (rows == 0 || cols == 0) return LRC_OK;
@@ -152,15 +154,16 @@ lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X
     if (!aligned16(X)) return misaligned("X");
     if (!aligned16(Y)) return misaligned("Y");
     cudaStream_t s = as_stream(stream);
-    if (apply_skinny_takes(fmt, b, k))
-        return launch_apply_skinny(U, S, Vt, X, Y, m, n, k, b, fmt, s);
+    if (apply_skinny_takes(plain_fmt(fmt), b, k))
+        return launch_apply_skinny(U, S, Vt, X, Y, m, n, k, b, plain_fmt(fmt), s);
     switch (fmt) {
         case LRC_F64:
             return launch_apply_f64((const double*)U, (const double*)S, (const double*)Vt,
                                     (const double*)X, (double*)Y, m, n, k, b, s);
         case LRC_F32:
+        case LRC_F32_TC:
             return launch_apply_f32((const float*)U, (const float*)S, (const float*)Vt,
-                                    (const float*)X, (float*)Y, m, n, k, b, s);
+                                    (const float*)X, (float*)Y, m, n, k, b, fmt == LRC_F32_TC, s);
         case LRC_F16:
         case LRC_F16_O16:
             return launch_apply_f16(U, S, Vt, X, Y, m, n, k, b, fmt == LRC_F16_O16, s);
@@ -180,7 +183,12 @@ lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims, const i
     if (!aligned16(out)) return misaligned("out");
     cudaStream_t s = as_stream(stream);
     if (fmt == LRC_F16 || fmt == LRC_F16_O16) return launch_tt_f16(sh, fmt == LRC_F16_O16, out, s);
-    if (fmt == LRC_F32) return launch_tt_chain_f32(sh, static_cast<float*>(out), s);
+    if (fmt == LRC_F32_TC) {
+        bool handled = false;
+        st = launch_tt_split_f32tc(sh, static_cast<float*>(out), s, &handled);
+        if (st != LRC_OK || handled) return st;
+    }
+    if (fmt == LRC_F32 || fmt == LRC_F32_TC) return launch_tt_chain_f32(sh, static_cast<float*>(out), s);
     if (tt_chain_saves(sh)) return launch_tt_chain_f64(sh, static_cast<double*>(out), s);
     return launch_tt_cc(sh, fmt, out, s);
 }
@@ -188,6 +196,7 @@ lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims, const i
 lrc_status tt_gather(const void* const* cores, const int64_t* dims, const int64_t* ranks, int d, lrc_fmt fmt,
                      const int64_t* idx, int64_t count, void* out, lrc_stream_t stream) {
     if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    fmt = plain_fmt(fmt);
     if (count < 0) return invalid("negative count");
     TTShape sh;
     lrc_status st = tt_shape(cores, dims, ranks, d, storage_bytes(fmt), "cores", &sh);
@@ -218,6 +227,7 @@ lrc_status lrc_lowrank_eta(const double* U, const double* S, const double* Vt, c
                            const void* Vht, lrc_fmt fmt, int64_t m, int64_t n, int64_t k, double* eta_out,
                            double* norm_out, lrc_stream_t stream) {
     if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    fmt = plain_fmt(fmt);
     if (m <= 0 || n <= 0 || k <= 0)
         return invalid("sizes must be positive (m=%lld n=%lld k=%lld)", (long long)m, (long long)n, (long long)k);
     if (k > 4096) return invalid("k = %lld exceeds 4096", (long long)k);
@@ -240,6 +250,7 @@ lrc_status lrc_tt_eta(const double* const* cores, const void* const* cores_hat, 
                       const int64_t* ranks, int d, lrc_fmt fmt, double* eta_out, double* norm_out,
                       lrc_stream_t stream) {
     if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    fmt = plain_fmt(fmt);
     if (!eta_out) return invalid("null eta_out");
     TTShape sh, shh;
     lrc_status st = tt_shape((const void* const*)cores, dims, ranks, d, 8, "cores", &sh);
@@ -258,6 +269,8 @@ lrc_status lrc_tt_eta(const double* const* cores, const void* const* cores_hat, 
 lrc_status lrc_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
                         double* diff_out, double* normA_out, lrc_stream_t stream) {
     if (!valid_fmt(fa) || !valid_fmt(fb)) return invalid("unknown format");
+    fa = plain_fmt(fa);
+    fb = plain_fmt(fb);
     if (count < 0) return invalid("negative count");
     if (!diff_out) return invalid("null diff_out");
     int64_t t;
@@ -276,6 +289,8 @@ lrc_status lrc_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, in
 lrc_status lrc_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
                                 double* diff_out, double* normA_out, lrc_stream_t stream) {
     if (!valid_fmt(fa) || !valid_fmt(fb)) return invalid("unknown format");
+    fa = plain_fmt(fa);
+    fb = plain_fmt(fb);
     if (count < 0) return invalid("negative count");
     if (!diff_out) return invalid("null diff_out");
     if (count > fro_diff_noalloc_max_count())

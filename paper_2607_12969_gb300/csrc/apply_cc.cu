@@ -25,7 +25,20 @@
 // sums of at most 1024 terms, added in split order by
 // reduce_scale_f32_kernel, which also applies diag(s)), phase 2 over
 // 128 x 128 tiles of Y.  W (b x k') passes through the stream's workspace.
+//
+// LRC_F32_TC (a variant): phase 2 on the tensor cores.  W (per row: queries
+// may differ in magnitude by any factor) and U (per 32 rows) are scaled by
+// powers of two that bring each group's largest magnitude into [2^14, 2^15)
+// and split into binary16 parts hi = fp16(x), lo = fp16(x - hi)
+// laid side by side along the reduction, W as [W_hi | W_lo | W_hi] in the
+// product's 128-row operand image and U as [U_hi | U_hi | U_lo] rows, so
+// that one binary16 product with binary32 accumulation (apply_tc.cu) forms
+// W U^T ~ W_hi U_hi + W_lo U_hi + W_hi U_lo; its epilogue multiplies each
+// entry by the inverse scales (exact).
+#include <cuda_fp16.h>
+
 #include "common.cuh"
+#include "tc.cuh"
 
 namespace lrc {
 namespace {
@@ -269,7 +282,110 @@ lrc_status launch_reduce_scale_f32(const float* part, int splits, int64_t split_
     return after_launch("reduce_scale_f32_kernel");
 }
 
+// ---------------------------------------------------------------- LRC_F32_TC
+constexpr int kSplitRows = 32;     // rows per scale group (one CTA)
+
+// e with max * 2^e in [2^14, 2^15), clamped to [-60, 60] (the product's
+// epilogue factor 2^-(e_w + e_u) stays a normal binary32 number); 0 for a
+// zero or non-finite group
+__device__ __forceinline__ int group_exp(float maxabs) {
+    if (!(maxabs > 0.0f) || !(maxabs <= 3.0e38f)) return 0;
+    const int e = 14 - (((__float_as_int(maxabs) >> 23) & 0xff) - 127);
+    return e < -60 ? -60 : (e > 60 ? 60 : e);
+}
+
+// A CTA per 32 rows of a binary32 matrix (rows x cols, row pitch lds, columns
+// from cols on read as zero): scales the rows by powers of two -- one per row
+// when PER_ROW (the queries of W may differ in magnitude by any factor), else
+// one for the 32 rows -- writes the exponents to esc (index = row, or group)
+// and three binary16 parts of every row, part p at columns [p kq, (p + 1) kq),
+// the lo half where bit p of lomask is set, else the hi half.  IMG: the output
+// is the canonical 128-row operand image of the tensor-core product
+// (tile_bytes per tile, rows up to the end of the last tile written, zero past
+// `rows`); else row-major with row pitch ldo (rows < `rows` only).  A thread
+// converts eight consecutive columns of one row and stores each part with one
+// 16-byte store.
+template <bool IMG, bool PER_ROW>
+__global__ void __launch_bounds__(256)
+split_parts_kernel(const float* __restrict__ src, int64_t rows, int cols, int64_t lds, int kq, int lomask,
+                   unsigned char* __restrict__ dst, int64_t ldo, uint32_t tile_bytes, int* __restrict__ esc) {
+    __shared__ float wmax[8];
+    __shared__ int rexp[kSplitRows];
+    const int64_t r0 = (int64_t)blockIdx.x * kSplitRows;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    if (PER_ROW) {
+        // warp w: rows 4w .. 4w + 3
+        for (int rr = 0; rr < kSplitRows / 8; ++rr) {
+            const int r = warp * (kSplitRows / 8) + rr;
+            float mx = 0.0f;
+            if (r0 + r < rows)
+                for (int c = lane; c < cols; c += 32) mx = fmaxf(mx, fabsf(src[(r0 + r) * lds + c]));
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            if (lane == 0) {
+                const int ex = group_exp(mx);
+                rexp[r] = ex;
+                if (r0 + r < rows) esc[r0 + r] = ex;
+            }
+        }
+    } else {
+        float mx = 0.0f;
+        for (int e = tid; e < kSplitRows * cols; e += 256) {
+            const int r = e / cols, c = e - r * cols;
+            if (r0 + r < rows) mx = fmaxf(mx, fabsf(src[(r0 + r) * lds + c]));
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        if (lane == 0) wmax[warp] = mx;
+        __syncthreads();
+        if (tid < kSplitRows) {
+            float gm = 0.0f;
+#pragma unroll
+            for (int w = 0; w < 8; ++w) gm = fmaxf(gm, wmax[w]);
+            rexp[tid] = group_exp(gm);
+            if (tid == 0) esc[blockIdx.x] = rexp[0];
+        }
+    }
+    __syncthreads();
+    const int g8 = kq / 8;
+    for (int e = tid; e < kSplitRows * g8; e += 256) {
+        const int r = e / g8, c0 = (e - r * g8) * 8;
+        const int64_t row = r0 + r;
+        if (!IMG && row >= rows) continue;
+        const float f = __int_as_float((127 + rexp[r]) << 23);
+        uint32_t hi[4], lo[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            float x[2];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int c = c0 + 2 * j + h;
+                x[h] = (row < rows && c < cols) ? __fmul_rn(src[row * lds + c], f) : 0.0f;
+            }
+            const __half h0 = __float2half_rn(x[0]), h1 = __float2half_rn(x[1]);
+            const __half l0 = __float2half_rn(__fsub_rn(x[0], __half2float(h0)));
+            const __half l1 = __float2half_rn(__fsub_rn(x[1], __half2float(h1)));
+            hi[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+            lo[j] = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
+        }
+        const uint4 vh = make_uint4(hi[0], hi[1], hi[2], hi[3]), vl = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+#pragma unroll
+        for (int p = 0; p < 3; ++p) {
+            const int col = p * kq + c0;
+            unsigned char* q = IMG ? dst + (size_t)(row / 128) * tile_bytes +
+                                         tc::w_image_off((uint32_t)(row % 128), (uint32_t)col)
+                                   : dst + ((size_t)row * ldo + col) * 2;
+            *reinterpret_cast<uint4*>(q) = ((lomask >> p) & 1) ? vl : vh;
+        }
+    }
+}
+
 }  // namespace
+
+// Ranks for which the tensor-core second product of LRC_F32_TC applies: the
+// three-part W image of a 128-row tile (128 x 3 k16 binary16) leaves room in
+// shared memory for the product's U ring and epilogue staging.
+constexpr int64_t kF32TcMaxRank = 192;
 
 // Batches below these sizes leave the fused kernels' row tiles too few to
 // fill the GPU; they take the split path of apply_split.cu (ranks up to 1024).
@@ -282,7 +398,7 @@ lrc_status launch_apply_f64(const double* U, const double* S, const double* Vt, 
 }
 
 lrc_status launch_apply_f32(const float* U, const float* S, const float* Vt, const float* X,
-                            float* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s) {
+                            float* Y, int64_t m, int64_t n, int64_t k, int64_t b, bool tc, cudaStream_t s) {
     if (b <= kSplitMaxBatchF32 && k <= kSplitMaxRank) return launch_apply_split_f32(U, S, Vt, X, Y, m, n, k, b, s);
     // phase 1: partial products of W = X V over n-splits, with V = (V^T)^T read
     // from the stored V^T rows; phase 2 after the ordered reduction and diag(s)
@@ -309,14 +425,35 @@ lrc_status launch_apply_f32(const float* U, const float* S, const float* Vt, con
         set_error("apply_f32: workspace size overflow");
         return LRC_ERR_INVALID_ARG;
     }
+    // LRC_F32_TC: room for the binary16 parts of W (operand images of 128-row
+    // tiles) and of U (rows of 3 k16) and the groups' exponents
+    tc = tc && k <= kF32TcMaxRank;
+    const int64_t kp3 = 3 * kp16;
+    const int64_t btiles = (b + 127) / 128;
+    const size_t tc_w = tc ? (size_t)btiles * 128 * kp3 * 2 : 0, tc_u = tc ? (size_t)m * kp3 * 2 : 0;
+    const int64_t ew = btiles * 128, eu = (m + kSplitRows - 1) / kSplitRows;   // W: a scale per row
+    const size_t tc_e = tc ? (size_t)(ew + eu) * sizeof(int) : 0;
+    const size_t base = ((size_t)(part_elems + w_elems) * sizeof(float) + 255) / 256 * 256;
     void* ws = nullptr;
-    lrc_status st = stream_workspace(s, (size_t)(part_elems + w_elems) * sizeof(float), &ws);
+    lrc_status st = stream_workspace(s, base + (tc_w + 255) / 256 * 256 + (tc_u + 255) / 256 * 256 + tc_e, &ws);
     if (st != LRC_OK) return st;
     float* part = static_cast<float*>(ws);
     float* Wd = part + part_elems;
     if ((st = gemm_cc_f32(X, ldn, Vt, ldn, true, part, kp16, b, k, n, (int)splits, w_elems, s)) != LRC_OK) return st;
     if ((st = launch_reduce_scale_f32(part, (int)splits, w_elems, b, k, kp16, S, Wd, s)) != LRC_OK) return st;
-    return gemm_cc_f32(Wd, kp16, U, ldk, true, Y, m, b, m, k, 1, 0, s);
+    if (!tc) return gemm_cc_f32(Wd, kp16, U, ldk, true, Y, m, b, m, k, 1, 0, s);
+    unsigned char* wimg = static_cast<unsigned char*>(ws) + base;
+    unsigned char* uimg = wimg + (tc_w + 255) / 256 * 256;
+    int* esc_w = reinterpret_cast<int*>(uimg + (tc_u + 255) / 256 * 256);
+    int* esc_u = esc_w + ew;
+    const uint32_t tile_bytes = (uint32_t)(128 * kp3 * 2);
+    split_parts_kernel<true, true><<<(unsigned)(btiles * 4), 256, 0, s>>>(Wd, b, (int)k, kp16, (int)kp16, 0b010, wimg,
+                                                                          0, tile_bytes, esc_w);
+    if ((st = after_launch("split_parts_kernel")) != LRC_OK) return st;
+    split_parts_kernel<false, false><<<(unsigned)eu, 256, 0, s>>>(U, m, (int)k, ldk, (int)kp16, 0b100, uimg, kp3, 0,
+                                                                  esc_u);
+    if ((st = after_launch("split_parts_kernel")) != LRC_OK) return st;
+    return launch_y_product(wimg, (int)kp3, uimg, kp3, m, b, false, Y, esc_w, esc_u, s, true);
 }
 
 }  // namespace lrc

@@ -482,8 +482,10 @@ struct YArgs {
     void* Y;
     // optional power-of-two scales of the operands, in groups of 32 rows of W
     // and 32 rows of U: entry (i, j) of the product is multiplied by
-    // 2^-(esc_w[i / 32] + esc_u[j / 32]) (exact in binary32)
+    // 2^-(esc_w[i / 32] + esc_u[j / 32]) (exact in binary32); esc_w[i] when
+    // esc_w_rows is set
     const int* esc_w;
+    int esc_w_rows;
     const int* esc_u;
 };
 
@@ -628,12 +630,14 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
             const int64_t row0 = bt * BM;
             const int ab = tl & 1;
             const bool scaled = a.esc_w != nullptr;
-            // this warp's 32 rows are one scale group of W; lane j holds the
-            // scale of the tile's j-th group of 32 columns (read before the
-            // accumulator wait, so the loads overlap it)
+            // this warp's 32 rows are one scale group of W (or the thread's row
+            // has its own scale); lane j holds the scale of the tile's j-th
+            // group of 32 columns (read before the accumulator wait, so the
+            // loads overlap it)
             int ew = 0, eu_lane = 0;
             if (scaled) {
-                ew = row0 + g * 32 < a.b ? a.esc_w[(row0 >> 5) + g] : 0;
+                if (a.esc_w_rows) ew = row0 + r < a.b ? a.esc_w[row0 + r] : 0;
+                else ew = row0 + g * 32 < a.b ? a.esc_w[(row0 >> 5) + g] : 0;
                 const int64_t cl = (int64_t)mt * a.n2 + lane * 32;
                 eu_lane = (lane < (a.n2 >> 5) && cl < a.m) ? a.esc_u[cl >> 5] : 0;
             }
@@ -1001,7 +1005,8 @@ lrc_status y_product_plan(int64_t m, int64_t b, int kp, bool out16, int* n2) {
 }
 
 lrc_status launch_y_product(const unsigned char* Wimg, int kp, const void* U, int64_t ldu, int64_t m, int64_t b,
-                            bool out16, void* Y, const int* esc_w, const int* esc_u, cudaStream_t s) {
+                            bool out16, void* Y, const int* esc_w, const int* esc_u, cudaStream_t s,
+                            bool w_per_row) {
     lrc_status st = get_encoder();
     if (st != LRC_OK) return st;
     YArgs a3{};
@@ -1011,6 +1016,7 @@ lrc_status launch_y_product(const unsigned char* Wimg, int kp, const void* U, in
     a3.W = Wimg;
     a3.Y = Y;
     a3.esc_w = esc_w;
+    a3.esc_w_rows = w_per_row ? 1 : 0;
     a3.esc_u = esc_u;
     CUtensorMap tu, ty;
     if ((st = make_map(&tu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, U, kp, m, ldu * 2, BK, (uint32_t)a3.n2, "U")) != LRC_OK)

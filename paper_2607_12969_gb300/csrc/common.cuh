@@ -49,14 +49,18 @@ inline cudaStream_t as_stream(lrc_stream_t s) { return reinterpret_cast<cudaStre
 inline int64_t storage_bytes(lrc_fmt f) {
     switch (f) {
         case LRC_F64: return 8;
-        case LRC_F32: return 4;
+        case LRC_F32:
+        case LRC_F32_TC: return 4;
         case LRC_F16:
         case LRC_F16_O16: return 2;
     }
     return 0;
 }
 
-inline bool valid_fmt(int f) { return f >= LRC_F64 && f <= LRC_F16_O16; }
+inline bool valid_fmt(int f) { return f >= LRC_F64 && f <= LRC_F32_TC; }
+// LRC_F32_TC is LRC_F32 everywhere but in the output products of lrc_apply
+// and tt_reconstruct
+inline lrc_fmt plain_fmt(lrc_fmt f) { return f == LRC_F32_TC ? LRC_F32 : f; }
 
 // a * b with overflow detection (both >= 0).
 inline bool mul_ok(int64_t a, int64_t b, int64_t* out) {
@@ -73,8 +77,9 @@ lrc_status launch_widen(const void* src, lrc_fmt fmt, int64_t rows, int64_t cols
                         double* dst, int64_t ld_dst, cudaStream_t s);
 lrc_status launch_apply_f64(const double* U, const double* S, const double* Vt, const double* X,
                             double* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
+// tc: the second product on the tensor cores (LRC_F32_TC) where it applies
 lrc_status launch_apply_f32(const float* U, const float* S, const float* Vt, const float* X,
-                            float* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
+                            float* Y, int64_t m, int64_t n, int64_t k, int64_t b, bool tc, cudaStream_t s);
 // small-batch split path of the CUDA-core apply (apply_split.cu)
 lrc_status launch_apply_split_f64(const double* U, const double* S, const double* Vt, const double* X, double* Y,
                                   int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
@@ -106,11 +111,13 @@ lrc_status gemm_cc_f32(const float* A, int64_t lda, const float* B, int64_t ldb,
 // binary16 output.  W is given as 128-row tile images (canonical K-major
 // layout, tc::w_image_off, 128 x kp binary16 each), U as m rows of kp
 // binary16 with row pitch ldu elements.  esc_w / esc_u (nullable together)
-// scale entry (i, j) by 2^-(esc_w[i / 32] + esc_u[j / 32]), each in
-// [-60, 60]; y_product_plan checks that the product fits the kernel.
+// scale entry (i, j) by 2^-(esc_w[i / 32] + esc_u[j / 32]) -- esc_w[i] when
+// w_per_row -- each in [-60, 60]; y_product_plan checks that the product
+// fits the kernel.
 lrc_status y_product_plan(int64_t m, int64_t b, int kp, bool out16, int* n2);
 lrc_status launch_y_product(const unsigned char* Wimg, int kp, const void* U, int64_t ldu, int64_t m, int64_t b,
-                            bool out16, void* Y, const int* esc_w, const int* esc_u, cudaStream_t s);
+                            bool out16, void* Y, const int* esc_w, const int* esc_u, cudaStream_t s,
+                            bool w_per_row = false);
 
 struct TTShape {
     int d;
@@ -132,6 +139,9 @@ lrc_status launch_tt_f16(const TTShape& sh, bool out16, void* out, cudaStream_t 
 // binary16 TT as a product chain with the output product on the tensor cores
 // (tt_split.cu); *handled = false when the shape is outside it (nothing launched)
 lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled);
+// the same product chain for binary32 cores (LRC_F32_TC): both operands split
+// into scaled hi/lo binary16 parts; *handled = false when the shape is outside it
+lrc_status launch_tt_split_f32tc(const TTShape& sh, float* out, cudaStream_t s, bool* handled);
 // binary32 TT whose chain has several small products at its ends: one side
 // launch forms Z and S, one product forms the tensor (tt_split.cu);
 // *handled = false when the shape is outside it

@@ -13,7 +13,8 @@
 // the output traffic.
 //
 // Operands of that product are binary16 with binary32 accumulation (Sec. 3.4).
-// An operand that is a stored core is exact in binary16.  An operand the
+// An operand that is a stored binary16 core is exact in binary16; binary32
+// cores (the LRC_F32_TC variant) take the hi/lo split below on both sides.  An operand the
 // chain computed is binary32; for a binary32 output it enters the product as
 // a pair hi = fp16(x), lo = fp16(x - hi) laid side by side along the
 // reduction, so one product of concatenated operands forms
@@ -384,14 +385,20 @@ size_t side_smem(const TTShape& sh, const SideArgs& a) {
 
 }  // namespace
 
-lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled) {
+namespace {
+
+// The split product chain for binary16 cores (TC = __half, stored cores exact
+// in binary16) or binary32 cores (TC = float: every operand split and scaled).
+template <typename TC>
+lrc_status launch_split_t(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled) {
+    constexpr bool kExactCores = sizeof(TC) == 2;
     *handled = false;
     const int d = sh.d;
     if (d > 16) return LRC_OK;
     const int c = tt_chain_bond(sh);
     const int r = (int)sh.ranks[c];
     const int rp = (r + 15) / 16 * 16;
-    const bool z_core = (c == 1), s_core = (c == d - 1);     // operands that are stored cores
+    const bool z_core = kExactCores && (c == 1), s_core = kExactCores && (c == d - 1);   // operands exact in binary16
     // parts along the reduction (see the file comment)
     Parts pw{1, 0}, pu{1, 0};
     if (!out16) {
@@ -430,13 +437,23 @@ lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStr
     a.Uimg = reinterpret_cast<__half*>(ws + w_bytes);
     a.esc_w = reinterpret_cast<int*>(ws + w_bytes + u_bytes);
     a.esc_u = a.esc_w + a.wunits;
-    cudaError_t e = cudaFuncSetAttribute(tt_side_kernel<__half, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(tt_side_kernel<TC, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "tt_side_kernel smem attribute");
-    e = launch_pdl(tt_side_kernel<__half, true>, dim3((unsigned)(a.wunits + uunits)), dim3(256), smem, s, a);
+    e = launch_pdl(tt_side_kernel<TC, true>, dim3((unsigned)(a.wunits + uunits)), dim3(256), smem, s, a);
     if (e != cudaSuccess) return cuda_fail(e, "tt_side_kernel launch");
     if ((st = after_launch("tt_side_kernel")) != LRC_OK) return st;
     return launch_y_product(a.Wimg, kp, a.Uimg, kp, a.Q, a.P, out16, out, a.esc_w, a.esc_u, s);
+}
+
+}  // namespace
+
+lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled) {
+    return launch_split_t<__half>(sh, out16, out, s, handled);
+}
+
+lrc_status launch_tt_split_f32tc(const TTShape& sh, float* out, cudaStream_t s, bool* handled) {
+    return launch_split_t<float>(sh, false, out, s, handled);
 }
 
 lrc_status launch_tt_side_f32(const TTShape& sh, float* out, cudaStream_t s, bool* handled) {

@@ -5,12 +5,13 @@ import numpy as np
 import oracle
 
 # relative Frobenius tolerances per path
-TOL = {"f64": 1e-12, "f32": 1e-5, "f16": 1e-5, "f16_o16": 2e-3}
+TOL = {"f64": 1e-12, "f32": 1e-5, "f16": 1e-5, "f16_o16": 2e-3, "f32tc": 1e-5}
 BITS_DTYPE = {"f64": np.float64, "f32": np.uint32, "f16": np.uint16}
 
 
 def base_fmt(fmt: str) -> str:
-    return "f16" if fmt.startswith("f16") else fmt
+    """Storage format whose rounding the oracle applies (f32tc stores binary32)."""
+    return "f16" if fmt.startswith("f16") else ("f32" if fmt == "f32tc" else fmt)
 
 
 def rel_fro(got: np.ndarray, want: np.ndarray) -> float:

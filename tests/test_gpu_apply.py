@@ -10,7 +10,7 @@ from parity import TOL, base_fmt, oracle_inputs, packed, rel_fro
 
 pytestmark = pytest.mark.gpu
 
-FMTS = ["f64", "f32", "f16", "f16_o16"]
+FMTS = ["f64", "f32", "f16", "f16_o16", "f32tc"]
 
 
 def run_apply(lrc, dev, U, s, Vt, X, fmt):
@@ -106,7 +106,7 @@ def test_identity_queries_reconstruct_dense_f64(lrc, cuda):
     assert np.max(np.abs(got - want)) <= 1e-14 * np.max(np.abs(want))
 
 
-@pytest.mark.parametrize("fmt", ["f32", "f64"])
+@pytest.mark.parametrize("fmt", ["f32", "f64", "f32tc"])
 @pytest.mark.parametrize("m,n,k,b", [
     (257, 1100, 136, 300),     # several n-splits, one 160-wide rank tile
     (130, 3000, 161, 517),     # rank above 160: two rank tiles, ragged everything
@@ -163,3 +163,37 @@ def test_apply_bitwise_reproducible(lrc, cuda, fmt, b):
     assert lrc.lrc_device_status() == 0
     assert torch.equal(outs[0].view(torch.int8), outs[1].view(torch.int8)), (fmt, b)
     assert not torch.isnan(outs[0].double()).any()
+
+
+@pytest.mark.parametrize("m,n,k,b", [
+    (2048, 1536, 136, 300),    # rank of the large-batch workload, ragged batch: the tensor-core product
+    (1000, 700, 192, 129),     # largest rank of the tensor-core product
+    (900, 600, 200, 64),       # rank above it: the binary32 product kernel
+])
+def test_f32tc_matches_f32_path(lrc, cuda, m, n, k, b):
+    """LRC_F32_TC (second product on the tensor cores through the scaled
+    binary16 hi/lo split) stays within the binary32 tolerance of the oracle
+    and of the LRC_F32 result on the same inputs."""
+    f = W.random_factors(m, n, k, seed=m + k + 7)
+    X = W.gaussian((b, n), b + 3)
+    want = oracle.apply(*oracle_inputs(f.U, f.s, f.Vt, X, "f32"))
+    got_tc = run_apply(lrc, cuda, f.U, f.s, f.Vt, X, "f32tc")
+    got_32 = run_apply(lrc, cuda, f.U, f.s, f.Vt, X, "f32")
+    assert rel_fro(got_tc, want) <= TOL["f32tc"]
+    assert rel_fro(got_tc, got_32) <= 2 * TOL["f32"]
+
+
+def test_f32tc_wide_dynamic_range(lrc, cuda):
+    """Queries spanning 40 binades and factor rows spanning 16: W takes a
+    power-of-two scale per row and U one per 32 rows, so every part stays a
+    normal binary16 number and each query keeps binary32 accuracy."""
+    m, n, k, b = 512, 384, 96, 256
+    f = W.random_factors(m, n, k, seed=77)
+    rng = np.random.default_rng(78)
+    U = f.U * np.exp2(rng.integers(-8, 8, size=(m, 1)))
+    X = W.gaussian((b, n), 79) * np.exp2(rng.integers(-20, 20, size=(b, 1)))
+    want = oracle.apply(*oracle_inputs(U, f.s, f.Vt, X, "f32"))
+    got = run_apply(lrc, cuda, U, f.s, f.Vt, X, "f32tc")
+    # per-row relative error: every query row is judged against its own scale
+    err = np.linalg.norm(got - want, axis=1) / np.linalg.norm(want, axis=1)
+    assert err.max() <= 1e-5, err.max()

@@ -10,7 +10,7 @@ from parity import TOL, base_fmt, rel_fro, to_dev
 
 pytestmark = pytest.mark.gpu
 
-FMTS = ["f64", "f32", "f16", "f16_o16"]
+FMTS = ["f64", "f32", "f16", "f16_o16", "f32tc"]
 
 
 def run_tt(lrc, dev, cores64, fmt):
