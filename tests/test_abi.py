@@ -54,6 +54,10 @@ def test_validation_rejects_before_launch(L):
     assert st == -1
     st = L.lrc_apply(16, 16, 16, 16, 16, 4, 4, 2, 1, 7, None)
     assert st == -1
+    st = L.lrc_apply(16, 16, 16, 16, 16, 4, 4, 2, 1, 5, None)       # one past LRC_F32_TC
+    assert st == -1
+    st = L.lrc_apply(17, 16, 16, 16, 16, 4, 4, 2, 1, 4, None)       # LRC_F32_TC is a format: checks go on
+    assert st == -2
     st = L.lrc_apply(17, 16, 16, 16, 16, 4, 4, 2, 1, 0, None)      # misaligned U
     assert st == -2
     st = L.lrc_round_factors(16, 4, 8, 4, 16, 8, 1, None)           # ld_src < cols
@@ -102,6 +106,9 @@ def test_host_helpers_agree_with_oracle(L):
         dims, base, aug = (256, 256, 256), (1, 32, 32, 1), (1, 34, 34, 1)
         assert abs(lrc.lrc_tt_storage_bytes(dims, aug, fmt) * 8 - oracle.tt_storage_bits(dims, aug, fmt)) < 1e-6
     assert lrc.lrc_matrix_storage_ratio(10, 10, 40, 41, "f16") == pytest.approx(0.25625)
+    # the binary32 tensor-core variant stores binary32
+    assert lrc.lrc_matrix_storage_ratio(16384, 8192, 128, 136, "f32tc") == \
+        lrc.lrc_matrix_storage_ratio(16384, 8192, 128, 136, "f32")
 
 
 def test_eta_validation_rejects_before_launch(L):
