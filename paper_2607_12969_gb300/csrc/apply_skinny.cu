@@ -13,8 +13,7 @@
 //                     shared memory; each warp takes 4 rows of V^T, each lane
 //                     keeps the b partial dot products of every row over its
 //                     16-byte columns, a recursive halving adds them across
-//                     the warp.  One partial W per chunk.  The CTAs also bring U
-//                     into L2 for the last kernel.
+//                     the warp.  One partial W per chunk.
 //   skinny_w2_kernel  W = (sum of the chunks' partials) diag(s), a warp per
 //                     entry; for binary16 output W is rounded to binary16 (the
 //                     method-precision workspace of Sec. 3.4).
@@ -42,7 +41,6 @@ constexpr int kRows = 4;                      // factor rows per warp (first pro
 constexpr int kBox = 256;                     // columns per TMA box of the first product
 constexpr size_t kSmemW1 = 100 * 1024;        // shared-memory budget of a first-product CTA
 constexpr size_t kSmemMaxS = 220 * 1024;      // largest dynamic shared memory a CTA asks for
-constexpr uint64_t kPrefetchMaxBytes = 64ull << 20;   // U prefetched into L2 up to this size
 
 template <typename TS>
 struct EVof {
@@ -185,7 +183,7 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
 template <typename TS, typename T, int B, int RW>
 __global__ void __launch_bounds__(kThreadsS, 2)
 skinny_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_v, int k, int b,
-                 int L, T* __restrict__ Wp, const void* upf, uint64_t upf_bytes) {
+                 int L, T* __restrict__ Wp) {
     constexpr int EV = EVof<TS>::v;
     constexpr int BR = kWarps * RW;              // rows of V^T per CTA
     extern __shared__ unsigned char smem_raw[];
@@ -208,8 +206,6 @@ skinny_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
             tc::tma_load_2d(vs + (size_t)q * BR * kBox, &tm_v, i0 + q * kBox, jb, &bar[q]);
             tc::tma_load_2d(xs + (size_t)q * B * kBox, &tm_x, i0 + q * kBox, 0, &bar[q]);
         }
-        // U, read by the last kernel, comes into L2 alongside this kernel's stream
-        if (upf) tc::bulk_prefetch_share(upf, upf_bytes, blockIdx.y * gridDim.x + blockIdx.x, gridDim.x * gridDim.y);
     }
     __syncthreads();
     const int jl = warp * RW;                 // first local row of the warp
@@ -431,9 +427,8 @@ lrc_status launch_skinny_b(const TS* U, const TS* S, const TS* Vt, const TS* X, 
     cudaError_t ce = cudaFuncSetAttribute(skinny_w1_kernel<TS, T, B, RW>,
                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem1);
     if (ce != cudaSuccess) return cuda_fail(ce, "skinny_w1_kernel smem attribute");
-    const uint64_t u_bytes = ((uint64_t)(m - 1) * (uint64_t)ldk + (uint64_t)k) * (uint64_t)e;
     skinny_w1_kernel<TS, T, B, RW><<<dim3((unsigned)p.nchunks, (unsigned)p.jblocks), kThreadsS, p.smem1, s>>>(
-        tx, tv, (int)k, (int)b, (int)p.L, Wp, u_bytes <= kPrefetchMaxBytes ? (const void*)U : nullptr, u_bytes);
+        tx, tv, (int)k, (int)b, (int)p.L, Wp);
     if ((st = after_launch("skinny_w1_kernel")) != LRC_OK) return st;
     ce = launch_pdl(skinny_w2_kernel<TS, T>, dim3((unsigned)((b * p.kv * 32 + 255) / 256)), dim3(256), 0, s,
                     (const T*)Wp, (int)p.nchunks, (int)b, (int)k, (int)p.kv, S, round16 ? 1 : 0, Wd);

@@ -61,8 +61,6 @@ constexpr uint32_t kXBytes = BM * BK * 2;    // one X box
 constexpr int kChunkBlocks = 8;              // k-blocks per accumulation chunk (FP32 output)
 constexpr int kPfBlocks = 4;                 // k-blocks per L2 prefetch box (512-byte rows)
 constexpr int kStageBlocks = 2;              // k-blocks per phase-1 ring stage
-constexpr int64_t kPrefetchMaxBatch = 1024;  // U prefetched into L2 by phase 1 up to this batch
-constexpr uint64_t kPrefetchMaxBytes = 48ull << 20;
 
 __device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
     return reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -84,8 +82,6 @@ struct W1Args {
     uint32_t sum_col;         // tensor-memory column of the running sum (FP32 output)
     uint32_t tmem_cols;
     float* P;                 // partials: [segment id][kgp columns][128 rows]
-    const void* upf;          // optional: buffer (U) that the CTAs prefetch into L2 for the next product
-    uint64_t upf_bytes;
 };
 
 // Next accumulation chunk of the k-block range [qbeg, qend): a chunk lies in
@@ -156,7 +152,6 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
             bool ok = true;
             int64_t q = qbeg, q0, q1, row;
             bool first, last;
-            if (a.upf) bulk_prefetch_share(a.upf, a.upf_bytes, blockIdx.x, gridDim.x);
             while (ok && next_chunk(q, qbeg, qend, a.nkb, a.chunk_blocks, q0, q1, row, first, last)) {
                 const int grp = (int)(row / a.btiles);
                 const int64_t bt = row - (int64_t)grp * a.btiles;
@@ -930,13 +925,6 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
     a3.W = Wimg;
 
     const int64_t ldn = lrc_packed_ld(n), ldk = lrc_packed_ld(k);
-    // small batches: the second product reads U a few times only, so phase 1
-    // brings it into L2 alongside its own stream
-    const uint64_t u_bytes = ((uint64_t)(m - 1) * (uint64_t)ldk + (uint64_t)k) * 2u;
-    if (b <= kPrefetchMaxBatch && u_bytes <= kPrefetchMaxBytes) {
-        a1.upf = U;
-        a1.upf_bytes = u_bytes;
-    }
     CUtensorMap tx, tv, tu, ty, txp, tvp;
     if ((st = make_map(&tx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, X, n, b, ldn * 2, BK, BM, "X")) != LRC_OK) return st;
     if ((st = make_map(&tv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, Vt, n, k, ldn * 2, BK, (uint32_t)a1.kgp, "Vt")) != LRC_OK)

@@ -138,22 +138,6 @@ __device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int32_t 
                  : "memory");
 }
 
-// L2 prefetch of this CTA's share of a contiguous buffer: the buffer is cut
-// into `parts` equal 16-byte-aligned ranges and range `part` is requested in
-// pieces of at most 64 KB (no shared memory, no barrier).  base must be
-// 16-byte aligned.
-__device__ __forceinline__ void bulk_prefetch_share(const void* base, uint64_t bytes, uint32_t part, uint32_t parts) {
-    const uint64_t units = bytes / 16;
-    uint64_t u0 = units * part / parts, u1 = units * (part + 1) / parts;
-    const unsigned char* p = static_cast<const unsigned char*>(base);
-    while (u0 < u1) {
-        const uint64_t nu = (u1 - u0) < 4096 ? (u1 - u0) : 4096;
-        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p + u0 * 16), "r"((uint32_t)(nu * 16))
-                     : "memory");
-        u0 += nu;
-    }
-}
-
 // 2-D tiled store of a shared-memory box to (x, y); elements outside the
 // tensor are not written.  x, y >= 0.
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int32_t x, int32_t y, const void* src) {
