@@ -187,6 +187,7 @@ lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims, const i
         bool handled = false;
         st = launch_tt_split_f32tc(sh, static_cast<float*>(out), s, &handled);
         if (st != LRC_OK || handled) return st;
+        return launch_tt_chain_f32tc(sh, static_cast<float*>(out), s);
     }
     if (fmt == LRC_F32 || fmt == LRC_F32_TC) return launch_tt_chain_f32(sh, static_cast<float*>(out), s);
     if (tt_chain_saves(sh)) return launch_tt_chain_f64(sh, static_cast<double*>(out), s);

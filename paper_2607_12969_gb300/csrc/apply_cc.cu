@@ -294,45 +294,49 @@ __device__ __forceinline__ int group_exp(float maxabs) {
     return e < -60 ? -60 : (e > 60 ? 60 : e);
 }
 
-// A CTA per 32 rows of a binary32 matrix (rows x cols, row pitch lds, columns
-// from cols on read as zero): scales the rows by powers of two -- one per row
-// when PER_ROW (the queries of W may differ in magnitude by any factor), else
-// one for the 32 rows -- writes the exponents to esc (index = row, or group)
-// and three binary16 parts of every row, part p at columns [p kq, (p + 1) kq),
-// the lo half where bit p of lomask is set, else the hi half.  IMG: the output
-// is the canonical 128-row operand image of the tensor-core product
-// (tile_bytes per tile, rows up to the end of the last tile written, zero past
-// `rows`); else row-major with row pitch ldo (rows < `rows` only).  A thread
-// converts eight consecutive columns of one row and stores each part with one
-// 16-byte store.
-template <bool IMG, bool PER_ROW>
-__global__ void __launch_bounds__(256)
-split_parts_kernel(const float* __restrict__ src, int64_t rows, int cols, int64_t lds, int kq, int lomask,
-                   unsigned char* __restrict__ dst, int64_t ldo, uint32_t tile_bytes, int* __restrict__ esc) {
+// A CTA per 32 rows of a binary32 matrix whose entry (row, c) is
+// src[row * rs + c * cs] (columns from cols on read as zero; TRANS: the
+// matrix is the transpose of a row-major one, cs its row pitch, so threads
+// take consecutive rows for coalesced reads): scales the rows by powers of two
+// -- one per row when PER_ROW (the queries of W may differ in magnitude by any
+// factor), else one for the 32 rows -- writes the exponents to esc (index =
+// row, or group) and three binary16 parts of every row, part p at columns
+// [p kq, (p + 1) kq), the lo half where bit p of lomask is set, else the hi
+// half.  IMG: the output is the canonical 128-row operand image of the
+// tensor-core product (tile_bytes per tile, rows up to the end of the last
+// tile written, zero past `rows`); else row-major with row pitch ldo (rows <
+// `rows` only).  A thread converts eight consecutive columns of one row and
+// stores each part with one 16-byte store.
+template <bool IMG, bool PER_ROW, bool TRANS>
+__device__ __forceinline__ void split_parts_block(int64_t blk, const float* __restrict__ src, int64_t rows, int cols,
+                                                  int64_t rs, int64_t cs, int kq, int lomask,
+                                                  unsigned char* __restrict__ dst, int64_t ldo, uint32_t tile_bytes,
+                                                  int* __restrict__ esc) {
     __shared__ float wmax[8];
     __shared__ int rexp[kSplitRows];
-    const int64_t r0 = (int64_t)blockIdx.x * kSplitRows;
+    __shared__ int rmax[kSplitRows];    // row maxima as bits (|x| >= 0 orders as an integer)
+    const int64_t r0 = blk * kSplitRows;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    auto at = [&](int64_t row, int c) { return src[row * rs + (int64_t)c * cs]; };
     if (PER_ROW) {
-        // warp w: rows 4w .. 4w + 3
-        for (int rr = 0; rr < kSplitRows / 8; ++rr) {
-            const int r = warp * (kSplitRows / 8) + rr;
-            float mx = 0.0f;
-            if (r0 + r < rows)
-                for (int c = lane; c < cols; c += 32) mx = fmaxf(mx, fabsf(src[(r0 + r) * lds + c]));
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-            if (lane == 0) {
-                const int ex = group_exp(mx);
-                rexp[r] = ex;
-                if (r0 + r < rows) esc[r0 + r] = ex;
-            }
+        // one coalesced pass over the 32 rows, maxima gathered by shared atomics
+        if (tid < kSplitRows) rmax[tid] = 0;
+        __syncthreads();
+        for (int e = tid; e < kSplitRows * cols; e += 256) {
+            const int r = TRANS ? e % kSplitRows : e / cols, c = TRANS ? e / kSplitRows : e % cols;
+            if (r0 + r < rows) atomicMax(&rmax[r], __float_as_int(fabsf(at(r0 + r, c))));
+        }
+        __syncthreads();
+        if (tid < kSplitRows) {
+            const int ex = group_exp(__int_as_float(rmax[tid]));
+            rexp[tid] = ex;
+            if (r0 + tid < rows) esc[r0 + tid] = ex;
         }
     } else {
         float mx = 0.0f;
         for (int e = tid; e < kSplitRows * cols; e += 256) {
-            const int r = e / cols, c = e - r * cols;
-            if (r0 + r < rows) mx = fmaxf(mx, fabsf(src[(r0 + r) * lds + c]));
+            const int r = TRANS ? e % kSplitRows : e / cols, c = TRANS ? e / kSplitRows : e % cols;
+            if (r0 + r < rows) mx = fmaxf(mx, fabsf(at(r0 + r, c)));
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
@@ -343,13 +347,14 @@ split_parts_kernel(const float* __restrict__ src, int64_t rows, int cols, int64_
 #pragma unroll
             for (int w = 0; w < 8; ++w) gm = fmaxf(gm, wmax[w]);
             rexp[tid] = group_exp(gm);
-            if (tid == 0) esc[blockIdx.x] = rexp[0];
+            if (tid == 0) esc[blk] = rexp[0];
         }
     }
     __syncthreads();
     const int g8 = kq / 8;
     for (int e = tid; e < kSplitRows * g8; e += 256) {
-        const int r = e / g8, c0 = (e - r * g8) * 8;
+        const int r = TRANS ? e % kSplitRows : e / g8;
+        const int c0 = (TRANS ? e / kSplitRows : e - r * g8) * 8;
         const int64_t row = r0 + r;
         if (!IMG && row >= rows) continue;
         const float f = __int_as_float((127 + rexp[r]) << 23);
@@ -360,7 +365,7 @@ split_parts_kernel(const float* __restrict__ src, int64_t rows, int cols, int64_
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
                 const int c = c0 + 2 * j + h;
-                x[h] = (row < rows && c < cols) ? __fmul_rn(src[row * lds + c], f) : 0.0f;
+                x[h] = (row < rows && c < cols) ? __fmul_rn(at(row, c), f) : 0.0f;
             }
             const __half h0 = __float2half_rn(x[0]), h1 = __float2half_rn(x[1]);
             const __half l0 = __float2half_rn(__fsub_rn(x[0], __half2float(h0)));
@@ -380,12 +385,100 @@ split_parts_kernel(const float* __restrict__ src, int64_t rows, int cols, int64_
     }
 }
 
+// One launch splits both operands of a product: blocks [0, wblocks) form the
+// W image (A: a scale per row, parts [hi | lo | hi]), the rest the U rows
+// (B: a scale per 32 rows, parts [hi | hi | lo]).
+struct SplitPair {
+    const float* A;
+    int64_t a_rows, a_rs, a_cs;
+    const float* B;
+    int64_t b_rows, b_rs, b_cs;
+    int cols, kq;
+    int64_t wblocks, ldu;
+    uint32_t tile_bytes;
+    unsigned char* wimg;
+    unsigned char* uimg;
+    int* esc_w;
+    int* esc_u;
+};
+
+template <bool TA, bool TB>
+__global__ void __launch_bounds__(256) split_pair_kernel(const SplitPair a) {
+    if ((int64_t)blockIdx.x < a.wblocks)
+        split_parts_block<true, true, TA>(blockIdx.x, a.A, a.a_rows, a.cols, a.a_rs, a.a_cs, a.kq, 0b010, a.wimg, 0,
+                                          a.tile_bytes, a.esc_w);
+    else
+        split_parts_block<false, false, TB>(blockIdx.x - a.wblocks, a.B, a.b_rows, a.cols, a.b_rs, a.b_cs, a.kq,
+                                            0b100, a.uimg, a.ldu, 0, a.esc_u);
+}
+
 }  // namespace
 
 // Ranks for which the tensor-core second product of LRC_F32_TC applies: the
 // three-part W image of a 128-row tile (128 x 3 k16 binary16) leaves room in
 // shared memory for the product's U ring and epilogue staging.
 constexpr int64_t kF32TcMaxRank = 192;
+
+// C (P x Q, row pitch Q) = A B^T on the tensor cores through the scaled
+// binary16 split: A(i, j) = A[i a_rs + j a_cs] (P x k, scaled per row), B(i, j)
+// = B[i b_rs + j b_cs] (Q x k, scaled per 32 rows).
+lrc_status launch_split_product(const float* A, int64_t a_rs, int64_t a_cs, const float* B, int64_t b_rs,
+                                int64_t b_cs, int64_t P, int64_t Q, int64_t k, unsigned char* wimg,
+                                unsigned char* uimg, int* esc_w, int* esc_u, float* C, cudaStream_t s) {
+    const int64_t kp16 = (k + 15) / 16 * 16, kp3 = 3 * kp16;
+    const int64_t ptiles = (P + 127) / 128;
+    SplitPair sp{};
+    sp.A = A;
+    sp.a_rows = P;
+    sp.a_rs = a_rs;
+    sp.a_cs = a_cs;
+    sp.B = B;
+    sp.b_rows = Q;
+    sp.b_rs = b_rs;
+    sp.b_cs = b_cs;
+    sp.cols = (int)k;
+    sp.kq = (int)kp16;
+    sp.wblocks = ptiles * 4;
+    sp.ldu = kp3;
+    sp.tile_bytes = (uint32_t)(128 * kp3 * 2);
+    sp.wimg = wimg;
+    sp.uimg = uimg;
+    sp.esc_w = esc_w;
+    sp.esc_u = esc_u;
+    const unsigned grid = (unsigned)(ptiles * 4 + (Q + kSplitRows - 1) / kSplitRows);
+    if (a_cs == 1 && b_cs == 1) split_pair_kernel<false, false><<<grid, 256, 0, s>>>(sp);
+    else if (a_cs == 1) split_pair_kernel<false, true><<<grid, 256, 0, s>>>(sp);
+    else if (b_cs == 1) split_pair_kernel<true, false><<<grid, 256, 0, s>>>(sp);
+    else split_pair_kernel<true, true><<<grid, 256, 0, s>>>(sp);
+    lrc_status st = after_launch("split_pair_kernel");
+    if (st != LRC_OK) return st;
+    return launch_y_product(wimg, (int)kp3, uimg, kp3, Q, P, false, C, esc_w, esc_u, s, true);
+}
+
+size_t split_product_bytes(int64_t P, int64_t Q, int64_t k) {
+    const int64_t kp3 = 3 * ((k + 15) / 16 * 16);
+    const int64_t ptiles = (P + 127) / 128;
+    return ((size_t)ptiles * 128 * kp3 * 2 + 255) / 256 * 256 + ((size_t)Q * kp3 * 2 + 255) / 256 * 256 +
+           (size_t)(ptiles * 128 + (Q + kSplitRows - 1) / kSplitRows) * sizeof(int);
+}
+
+bool split_product_fits(int64_t P, int64_t Q, int64_t k) {
+    int n2 = 0;
+    return k <= kF32TcMaxRank && y_product_plan(Q, P, (int)(3 * ((k + 15) / 16 * 16)), false, &n2) == LRC_OK;
+}
+
+lrc_status launch_split_product(const float* A, int64_t a_rs, int64_t a_cs, const float* B, int64_t b_rs,
+                                int64_t b_cs, int64_t P, int64_t Q, int64_t k, unsigned char* ws, float* C,
+                                cudaStream_t s) {
+    const int64_t kp16 = (k + 15) / 16 * 16, kp3 = 3 * kp16;
+    const int64_t ptiles = (P + 127) / 128;
+    unsigned char* wimg = ws;
+    unsigned char* uimg = wimg + ((size_t)ptiles * 128 * kp3 * 2 + 255) / 256 * 256;
+    int* esc_w = reinterpret_cast<int*>(uimg + ((size_t)Q * kp3 * 2 + 255) / 256 * 256);
+    int* esc_u = esc_w + ptiles * 128;
+    return launch_split_product(A, a_rs, a_cs, B, b_rs, b_cs, P, Q, k, wimg, uimg, esc_w, esc_u, C, s);
+}
+
 
 // Batches below these sizes leave the fused kernels' row tiles too few to
 // fill the GPU; they take the split path of apply_split.cu (ranks up to 1024).
@@ -446,14 +539,9 @@ lrc_status launch_apply_f32(const float* U, const float* S, const float* Vt, con
     unsigned char* uimg = wimg + (tc_w + 255) / 256 * 256;
     int* esc_w = reinterpret_cast<int*>(uimg + (tc_u + 255) / 256 * 256);
     int* esc_u = esc_w + ew;
-    const uint32_t tile_bytes = (uint32_t)(128 * kp3 * 2);
-    split_parts_kernel<true, true><<<(unsigned)(btiles * 4), 256, 0, s>>>(Wd, b, (int)k, kp16, (int)kp16, 0b010, wimg,
-                                                                          0, tile_bytes, esc_w);
-    if ((st = after_launch("split_parts_kernel")) != LRC_OK) return st;
-    split_parts_kernel<false, false><<<(unsigned)eu, 256, 0, s>>>(U, m, (int)k, ldk, (int)kp16, 0b100, uimg, kp3, 0,
-                                                                  esc_u);
-    if ((st = after_launch("split_parts_kernel")) != LRC_OK) return st;
-    return launch_y_product(wimg, (int)kp3, uimg, kp3, m, b, false, Y, esc_w, esc_u, s, true);
+    if ((st = launch_split_product(Wd, kp16, 1, U, ldk, 1, b, m, k, wimg, uimg, esc_w, esc_u, Y, s)) != LRC_OK)
+        return st;
+    return LRC_OK;
 }
 
 }  // namespace lrc

@@ -77,6 +77,17 @@ lrc_status launch_widen(const void* src, lrc_fmt fmt, int64_t rows, int64_t cols
                         double* dst, int64_t ld_dst, cudaStream_t s);
 lrc_status launch_apply_f64(const double* U, const double* S, const double* Vt, const double* X,
                             double* Y, int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
+// LRC_F32_TC output product C (P x Q, row pitch Q) = A B^T on the tensor
+// cores through the scaled binary16 split (apply_cc.cu): A(i, j) =
+// A[i a_rs + j a_cs] is P x k (a scale per row), B(i, j) = B[i b_rs + j b_cs]
+// is Q x k (a scale per 32 rows); ws holds split_product_bytes(P, Q, k)
+// bytes (256-byte aligned); split_product_fits says whether the product
+// kernel takes the shape.
+size_t split_product_bytes(int64_t P, int64_t Q, int64_t k);
+bool split_product_fits(int64_t P, int64_t Q, int64_t k);
+lrc_status launch_split_product(const float* A, int64_t a_rs, int64_t a_cs, const float* B, int64_t b_rs,
+                                int64_t b_cs, int64_t P, int64_t Q, int64_t k, unsigned char* ws, float* C,
+                                cudaStream_t s);
 // tc: the second product on the tensor cores (LRC_F32_TC) where it applies
 lrc_status launch_apply_f32(const float* U, const float* S, const float* Vt, const float* X,
                             float* Y, int64_t m, int64_t n, int64_t k, int64_t b, bool tc, cudaStream_t s);
@@ -142,6 +153,9 @@ lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStr
 // the same product chain for binary32 cores (LRC_F32_TC): both operands split
 // into scaled hi/lo binary16 parts; *handled = false when the shape is outside it
 lrc_status launch_tt_split_f32tc(const TTShape& sh, float* out, cudaStream_t s, bool* handled);
+// the FP32 product chain with its output product on the tensor cores
+// (LRC_F32_TC) when split_product_fits, else on the CUDA cores (tt_chain.cu)
+lrc_status launch_tt_chain_f32tc(const TTShape& sh, float* out, cudaStream_t s);
 // binary32 TT whose chain has several small products at its ends: one side
 // launch forms Z and S, one product forms the tensor (tt_split.cu);
 // *handled = false when the shape is outside it

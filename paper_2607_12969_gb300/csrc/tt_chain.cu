@@ -72,8 +72,10 @@ lrc_status product(const double* A, int64_t lda, const double* B, int64_t ldb, d
     return gemm_cc_f64(A, lda, B, ldb, C, ldc, M, N, K, s);
 }
 
+// tc_final (binary32 only): the output product on the tensor cores through
+// the scaled binary16 split (LRC_F32_TC) when the product kernel takes it.
 template <typename T>
-lrc_status launch_chain(const TTShape& sh, T* out, cudaStream_t s) {
+lrc_status launch_chain(const TTShape& sh, T* out, cudaStream_t s, bool tc_final = false) {
     const int d = sh.d;
     const int c = plan_chain(sh).c;
     const T* const* G = reinterpret_cast<const T* const*>(sh.cores);
@@ -93,7 +95,10 @@ lrc_status launch_chain(const TTShape& sh, T* out, cudaStream_t s) {
         if (b > rsz[j & 1]) rsz[j & 1] = b;
     }
     unsigned char* ws = nullptr;
-    const size_t total = lsz[0] + lsz[1] + rsz[0] + rsz[1];
+    const int64_t rc = sh.ranks[c];
+    const bool tc = tc_final && sizeof(T) == 4 && split_product_fits(P[c], Q[c], rc);
+    const size_t tsz = tc ? round256(split_product_bytes(P[c], Q[c], rc)) : 0;
+    const size_t total = lsz[0] + lsz[1] + rsz[0] + rsz[1] + tsz;
     if (total > 0) {
         void* p = nullptr;
         lrc_status st = stream_workspace(s, total, &p);
@@ -118,6 +123,12 @@ lrc_status launch_chain(const TTShape& sh, T* out, cudaStream_t s) {
             return st;
         S = dst;
     }
+    if constexpr (sizeof(T) == 4) {
+        // Z is P x r (row pitch r), S is r x Q (row pitch Q): B = S^T
+        if (tc)
+            return launch_split_product(Z, rc, 1, S, 1, Q[c], P[c], Q[c], rc,
+                                        ws + lsz[0] + lsz[1] + rsz[0] + rsz[1], out, s);
+    }
     return product(Z, sh.ranks[c], S, Q[c], out, Q[c], P[c], Q[c], sh.ranks[c], s);
 }
 
@@ -128,6 +139,10 @@ lrc_status launch_tt_chain_f32(const TTShape& sh, float* out, cudaStream_t s) {
     const lrc_status st = launch_tt_side_f32(sh, out, s, &handled);
     if (handled) return st;
     return launch_chain<float>(sh, out, s);
+}
+
+lrc_status launch_tt_chain_f32tc(const TTShape& sh, float* out, cudaStream_t s) {
+    return launch_chain<float>(sh, out, s, true);
 }
 
 lrc_status launch_tt_chain_f64(const TTShape& sh, double* out, cudaStream_t s) {
