@@ -4,35 +4,40 @@
 //
 // Three launches on the caller's stream:
 //  1. apply_w1_kernel -- W = X V in FP32 partials.  For every 128-row tile of
-//     X and every column group of W (at most 160 ranks for FP32 output, so that a
-//     running sum fits in shared memory) the reduction over n is a row of
-//     64-wide k-blocks.  The rows are laid end to end and cut into equal
-//     contiguous ranges, one per CTA of a persistent grid: every SM gets the
-//     same share of the product whatever b is (one row tile or hundreds).
-//     A CTA's range crosses a few rows; each piece (segment) accumulates in
-//     tensor memory -- for FP32 output in chunks of at most kChunkBlocks
-//     k-blocks whose results the epilogue adds with IEEE binary32 additions
-//     (the tensor core's own accumulation error grows with the number of
-//     accumulation steps) -- and is written to the workspace as an FP32
-//     partial.  Column groups are the slower index of the rows, so the CTAs
-//     working on the two groups of one row tile run side by side and the
-//     second read of an X tile hits L2.
+//     X and every column group of W (at most 160 ranks for FP32 output, so that
+//     two accumulators and a running sum fit in tensor memory) the reduction
+//     over n is a row of 64-wide k-blocks.  The rows are laid end to end and
+//     cut into equal contiguous ranges, one per CTA of a persistent grid:
+//     every SM gets the same share of the product whatever b is (one row tile
+//     or hundreds).  A CTA's range crosses a few rows; each piece (segment)
+//     accumulates in tensor memory -- for FP32 output in chunks of at most
+//     kChunkBlocks k-blocks whose results the epilogue adds with IEEE
+//     binary32 additions into a running sum kept in tensor memory (the tensor
+//     core's own accumulation error grows with the number of accumulation
+//     steps) -- and is written to the workspace as an FP32 partial.  Column
+//     groups are the slower index of the rows, so the CTAs working on the two
+//     groups of one row tile run side by side and the second read of an X
+//     tile hits L2.
 //  2. apply_w2_kernel -- every W entry adds its tile's partials in a fixed
 //     order (deterministic), is scaled by diag(s) in FP32 and written as
 //     binary16: a hi/lo pair (hi = fp16(w), lo = fp16(w - hi)) for FP32
 //     output, which keeps about 22 significand bits through the second
 //     product, or one rounding for FP16 output (the method-precision
 //     workspace of Sec. 3.4).  The layout is the shared-memory image of the
-//     second product's A operand, so it is loaded with one bulk copy.
+//     second product's A operand, so it is loaded with one bulk copy.  With
+//     many partials per row (small b) apply_w2_slice_kernel spreads each
+//     entry's partials over 16 warps.
 //  3. apply_y_kernel -- Y tiles = W U^T.  A persistent grid takes equal
 //     contiguous ranges of (row tile, column tile) pairs; W of the current
 //     row tile sits in shared memory, U streams through a TMA ring, and two
 //     tensor-memory accumulators let the epilogue drain one tile (TMEM ->
-//     registers -> swizzled shared memory -> TMA store, each epilogue warp
-//     storing its own 32 rows) while the next is multiplied.
-// Warp roles of kernels 1 and 3: warp 0 TMA producer, warp 1 tensor-memory
-// owner and MMA issuer (one thread), warps 2..5 epilogue (one TMEM lane = one
-// row per thread).  W is b x k' values, a few percent of the traffic.
+//     registers -> swizzled shared memory -> TMA stores of 128-row boxes, two
+//     warps per lane quarter on alternate column chunks) while the next is
+//     multiplied.
+// Warp roles: warp 0 TMA producer, warp 1 tensor-memory owner and MMA issuer
+// (one thread), then the epilogue warps (one TMEM lane = one row per thread;
+// four in kernel 1, eight in kernel 3).  W is b x k' values, a few percent of
+// the traffic.
 #include <cudaTypedefs.h>
 
 #include <mutex>
