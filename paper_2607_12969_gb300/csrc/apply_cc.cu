@@ -518,30 +518,19 @@ lrc_status launch_apply_f32(const float* U, const float* S, const float* Vt, con
         set_error("apply_f32: workspace size overflow");
         return LRC_ERR_INVALID_ARG;
     }
-    // LRC_F32_TC: room for the binary16 parts of W (operand images of 128-row
-    // tiles) and of U (rows of 3 k16) and the groups' exponents
-    tc = tc && k <= kF32TcMaxRank;
-    const int64_t kp3 = 3 * kp16;
-    const int64_t btiles = (b + 127) / 128;
-    const size_t tc_w = tc ? (size_t)btiles * 128 * kp3 * 2 : 0, tc_u = tc ? (size_t)m * kp3 * 2 : 0;
-    const int64_t ew = btiles * 128, eu = (m + kSplitRows - 1) / kSplitRows;   // W: a scale per row
-    const size_t tc_e = tc ? (size_t)(ew + eu) * sizeof(int) : 0;
+    // LRC_F32_TC: room for the binary16 parts of W and U (split_product_bytes)
+    tc = tc && split_product_fits(b, m, k);
     const size_t base = ((size_t)(part_elems + w_elems) * sizeof(float) + 255) / 256 * 256;
     void* ws = nullptr;
-    lrc_status st = stream_workspace(s, base + (tc_w + 255) / 256 * 256 + (tc_u + 255) / 256 * 256 + tc_e, &ws);
+    lrc_status st = stream_workspace(s, base + (tc ? split_product_bytes(b, m, k) : 0), &ws);
     if (st != LRC_OK) return st;
     float* part = static_cast<float*>(ws);
     float* Wd = part + part_elems;
     if ((st = gemm_cc_f32(X, ldn, Vt, ldn, true, part, kp16, b, k, n, (int)splits, w_elems, s)) != LRC_OK) return st;
     if ((st = launch_reduce_scale_f32(part, (int)splits, w_elems, b, k, kp16, S, Wd, s)) != LRC_OK) return st;
     if (!tc) return gemm_cc_f32(Wd, kp16, U, ldk, true, Y, m, b, m, k, 1, 0, s);
-    unsigned char* wimg = static_cast<unsigned char*>(ws) + base;
-    unsigned char* uimg = wimg + (tc_w + 255) / 256 * 256;
-    int* esc_w = reinterpret_cast<int*>(uimg + (tc_u + 255) / 256 * 256);
-    int* esc_u = esc_w + ew;
-    if ((st = launch_split_product(Wd, kp16, 1, U, ldk, 1, b, m, k, wimg, uimg, esc_w, esc_u, Y, s)) != LRC_OK)
-        return st;
-    return LRC_OK;
+    // Y (b x m) = W U^T with W = Wd (b x k, row pitch kp16) and U (m x k, row pitch ldk)
+    return launch_split_product(Wd, kp16, 1, U, ldk, 1, b, m, k, static_cast<unsigned char*>(ws) + base, Y, s);
 }
 
 }  // namespace lrc
