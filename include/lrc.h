@@ -199,9 +199,17 @@ LRC_API lrc_status tt_gather(const void* const* cores, const int64_t* dims, cons
  *   A, B        device arrays of `count` elements in formats fa, fb
  *               (LRC_F64, LRC_F32, or LRC_F16 / LRC_F16_O16 = binary16);
  *               B may be NULL, meaning B = 0
- *   diff_out    host: sqrt(sum_i (A_i - B_i)^2), differences and squares in
- *               binary64
+ *   diff_out    host: sqrt(sum_i (A_i - B_i)^2), sums in binary64
  *   normA_out   host, may be NULL: sqrt(sum_i A_i^2)
+ *
+ * Arithmetic: differences are binary64.  When both inputs are binary64, each
+ * square d^2 with 2^-48 <= |d| < 2^60 is formed from a binary32 pair split of
+ * d (its leading 24 and next 23 significand bits; the last 6 bits are
+ * dropped, a relative change of d of at most 2^-47) as an exact binary32
+ * two-product plus correction terms, summed in binary32 pairs and flushed to
+ * binary64 every 128 elements; other squares, and all squares of binary32 or
+ * binary16 inputs, are binary64 FMAs.  The result is within about 2^-46
+ * relative of the exactly rounded binary64 sum of squares.
  *
  * Summation is deterministic: fixed per-block partial sums reduced in a
  * fixed order, so repeated calls on the same data give identical bits.
@@ -232,7 +240,9 @@ LRC_API lrc_status lrc_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fm
  * share the one array and every call overwrites the entries it uses, so no
  * state carries over between calls, but calls whose kernels overlap on the
  * GPU (different streams, other threads) race on it and must be serialised by
- * the caller.  Synchronises `stream`.
+ * the caller.  The looked-up address is cached per device; a caller that
+ * resets a device (cudaDeviceReset) calls lrc_shutdown first, which forgets
+ * it.  Synchronises `stream`.
  */
 LRC_API lrc_status lrc_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb,
                                         int64_t count, double* diff_out, double* normA_out,

@@ -4,9 +4,10 @@ Argument marshalling only: every entry point forwards device pointers of
 torch tensors (torch is used for device memory and streams) and sizes to the
 C ABI declared in include/lrc.h, where every step runs in the library's own
 CUDA kernels.  Before forwarding, it refuses tensors that are not CUDA
-tensors of the format's element type with storage for the extent the call
-reads or writes (the C ABI cannot see buffer sizes).  There is no CPU fallback: if the library is missing or fails
-to load, every call raises.
+tensors of the format's element type, on the GPU the call runs on, with
+storage for the extent the call reads or writes (the C ABI cannot see buffer
+sizes or devices).  There is no CPU fallback: if the library is missing or
+fails to load, every call raises.
 
 Names follow the C ABI: lrc_round_factors, lrc_widen_factors, lrc_apply,
 tt_reconstruct, lrc_fro_diff, plus the host helpers lrc_certified,
@@ -138,17 +139,33 @@ def _span(t) -> int:
     return t.untyped_storage().nbytes() // t.element_size() - t.storage_offset()
 
 
-def _need(t, what: str, dtype=None, elems: int = 0) -> None:
+def _call_device(stream) -> int:
+    """Ordinal of the GPU a call runs on: the stream's device when a torch
+    stream is given, else the current device (whose stream a raw handle or
+    None names)."""
+    dev = getattr(stream, "device", None)
+    if dev is not None:
+        return dev.index if hasattr(dev, "index") else int(dev)
+    import torch
+    return torch.cuda.current_device()
+
+
+def _need(t, what: str, dtype=None, elems: int = 0, stream=None) -> None:
     """Marshalling checks that keep a call from reaching memory it does not
-    own: a CUDA tensor of the format's element type whose storage holds at
-    least `elems` elements from its first one.  (Layout and values are the
-    library's to check; sizes <= 0 are left to its validation.)"""
+    own: a CUDA tensor of the format's element type, on the GPU the call runs
+    on, whose storage holds at least `elems` elements from its first one.
+    (Layout and values are the library's to check; sizes <= 0 are left to its
+    validation.)"""
     if t is None:
         raise ValueError(f"{what}: a tensor is required")
     if not t.is_cuda:
         raise ValueError(f"{what}: must be a CUDA tensor (got device {t.device})")
     if dtype is not None and t.dtype != dtype:
         raise ValueError(f"{what}: element type {t.dtype}, the format needs {dtype}")
+    want = _call_device(stream)
+    if t.device.index is not None and t.device.index != want:
+        raise ValueError(f"{what}: on {t.device}, but the call runs on cuda:{want} (a kernel there "
+                         "cannot address another GPU's memory)")
     if elems > 0 and _span(t) < elems:
         raise ValueError(f"{what}: storage holds {_span(t)} elements from its start, the call reads or "
                          f"writes {elems}")
@@ -169,16 +186,16 @@ def lrc_packed_ld(cols: int) -> int:
 
 def lrc_round_factors(src, rows: int, cols: int, ld_src: int, dst, ld_dst: int, fmt, stream=None):
     import torch
-    _need(src, "src", torch.float64, _extent(rows, cols, ld_src))
-    _need(dst, "dst", storage_dtype(fmt), _extent(rows, ld_dst, ld_dst))
+    _need(src, "src", torch.float64, _extent(rows, cols, ld_src), stream=stream)
+    _need(dst, "dst", storage_dtype(fmt), _extent(rows, ld_dst, ld_dst), stream=stream)
     _check(load().lrc_round_factors(_ptr(src), rows, cols, ld_src, _ptr(dst), ld_dst, _fmt(fmt),
                                     _stream(stream)))
 
 
 def lrc_widen_factors(src, fmt, rows: int, cols: int, ld_src: int, dst, ld_dst: int, stream=None):
     import torch
-    _need(src, "src", storage_dtype(fmt), _extent(rows, cols, ld_src))
-    _need(dst, "dst", torch.float64, _extent(rows, ld_dst, ld_dst))
+    _need(src, "src", storage_dtype(fmt), _extent(rows, cols, ld_src), stream=stream)
+    _need(dst, "dst", torch.float64, _extent(rows, ld_dst, ld_dst), stream=stream)
     _check(load().lrc_widen_factors(_ptr(src), _fmt(fmt), rows, cols, ld_src, _ptr(dst), ld_dst,
                                     _stream(stream)))
 
@@ -186,29 +203,29 @@ def lrc_widen_factors(src, fmt, rows: int, cols: int, ld_src: int, dst, ld_dst: 
 def lrc_apply(U, S, Vt, X, Y, m: int, n: int, k: int, b: int, fmt, stream=None):
     if m > 0 and n > 0 and k > 0 and b > 0:
         st, ldk, ldn = storage_dtype(fmt), lrc_packed_ld(k), lrc_packed_ld(n)
-        _need(U, "U", st, _extent(m, k, ldk))
-        _need(S, "S", st, k)
-        _need(Vt, "Vt", st, _extent(k, n, ldn))
-        _need(X, "X", st, _extent(b, n, ldn))
-        _need(Y, "Y", output_dtype(fmt), b * m)
+        _need(U, "U", st, _extent(m, k, ldk), stream=stream)
+        _need(S, "S", st, k, stream=stream)
+        _need(Vt, "Vt", st, _extent(k, n, ldn), stream=stream)
+        _need(X, "X", st, _extent(b, n, ldn), stream=stream)
+        _need(Y, "Y", output_dtype(fmt), b * m, stream=stream)
     _check(load().lrc_apply(_ptr(U), _ptr(S), _ptr(Vt), _ptr(X), _ptr(Y), m, n, k, b, _fmt(fmt),
                             _stream(stream)))
 
 
-def _need_cores(cores, dims, ranks, fmt) -> bool:
+def _need_cores(cores, dims, ranks, fmt, stream=None) -> bool:
     """Checks the cores; True when dims and ranks describe them (else the
     library's validation reports the mismatch)."""
     d = len(cores)
     shaped = len(dims) == d and len(ranks) == d + 1 and all(int(x) > 0 for x in list(dims) + list(ranks))
     for l, c in enumerate(cores):
         _need(c, f"cores[{l}]", storage_dtype(fmt),
-              int(ranks[l]) * int(dims[l]) * int(ranks[l + 1]) if shaped else 0)
+              int(ranks[l]) * int(dims[l]) * int(ranks[l + 1]) if shaped else 0, stream=stream)
     return shaped
 
 
 def tt_reconstruct(cores: Sequence, dims: Sequence[int], ranks: Sequence[int], fmt, out, stream=None):
-    if _need_cores(cores, dims, ranks, fmt):
-        _need(out, "out", output_dtype(fmt), int(np_prod(dims)))
+    if _need_cores(cores, dims, ranks, fmt, stream):
+        _need(out, "out", output_dtype(fmt), int(np_prod(dims)), stream=stream)
     d = len(cores)
     ptrs = (ctypes.c_void_p * d)(*[c.data_ptr() for c in cores])
     dd = (ctypes.c_int64 * d)(*[int(x) for x in dims])
@@ -221,10 +238,10 @@ def tt_reconstruct(cores: Sequence, dims: Sequence[int], ranks: Sequence[int], f
 def tt_gather(cores: Sequence, dims: Sequence[int], ranks: Sequence[int], fmt, idx, out, stream=None):
     """Entries of the TT at the flat indices `idx` (int64 CUDA tensor) into `out`."""
     import torch
-    _need_cores(cores, dims, ranks, fmt)
-    _need(idx, "idx", torch.int64)
+    _need_cores(cores, dims, ranks, fmt, stream)
+    _need(idx, "idx", torch.int64, stream=stream)
     gather_dtype = {F64: torch.float64, F16_O16: torch.float16}.get(_fmt(fmt), torch.float32)
-    _need(out, "out", gather_dtype, int(idx.numel()))
+    _need(out, "out", gather_dtype, int(idx.numel()), stream=stream)
     d = len(cores)
     ptrs = (ctypes.c_void_p * d)(*[c.data_ptr() for c in cores])
     dd = (ctypes.c_int64 * d)(*[int(x) for x in dims])
@@ -238,9 +255,9 @@ def lrc_fro_diff(A, fa, B, fb, count: int, stream=None, want_norm: bool = True) 
     """Returns (||A - B||_F, ||A||_F); B may be None.  With want_norm=False
     ||A||_F is not computed (NaN is returned in its place)."""
     if count > 0:
-        _need(A, "A", storage_dtype(fa), count)
+        _need(A, "A", storage_dtype(fa), count, stream=stream)
         if B is not None:
-            _need(B, "B", storage_dtype(fb), count)
+            _need(B, "B", storage_dtype(fb), count, stream=stream)
     diff = ctypes.c_double(0.0)
     norm = ctypes.c_double(float("nan"))
     _check(load().lrc_fro_diff(_ptr(A), _fmt(fa), _ptr(B), _fmt(fb) if B is not None else 0, count,
@@ -253,9 +270,9 @@ def lrc_fro_diff_noalloc(A, fa, B, fb, count: int, stream=None) -> Tuple[float, 
     """lrc_fro_diff without any device allocation (scratch is a fixed array
     inside the library); at most 268435456 elements.  Returns (||A - B||_F, ||A||_F)."""
     if count > 0:
-        _need(A, "A", storage_dtype(fa), count)
+        _need(A, "A", storage_dtype(fa), count, stream=stream)
         if B is not None:
-            _need(B, "B", storage_dtype(fb), count)
+            _need(B, "B", storage_dtype(fb), count, stream=stream)
     diff = ctypes.c_double(0.0)
     norm = ctypes.c_double(0.0)
     _check(load().lrc_fro_diff_noalloc(_ptr(A), _fmt(fa), _ptr(B), _fmt(fb) if B is not None else 0, count,
@@ -274,11 +291,11 @@ def lrc_lowrank_eta(U, S, Vt, Uh, Sh, Vht, fmt, m: int, n: int, k: int, stream=N
         import torch
         ldk, ldn, st = lrc_packed_ld(k), lrc_packed_ld(n), storage_dtype(fmt)
         for t, what, dt in ((U, "U", torch.float64), (Uh, "Uh", st)):
-            _need(t, what, dt, _extent(m, k, ldk))
+            _need(t, what, dt, _extent(m, k, ldk), stream=stream)
         for t, what, dt in ((S, "S", torch.float64), (Sh, "Sh", st)):
-            _need(t, what, dt, k)
+            _need(t, what, dt, k, stream=stream)
         for t, what, dt in ((Vt, "Vt", torch.float64), (Vht, "Vht", st)):
-            _need(t, what, dt, _extent(k, n, ldn))
+            _need(t, what, dt, _extent(k, n, ldn), stream=stream)
     _check(load().lrc_lowrank_eta(_ptr(U), _ptr(S), _ptr(Vt), _ptr(Uh), _ptr(Sh), _ptr(Vht), _fmt(fmt),
                                   m, n, k, ctypes.addressof(eta),
                                   ctypes.addressof(norm) if want_norm else None, _stream(stream)))
@@ -293,9 +310,9 @@ def lrc_tt_eta(cores: Sequence, cores_hat: Sequence, dims: Sequence[int], ranks:
     shaped = len(dims) == d and len(ranks) == d + 1 and all(int(x) > 0 for x in list(dims) + list(ranks))
     for l, c in enumerate(cores):
         _need(c, f"cores[{l}]", torch.float64,
-              int(ranks[l]) * int(dims[l]) * int(ranks[l + 1]) if shaped else 0)
+              int(ranks[l]) * int(dims[l]) * int(ranks[l + 1]) if shaped else 0, stream=stream)
     if len(cores_hat) == d:
-        _need_cores(cores_hat, dims, ranks, fmt)
+        _need_cores(cores_hat, dims, ranks, fmt, stream)
     d = len(cores)
     if len(cores_hat) != d:
         raise ValueError("cores and cores_hat differ in length")

@@ -107,8 +107,11 @@ __device__ __forceinline__ void block_sum2(double& a, double& b, double* sh) {
 // and d^2 = hi^2 + (2 hi lo + lo^2) is formed with an exact two-product
 // (hi^2 = p + e, e = fma(hi, hi, -p)) and added to a binary32 pair sum with
 // two-sum.  Every 16 groups the pair sum is added to a binary64 accumulator.
-// Elements with |d| outside [2^-60, 2^60) (where hi^2 or a sum of them could
-// leave the binary32 range) are squared in binary64 instead.
+// Elements with |d| outside [2^-48, 2^60) are squared in binary64 instead:
+// above, a sum of hi^2 terms could overflow binary32; below, the correction
+// terms 2 hi lo and fma(hi, hi, -p) (about 2^-23 d^2) would fall under 2^-126,
+// into binary32 subnormals whose fixed spacing 2^-149 would cost more than
+// 2^-54 of d^2.
 // ---------------------------------------------------------------------------
 struct Pair {
     float hi = 0.0f, lo = 0.0f;
@@ -118,7 +121,7 @@ struct Pair {
 __device__ __forceinline__ bool split_hi_lo(double d, float& hi, float& lo) {
     const unsigned long long b = (unsigned long long)__double_as_longlong(d);
     const int e = (int)((b >> 52) & 0x7ffu);
-    if (e < 1023 - 60 || e >= 1023 + 60) {
+    if (e < 1023 - 48 || e >= 1023 + 60) {
         hi = lo = 0.0f;
         return (b << 1) == 0ull;
     }
@@ -304,8 +307,9 @@ lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, in
 // ---------------------------------------------------------------------------
 // Allocation-free variant.  The per-block partial sums go to a fixed array in
 // device memory that is part of the loaded library image, so the call never
-// allocates.  Its size caps the element count: one block per
-// kStaticElemsPerBlock elements, at most kStaticBlocks blocks.
+// allocates.  It holds kStaticBlocks block slots; the documented element
+// limit (kStaticBlocks x kStaticElemsPerBlock) is kept as the interface's
+// bound, the grid itself is that of the allocating path.
 // ---------------------------------------------------------------------------
 namespace {
 constexpr int kStaticBlocks = 4096;
@@ -344,13 +348,19 @@ lrc_status run_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fm
         }
         partial = g_static_ptr[dev];
     }
-    int grid = (int)((count + kStaticElemsPerBlock - 1) / kStaticElemsPerBlock);
-    if (grid < 1) grid = 1;
+    // the grid of the allocating path (the kernel strides over the groups),
+    // capped by the array's kStaticBlocks slots
+    const int64_t groups = count / kGroup;
+    const int64_t want = (groups + kThreads - 1) / kThreads;
+    int64_t cap = (int64_t)sm_count() * 4;
+    if (cap > kStaticBlocks) cap = kStaticBlocks;
+    const int grid = (int)(want < cap ? (want > 0 ? want : 1) : cap);
     const int a = fcode(fa), b = B ? fcode(fb) : -1;
+    const bool norm = normA_out != nullptr;
     switch (a) {
-        case 0: launch_partial<0>(b, grid, A, B, count, partial, s); break;
-        case 1: launch_partial<1>(b, grid, A, B, count, partial, s); break;
-        default: launch_partial<2>(b, grid, A, B, count, partial, s); break;
+        case 0: launch_partial<0>(b, grid, A, B, count, partial, s, norm); break;
+        case 1: launch_partial<1>(b, grid, A, B, count, partial, s, norm); break;
+        default: launch_partial<2>(b, grid, A, B, count, partial, s, norm); break;
     }
     lrc_status st = after_launch("fro_partial_kernel (no-alloc)");
     if (st != LRC_OK) return st;
@@ -369,6 +379,12 @@ lrc_status run_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fm
 }
 
 void release_scratch() {
+    {
+        // forget the looked-up array addresses: after a device reset the
+        // module is loaded again and the array may live elsewhere
+        std::lock_guard<std::mutex> lock(g_static_mu);
+        for (int d = 0; d < 64; ++d) g_static_ptr[d] = nullptr;
+    }
     std::lock_guard<std::mutex> lock(g_mu);
     int prev = -1;
     cudaGetDevice(&prev);

@@ -1,5 +1,6 @@
 """Host logic of bench.py that every reported fraction rests on: the
-algorithmic bytes and flops of each call (SURVEY 8(d) formulas) and the
+algorithmic bytes and flops of each call (the roofline formulas for the apply,
+the TT reconstruction, rounding and the Frobenius difference) and the
 cheapest contraction of a TT chain -- checked without a GPU."""
 import itertools
 

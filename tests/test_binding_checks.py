@@ -11,12 +11,13 @@ import paper_2607_12969_gb300 as lrc
 
 
 class AsCuda:
-    """A host tensor presented as a CUDA tensor to the binding's checks."""
+    """A host tensor presented as a CUDA tensor (on cuda:`index`) to the
+    binding's checks."""
 
-    def __init__(self, t):
+    def __init__(self, t, index: int = 0):
         self.t = t
         self.is_cuda = True
-        self.device = torch.device("cuda", 0)
+        self.device = torch.device("cuda", index)
         self.dtype = t.dtype
 
     def untyped_storage(self):
@@ -32,10 +33,16 @@ class AsCuda:
         return self.t.numel()
 
     def half(self):
-        return AsCuda(self.t.half())
+        return AsCuda(self.t.half(), self.device.index)
 
     def __getitem__(self, key):
-        return AsCuda(self.t[key])
+        return AsCuda(self.t[key], self.device.index)
+
+
+@pytest.fixture(autouse=True)
+def current_device_0(monkeypatch):
+    """The calls run on cuda:0 (the machine may have no GPU to ask)."""
+    monkeypatch.setattr(torch.cuda, "current_device", lambda: 0)
 
 
 def test_host_tensors_are_refused():
@@ -87,3 +94,28 @@ def test_views_are_measured_from_their_first_element():
     base = torch.zeros((5, 64))
     assert lrc._span(base[:, 1:]) == 5 * 64 - 1
     assert lrc._span(base[1:]) == 4 * 64
+
+
+def test_tensor_on_another_gpu_is_refused():
+    """A tensor on cuda:1 passed to a call that runs on cuda:0 would hand a
+    kernel a pointer into another GPU's memory: it is refused."""
+    m, n, k, b = 64, 48, 8, 5
+    h = lambda shape, dt, i=0: AsCuda(torch.zeros(shape, dtype=dt), i)    # noqa: E731
+    U, S = h((m, 16), torch.float32), h((1, 16), torch.float32)
+    Vt, X, Y = h((k, n), torch.float32), h((b, n), torch.float32), h((b, m), torch.float32)
+    with pytest.raises(ValueError, match="cuda:1"):
+        lrc.lrc_apply(U, S, Vt, h((b, n), torch.float32, 1), Y, m, n, k, b, "f32")
+    with pytest.raises(ValueError, match="cuda:1"):
+        lrc.lrc_apply(U, S, Vt, X, h((b, m), torch.float32, 1), m, n, k, b, "f32")
+    with pytest.raises(ValueError, match="cuda:1"):
+        lrc.tt_reconstruct([h((1, 6, 2), torch.float32), h((2, 5, 1), torch.float32, 1)], [6, 5], [1, 2, 1],
+                           "f32", h((30,), torch.float32))
+    with pytest.raises(ValueError, match="cuda:1"):
+        lrc.lrc_fro_diff(h((100,), torch.float64), "f64", h((100,), torch.float64, 1), "f64", 100)
+
+    class OnDevice1:
+        device = torch.device("cuda", 1)
+        cuda_stream = 0
+    # a stream of cuda:1 with tensors on cuda:0
+    with pytest.raises(ValueError, match="cuda:0, but the call runs on cuda:1"):
+        lrc.lrc_fro_diff(h((100,), torch.float64), "f64", None, "f64", 100, stream=OnDevice1())

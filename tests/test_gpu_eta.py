@@ -37,7 +37,7 @@ def test_fro_diff_mixed_formats(lrc, cuda, fa, fb):
 @pytest.mark.parametrize("lo,hi", [(-63, 63), (-62, -58), (58, 62), (-1074, -1000)])
 def test_fro_diff_f64_magnitude_ranges(lrc, cuda, lo, hi):
     """Values and differences whose binary exponents straddle the limits of
-    the binary32-pair squaring (|d| in [2^-60, 2^60)), binary64 subnormals,
+    the binary32-pair squaring (|d| in [2^-48, 2^60)), binary64 subnormals,
     zeros and both signs: the sum of squares stays within 1e-12 relative."""
     rng = np.random.default_rng(lo + 2000)
     count = 400_003
@@ -47,6 +47,19 @@ def test_fro_diff_f64_magnitude_ranges(lrc, cuda, lo, hi):
     a[::97] = 0.0
     b[::89] = a[::89]
     d, na = lrc.lrc_fro_diff(to_dev(a, cuda), "f64", to_dev(b, cuda), "f64", count)
+    wd, wna = oracle.fro_diff(a, b)
+    assert abs(d - wd) <= 1e-12 * wd and abs(na - wna) <= 1e-12 * wna
+
+
+@pytest.mark.parametrize("e", [-59, -54, -49, -48, -47])
+def test_fro_diff_few_small_differences(lrc, cuda, e):
+    """Eight differences of one size near the lower limit of the binary32-pair
+    squaring: no averaging over many elements hides a per-element error, so
+    each square must be accurate to well under 1e-12 on its own."""
+    rng = np.random.default_rng(50 - e)
+    a = rng.uniform(0.5, 1.0, 8)
+    b = a - np.ldexp(rng.uniform(0.5, 1.0, 8) * rng.choice([-1.0, 1.0], 8), e)
+    d, na = lrc.lrc_fro_diff(to_dev(a, cuda), "f64", to_dev(b, cuda), "f64", 8)
     wd, wna = oracle.fro_diff(a, b)
     assert abs(d - wd) <= 1e-12 * wd and abs(na - wna) <= 1e-12 * wna
 

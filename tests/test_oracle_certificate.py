@@ -125,3 +125,39 @@ def test_paper_rank_capping_example():
     # Sec. 7.4: Salinas-A (83 x 86 x 204) at nominal rank 160 gives R = (83, 160)
     assert W.capped_ranks((83, 86, 204), 160) == (1, 83, 160, 1)
     assert W.capped_ranks((83, 86, 204), 161) == (1, 83, 161, 1)
+
+
+def test_matrix_bound_pinned_to_eckart_young_equality():
+    """Thm 4.1 Eq. matrix_universal_bound at its equality case.  With eta = 0
+    the compensated factors are the exact rank-(k+1) truncation, whose error is
+    E_{k+1} = (E_k^2 - sigma_{k+1}^2)^(1/2) (Sec. 4, Eckart-Young), so the
+    bound must equal (i) the oracle's tail error at k + 1, (ii) the closed-form
+    geometric tail of the tiny workload's spectrum sigma_j = 2^(-j/16), and
+    (iii) the dense error ||A - A_{k+1}||_F itself; and it must grow with eta
+    at unit slope.  A dropped square root, a + in place of the -, the wrong
+    sigma index or a scaled eta each fail one of these."""
+    cfg = W.MATRIX_CONFIGS["tiny"]
+    q1, sig, q2 = W.matrix_bases(cfg, k_max=512)
+    ln2 = math.log(2.0)
+
+    def geo_tail(k):   # (sum_{j=k+1}^{512} 2^(-j/8))^(1/2), 1-based j
+        t2 = math.exp2(-(k + 1) / 8.0) * -math.expm1(-(512 - k) / 8.0 * ln2) / -math.expm1(-ln2 / 8.0)
+        return math.sqrt(t2)
+
+    for k in (0, 1, 31, 32, 33, 100, 255, 400, 510):
+        ek = oracle.tail_error(sig, k)
+        b0 = oracle.matrix_bound(ek, sig[k], 0.0)             # sig[k] = sigma_{k+1}
+        e_next = oracle.tail_error(sig, k + 1)
+        assert abs(b0 - e_next) <= 1e-14 * e_next, k
+        # closed form, with E_k also taken from the closed form
+        b0c = oracle.matrix_bound(geo_tail(k), math.exp2(-(k + 1) / 16.0), 0.0)
+        assert abs(b0c - geo_tail(k + 1)) <= 1e-13 * geo_tail(k + 1), k
+        for eta in (1e-9, 3.7e-4, 0.25):
+            assert abs(oracle.matrix_bound(ek, sig[k], eta) - (b0 + eta)) <= 1e-15 * (b0 + eta), (k, eta)
+    # (iii) the bound is attained: ||A - A_{k+1}||_F from the dense oracle products
+    A_T = (q2 * sig) @ q1.T
+    for k in (31, 32, 33):
+        f = W.truncate(q1, sig, q2, k + 1)
+        err, _ = oracle.fro_diff(A_T, oracle.apply(f.U, f.s, f.Vt, np.eye(512)))
+        b0 = oracle.matrix_bound(oracle.tail_error(sig, k), sig[k], 0.0)
+        assert abs(err - b0) <= 1e-12 * b0, k
