@@ -1,26 +1,37 @@
 #!/usr/bin/env python
 """Benchmark of the rank-compensation hot path on GB300.
 
-One step is one pass of the whole hot path over one synthetic batch:
+One step is one pass of the rank-compensated path (the paper's FP32 and FP16
+methods at the compensated ranks) over every workload of the benchmark
+definition, inputs resident in HBM:
 
-  round/pack  the FP64 factors U, s, V^T of every format (FP64 rank k = 128,
-              FP32 rank k' = 136, FP16 rank k' = 144), the query batch X
-              (8192 x 8192) and the TT cores, with lrc_round_factors;
-  apply       Y = [(X V) diag(s)] U^T in FP64 / FP32 / FP16 (FP32 out) /
-              FP16 (FP16 out), m = 16384, n = 8192, b = 8192 (lrc_apply);
-  TT          dense 256^3 reconstruction, ranks (1,32,32,1) FP64 and
-              (1,34,34,1) FP32 / FP16 / FP16-out (tt_reconstruct);
-  eta         FP64 dense reconstruction of the unrounded and of the widened
-              rounded factors / cores, then lrc_fro_diff (matrix and TT, FP32
-              and FP16);
-  certificate E_k' + eta <= E_k with E_k from the spectrum (lrc_certified).
+  matrices   tiny      m = n = 512,     b = 64,    k' = 33 (FP32) / 34 (FP16)
+             large     m = 16384, n = 8192, b = 8192,  k' = 136 / 144
+             sweep     m = n = 16384,   b = 32768, k' = 272 / 272
+  TT         256^3     ranks (1,34,34,1)
+             16^6      ranks (1,16,26|28,26|28,26|28,16,1)
+             512^2x224 ranks (1,70,52,1)
 
-The metric is the fraction of the GB300 roofline the step achieves:
-value = 100 * sum over calls of max(bytes / HBM peak, flops / format peak)
-divided by the step time, summed over GPUs (each GPU runs an independent
-replica of the step: weak scaling, no collective on the data path).
+  a1 round/pack the FP64 factors (U, s, V^T; TT cores) and query batches X to
+     FP32 and FP16 (and pack the FP64 factors at rank k' for eta)
+  a2-a4 apply Y = [(X V) diag(s)] U^T in FP32, FP16 (FP32 out), FP16 (FP16 out)
+  a5 TT reconstruction in the same three formats (outputs written to a
+     rotation of buffers larger than L2, so every call is judged against HBM)
+  a6 eta and eta_TT of the FP32 and FP16 storage (fused Gram-block route)
+  a7 the certificate E_k' + eta <= E_k (matrices).
+
+value = 100 x sum over the step's calls of max(bytes / HBM peak, flops /
+format peak), divided by the step time: the percentage of the GB300 roofline
+the whole step reaches, summed over GPUs (each GPU runs an independent
+replica with its own query batches: weak scaling, no collective).
+
+The FP64 baseline (rank k), the compensated calls and torch.matmul (the
+paper's own method, cuBLAS) are then timed in randomised paired blocks, as in
+the paper's Sec. 3.4 protocol: speedup = median over blocks of the paired
+ratio t(FP64, k) / t(fmt, k').
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+  python bench.py --case {apply,tt,round,fro,eta_matrix,eta_tt,eta_dense,gather,peaks} ...
 """
 from __future__ import annotations
 
@@ -43,13 +54,15 @@ import workloads as W  # noqa: E402
 
 METRIC = "rank-compensated apply / TT reconstruct: % of roofline, speedup vs FP64"
 UNIT = "% of GB300 roofline (summed over GPUs)"
-WORKLOAD = ("large-batch apply m=16384 n=8192 b=8192 k=128/136/144 + 3-way TT 256^3 "
-            "r=32/34, FP64/FP32/FP16/FP16-out, with rounding, eta and certificate")
+WORKLOAD = ("rank-compensated FP32/FP16/FP16-out path on all five configurations: apply m=n=512 b=64 "
+            "k'=33/34; apply m=16384 n=8192 b=8192 k'=136/144; apply m=n=16384 b=32768 k'=272; "
+            "TT 256^3 r=34, 16^6 r=26/28, 512x512x224 r=(70,52); with rounding, fused eta and certificate")
 
 # Peaks (per GPU).  HBM and the bf16 tensor peak are the driver's measured
 # copy / cuBLAS numbers; the CUDA-core FP32 and FP64 peaks are derived from
-# unit counts x maximum SM clock (152 SMs x 128 FP32 FMA/clk; FP64 at the
-# GB300's nominal 1.25 TFLOP/s).
+# unit counts x maximum SM clock: 152 SMs x 128 FP32 FMA/clk and 152 SMs x 2
+# FP64 FMA/clk (the GB300's nominal 1.25 TFLOP/s).  bench.py --case peaks
+# measures them (FMA-chain kernels and torch.matmul).
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "sm_max_mhz": 2070.0}
 
 
@@ -67,7 +80,7 @@ def load_peaks():
         "hbm": float(d.get("hbm_gbs", FALLBACK["hbm_gbs"])) * 1e9,                 # B/s
         "f16": float(d.get("bf16_tflops_sustained", FALLBACK["bf16_tflops_sustained"])) * 1e12,
         "f32": 152 * 128 * 2 * mhz * 1e6,                                          # FFMA
-        "f64": 1.25e12,                                                            # DFMA, nominal
+        "f64": 152 * 2 * 2 * mhz * 1e6,                                            # DFMA
     }
 
 
@@ -79,6 +92,12 @@ ALU = {"f64": "f64", "f32": "f32", "f16": "f16", "f16_o16": "f16", "f32tc": None
 # three binary16 products (hi/lo split), the rest on the CUDA cores.  Its
 # arithmetic bound is the sum of the two engines' times (alu_time).
 F32TC_PASSES = 3
+COMP = ("f32", "f16", "f16_o16")          # the compensated formats
+STORE = ("f32", "f16")                   # their storage formats
+
+
+def store_of(fmt: str) -> str:
+    return "f16" if fmt.startswith("f16") else ("f32" if fmt == "f32tc" else fmt)
 
 
 # ---------------------------------------------------------------------------
@@ -86,10 +105,9 @@ F32TC_PASSES = 3
 # ---------------------------------------------------------------------------
 
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from
-# one ncu capture of the call type's kernel as it stands; an entry is removed
-# when its kernel changes.  apply_f64_dense: profiles/
-# apply_cc_kernel_f64_m16384_n8192_b8192_k144.md.
-MEASURED_TRAFFIC = {"apply_f64_dense": 604_804_096 + 1_014_732_288}
+# one ncu capture of the call type's kernels as they stand; an entry is
+# removed when its kernels change.
+MEASURED_TRAFFIC: dict = {}
 
 
 def work_round(rows, cols, ld, fmt):
@@ -190,69 +208,149 @@ def bound_of(w):
     return "tensor" if w["alu"] == "f16" else "alu"
 
 
+def rotation(nbytes: int, floor: int = 2 * 129 * 2 ** 20) -> int:
+    """Number of output buffers of `nbytes` that together exceed `floor`
+    bytes (twice the GB300's 129 MB L2): writing them in turn makes every
+    call's output miss L2, as a single call on a cold GPU would."""
+    return max(1, -(-floor // max(1, nbytes)) + (1 if nbytes < floor else 0))
+
+
 # ---------------------------------------------------------------------------
-# the step
+# workloads of the step
 # ---------------------------------------------------------------------------
 
-class Step:
-    """Holds the resident inputs/outputs and issues one pass of the hot path."""
+MATRIX_WL = ("tiny", "large", "sweep")     # cfg 1, cfg 2, cfg 5 (b = 32768)
+TT_WL = ("tt3", "tt6", "tt_hsi")           # cfg 3, cfg 4, cfg 5
 
-    def __init__(self, lrc, dev, seed_offset=0):
-        import torch
-        self.lrc, self.dev, self.torch = lrc, dev, torch
-        cfg = W.MATRIX_CONFIGS["large"]
+
+def matrix_cfg(name):
+    return W.sweep_config(32768) if name == "sweep" else W.MATRIX_CONFIGS[name]
+
+
+class MatrixWL:
+    """Resident inputs and outputs of one matrix workload."""
+
+    def __init__(self, lrc, torch, dev, name, replica):
+        self.name = name
+        cfg = matrix_cfg(name)
         self.cfg = cfg
         q1, sig, q2 = W.matrix_bases(cfg)
         self.sigma = sig
-        X = W.queries(cfg, replica=seed_offset)   # every rank: its own batch of the same shape
-        self.host = {"Q1": np.ascontiguousarray(q1), "Q2t": np.ascontiguousarray(q2.T), "s": sig[:cfg.k_max].copy(),
-                     "X": X}
-        ttc = W.TT_CONFIGS["tt3"]
-        self.tt = ttc
-        self.host_tt = {f: W.tt_cores(ttc, f) for f in ("f64", "f32", "f16")}
-        self.timers = []
-        self.alloc()
-
-    def alloc(self):
-        torch, lrc, dev, cfg = self.torch, self.lrc, self.dev, self.cfg
+        self.host = {"Q1": np.ascontiguousarray(q1), "Q2t": np.ascontiguousarray(q2.T),
+                     "s": sig[:cfg.k_max][None, :].copy(), "X": W.queries(cfg, replica=replica)}
         m, n, b = cfg.m, cfg.n, cfg.b
         T = lambda shape, dt: torch.empty(shape, dtype=dt, device=dev)  # noqa: E731
-        h = self.host
-        self.d_Q1 = torch.from_numpy(h["Q1"]).to(dev)            # m x 144 (ld 144)
-        self.d_Q2t = torch.from_numpy(h["Q2t"]).to(dev)          # 144 x n
-        self.d_s = torch.from_numpy(h["s"][None, :]).to(dev)     # 1 x 144
-        self.d_X = torch.from_numpy(h["X"]).to(dev)              # b x n FP64 (ld = n)
-        self.d_I = torch.eye(n, dtype=torch.float64, device=dev)
+        self.d = {k: torch.from_numpy(v).to(dev) for k, v in self.host.items()}
+        self.kp = {s: cfg.ranks[s] for s in STORE}
+        self.k = cfg.ranks["f64"]
+        ld = lrc.lrc_packed_ld
         self.fac = {}
-        for fmt in ("f64", "f32", "f16", "f16_o16"):
-            base = "f16" if fmt.startswith("f16") else fmt
-            k = cfg.ranks[base]
-            dt = lrc.storage_dtype(fmt)
-            self.fac[fmt] = {
-                "k": k,
-                "U": T((m, lrc.lrc_packed_ld(k)), dt),
-                "S": T((1, lrc.lrc_packed_ld(k)), dt),
-                "Vt": T((k, lrc.lrc_packed_ld(n)), dt),
-                "Y": T((b, m), lrc.output_dtype(fmt)),
-            }
-        self.Xr = {"f32": T((b, n), torch.float32), "f16": T((b, n), torch.float16)}
-        self.wide = {f: {"U": T((m, lrc.lrc_packed_ld(cfg.ranks[f])), torch.float64),
-                         "S": T((1, lrc.lrc_packed_ld(cfg.ranks[f])), torch.float64),
-                         "Vt": T((cfg.ranks[f], n), torch.float64)} for f in ("f32", "f16")}
-        self.dense = T((n, m), torch.float64)
-        self.dense_hat = T((n, m), torch.float64)
-        # TT
-        tt = self.tt
-        N = int(np.prod(tt.dims))
-        self.tt_dev = {f: [torch.from_numpy(c).to(dev) for c in self.host_tt[f]] for f in ("f64", "f32", "f16")}
-        self.tt_low = {f: [T(c.shape, lrc.storage_dtype(f)) for c in self.host_tt[f]] for f in ("f32", "f16")}
-        self.tt_wide = {f: [T(c.shape, torch.float64) for c in self.host_tt[f]] for f in ("f32", "f16")}
-        self.tt_out = {f: T((N,), lrc.output_dtype(f)) for f in ("f64", "f32", "f16", "f16_o16")}
-        self.tt_T = T((N,), torch.float64)
-        self.tt_That = T((N,), torch.float64)
+        for s in STORE:
+            k = self.kp[s]
+            dt = lrc.storage_dtype(s)
+            self.fac[s] = {"U": T((m, ld(k)), dt), "S": T((1, ld(k)), dt), "Vt": T((k, ld(n)), dt),
+                           "X": T((b, ld(n)), dt), "U64": T((m, ld(k)), torch.float64)}
+        self.Y = {f: T((b, m), lrc.output_dtype(f)) for f in COMP}
         self.results = {}
 
-    # -- timing helpers ------------------------------------------------------
+    def calls(self, lrc, step):
+        """Rounding (a1) and applies (a2-a4) of this workload."""
+        cfg, d = self.cfg, self.d
+        m, n, b = cfg.m, cfg.n, cfg.b
+        kmax = d["Q1"].shape[1]
+        for s in STORE:
+            F, k = self.fac[s], self.kp[s]
+            step.timed(f"round@{self.name}", work_round(m, k, F["U64"].shape[1], "f64"),
+                       lambda: lrc.lrc_round_factors(d["Q1"], m, k, kmax, F["U64"], F["U64"].shape[1], "f64"))
+            step.timed(f"round@{self.name}", work_round(m, k, F["U"].shape[1], s),
+                       lambda: lrc.lrc_round_factors(d["Q1"], m, k, kmax, F["U"], F["U"].shape[1], s))
+            step.timed(f"round@{self.name}", work_round(1, k, F["S"].shape[1], s),
+                       lambda: lrc.lrc_round_factors(d["s"], 1, k, kmax, F["S"], F["S"].shape[1], s))
+            step.timed(f"round@{self.name}", work_round(k, n, F["Vt"].shape[1], s),
+                       lambda: lrc.lrc_round_factors(d["Q2t"], k, n, n, F["Vt"], F["Vt"].shape[1], s))
+            step.timed(f"round@{self.name}", work_round(b, n, F["X"].shape[1], s),
+                       lambda: lrc.lrc_round_factors(d["X"], b, n, n, F["X"], F["X"].shape[1], s))
+        for f in COMP:
+            F, k = self.fac[store_of(f)], self.kp[store_of(f)]
+            step.timed(f"apply_{f}@{self.name}", work_apply(m, n, k, b, f),
+                       lambda: lrc.lrc_apply(F["U"], F["S"], F["Vt"], F["X"], self.Y[f], m, n, k, b, f))
+
+    def eta_calls(self, lrc, step):
+        """eta of each storage format (a6, fused route) and the certificate (a7)."""
+        cfg, d = self.cfg, self.d
+        m, n = cfg.m, cfg.n
+        Ek = lrc.lrc_tail_error(self.sigma, self.k)
+        for s in STORE:
+            F, k = self.fac[s], self.kp[s]
+            res = {}
+            step.timed(f"eta_matrix@{self.name}", work_eta_lowrank(m, n, k, s), lambda: res.update(
+                eta=lrc.lrc_lowrank_eta(F["U64"], d["s"], d["Q2t"][:k], F["U"], F["S"], F["Vt"], s, m, n, k,
+                                        want_norm=False)[0]))
+            Ekp = lrc.lrc_tail_error(self.sigma, k)
+            self.results[f"eta_{s}"] = res["eta"]
+            self.results[f"certified_{s}"] = lrc.lrc_certified(Ek, Ekp, res["eta"])
+        self.results["E_k"] = Ek
+
+
+class TTWL:
+    """Resident cores and rotating outputs of one TT workload."""
+
+    def __init__(self, lrc, torch, dev, name):
+        self.name = name
+        cfg = W.TT_CONFIGS[name]
+        self.cfg = cfg
+        self.host = {s: W.tt_cores(cfg, s) for s in ("f64",) + STORE}
+        self.c64 = {s: [torch.from_numpy(c).to(dev) for c in self.host[s]] for s in STORE}
+        self.low = {s: [torch.empty(c.shape, dtype=lrc.storage_dtype(s), device=dev) for c in self.host[s]]
+                    for s in STORE}
+        N = int(np.prod(cfg.dims))
+        self.N = N
+        self.out = {}
+        for f in COMP:
+            dt = lrc.output_dtype(f)
+            nb = N * torch.empty((), dtype=dt).element_size()
+            self.out[f] = [torch.empty(N, dtype=dt, device=dev) for _ in range(rotation(nb))]
+        self.turn = 0
+        self.results = {}
+
+    def calls(self, lrc, step):
+        cfg = self.cfg
+        for s in STORE:
+            for src, dst in zip(self.c64[s], self.low[s]):
+                cnt = src.numel()
+                step.timed(f"round@{self.name}", work_round(1, cnt, cnt, s),
+                           lambda: lrc.lrc_round_factors(src, 1, cnt, cnt, dst, cnt, s))
+        for f in COMP:
+            s = store_of(f)
+            outs = self.out[f]
+            o = outs[self.turn % len(outs)]
+            step.timed(f"tt_{f}@{self.name}", work_tt(cfg.dims, cfg.ranks[s], f),
+                       lambda: lrc.tt_reconstruct(self.low[s], cfg.dims, cfg.ranks[s], f, o))
+        self.turn += 1
+
+    def last_outputs(self):
+        return {f: self.out[f][(self.turn - 1) % len(self.out[f])] for f in COMP}
+
+    def eta_calls(self, lrc, step):
+        cfg = self.cfg
+        for s in STORE:
+            res = {}
+            step.timed(f"eta_tt@{self.name}", work_eta_tt(cfg.dims, cfg.ranks[s], s), lambda: res.update(
+                eta=lrc.lrc_tt_eta(self.c64[s], self.low[s], cfg.dims, cfg.ranks[s], s, want_norm=False)[0]))
+            self.results[f"eta_{s}"] = res["eta"]
+
+
+class Step:
+    """One pass of the rank-compensated path over every workload."""
+
+    def __init__(self, lrc, dev, replica=0):
+        import torch
+        self.lrc, self.dev, self.torch = lrc, dev, torch
+        self.mats = [MatrixWL(lrc, torch, dev, n, replica) for n in MATRIX_WL]
+        self.tts = [TTWL(lrc, torch, dev, n) for n in TT_WL]
+        self.timers = []
+        self.record = False
+
     def timed(self, name, work, fn):
         torch = self.torch
         if self.record:
@@ -265,104 +363,30 @@ class Step:
         else:
             fn()
 
-    def run(self, record=False, on_outputs=None):
-        """One pass of the path.  on_outputs, if given, is called once the
+    def run(self, record=False, on_outputs=None, wait_inputs=None):
+        """One pass.  wait_inputs(workload), if given, is called before a
+        workload's first call (the end-to-end run makes the stream wait for
+        that workload's input copies there); on_outputs, if given, once the
         apply and TT outputs are enqueued (the eta and certificate work that
         follows reads none of them)."""
         self.record = record
-        lrc, cfg = self.lrc, self.cfg
-        m, n, b = cfg.m, cfg.n, cfg.b
-        # a1: round / pack factors of every format and the query batch
-        for fmt, F in self.fac.items():
-            k = F["k"]
-            self.timed("round", work_round(m, k, F["U"].shape[1], fmt), lambda: lrc.lrc_round_factors(
-                self.d_Q1, m, k, self.d_Q1.shape[1], F["U"], F["U"].shape[1], fmt))
-            self.timed("round", work_round(1, k, F["S"].shape[1], fmt), lambda: lrc.lrc_round_factors(
-                self.d_s, 1, k, self.d_s.shape[1], F["S"], F["S"].shape[1], fmt))
-            self.timed("round", work_round(k, n, n, fmt), lambda: lrc.lrc_round_factors(
-                self.d_Q2t, k, n, n, F["Vt"], n, fmt))
-        for fmt, Xr in self.Xr.items():
-            self.timed("round", work_round(b, n, n, fmt), lambda: lrc.lrc_round_factors(
-                self.d_X, b, n, n, Xr, n, fmt))
-        for fmt in ("f32", "f16"):
-            for src, dst in zip(self.tt_dev[fmt], self.tt_low[fmt]):
-                cnt = src.numel()
-                self.timed("round", work_round(1, cnt, cnt, fmt), lambda: lrc.lrc_round_factors(
-                    src, 1, cnt, cnt, dst, cnt, fmt))
-        # a2-a4: the four applies
-        for fmt, F in self.fac.items():
-            X = self.d_X if fmt == "f64" else (self.Xr["f32"] if fmt == "f32" else self.Xr["f16"])
-            self.timed(f"apply_{fmt}", work_apply(m, n, F["k"], b, fmt), lambda: lrc.lrc_apply(
-                F["U"], F["S"], F["Vt"], X, F["Y"], m, n, F["k"], b, fmt))
-        # a5: TT reconstructions
-        tt = self.tt
-        for fmt in ("f64", "f32", "f16", "f16_o16"):
-            base = "f16" if fmt.startswith("f16") else fmt
-            cores = self.tt_dev["f64"] if fmt == "f64" else self.tt_low[base]
-            ranks = tt.ranks[base]
-            self.timed(f"tt_{fmt}", work_tt(tt.dims, ranks, fmt), lambda: lrc.tt_reconstruct(
-                cores, tt.dims, ranks, fmt, self.tt_out[fmt]))
+        lrc = self.lrc
+        order = [self.mats[1]] + self.tts + [self.mats[0], self.mats[2]]
+        for wl in order:
+            if wait_inputs is not None:
+                wait_inputs(wl)
+            wl.calls(lrc, self)
         if on_outputs is not None:
             on_outputs()
-        # a6: eta for the matrix (FP64 dense products of unrounded and widened factors)
-        for fmt in ("f32", "f16"):
-            F = self.fac[fmt]
-            k = F["k"]
-            Wd = self.wide[fmt]
-            self.timed("apply_f64_dense", work_apply(m, n, k, n, "f64"), lambda: lrc.lrc_apply(
-                self.fac_f64_view(k, "U"), self.fac_f64_view(k, "S"), self.fac_f64_view(k, "Vt"),
-                self.d_I, self.dense, m, n, k, n, "f64"))
-            self.timed("widen", work_widen(m, k, Wd["U"].shape[1], fmt), lambda: lrc.lrc_widen_factors(
-                F["U"], fmt, m, k, F["U"].shape[1], Wd["U"], Wd["U"].shape[1]))
-            self.timed("widen", work_widen(1, k, Wd["S"].shape[1], fmt), lambda: lrc.lrc_widen_factors(
-                F["S"], fmt, 1, k, F["S"].shape[1], Wd["S"], Wd["S"].shape[1]))
-            self.timed("widen", work_widen(k, n, n, fmt), lambda: lrc.lrc_widen_factors(
-                F["Vt"], fmt, k, n, n, Wd["Vt"], n))
-            self.timed("apply_f64_dense", work_apply(m, n, k, n, "f64"), lambda: lrc.lrc_apply(
-                Wd["U"], Wd["S"], Wd["Vt"], self.d_I, self.dense_hat, m, n, k, n, "f64"))
-            res = {}
-            self.timed("fro_diff", work_fro(m * n, "f64", "f64"), lambda: res.update(
-                eta=lrc.lrc_fro_diff(self.dense, "f64", self.dense_hat, "f64", m * n, want_norm=False)[0]))
-            self.results[f"eta_matrix_{fmt}"] = res["eta"]
-        # a6: eta for the TT
-        N = int(np.prod(tt.dims))
-        for fmt in ("f32", "f16"):
-            ranks = tt.ranks[fmt]
-            self.timed("tt_f64_eta", work_tt(tt.dims, ranks, "f64"), lambda: lrc.tt_reconstruct(
-                self.tt_dev[fmt], tt.dims, ranks, "f64", self.tt_T))
-            for src, dst in zip(self.tt_low[fmt], self.tt_wide[fmt]):
-                cnt = src.numel()
-                self.timed("widen", work_widen(1, cnt, cnt, fmt), lambda: lrc.lrc_widen_factors(
-                    src, fmt, 1, cnt, cnt, dst, cnt))
-            self.timed("tt_f64_eta", work_tt(tt.dims, ranks, "f64"), lambda: lrc.tt_reconstruct(
-                self.tt_wide[fmt], tt.dims, ranks, "f64", self.tt_That))
-            res = {}
-            self.timed("fro_diff", work_fro(N, "f64", "f64"), lambda: res.update(
-                eta=lrc.lrc_fro_diff(self.tt_T, "f64", self.tt_That, "f64", N, want_norm=False)[0]))
-            self.results[f"eta_tt_{fmt}"] = res["eta"]
-        # a7: certificate (Eq. matrix_condition)
-        Ek = lrc.lrc_tail_error(self.sigma, cfg.ranks["f64"])
-        for fmt in ("f32", "f16"):
-            Ekp = lrc.lrc_tail_error(self.sigma, cfg.ranks[fmt])
-            self.results[f"certified_{fmt}"] = lrc.lrc_certified(Ek, Ekp, self.results[f"eta_matrix_{fmt}"])
-        self.results["E_k"] = Ek
+        for wl in self.mats + self.tts:
+            wl.eta_calls(lrc, self)
 
-    def fac_f64_view(self, k, what):
-        """Packed FP64 factors at rank k (the unrounded factors used for eta)."""
-        key = f"_f64_{what}_{k}"
-        if not hasattr(self, key):
-            lrc, cfg, torch = self.lrc, self.cfg, self.torch
-            m, n = cfg.m, cfg.n
-            if what == "U":
-                t = torch.empty((m, lrc.lrc_packed_ld(k)), dtype=torch.float64, device=self.dev)
-                lrc.lrc_round_factors(self.d_Q1, m, k, self.d_Q1.shape[1], t, t.shape[1], "f64")
-            elif what == "S":
-                t = torch.empty((1, lrc.lrc_packed_ld(k)), dtype=torch.float64, device=self.dev)
-                lrc.lrc_round_factors(self.d_s, 1, k, self.d_s.shape[1], t, t.shape[1], "f64")
-            else:
-                t = self.d_Q2t[:k]
-            setattr(self, key, t)
-        return getattr(self, key)
+    def results(self):
+        out = {}
+        for wl in self.mats + self.tts:
+            for k, v in wl.results.items():
+                out[f"{k}@{wl.name}"] = v if isinstance(v, bool) else float(v)
+        return out
 
     def summarize(self):
         """Per-call-type durations (ms) of the recorded calls and roofline time."""
@@ -380,6 +404,139 @@ class Step:
             p["flops"] += work["flops"]
             p["rt_s"] += rt
         return per, total_rt
+
+
+# ---------------------------------------------------------------------------
+# paired protocol: FP64 baseline, compensated formats and torch.matmul
+# ---------------------------------------------------------------------------
+
+def torch_apply(torch, X, Vt, S, U, k, n, W_, Y):
+    """The paper's GPU apply (Sec. 4.4): two library GEMMs and a column
+    scaling, in the storage precision (binary16 workspace for FP16)."""
+    torch.matmul(X[:, :n], Vt[:k, :n].t(), out=W_)
+    W_.mul_(S[0, :k])
+    torch.matmul(W_, U[:, :k].t(), out=Y)
+
+
+def torch_tt(torch, cores, dims, ranks, bufs):
+    """The paper's GPU TT reconstruction (Sec. 7.5): a chain of library GEMMs
+    Z_l = reshape(Z_{l-1}) K_l, left to right, in the storage precision."""
+    Z = cores[0].reshape(dims[0], ranks[1])
+    for l in range(1, len(dims)):
+        K = cores[l].reshape(ranks[l], dims[l] * ranks[l + 1])
+        torch.matmul(Z, K, out=bufs[l - 1])
+        Z = bufs[l - 1].view(-1, ranks[l + 1])
+    return Z
+
+
+class Paired:
+    """Calls of the paired blocks: for every workload, the FP64 call at rank k
+    and the compensated calls at rank k' through this library, and
+    torch.matmul in FP64, FP32 and FP16 (FP16 output)."""
+
+    def __init__(self, lrc, torch, dev, step):
+        self.calls = []       # (workload, method, impl, fn)
+        ld = lrc.lrc_packed_ld
+        self.keep = []
+        for wl in step.mats:
+            cfg, d = wl.cfg, wl.d
+            m, n, b, k = cfg.m, cfg.n, cfg.b, wl.k
+            kmax = d["Q1"].shape[1]
+            U64 = torch.empty((m, ld(k)), dtype=torch.float64, device=dev)
+            S64 = torch.empty((1, ld(k)), dtype=torch.float64, device=dev)
+            lrc.lrc_round_factors(d["Q1"], m, k, kmax, U64, U64.shape[1], "f64")
+            lrc.lrc_round_factors(d["s"], 1, k, kmax, S64, S64.shape[1], "f64")
+            Vt64 = d["Q2t"][:k]
+            Y64 = torch.empty((b, m), dtype=torch.float64, device=dev)
+            self.keep += [U64, S64, Y64]
+            self.calls.append((wl.name, "f64", "ours", lambda U64=U64, S64=S64, Vt64=Vt64, Y64=Y64, d=d, m=m, n=n,
+                               k=k, b=b: lrc.lrc_apply(U64, S64, Vt64, d["X"], Y64, m, n, k, b, "f64")))
+            for f in COMP:
+                F, kp = wl.fac[store_of(f)], wl.kp[store_of(f)]
+                self.calls.append((wl.name, f, "ours", lambda F=F, kp=kp, f=f, wl=wl, m=m, n=n, b=b: lrc.lrc_apply(
+                    F["U"], F["S"], F["Vt"], F["X"], wl.Y[f], m, n, kp, b, f)))
+            # torch.matmul in each storage precision
+            for f, (U, S, Vt, X, kk) in (("f64", (U64, S64, Vt64, d["X"], k)),
+                                         ("f32", (wl.fac["f32"]["U"], wl.fac["f32"]["S"], wl.fac["f32"]["Vt"],
+                                                  wl.fac["f32"]["X"], wl.kp["f32"])),
+                                         ("f16_o16", (wl.fac["f16"]["U"], wl.fac["f16"]["S"], wl.fac["f16"]["Vt"],
+                                                      wl.fac["f16"]["X"], wl.kp["f16"]))):
+                Wt = torch.empty((b, kk), dtype=U.dtype, device=dev)
+                Yt = torch.empty((b, m), dtype=U.dtype, device=dev)
+                self.keep += [Wt, Yt]
+                self.calls.append((wl.name, f, "torch", lambda U=U, S=S, Vt=Vt, X=X, kk=kk, Wt=Wt, Yt=Yt, n=n:
+                                   torch_apply(torch, X, Vt, S, U, kk, n, Wt, Yt)))
+        for wl in step.tts:
+            cfg = wl.cfg
+            c64 = [torch.from_numpy(c).to(dev) for c in wl.host["f64"]]
+            r64 = cfg.ranks["f64"]
+            outs64 = [torch.empty(wl.N, dtype=torch.float64, device=dev) for _ in range(rotation(wl.N * 8))]
+            self.keep += c64 + outs64
+            turn = {"i": 0}
+
+            def tt64(c64=c64, r64=r64, outs64=outs64, turn=turn, cfg=cfg):
+                turn["i"] += 1
+                lrc.tt_reconstruct(c64, cfg.dims, r64, "f64", outs64[turn["i"] % len(outs64)])
+            self.calls.append((wl.name, "f64", "ours", tt64))
+            for f in COMP:
+                s = store_of(f)
+
+                def ttf(f=f, s=s, wl=wl, cfg=cfg):
+                    outs = wl.out[f]
+                    wl.turn += 1
+                    lrc.tt_reconstruct(wl.low[s], cfg.dims, cfg.ranks[s], f, outs[wl.turn % len(outs)])
+                self.calls.append((wl.name, f, "ours", ttf))
+            for f, cores, ranks in (("f64", c64, r64), ("f32", wl.low["f32"], cfg.ranks["f32"]),
+                                    ("f16_o16", wl.low["f16"], cfg.ranks["f16"])):
+                bufs, rows = [], cfg.dims[0]
+                for l in range(1, len(cfg.dims)):
+                    bufs.append(torch.empty((rows, cfg.dims[l] * ranks[l + 1]), dtype=cores[0].dtype, device=dev))
+                    rows *= cfg.dims[l]
+                self.keep += bufs
+                self.calls.append((wl.name, f, "torch", lambda cores=cores, ranks=ranks, bufs=bufs, cfg=cfg:
+                                   torch_tt(torch, cores, cfg.dims, ranks, bufs)))
+
+    def run(self, torch, blocks, seed=20260):
+        """Randomised blocks; returns {(workload, method, impl): [ms per block]}."""
+        rng = np.random.default_rng(seed)
+        times = {(w, f, i): [] for w, f, i, _ in self.calls}
+        for _ in range(blocks):
+            order = rng.permutation(len(self.calls))
+            evs = []
+            torch.cuda.synchronize()
+            # queue the block behind a GPU-side wait so host-side marshalling
+            # opens no gaps between the calls
+            torch.cuda._sleep(int(2.0e6 + 1.5e5 * len(self.calls)))
+            for j in order:
+                w, f, i, fn = self.calls[j]
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                fn()
+                e1.record()
+                evs.append(((w, f, i), e0, e1))
+            torch.cuda.synchronize()
+            for key, e0, e1 in evs:
+                times[key].append(e0.elapsed_time(e1))
+        return times
+
+
+def paired_report(times, kind_of):
+    """Median over blocks of paired ratios (Sec. 3.4 protocol)."""
+    speed, vs_torch, ms, torch_ms = {}, {}, {}, {}
+    for (w, f, i), ts in times.items():
+        key = f"{kind_of[w]}_{f}@{w}"
+        (ms if i == "ours" else torch_ms)[key] = statistics.median(ts)
+    for (w, f, i), ts in times.items():
+        if i != "ours":
+            continue
+        key = f"{kind_of[w]}_{f}@{w}"
+        if f != "f64":
+            base = times[(w, "f64", "ours")]
+            speed[key] = statistics.median(b / t for b, t in zip(base, ts))
+        tk = (w, f, "torch")
+        if tk in times:
+            vs_torch[key] = statistics.median(tt / t for tt, t in zip(times[tk], ts))
+    return speed, vs_torch, ms, torch_ms
 
 
 # ---------------------------------------------------------------------------
@@ -485,67 +642,96 @@ def aggregate_value(rt_sum_all_ranks: float, ms_per_step_max: float) -> float:
 # CPU oracle (the reference arm and the cpu_baseline)
 # ---------------------------------------------------------------------------
 
-ORACLE_ROWS = 256        # query rows per apply in the sampled oracle step
-ORACLE_TT_SLAB = 8       # i_1 slices of the 256^3 tensor per TT reconstruction
+# bounded sample of one step: query rows per apply and rows of the dense
+# products behind eta, per matrix workload; leading-index slabs per TT
+ORACLE_ROWS = {"tiny": None, "large": 256, "sweep": 96}     # None: the whole workload
+ORACLE_SLABS = {"tt3": 32, "tt6": 4, "tt_hsi": 16}
+
+
+def oracle_context():
+    ctx = {"mat": {}, "tt": {}}
+    for name in MATRIX_WL:
+        cfg = matrix_cfg(name)
+        q1, sig, q2 = W.matrix_bases(cfg)
+        rows = ORACLE_ROWS[name]
+        ctx["mat"][name] = {"cfg": cfg, "U": q1, "s": sig, "Vt": np.ascontiguousarray(q2.T),
+                            "X": W.queries(cfg, b=rows if rows is not None else cfg.b)}
+    for name in TT_WL:
+        cfg = W.TT_CONFIGS[name]
+        ctx["tt"][name] = {"cfg": cfg, "cores": {s: W.tt_cores(cfg, s) for s in STORE}}
+    return ctx
 
 
 def oracle_sample_step(ctx):
     """One bounded sample of the step on the CPU oracle; returns the GPU
     roofline time (s) of the sampled work."""
     import oracle
-    cfg = W.MATRIX_CONFIGS["large"]
-    m, n, b = cfg.m, cfg.n, cfg.b
-    rows = np.arange(ORACLE_ROWS)
-    frac_rows = ORACLE_ROWS / b
     rt = 0.0
-    X = ctx["X"][:ORACLE_ROWS]
-    for fmt in ("f64", "f32", "f16", "f16_o16"):
-        base = "f16" if fmt.startswith("f16") else fmt
-        k = cfg.ranks[base]
-        U, s, Vt = ctx["U"][:, :k], ctx["s"][:k], ctx["Vt"][:k]
-        Ur, sr, Vr = oracle.rounded(U, base), oracle.rounded(s, base), oracle.rounded(Vt, base)
-        Xr = oracle.rounded(X, base)
-        rt += roofline_time(work_round(ORACLE_ROWS, n, n, fmt))
-        oracle.apply_rows(Ur, sr, Vr, Xr, rows)
-        w = work_apply(m, n, k, b, fmt)
-        rt += roofline_time(w) * frac_rows
-    for fmt in ("f32", "f16"):
-        k = cfg.ranks[fmt]
-        U, s, Vt = ctx["U"][:, :k], ctx["s"][:k], ctx["Vt"][:k]
-        I = np.zeros((ORACLE_ROWS, n))
-        I[rows, rows] = 1.0                       # the first rows of I_n
-        A = oracle.apply_rows(U, s, Vt, I, rows)
-        Ah = oracle.apply_rows(oracle.rounded(U, fmt), oracle.rounded(s, fmt), oracle.rounded(Vt, fmt), I, rows)
-        oracle.fro_diff(A, Ah)
-        w = work_apply(m, n, k, n, "f64")
-        rt += 2 * roofline_time(w) * (ORACLE_ROWS / n) + roofline_time(work_fro(m * n, "f64", "f64")) * (ORACLE_ROWS / n)
-    tt = W.TT_CONFIGS["tt3"]
-    frac_tt = ORACLE_TT_SLAB / tt.dims[0]
-    for fmt in ("f64", "f32", "f16", "f16_o16"):
-        base = "f16" if fmt.startswith("f16") else fmt
-        cores = ctx["tt"][base]
-        sl = [oracle.rounded(cores[0][:, :ORACLE_TT_SLAB, :], base)] + [oracle.rounded(c, base) for c in cores[1:]]
-        oracle.tt_full(sl)
-        rt += roofline_time(work_tt(tt.dims, tt.ranks[base], fmt)) * frac_tt
+    for name, c in ctx["mat"].items():
+        cfg = c["cfg"]
+        m, n, b = cfg.m, cfg.n, cfg.b
+        rows = ORACLE_ROWS[name]
+        nb = b if rows is None else rows
+        X = c["X"][:nb]
+        for s in STORE:
+            k = cfg.ranks[s]
+            U, sg, Vt = c["U"][:, :k], c["s"][:k], c["Vt"][:k]
+            Ur, sr, Vr, Xr = (oracle.rounded(a, s) for a in (U, sg, Vt, X))
+            rt += (roofline_time(work_round(m, k, k, s)) + roofline_time(work_round(k, n, n, s))
+                   + roofline_time(work_round(b, n, n, s)) * nb / b)
+            Yr = oracle.apply(Ur, sr, Vr, Xr) if rows is None else oracle.apply_rows(Ur, sr, Vr, Xr, range(nb))
+            for f in COMP:
+                if store_of(f) == s:
+                    if f == "f16_o16":
+                        oracle.rounded(Yr, "f16")
+                    rt += roofline_time(work_apply(m, n, k, b, f)) * nb / b
+            # eta: rows of both dense FP64 products (rows of A_k'^T), then the difference
+            if rows is None:
+                oracle.eta_matrix(U, sg, Vt, s)
+                frac = 1.0
+            else:
+                I = np.zeros((nb, n))
+                I[np.arange(nb), np.arange(nb)] = 1.0
+                A = oracle.apply_rows(U, sg, Vt, I, range(nb))
+                Ah = oracle.apply_rows(Ur, sr, Vr, I, range(nb))
+                oracle.fro_diff(A, Ah)
+                frac = nb / n
+            rt += roofline_time(work_eta_lowrank(m, n, k, s)) * frac
+    for name, c in ctx["tt"].items():
+        cfg = c["cfg"]
+        sl = ORACLE_SLABS[name]
+        frac = sl / cfg.dims[0]
+        for s in STORE:
+            cores = c["cores"][s]
+            part = [cores[0][:, :sl, :]] + list(cores[1:])
+            rounded = [oracle.rounded(g, s) for g in part]
+            T = oracle.tt_full(part)
+            Th = oracle.tt_full(rounded)
+            oracle.fro_diff(T, Th)
+            rt += roofline_time(work_eta_tt(cfg.dims, cfg.ranks[s], s)) * frac
+            for f in COMP:
+                if store_of(f) == s:
+                    if f == "f16_o16":
+                        oracle.rounded(Th, "f16")
+                    rt += roofline_time(work_tt(cfg.dims, cfg.ranks[s], f)) * frac
     return rt
 
 
-def oracle_context():
-    cfg = W.MATRIX_CONFIGS["large"]
-    q1, sig, q2 = W.matrix_bases(cfg)
-    return {"U": q1, "s": sig, "Vt": np.ascontiguousarray(q2.T), "X": W.queries(cfg, b=ORACLE_ROWS),
-            "tt": {f: W.tt_cores(W.TT_CONFIGS["tt3"], f) for f in ("f64", "f32", "f16")}}
-
-
 def oracle_sample_desc():
-    return (f"per step: {ORACLE_ROWS} of 8192 query rows for each of the 4 applies and of the 4 FP64 "
-            f"dense reconstructions for eta (rows of A_k'^T), {ORACLE_TT_SLAB} of 256 i_1-slabs of each "
-            "of the 4 TT reconstructions; value scaled by the GPU roofline time of the sampled work")
+    parts = [f"{name}: {'all' if r is None else r} of {matrix_cfg(name).b} query rows per apply and "
+             f"{'all' if r is None else r} rows of the two dense FP64 products behind eta"
+             for name, r in ORACLE_ROWS.items()]
+    parts += [f"{name}: {sl} of {W.TT_CONFIGS[name].dims[0]} leading-index slabs of each reconstruction "
+              "and of the eta_TT pair" for name, sl in ORACLE_SLABS.items()]
+    return ("per step, each storage format: " + "; ".join(parts)
+            + "; value scaled by the GPU roofline time of the sampled work")
 
 
-def run_oracle_timing(steps: int, warmup: int):
+def run_oracle_timing(steps: int, warmup: int, threads: int | None = None):
     import oracle
     oracle.build()
+    if threads is not None:
+        oracle.set_threads(threads)
     ctx = oracle_context()
     for _ in range(warmup):
         oracle_sample_step(ctx)
@@ -559,19 +745,54 @@ def run_oracle_timing(steps: int, warmup: int):
 
 
 # ---------------------------------------------------------------------------
-# main
+# single-call mode (the commands the ncu captures in profiles/ run)
 # ---------------------------------------------------------------------------
 
+def run_peaks(lrc, torch, dev, reps):
+    """Measured arithmetic rates: the library's FMA-chain probes and
+    torch.matmul (cuBLAS) per dtype at 8192^3."""
+    out = {}
+    for kind in ("ffma", "ffma2", "dfma", "dmma"):
+        iters = 1 << 22 if kind.startswith("ffma") else 1 << 17
+        out[f"probe_{kind}_tflops"] = max(lrc.lrc_probe_peak(kind, iters) for _ in range(reps)) / 1e12
+    torch.backends.cuda.matmul.allow_tf32 = False
+    torch.backends.cuda.matmul.allow_fp16_reduced_precision_reduction = False
+    N = 8192
+    for name, dt in (("f64", torch.float64), ("f32", torch.float32), ("f16", torch.float16),
+                     ("bf16", torch.bfloat16)):
+        a = torch.randn(N, N, device=dev).to(dt)
+        b = torch.randn(N, N, device=dev).to(dt)
+        c = torch.empty(N, N, device=dev, dtype=dt)
+        torch.matmul(a, b, out=c)
+        torch.cuda.synchronize()
+        best = None
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            torch.matmul(a, b, out=c)
+            e1.record()
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1)
+            best = ms if best is None else min(best, ms)
+        out[f"torch_matmul_{name}_tflops"] = 2 * N ** 3 / (best * 1e-3) / 1e12
+        del a, b, c
+    out["derived_f32_tflops"] = PEAKS["f32"] / 1e12
+    out["derived_f64_tflops"] = PEAKS["f64"] / 1e12
+    print(json.dumps({"case": "peaks", **out}))
+    return 0
+
+
 def run_case(args):
-    """One call type at chosen sizes, launched `--reps` times after one warm-up
-    (the command ncu captures)."""
+    """One call type at chosen sizes, launched `--reps` times after one warm-up."""
     import torch
     import paper_2607_12969_gb300 as lrc
     lrc.load()
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
+    if args.case == "peaks":
+        return run_peaks(lrc, torch, dev, max(args.reps, 3))
     fmt = args.fmt
-    base = "f16" if fmt.startswith("f16") else ("f32" if fmt == "f32tc" else fmt)
+    base = store_of(fmt)
     if args.case == "apply":
         m, n, b, k = args.m, args.n, args.b, args.k
         f = W.random_factors(m, n, k, seed=7)
@@ -585,8 +806,15 @@ def run_case(args):
         cfg = W.TT_CONFIGS[args.tt]
         cores = [torch.from_numpy(c).to(dev).to(lrc.storage_dtype(fmt)).contiguous() for c in W.tt_cores(cfg, base)]
         ranks = cfg.ranks[base]
-        out = torch.empty(int(np.prod(cfg.dims)), dtype=lrc.output_dtype(fmt), device=dev)
-        call = lambda: lrc.tt_reconstruct(cores, cfg.dims, ranks, fmt, out)  # noqa: E731
+        N = int(np.prod(cfg.dims))
+        dt = lrc.output_dtype(fmt)
+        outs = [torch.empty(N, dtype=dt, device=dev)
+                for _ in range(rotation(N * torch.empty((), dtype=dt).element_size()) if args.rotate else 1)]
+        turn = {"i": 0}
+
+        def call():
+            turn["i"] += 1
+            lrc.tt_reconstruct(cores, cfg.dims, ranks, fmt, outs[turn["i"] % len(outs)])
         work = work_tt(cfg.dims, ranks, fmt)
     elif args.case == "eta_matrix":
         m, n, k = args.m, args.n, args.k
@@ -596,6 +824,26 @@ def run_case(args):
         low = [mk(a, fmt) for a in (f.U, f.s, f.Vt)]
         call = lambda: lrc.lrc_lowrank_eta(*f64, *low, fmt, m, n, k)  # noqa: E731
         work = work_eta_lowrank(m, n, k, fmt)
+    elif args.case == "eta_dense":
+        # eta by the dense route: both FP64 products with identity queries
+        # (lrc_apply), then lrc_fro_diff
+        m, n, k = args.m, args.n, args.k
+        f = W.random_factors(m, n, k, seed=7)
+        mk = lambda a, ft: lrc.round_matrix(torch.from_numpy(a if a.ndim == 2 else a[None, :]).to(dev), ft)  # noqa: E731
+        f64 = [mk(a, "f64") for a in (f.U, f.s, f.Vt)]
+        low = [mk(a, fmt) for a in (f.U, f.s, f.Vt)]
+        wide = [lrc.widen_matrix(low[0], fmt, k), lrc.widen_matrix(low[1], fmt, k), lrc.widen_matrix(low[2], fmt, n)]
+        I = lrc.round_matrix(torch.eye(n, dtype=torch.float64, device=dev), "f64")
+        A = torch.empty((n, m), dtype=torch.float64, device=dev)
+        Ah = torch.empty_like(A)
+
+        def call():
+            lrc.lrc_apply(*f64, I, A, m, n, k, n, "f64")
+            lrc.lrc_apply(*wide, I, Ah, m, n, k, n, "f64")
+            return lrc.lrc_fro_diff(A, "f64", Ah, "f64", A.numel(), want_norm=False)
+        w1 = work_apply(m, n, k, n, "f64")
+        w2 = work_fro(m * n, "f64", "f64")
+        work = {"bytes": 2 * w1["bytes"] + w2["bytes"], "flops": 2 * w1["flops"], "alu": "f64"}
     elif args.case == "eta_tt":
         cfg = W.TT_CONFIGS[args.tt]
         c64 = [torch.from_numpy(c).to(dev).contiguous() for c in W.tt_cores(cfg, base)]
@@ -648,14 +896,20 @@ def run_case(args):
     return 0 if st == 0 else 1
 
 
+# ---------------------------------------------------------------------------
+# main
+# ---------------------------------------------------------------------------
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--blocks", type=int, default=5, help="paired blocks of the speedup protocol")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", choices=["apply", "tt", "fro", "round", "eta_matrix", "eta_tt", "gather"], default=None,
+    ap.add_argument("--case", choices=["apply", "tt", "fro", "round", "eta_matrix", "eta_tt", "eta_dense",
+                                       "gather", "peaks"], default=None,
                     help="time one call type instead of the step (profiling captures)")
     ap.add_argument("--fmt", default="f16")
     ap.add_argument("--m", type=int, default=16384)
@@ -663,6 +917,7 @@ def main():
     ap.add_argument("--b", type=int, default=2048)
     ap.add_argument("--k", type=int, default=144)
     ap.add_argument("--tt", default="tt3")
+    ap.add_argument("--rotate", action="store_true", help="TT case: rotate outputs over more than 2 x L2")
     ap.add_argument("--count", type=int, default=1 << 26)
     ap.add_argument("--reps", type=int, default=3)
     args = ap.parse_args()
@@ -691,10 +946,12 @@ def main():
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
+    torch.backends.cuda.matmul.allow_tf32 = False
+    torch.backends.cuda.matmul.allow_fp16_reduced_precision_reduction = False
     import paper_2607_12969_gb300 as lrc
     lrc.load()
 
-    step = Step(lrc, dev, seed_offset=rank)
+    step = Step(lrc, dev, replica=rank)
     for _ in range(max(args.warmup, 3)):
         step.run(record=False)
     torch.cuda.synchronize()
@@ -722,38 +979,72 @@ def main():
     ms_max = reduce_max(ms, world, dev)
     rt_all = reduce_sum(rt_step, world, dev)
     value = aggregate_value(rt_all, ms_max)
+    results = step.results()
+
+    # ---- paired blocks: FP64 baseline, compensated calls, torch.matmul ----
+    paired = Paired(lrc, torch, dev, step)
+    paired.run(torch, 1)                          # warm-up block
+    ptimes = paired.run(torch, max(args.blocks, 1))
+    kind_of = {n: "apply" for n in MATRIX_WL}
+    kind_of.update({n: "tt" for n in TT_WL})
+    speed, vs_torch, paired_ms, torch_ms = paired_report(ptimes, kind_of)
+    del paired
+    torch.cuda.empty_cache()
 
     # ---- end to end: host inputs in, results out, through the same API ----
     h2d, d2h = e2e_bytes(step)
-    pinned = {k: torch.from_numpy(v).pin_memory() for k, v in step.host.items()}
-    pinned_tt = {f: [torch.from_numpy(c).pin_memory() for c in cs] for f, cs in step.host_tt.items()}
-    outs = {f: torch.empty(F["Y"].shape, dtype=F["Y"].dtype, pin_memory=True) for f, F in step.fac.items()}
-    outs_tt = {f: torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for f, t in step.tt_out.items()}
+    pin = {}
+    for wl in step.mats:
+        pin[wl.name] = {k: torch.from_numpy(v).pin_memory() for k, v in wl.host.items()}
+    for wl in step.tts:
+        pin[wl.name] = {s: [torch.from_numpy(c).pin_memory() for c in wl.host[s]] for s in STORE}
+    outs = {}
+    for wl in step.mats:
+        outs[wl.name] = {f: torch.empty(y.shape, dtype=y.dtype, pin_memory=True) for f, y in wl.Y.items()}
+    for wl in step.tts:
+        outs[wl.name] = {f: torch.empty(wl.N, dtype=lrc.output_dtype(f), pin_memory=True) for f in COMP}
+    h2d_stream, d2h_stream = torch.cuda.Stream(), torch.cuda.Stream()
+    main_stream = torch.cuda.current_stream()
+    ready = {}
 
-    copy_stream = torch.cuda.Stream()
+    def copy_inputs():
+        # every workload's FP64 inputs on a copy stream, in the order the step
+        # uses them; the step waits for each workload's own copies only
+        h2d_stream.wait_stream(main_stream)
+        with torch.cuda.stream(h2d_stream):
+            for wl in [step.mats[1]] + step.tts + [step.mats[0], step.mats[2]]:
+                if isinstance(wl, MatrixWL):
+                    for k, h in pin[wl.name].items():
+                        wl.d[k].copy_(h, non_blocking=True)
+                else:
+                    for s in STORE:
+                        for dd, h in zip(wl.c64[s], pin[wl.name][s]):
+                            dd.copy_(h, non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record()
+                ready[wl.name] = ev
+
+    def wait_inputs(wl):
+        main_stream.wait_event(ready[wl.name])
 
     def read_back():
-        # the outputs come back on a copy stream while the eta work runs
-        ready = torch.cuda.Event()
-        ready.record()
-        copy_stream.wait_event(ready)
-        with torch.cuda.stream(copy_stream):
-            for f, F in step.fac.items():
-                outs[f].copy_(F["Y"], non_blocking=True)
-            for f, t in step.tt_out.items():
-                outs_tt[f].copy_(t, non_blocking=True)
+        # outputs come back on a second copy stream while the eta work runs
+        done = torch.cuda.Event()
+        done.record()
+        d2h_stream.wait_event(done)
+        with torch.cuda.stream(d2h_stream):
+            for wl in step.mats:
+                for f, y in wl.Y.items():
+                    outs[wl.name][f].copy_(y, non_blocking=True)
+            for wl in step.tts:
+                for f, o in wl.last_outputs().items():
+                    outs[wl.name][f].copy_(o, non_blocking=True)
 
     def e2e_once():
-        step.d_Q1.copy_(pinned["Q1"], non_blocking=True)
-        step.d_Q2t.copy_(pinned["Q2t"], non_blocking=True)
-        step.d_s.copy_(pinned["s"][None, :], non_blocking=True)
-        step.d_X.copy_(pinned["X"], non_blocking=True)
-        for f in pinned_tt:
-            for d, h in zip(step.tt_dev[f], pinned_tt[f]):
-                d.copy_(h, non_blocking=True)
-        step.run(record=False, on_outputs=read_back)
-        torch.cuda.current_stream().synchronize()
-        copy_stream.synchronize()
+        copy_inputs()
+        step.run(record=False, on_outputs=read_back, wait_inputs=wait_inputs)
+        main_stream.synchronize()
+        d2h_stream.synchronize()
 
     e2e_once()
     barrier(world)
@@ -765,11 +1056,12 @@ def main():
     e2e_ms = (time.perf_counter() - t0) * 1e3 / args.steps
     e2e_ms_max = reduce_max(e2e_ms, world, dev)
     e2e_value = aggregate_value(rt_all, e2e_ms_max)
+    st = lrc.lrc_device_status()
 
     # ---- report -------------------------------------------------------------
     if rank == 0:
         kernels = {}
-        for name, p in per.items():
+        for name, p in sorted(per.items(), key=lambda kv: -kv[1]["ms"]):
             avg_ms = p["ms"] / p["calls"]
             kernels[name] = {
                 "ms_per_step": p["ms"] / args.steps, "calls_per_step": p["calls"] // args.steps,
@@ -777,40 +1069,47 @@ def main():
                 "GBps": p["bytes"] / p["calls"] / (avg_ms * 1e-3) / 1e9,
                 "TFLOPs": p["flops"] / p["calls"] / (avg_ms * 1e-3) / 1e12,
             }
-        dom = max(per.items(), key=lambda kv: kv[1]["ms"])
-        dname, dp = dom
+        dname, dp = max(per.items(), key=lambda kv: kv[1]["ms"])
         avg_s = dp["ms"] / dp["calls"] * 1e-3
         if dp["bound"] == "hbm":
             ach, peak, unit_r = dp["bytes"] / dp["calls"] / avg_s / 1e9, PEAKS["hbm"] / 1e9, "GB/s"
         else:
             ach, peak, unit_r = dp["flops"] / dp["calls"] / avg_s / 1e12, PEAKS[dp["alu"]] / 1e12, "TFLOP/s"
-        speed = {}
-        for grp in ("apply", "tt"):
-            base = kernels.get(f"{grp}_f64")
-            for f in ("f32", "f16", "f16_o16"):
-                k = kernels.get(f"{grp}_{f}")
-                if base and k:
-                    speed[f"{grp}_{f}"] = base["ms_per_step"] / k["ms_per_step"]
+        fp64_base = {k: v for k, v in paired_ms.items() if "_f64@" in k}
+        latency_us = {k: 1e3 * v for k, v in paired_ms.items() if k.endswith("@tiny")}
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": max(args.warmup, 3), "ms_per_step": ms_max, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f16/f32/f64", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "l2": "inputs larger than L2 (no flush needed)",
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32/f16 (eta in f64)", "data": "synthetic",
+            "config": {"workload": WORKLOAD,
+                       "l2": "inputs larger than L2 or rotated: TT outputs rotate over buffers > 2 x 129 MB; "
+                             "applies stream X and Y of 8 MB (tiny) to 5.4 GB",
                        "parallelism": f"replicas x{world} (independent batches, no collective)"},
             "roofline": {"kernel": dname, "bound": dp["bound"], "achieved": ach, "peak": peak, "unit": unit_r,
                          "frac": ach / peak, "traffic": MEASURED_TRAFFIC.get(dname),
-                         "peak_source": ("measured" if dp["bound"] == "hbm" or dp["alu"] == "f16" else "derived")
-                         + f" ({PEAKS['source']} file)"},
+                         "peak_source": ("measured" if dp["bound"] == "hbm" or dp["alu"] == "f16" else
+                                         "derived from unit counts x max SM clock") + f" ({PEAKS['source']} file)"},
             "kernels": kernels,
             "speedup_vs_fp64": speed,
-            "results": {k: (float(v) if not isinstance(v, bool) else v) for k, v in step.results.items()},
+            "speedup_protocol": (f"{max(args.blocks, 1)} randomised blocks, every call once per block, CUDA events "
+                                 "per call behind a GPU-side wait; median of paired per-block ratios "
+                                 "t(FP64, rank k) / t(fmt, rank k')"),
+            "fp64_baseline_ms": fp64_base,
+            "torch_matmul_ms": torch_ms,
+            "speedup_vs_torch_matmul": vs_torch,
+            "latency_us_tiny": latency_us,
+            "results": results,
+            "device_status": st,
             "gpu_launches": int(launches), "gpu_launches_per_step": int(launches // args.steps),
             "clocks": clk,
             "e2e": {"value": e2e_value, "unit": UNIT, "ms_per_step": e2e_ms_max,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         }
         if world == 1 and not args.no_cpu_baseline:
-            line["cpu_baseline"] = {k: v for k, v in run_oracle_timing(1, 0).items() if k != "seconds_per_step"}
+            r = run_oracle_timing(2, 0)
+            line["cpu_baseline"] = {k: v for k, v in r.items() if k != "seconds_per_step"}
+            r1 = run_oracle_timing(1, 0, threads=1)
+            line["cpu_baseline_1thread"] = {k: v for k, v in r1.items() if k not in ("seconds_per_step", "sample")}
         print(json.dumps(line))
     if world > 1:
         import torch.distributed as dist
@@ -819,9 +1118,10 @@ def main():
 
 
 def e2e_bytes(step):
-    h2d = sum(v.nbytes for v in step.host.values()) + sum(c.nbytes for cs in step.host_tt.values() for c in cs)
-    d2h = sum(F["Y"].numel() * F["Y"].element_size() for F in step.fac.values())
-    d2h += sum(t.numel() * t.element_size() for t in step.tt_out.values())
+    h2d = sum(v.nbytes for wl in step.mats for v in wl.host.values())
+    h2d += sum(c.nbytes for wl in step.tts for s in STORE for c in wl.host[s])
+    d2h = sum(y.numel() * y.element_size() for wl in step.mats for y in wl.Y.values())
+    d2h += sum(wl.N * E_OUT[f] for wl in step.tts for f in COMP)
     return int(h2d), int(d2h)
 
 

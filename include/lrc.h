@@ -341,6 +341,25 @@ LRC_API lrc_status lrc_device_status(lrc_stream_t stream);
  * arrives on.  The next lrc_device_status() returns LRC_ERR_TIMEOUT. */
 LRC_API lrc_status lrc_selftest_wait_timeout(int64_t limit_ns, lrc_stream_t stream);
 
+/*
+ * lrc_probe_peak -- measured rate of one arithmetic unit of this GPU, the
+ * denominator of the roofline fractions of the binary32 and binary64 paths
+ * (their products run on the CUDA cores' FMA units or on the binary64 tensor
+ * cores, Sec. 3.4 fixing only the precision).  Runs a kernel of independent
+ * multiply-add chains (no memory traffic in the loop) on every SM:
+ *
+ *   kind  0 = binary32 FMA, 1 = binary32 two-lane packed FMA,
+ *         2 = binary64 FMA, 3 = binary64 tensor-core MMA (m8n8k4)
+ *   iters loop steps per thread, 1 <= iters <= 2^30 (about 2^20 gives a
+ *         launch of a few to a few hundred milliseconds)
+ *   flops_out  host: flops per second, CUDA-event time of one launch after
+ *         a shorter warm-up launch
+ *
+ * Uses the stream's library workspace for one value per thread.
+ * SYNCHRONISES `stream`.
+ */
+LRC_API lrc_status lrc_probe_peak(int kind, int64_t iters, double* flops_out, lrc_stream_t stream);
+
 /* Release library-held scratch on every device; the library stays usable. */
 LRC_API lrc_status lrc_shutdown(void);
 

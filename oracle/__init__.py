@@ -78,6 +78,7 @@ def lib() -> ctypes.CDLL:
         L.oracle_tt_storage_bits.argtypes = [vp, vp, ip, ip]
         L.oracle_tt_storage_bits.restype = dbl
         L.oracle_threads.restype = ip
+        L.oracle_set_threads.argtypes = [ip]
         _lib = L
     return _lib
 
@@ -92,6 +93,11 @@ def _f64(a) -> np.ndarray:
 
 def threads() -> int:
     return int(lib().oracle_threads())
+
+
+def set_threads(n: int) -> None:
+    """Number of OpenMP threads the oracle's loops use (results unchanged)."""
+    lib().oracle_set_threads(int(n))
 
 
 # --------------------------------------------------------------------------

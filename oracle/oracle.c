@@ -338,6 +338,17 @@ double oracle_tt_storage_bits(const int64_t* dims, const int64_t* ranks, int d, 
     return s * (double)bits;
 }
 
+/* Thread count of the OpenMP loops (timing of the oracle on 1 and on all
+ * host cores); no effect on any result, every loop writes disjoint outputs. */
+void oracle_set_threads(int n)
+{
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+
 int oracle_threads(void)
 {
 #ifdef _OPENMP

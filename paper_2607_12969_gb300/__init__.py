@@ -82,6 +82,8 @@ def load() -> ctypes.CDLL:
     L.lrc_shutdown.restype = i32
     L.lrc_device_status.argtypes = [vp]
     L.lrc_device_status.restype = i32
+    L.lrc_probe_peak.argtypes = [i32, i64, vp, vp]
+    L.lrc_probe_peak.restype = i32
     L.lrc_selftest_wait_timeout.argtypes = [i64, vp]
     L.lrc_selftest_wait_timeout.restype = i32
     _lib = L
@@ -363,6 +365,17 @@ def lrc_device_status(stream=None) -> int:
     """Synchronises the stream; returns the lrc_status (0, or -6 if a bounded
     device wait gave up since the last call).  Does not raise."""
     return int(load().lrc_device_status(_stream(stream)))
+
+
+PROBE_KINDS = {"ffma": 0, "ffma2": 1, "dfma": 2, "dmma": 3}
+
+
+def lrc_probe_peak(kind, iters: int, stream=None) -> float:
+    """Measured flop/s of one arithmetic unit (kind: ffma, ffma2, dfma, dmma)."""
+    k = PROBE_KINDS[kind] if isinstance(kind, str) else int(kind)
+    out = ctypes.c_double(0.0)
+    _check(load().lrc_probe_peak(k, int(iters), ctypes.addressof(out), _stream(stream)))
+    return out.value
 
 
 def lrc_selftest_wait_timeout(limit_ns: int, stream=None) -> None:

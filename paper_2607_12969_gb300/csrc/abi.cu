@@ -379,6 +379,13 @@ lrc_status lrc_selftest_wait_timeout(int64_t limit_ns, lrc_stream_t stream) {
     return launch_wait_timeout_probe(limit_ns, as_stream(stream));
 }
 
+lrc_status lrc_probe_peak(int kind, int64_t iters, double* flops_out, lrc_stream_t stream) {
+    if (kind < 0 || kind > 3) return invalid("kind must be 0..3");
+    if (iters < 1 || iters > (1LL << 30)) return invalid("iters must be in [1, 2^30]");
+    if (!flops_out) return invalid("null flops_out");
+    return run_probe_peak(kind, iters, flops_out, as_stream(stream));
+}
+
 lrc_status lrc_shutdown(void) {
     release_scratch();
     release_workspaces();

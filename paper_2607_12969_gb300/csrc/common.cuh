@@ -207,4 +207,7 @@ lrc_status run_lowrank_eta(const double* U, const double* S, const double* Vt, c
 lrc_status run_tt_eta(const TTShape& sh, const void* const* hats, lrc_fmt fmt, double* eta_out, double* norm_out,
                       cudaStream_t s);
 
+// Measured rate of one arithmetic unit (peak_probe.cu); synchronises s.
+lrc_status run_probe_peak(int kind, int64_t iters, double* flops_out, cudaStream_t s);
+
 }  // namespace lrc
