@@ -26,10 +26,11 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "oracle.c")
 _LIB = os.path.join(_HERE, "liboracle.so")
 
-FMT_CODE = {"f64": 0, "f32": 1, "f16": 2}
-BITS = {"f64": 64, "f32": 32, "f16": 16}
+FMT_CODE = {"f64": 0, "f32": 1, "f16": 2, "bf16": 3}
+BITS = {"f64": 64, "f32": 32, "f16": 16, "bf16": 16}
 # unit roundoff u = 2^-p (Sec. 3.2, Table "precision comparison")
-UNIT_ROUNDOFF = {"f64": 2.0 ** -53, "f32": 2.0 ** -24, "f16": 2.0 ** -11}
+UNIT_ROUNDOFF = {"f64": 2.0 ** -53, "f32": 2.0 ** -24, "f16": 2.0 ** -11, "bf16": 2.0 ** -8}
+ENC_DTYPE = {"f64": np.float64, "f32": np.uint32, "f16": np.uint16, "bf16": np.uint16}
 
 
 def build(force: bool = False) -> str:
@@ -58,6 +59,8 @@ def lib() -> ctypes.CDLL:
         L.oracle_f64_to_f32_bits.argtypes = [dbl]
         L.oracle_f64_to_f16_bits.restype = ctypes.c_uint16
         L.oracle_f64_to_f16_bits.argtypes = [dbl]
+        L.oracle_f64_to_bf16_bits.restype = ctypes.c_uint16
+        L.oracle_f64_to_bf16_bits.argtypes = [dbl]
         L.oracle_round_pack.argtypes = [vp, i64, i64, i64, vp, i64, ip]
         L.oracle_decode.argtypes = [vp, i64, ip, vp]
         L.oracle_apply.argtypes = [vp, i64, vp, vp, i64, vp, i64, vp, i64, i64, i64, i64, i64]
@@ -112,14 +115,14 @@ def packed_ld(cols: int) -> int:
 def round_pack(src: np.ndarray, fmt: str, ld: Optional[int] = None) -> np.ndarray:
     """RN-even rounding of a 2-D FP64 array to fmt, rows padded with +0 to ld.
 
-    Returns the encodings: float64 for f64, uint32 for f32, uint16 for f16."""
+    Returns the encodings: float64 for f64, uint32 for f32, uint16 for f16
+    and bf16."""
     src = _f64(src)
     if src.ndim == 1:
         src = src[None, :]
     rows, cols = src.shape
     ld = cols if ld is None else ld
-    dt = {"f64": np.float64, "f32": np.uint32, "f16": np.uint16}[fmt]
-    out = np.empty((rows, ld), dtype=dt)
+    out = np.empty((rows, ld), dtype=ENC_DTYPE[fmt])
     lib().oracle_round_pack(_p(src), rows, cols, cols, _p(out), ld, FMT_CODE[fmt])
     return out
 
@@ -133,8 +136,7 @@ def round_bits(x: np.ndarray, fmt: str) -> np.ndarray:
 
 def decode(bits: np.ndarray, fmt: str) -> np.ndarray:
     """Exact FP64 values of encodings produced by round_bits / the GPU."""
-    dt = {"f64": np.float64, "f32": np.uint32, "f16": np.uint16}[fmt]
-    b = np.ascontiguousarray(bits, dtype=dt)
+    b = np.ascontiguousarray(bits, dtype=ENC_DTYPE[fmt])
     out = np.empty(b.shape, dtype=np.float64)
     lib().oracle_decode(_p(b), b.size, FMT_CODE[fmt], _p(out))
     return out

@@ -94,6 +94,8 @@ static uint64_t round_binary(double x, int p, int emin, int emax, int ebits, int
 
 uint32_t oracle_f64_to_f32_bits(double x) { return (uint32_t)round_binary(x, 24, -126, 127, 8, 32); }
 uint16_t oracle_f64_to_f16_bits(double x) { return (uint16_t)round_binary(x, 11, -14, 15, 5, 16); }
+/* bfloat16 (Sec. 3.2 precision table): 8 significand bits, binary32's exponent range */
+uint16_t oracle_f64_to_bf16_bits(double x) { return (uint16_t)round_binary(x, 8, -126, 127, 8, 16); }
 
 /* Value of a binary16 / binary32 encoding, from the format definition. */
 double oracle_f16_bits_to_f64(uint16_t h)
@@ -117,7 +119,18 @@ double oracle_f32_bits_to_f64(uint32_t w)
     return s ? -v : v;
 }
 
-/* fmt: 0 = binary64 (copy), 1 = binary32, 2 = binary16.  Packed layout:
+/* Value of a bfloat16 encoding: sign, 8-bit biased exponent, 7 fraction bits. */
+double oracle_bf16_bits_to_f64(uint16_t h)
+{
+    const int s = h >> 15, e = (h >> 7) & 0xff, f = h & 0x7f;
+    double v;
+    if (e == 0) v = ldexp((double)f, -133);
+    else if (e == 255) v = f ? NAN : INFINITY;
+    else v = ldexp((double)(f | 0x80), e - 134);
+    return s ? -v : v;
+}
+
+/* fmt: 0 = binary64 (copy), 1 = binary32, 2 = binary16, 3 = bfloat16.  Packed layout:
  * dst row r holds the rounded src[r, 0..cols) followed by +0 up to ld_dst. */
 void oracle_round_pack(const double* src, int64_t rows, int64_t cols, int64_t ld_src,
                        void* dst, int64_t ld_dst, int fmt)
@@ -127,6 +140,7 @@ void oracle_round_pack(const double* src, int64_t rows, int64_t cols, int64_t ld
             const double v = (c < cols) ? src[r * ld_src + c] : 0.0;
             if (fmt == 0) ((double*)dst)[r * ld_dst + c] = v;
             else if (fmt == 1) ((uint32_t*)dst)[r * ld_dst + c] = oracle_f64_to_f32_bits(v);
+            else if (fmt == 3) ((uint16_t*)dst)[r * ld_dst + c] = oracle_f64_to_bf16_bits(v);
             else ((uint16_t*)dst)[r * ld_dst + c] = oracle_f64_to_f16_bits(v);
         }
     }
@@ -137,6 +151,7 @@ void oracle_decode(const void* src, int64_t count, int fmt, double* dst)
     for (int64_t i = 0; i < count; ++i) {
         if (fmt == 0) dst[i] = ((const double*)src)[i];
         else if (fmt == 1) dst[i] = oracle_f32_bits_to_f64(((const uint32_t*)src)[i]);
+        else if (fmt == 3) dst[i] = oracle_bf16_bits_to_f64(((const uint16_t*)src)[i]);
         else dst[i] = oracle_f16_bits_to_f64(((const uint16_t*)src)[i]);
     }
 }

@@ -142,3 +142,82 @@ def test_round_pack_zero_fills_padding():
         assert np.all(out[:, 7:] == 0)
         assert np.array_equal(oracle.decode(out[:, :7], fmt), oracle.rounded(src, fmt))
     assert oracle.packed_ld(1) == 16 and oracle.packed_ld(16) == 16 and oracle.packed_ld(17) == 32
+
+
+# ---------------------------------------------------------------------------
+# bfloat16 (Sec. 3.2 precision table: 8 significand bits, binary32's exponent
+# range).  numpy has no bfloat16; its values are decoded here as the binary32
+# numbers whose upper 16 bits are the pattern, and the library pin is torch's
+# binary32 -> bfloat16 conversion on inputs that are binary32 numbers (so that
+# no intermediate rounding is involved).
+# ---------------------------------------------------------------------------
+
+def bf16_values(bits):
+    return (np.asarray(bits, dtype=np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def test_bf16_direct_conversion_not_double_rounding():
+    # 1 + 2^-8 + 2^-40 lies just above the midpoint between 1 and 1 + 2^-7:
+    # direct rounding gives 1 + 2^-7; via binary32 the 2^-40 is lost first and
+    # the tie then rounds to even (1.0)
+    x = 1.0 + 2.0 ** -8 + 2.0 ** -40
+    assert oracle.round_bits(np.array([x]), "bf16")[0] == 0x3F81
+    assert oracle.round_bits(np.array([1.0 + 2.0 ** -8]), "bf16")[0] == 0x3F80
+
+
+def test_exhaustive_bf16_values_roundtrip():
+    allbits = np.arange(65536, dtype=np.uint16)
+    vals = bf16_values(allbits)
+    finite = np.isfinite(vals)
+    assert np.array_equal(oracle.round_bits(vals[finite], "bf16"), allbits[finite])
+    dec = oracle.decode(allbits, "bf16")
+    assert np.array_equal(np.isnan(dec), np.isnan(vals))
+    ok = ~np.isnan(vals)
+    assert np.array_equal(dec[ok], vals[ok])
+
+
+def test_bf16_midpoints_ties_to_even():
+    pos = np.arange(0, 0x7F80, dtype=np.uint16)          # +0 .. max finite
+    lo, hi = bf16_values(pos[:-1]), bf16_values(pos[1:])
+    mid = (lo + hi) / 2.0                                 # exact in binary64
+    even = np.where(pos[:-1] % 2 == 0, pos[:-1], pos[1:])
+    assert np.array_equal(oracle.round_bits(mid, "bf16"), even)
+    assert np.array_equal(oracle.round_bits(np.nextafter(mid, np.inf), "bf16"), pos[1:])
+    assert np.array_equal(oracle.round_bits(np.nextafter(mid, -np.inf), "bf16"), pos[:-1])
+    assert np.array_equal(oracle.round_bits(-mid, "bf16"), even | 0x8000)
+
+
+def test_bf16_special_values_and_thresholds():
+    bmax = (2.0 - 2.0 ** -7) * 2.0 ** 127
+    cases = [
+        (0.0, 0x0000), (-0.0, 0x8000), (np.inf, 0x7F80), (-np.inf, 0xFF80),
+        (bmax, 0x7F7F),                                   # largest finite
+        ((2.0 - 2.0 ** -8) * 2.0 ** 127, 0x7F80),         # overflow midpoint ties to even -> inf
+        (np.nextafter((2.0 - 2.0 ** -8) * 2.0 ** 127, 0.0), 0x7F7F),
+        (2.0 ** -133, 0x0001),                            # smallest subnormal
+        (2.0 ** -134, 0x0000),                            # half of it: tie to even -> 0
+        (np.nextafter(2.0 ** -134, 1.0), 0x0001),
+        (3 * 2.0 ** -134, 0x0002),                        # tie between 1 and 2 quanta -> 2
+        (2.0 ** -126, 0x0080),                            # smallest normal
+        (5e-324, 0x0000), (1e300, 0x7F80), (-1e300, 0xFF80),
+    ]
+    for x, want in cases:
+        assert int(oracle.round_bits(np.array([x]), "bf16")[0]) == want, x
+    nan = oracle.round_bits(np.array([np.nan, -np.nan]), "bf16")
+    assert np.all((nan & 0x7F80) == 0x7F80) and np.all((nan & 0x007F) != 0)
+
+
+def test_bf16_matches_torch_on_binary32_inputs():
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(5)
+    x = (rng.standard_normal(300_000) * np.exp2(rng.uniform(-140, 120, 300_000))).astype(np.float32)
+    x[:2000] = rng.standard_normal(2000).astype(np.float32)
+    want = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(oracle.round_bits(x.astype(np.float64), "bf16"), want)
+
+
+def test_bf16_rounding_error_within_unit_roundoff():
+    x = np.random.default_rng(8).uniform(-1000, 1000, 100_000)
+    r = oracle.rounded(x, "bf16")
+    assert np.all(np.abs(r - x) <= oracle.UNIT_ROUNDOFF["bf16"] * np.abs(x))
+    assert np.max(np.abs(r - x) / np.abs(x)) > 0.9 * oracle.UNIT_ROUNDOFF["bf16"]   # the bound is attained
