@@ -85,9 +85,9 @@ def load_peaks():
 
 
 PEAKS = load_peaks()
-E = {"f64": 8, "f32": 4, "f16": 2, "f16_o16": 2, "f32tc": 4}
-E_OUT = {"f64": 8, "f32": 4, "f16": 4, "f16_o16": 2, "f32tc": 4}
-ALU = {"f64": "f64", "f32": "f32", "f16": "f16", "f16_o16": "f16", "f32tc": None}
+E = {"f64": 8, "f32": 4, "f16": 2, "f16_o16": 2, "f32tc": 4, "bf16": 2}
+E_OUT = {"f64": 8, "f32": 4, "f16": 4, "f16_o16": 2, "f32tc": 4, "bf16": 2}
+ALU = {"f64": "f64", "f32": "f32", "f16": "f16", "f16_o16": "f16", "f32tc": None, "bf16": "f16"}
 # LRC_F32_TC: binary32 storage; the output product on the tensor cores as
 # three binary16 products (hi/lo split), the rest on the CUDA cores.  Its
 # arithmetic bound is the sum of the two engines' times (alu_time).
@@ -98,6 +98,12 @@ STORE = ("f32", "f16")                   # their storage formats
 
 def store_of(fmt: str) -> str:
     return "f16" if fmt.startswith("f16") else ("f32" if fmt == "f32tc" else fmt)
+
+
+def rank_set(fmt: str) -> str:
+    """Rank set of the workloads a format takes: the 16-bit formats share the
+    binary16 compensated ranks."""
+    return "f16" if fmt == "bf16" else store_of(fmt)
 
 
 # ---------------------------------------------------------------------------
@@ -792,7 +798,7 @@ def run_case(args):
     if args.case == "peaks":
         return run_peaks(lrc, torch, dev, max(args.reps, 3))
     fmt = args.fmt
-    base = store_of(fmt)
+    base = rank_set(fmt)
     if args.case == "apply":
         m, n, b, k = args.m, args.n, args.b, args.k
         f = W.random_factors(m, n, k, seed=7)

@@ -49,12 +49,16 @@ typedef enum {
     LRC_F16 = 2,      /* binary16 storage, binary32 accumulation, binary32 output           */
     LRC_F16_O16 = 3,  /* binary16 storage, binary32 accumulation, binary16 workspaces and
                          output: the method-precision FP16 path of Sec. 3.4                 */
-    LRC_F32_TC = 4    /* binary32 storage and output; the output product of lrc_apply and
+    LRC_F32_TC = 4,   /* binary32 storage and output; the output product of lrc_apply and
                          tt_reconstruct on the tensor cores: each binary32 operand is scaled
                          by a power of two per 32 rows and split into binary16 parts
                          hi + lo, and Z S ~ Z_hi S_hi + Z_lo S_hi + Z_hi S_lo accumulates in
                          binary32 (about 22 significand bits per operand).  A variant of
                          LRC_F32; every other call treats it as LRC_F32                      */
+    LRC_BF16 = 5      /* bfloat16 storage (8 significand bits, binary32's exponent range:
+                         Sec. 3.2 precision table), binary32 accumulation, bfloat16
+                         workspaces and output: the method-precision policy of Sec. 3.4
+                         applied to bfloat16                                                  */
 } lrc_fmt;
 
 typedef enum {

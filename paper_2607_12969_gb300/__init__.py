@@ -22,8 +22,8 @@ from typing import Optional, Sequence, Tuple
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "liblrc.so")
 
-F64, F32, F16, F16_O16, F32_TC = 0, 1, 2, 3, 4
-FORMATS = {"f64": F64, "f32": F32, "f16": F16, "f16_o16": F16_O16, "f32tc": F32_TC}
+F64, F32, F16, F16_O16, F32_TC, BF16 = 0, 1, 2, 3, 4, 5
+FORMATS = {"f64": F64, "f32": F32, "f16": F16, "f16_o16": F16_O16, "f32tc": F32_TC, "bf16": BF16}
 STATUS = {0: "ok", -1: "invalid argument", -2: "misaligned pointer", -3: "unsupported",
           -4: "CUDA error", -5: "out of memory", -6: "device wait timed out"}
 
@@ -100,14 +100,14 @@ def storage_dtype(fmt):
     import torch
     f = _fmt(fmt)
     return {F64: torch.float64, F32: torch.float32, F16: torch.float16, F16_O16: torch.float16,
-            F32_TC: torch.float32}[f]
+            F32_TC: torch.float32, BF16: torch.bfloat16}[f]
 
 
 def output_dtype(fmt):
     import torch
     f = _fmt(fmt)
     return {F64: torch.float64, F32: torch.float32, F16: torch.float32, F16_O16: torch.float16,
-            F32_TC: torch.float32}[f]
+            F32_TC: torch.float32, BF16: torch.bfloat16}[f]
 
 
 def _check(status: int) -> None:
@@ -242,7 +242,7 @@ def tt_gather(cores: Sequence, dims: Sequence[int], ranks: Sequence[int], fmt, i
     import torch
     _need_cores(cores, dims, ranks, fmt, stream)
     _need(idx, "idx", torch.int64, stream=stream)
-    gather_dtype = {F64: torch.float64, F16_O16: torch.float16}.get(_fmt(fmt), torch.float32)
+    gather_dtype = {F64: torch.float64, F16_O16: torch.float16, BF16: torch.bfloat16}.get(_fmt(fmt), torch.float32)
     _need(out, "out", gather_dtype, int(idx.numel()), stream=stream)
     d = len(cores)
     ptrs = (ctypes.c_void_p * d)(*[c.data_ptr() for c in cores])

@@ -167,6 +167,8 @@ lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X
         case LRC_F16:
         case LRC_F16_O16:
             return launch_apply_f16(U, S, Vt, X, Y, m, n, k, b, fmt == LRC_F16_O16, s);
+        case LRC_BF16:
+            return launch_apply_f16(U, S, Vt, X, Y, m, n, k, b, true, s, true);
     }
     return invalid("unknown format");
 }
@@ -183,6 +185,7 @@ lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims, const i
     if (!aligned16(out)) return misaligned("out");
     cudaStream_t s = as_stream(stream);
     if (fmt == LRC_F16 || fmt == LRC_F16_O16) return launch_tt_f16(sh, fmt == LRC_F16_O16, out, s);
+    if (fmt == LRC_BF16) return launch_tt_bf16(sh, out, s);
     if (fmt == LRC_F32_TC) {
         bool handled = false;
         st = launch_tt_split_f32tc(sh, static_cast<float*>(out), s, &handled);
@@ -216,7 +219,7 @@ lrc_status tt_gather(const void* const* cores, const int64_t* dims, const int64_
         set_error("idx is not 8-byte aligned");
         return LRC_ERR_ALIGNMENT;
     }
-    const uintptr_t oa = (fmt == LRC_F16_O16) ? 2u : (fmt == LRC_F64 ? 8u : 4u);
+    const uintptr_t oa = (fmt == LRC_F16_O16 || fmt == LRC_BF16) ? 2u : (fmt == LRC_F64 ? 8u : 4u);
     if ((reinterpret_cast<uintptr_t>(out) % oa) != 0) {
         set_error("out is not aligned to its element size");
         return LRC_ERR_ALIGNMENT;

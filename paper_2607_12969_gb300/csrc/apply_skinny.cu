@@ -463,6 +463,7 @@ int64_t max_batch(lrc_fmt fmt) { return fmt == LRC_F16 || fmt == LRC_F16_O16 ? 4
 // to 4 for binary16 (whose tensor-core path is faster from 16 queries on);
 // ranks whose tiles fit in shared memory.
 bool apply_skinny_takes(lrc_fmt fmt, int64_t b, int64_t k) {
+    if (fmt == LRC_BF16) return false;    // bfloat16 takes the tensor-core path at every batch size
     if (b < 1 || b > max_batch(fmt) || k < 1 || k > 1024) return false;
     const int B = b <= 1 ? 1 : (b <= 4 ? 4 : (b <= 8 ? 8 : 16));
     const int64_t e = storage_bytes(fmt);

@@ -18,6 +18,8 @@
 //     groups are the slower index of the rows, so the CTAs working on the two
 //     groups of one row tile run side by side and the second read of an X
 //     tile hits L2.
+//     The same kernels take bfloat16 storage (LRC_BF16): bfloat16 tensor-core
+//     operands (the instruction descriptor's A/B format), bfloat16 W and output.
 //  2. apply_w2_kernel -- every W entry adds its tile's partials in a fixed
 //     order (deterministic), is scaled by diag(s) in FP32 and written as
 //     binary16: a hi/lo pair (hi = fp16(w), lo = fp16(w - hi)) for FP32
@@ -86,6 +88,7 @@ struct W1Args {
     uint32_t bar_off;
     uint32_t sum_col;         // tensor-memory column of the running sum (FP32 output)
     uint32_t tmem_cols;
+    uint32_t idesc_ab;        // operand-format bits of the MMA descriptor (0: binary16)
     float* P;                 // partials: [segment id][kgp columns][128 rows]
 };
 
@@ -221,7 +224,7 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
                 tc_fence_after();
                 const int grp = (int)(row / a.btiles);
                 const int kgw = min(a.kgp, a.kp - grp * a.kgp);
-                const uint32_t idesc = idesc_f16_f32(BM, (uint32_t)kgw);
+                const uint32_t idesc = idesc_f16_f32(BM, (uint32_t)kgw) | a.idesc_ab;
                 const uint32_t dacc = tmem + (uint32_t)(buf * a.kgp);
                 uint32_t accf = 0;
                 for (int64_t qs = q0; qs < q1; qs += kStageBlocks, ++it) {
@@ -325,9 +328,15 @@ struct W2Args {
     int G, kgp, kp, k, planes;
     uint32_t tile_bytes;      // one plane of one row tile: 128 x kp x 2
     const float* P;
-    const __half* S;
+    const uint16_t* S;        // binary16 or bfloat16 encodings
+    int bf16;                 // operands, W and output are bfloat16 (one plane)
     unsigned char* W;         // [row tile][plane][tile_bytes]
 };
+
+__device__ __forceinline__ float s_value(const W2Args& a, int j) {
+    const uint16_t h = a.S[j];
+    return a.bf16 ? bf16_bits_to_float(h) : __half2float(__ushort_as_half(h));
+}
 
 // CTA of the phase-1 grid whose range [floor(c Q / P1), floor((c+1) Q / P1))
 // holds k-block q.
@@ -337,11 +346,16 @@ __device__ __forceinline__ int64_t cta_of(int64_t q, int64_t Q, int64_t P1) { re
 // into the operand image(s).
 __device__ __forceinline__ void put_w8(const W2Args& a, int64_t bt, int r, int col0, const float (&w)[8]) {
     uint32_t hi[4], lo[4];
+    if (a.bf16) {
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const __half h0 = __float2half_rn(w[2 * j]), h1 = __float2half_rn(w[2 * j + 1]);
-        hi[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
-        lo[j] = pack_half2(w[2 * j] - __half2float(h0), w[2 * j + 1] - __half2float(h1));
+        for (int j = 0; j < 4; ++j) hi[j] = lo[j] = pack_bf162(w[2 * j], w[2 * j + 1]);
+    } else {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const __half h0 = __float2half_rn(w[2 * j]), h1 = __float2half_rn(w[2 * j + 1]);
+            hi[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+            lo[j] = pack_half2(w[2 * j] - __half2float(h0), w[2 * j + 1] - __half2float(h1));
+        }
     }
     unsigned char* base = a.W + (size_t)bt * a.planes * a.tile_bytes + w_image_off((uint32_t)r, (uint32_t)col0);
     *reinterpret_cast<uint4*>(base) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
@@ -391,7 +405,7 @@ apply_w2_kernel(const W2Args a) {
                 }
         }
 #pragma unroll
-        for (int i = 0; i < 8; ++i) w[i] = __fmul_rn(w[i], col0 + i < a.k ? __half2float(a.S[col0 + i]) : 0.0f);
+        for (int i = 0; i < 8; ++i) w[i] = __fmul_rn(w[i], col0 + i < a.k ? s_value(a, col0 + i) : 0.0f);
     }
     put_w8(a, bt, r, col0, w);
 }
@@ -458,7 +472,7 @@ apply_w2_slice_kernel(const W2Args a) {
             float v = red[0][i][lane];
 #pragma unroll
             for (int q = 1; q < kW2Slices; ++q) v = __fadd_rn(v, red[q][i][lane]);
-            w[i] = __fmul_rn(v, col0 + i < a.k ? __half2float(a.S[col0 + i]) : 0.0f);
+            w[i] = __fmul_rn(v, col0 + i < a.k ? s_value(a, col0 + i) : 0.0f);
         }
         if (bt * BM + r >= a.b) {
 #pragma unroll
@@ -477,6 +491,8 @@ struct YArgs {
     uint32_t u_bytes, slot_bytes, tile_bytes;
     uint32_t w_off, ystage_off, bar_off, tmem_cols;
     int out16, tma_store;
+    int bf16;                 // bfloat16 operands and output
+    uint32_t idesc_ab;        // operand-format bits of the MMA descriptor
     int ydepth;               // staging buffers per epilogue warp (1 or 2): TMA stores in flight
     const unsigned char* W;
     void* Y;
@@ -575,7 +591,7 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
             const uint32_t whi = smem_u32(smem + a.w_off);
             const uint64_t whd = smem_desc(whi, 2048, 128, 0);
             const uint64_t wld = smem_desc(whi + a.tile_bytes, 2048, 128, 0);
-            const uint32_t idesc2 = idesc_f16_f32(BM, (uint32_t)a.n2);
+            const uint32_t idesc2 = idesc_f16_f32(BM, (uint32_t)a.n2) | a.idesc_ab;
             for (int64_t t = tbeg; t < tend && ok; ++t, ++tl) {
                 const int64_t bt = t / a.mtiles;
                 if (bt != cur_bt) {
@@ -666,7 +682,11 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
                 }
                 if (a.tma_store) {
                     uint32_t packed[32];
-                    if (a.out16) {
+                    if (a.out16 && a.bf16) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            packed[j] = pack_bf162(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+                    } else if (a.out16) {
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
                             packed[j] = pack_half2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
@@ -697,9 +717,11 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
                     const int64_t grow = row0 + r;
                     if (grow < a.b) {
                         if (a.out16) {
-                            __half* yrow = static_cast<__half*>(a.Y) + grow * a.m;
+                            uint16_t* yrow = static_cast<uint16_t*>(a.Y) + grow * a.m;
                             for (int j = 0; j < 64; ++j)
-                                if (col0 + j < a.m) yrow[col0 + j] = __float2half_rn(__uint_as_float(v[j]));
+                                if (col0 + j < a.m)
+                                    yrow[col0 + j] = a.bf16 ? to_bf16_bits(__uint_as_float(v[j]))
+                                                            : __half_as_ushort(__float2half_rn(__uint_as_float(v[j])));
                         } else {
                             float* yrow = static_cast<float*>(a.Y) + grow * a.m;
                             for (int j = 0; j < 32; ++j)
@@ -839,10 +861,12 @@ lrc_status plan_y(YArgs& a3, size_t& smem3, int64_t m, int64_t b, int kp, int pl
     return LRC_OK;
 }
 
+CUtensorMapDataType t16(bool bf16) { return bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16; }
+
 lrc_status make_y_map(CUtensorMap* ty, const YArgs& a3, void* Y, int64_t m, int64_t b, bool out16) {
     if (!a3.tma_store) return LRC_OK;   // unused by the kernel
     const int e_out = out16 ? 2 : 4;
-    return make_map(ty, out16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, Y, m, b, m * e_out,
+    return make_map(ty, out16 ? t16(a3.bf16 != 0) : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, Y, m, b, m * e_out,
                     out16 ? 64 : 32, BM, "Y");
 }
 
@@ -858,9 +882,13 @@ lrc_status launch_y(const CUtensorMap& tu, const CUtensorMap& ty, const YArgs& a
 }  // namespace
 
 lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y, int64_t m,
-                            int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s) {
+                            int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s, bool bf16) {
     lrc_status st = get_encoder();
     if (st != LRC_OK) return st;
+    if (bf16 && !out16) {
+        set_error("bfloat16 apply: the output is bfloat16");
+        return LRC_ERR_UNSUPPORTED;
+    }
     const int kp = (int)((k + 15) / 16 * 16);
     if (kp > 512) {
         set_error("binary16 apply supports rank up to 512 (got %lld)", (long long)k);
@@ -881,6 +909,7 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
     a1.kgp = ((kp + a1.G - 1) / a1.G + 15) / 16 * 16;
     a1.kp = kp;
     a1.Q = btiles * a1.G * a1.nkb;
+    a1.idesc_ab = bf16 ? kIdescBF16 : 0u;
     a1.chunk_blocks = out16 ? (int)(a1.nkb < 0x7fffffff ? a1.nkb : 0x7fffffff) : kChunkBlocks;
     const bool use_sum = a1.chunk_blocks < a1.nkb;
     a1.slot_bytes = (uint32_t)round_up((size_t)kStageBlocks * (kXBytes + (size_t)a1.kgp * 128), 1024);
@@ -918,6 +947,8 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
     if ((st = plan_y(a3, smem3, m, b, kp, planes, out16, false)) != LRC_OK) return st;
     a3.tile_bytes = tile_bytes;
     a3.Y = Y;
+    a3.bf16 = bf16 ? 1 : 0;
+    a3.idesc_ab = bf16 ? kIdescBF16 : 0u;
     const int64_t P3 = a3.T < sms ? a3.T : sms;
 
     // ---- workspace: W images, then the phase-1 partials
@@ -931,17 +962,16 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
 
     const int64_t ldn = lrc_packed_ld(n), ldk = lrc_packed_ld(k);
     CUtensorMap tx, tv, tu, ty, txp, tvp;
-    if ((st = make_map(&tx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, X, n, b, ldn * 2, BK, BM, "X")) != LRC_OK) return st;
-    if ((st = make_map(&tv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, Vt, n, k, ldn * 2, BK, (uint32_t)a1.kgp, "Vt")) != LRC_OK)
+    const CUtensorMapDataType dt = t16(bf16);
+    if ((st = make_map(&tx, dt, X, n, b, ldn * 2, BK, BM, "X")) != LRC_OK) return st;
+    if ((st = make_map(&tv, dt, Vt, n, k, ldn * 2, BK, (uint32_t)a1.kgp, "Vt")) != LRC_OK) return st;
+    if ((st = make_map(&txp, dt, X, n, b, ldn * 2, kPfBlocks * BK, BM, "X prefetch", CU_TENSOR_MAP_SWIZZLE_NONE)) !=
+        LRC_OK)
         return st;
-    if ((st = make_map(&txp, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, X, n, b, ldn * 2, kPfBlocks * BK, BM, "X prefetch",
+    if ((st = make_map(&tvp, dt, Vt, n, k, ldn * 2, kPfBlocks * BK, (uint32_t)a1.kgp, "Vt prefetch",
                        CU_TENSOR_MAP_SWIZZLE_NONE)) != LRC_OK)
         return st;
-    if ((st = make_map(&tvp, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, Vt, n, k, ldn * 2, kPfBlocks * BK, (uint32_t)a1.kgp,
-                       "Vt prefetch", CU_TENSOR_MAP_SWIZZLE_NONE)) != LRC_OK)
-        return st;
-    if ((st = make_map(&tu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, U, k, m, ldk * 2, BK, (uint32_t)a3.n2, "U")) != LRC_OK)
-        return st;
+    if ((st = make_map(&tu, dt, U, k, m, ldk * 2, BK, (uint32_t)a3.n2, "U")) != LRC_OK) return st;
     if ((st = make_y_map(&ty, a3, Y, m, b, out16)) != LRC_OK) return st;
 
     cudaError_t e = cudaFuncSetAttribute(apply_w1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
@@ -962,7 +992,8 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
     a2.planes = planes;
     a2.tile_bytes = tile_bytes;
     a2.P = a1.P;
-    a2.S = static_cast<const __half*>(S);
+    a2.S = static_cast<const uint16_t*>(S);
+    a2.bf16 = bf16 ? 1 : 0;
     a2.W = Wimg;
     const int64_t n2items = btiles * (kp / 8) * BM;
     const int64_t max_parts = (a1.nkb * P1 + a1.Q - 1) / a1.Q + 1;     // CTAs sharing one row, at most
@@ -999,7 +1030,7 @@ lrc_status y_product_plan(int64_t m, int64_t b, int kp, bool out16, int* n2) {
 
 lrc_status launch_y_product(const unsigned char* Wimg, int kp, const void* U, int64_t ldu, int64_t m, int64_t b,
                             bool out16, void* Y, const int* esc_w, const int* esc_u, cudaStream_t s,
-                            bool w_per_row) {
+                            bool w_per_row, bool bf16) {
     lrc_status st = get_encoder();
     if (st != LRC_OK) return st;
     YArgs a3{};
@@ -1011,9 +1042,10 @@ lrc_status launch_y_product(const unsigned char* Wimg, int kp, const void* U, in
     a3.esc_w = esc_w;
     a3.esc_w_rows = w_per_row ? 1 : 0;
     a3.esc_u = esc_u;
+    a3.bf16 = bf16 ? 1 : 0;
+    a3.idesc_ab = bf16 ? kIdescBF16 : 0u;
     CUtensorMap tu, ty;
-    if ((st = make_map(&tu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, U, kp, m, ldu * 2, BK, (uint32_t)a3.n2, "U")) != LRC_OK)
-        return st;
+    if ((st = make_map(&tu, t16(bf16), U, kp, m, ldu * 2, BK, (uint32_t)a3.n2, "U")) != LRC_OK) return st;
     if ((st = make_y_map(&ty, a3, Y, m, b, out16)) != LRC_OK) return st;
     const int sms = sm_count();
     const int64_t P3 = a3.T < sms ? a3.T : sms;

@@ -52,12 +52,13 @@ inline int64_t storage_bytes(lrc_fmt f) {
         case LRC_F32:
         case LRC_F32_TC: return 4;
         case LRC_F16:
-        case LRC_F16_O16: return 2;
+        case LRC_F16_O16:
+        case LRC_BF16: return 2;
     }
     return 0;
 }
 
-inline bool valid_fmt(int f) { return f >= LRC_F64 && f <= LRC_F32_TC; }
+inline bool valid_fmt(int f) { return f >= LRC_F64 && f <= LRC_BF16; }
 // LRC_F32_TC is LRC_F32 everywhere but in the output products of lrc_apply
 // and tt_reconstruct
 inline lrc_fmt plain_fmt(lrc_fmt f) { return f == LRC_F32_TC ? LRC_F32 : f; }
@@ -96,8 +97,10 @@ lrc_status launch_apply_split_f64(const double* U, const double* S, const double
                                   int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
 lrc_status launch_apply_split_f32(const float* U, const float* S, const float* Vt, const float* X, float* Y,
                                   int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
+// bf16: bfloat16 operands and output (out16 must be set)
 lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y,
-                            int64_t m, int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s);
+                            int64_t m, int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s,
+                            bool bf16 = false);
 // small batches (at most 16 queries for binary32, 4 otherwise), ranks up to
 // 1024 whose tiles fit in shared memory, every format (apply_skinny.cu)
 bool apply_skinny_takes(lrc_fmt fmt, int64_t b, int64_t k);
@@ -128,7 +131,7 @@ lrc_status gemm_cc_f32(const float* A, int64_t lda, const float* B, int64_t ldb,
 lrc_status y_product_plan(int64_t m, int64_t b, int kp, bool out16, int* n2);
 lrc_status launch_y_product(const unsigned char* Wimg, int kp, const void* U, int64_t ldu, int64_t m, int64_t b,
                             bool out16, void* Y, const int* esc_w, const int* esc_u, cudaStream_t s,
-                            bool w_per_row = false);
+                            bool w_per_row = false, bool bf16 = false);
 
 struct TTShape {
     int d;
@@ -153,6 +156,10 @@ lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStr
 // the same product chain for binary32 cores (LRC_F32_TC): both operands split
 // into scaled hi/lo binary16 parts; *handled = false when the shape is outside it
 lrc_status launch_tt_split_f32tc(const TTShape& sh, float* out, cudaStream_t s, bool* handled);
+// bfloat16 cores, bfloat16 workspaces and output: the same product chain with
+// bfloat16 tensor-core operands where the shape fits it, else the CUDA-core
+// chain of tt_cc.cu
+lrc_status launch_tt_bf16(const TTShape& sh, void* out, cudaStream_t s);
 // the FP32 product chain with its output product on the tensor cores
 // (LRC_F32_TC) when split_product_fits, else on the CUDA cores (tt_chain.cu)
 lrc_status launch_tt_chain_f32tc(const TTShape& sh, float* out, cudaStream_t s);

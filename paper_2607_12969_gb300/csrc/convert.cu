@@ -1,7 +1,7 @@
-// convert.cu -- factor rounding / packing (binary64 -> binary32 / binary16)
-// and exact widening back to binary64.
+// convert.cu -- factor rounding / packing (binary64 -> binary32 / binary16 /
+// bfloat16) and exact widening back to binary64.
 //
-// Rounding is the hardware conversion cvt.rn.{f32,f16}.f64: IEEE 754
+// Rounding is the hardware conversion cvt.rn.{f32,f16,bf16}.f64: IEEE 754
 // round-to-nearest-even directly from binary64 (no intermediate format),
 // subnormals kept (no .ftz), overflow to infinity.  The kernels are
 // HBM-bound streams: each thread converts a group of 8 consecutive elements
@@ -21,6 +21,11 @@ __device__ __forceinline__ uint16_t cvt_f16(double x) {
     asm("cvt.rn.f16.f64 %0, %1;" : "=h"(h) : "d"(x));
     return h;
 }
+__device__ __forceinline__ uint16_t cvt_bf16(double x) {
+    uint16_t h;
+    asm("cvt.rn.bf16.f64 %0, %1;" : "=h"(h) : "d"(x));
+    return h;
+}
 __device__ __forceinline__ float cvt_f32(double x) {
     float f;
     asm("cvt.rn.f32.f64 %0, %1;" : "=f"(f) : "d"(x));
@@ -32,7 +37,7 @@ __device__ __forceinline__ double widen_f16(uint16_t h) {
     return d;
 }
 
-// FMT: 0 = binary64 copy, 1 = binary32, 2 = binary16
+// FMT: 0 = binary64 copy, 1 = binary32, 2 = binary16, 3 = bfloat16
 template <int FMT>
 __global__ void __launch_bounds__(kThreads)
 round_pack_kernel(const double* __restrict__ src, int64_t cols, int64_t ld_src,
@@ -56,11 +61,11 @@ round_pack_kernel(const double* __restrict__ src, int64_t cols, int64_t ld_src,
             for (int j = 0; j < kGroup; ++j) v[j] = (c0 + j < cols) ? __ldcs(srow + c0 + j) : 0.0;
         }
         const bool full = vec_dst && (c0 + kGroup <= ld_dst);
-        if (FMT == 2) {
+        if (FMT == 2 || FMT == 3) {
             uint16_t* drow = static_cast<uint16_t*>(dst) + r * ld_dst;
             uint16_t h[kGroup];
 #pragma unroll
-            for (int j = 0; j < kGroup; ++j) h[j] = cvt_f16(v[j]);
+            for (int j = 0; j < kGroup; ++j) h[j] = FMT == 2 ? cvt_f16(v[j]) : cvt_bf16(v[j]);
             if (full) {
                 uint4 q;
                 q.x = (uint32_t)h[0] | ((uint32_t)h[1] << 16);
@@ -126,12 +131,14 @@ widen_kernel(const void* __restrict__ src, int64_t cols, int64_t ld_src, double*
         const int64_t c0 = (g - r * groups_per_row) * kGroup;
         double v[kGroup];
         if (vec_src && c0 + kGroup <= cols) {
-            if (FMT == 2) {
+            if (FMT == 2 || FMT == 3) {
                 const uint4 q = __ldcs(reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(src) + r * ld_src + c0));
                 const uint32_t w[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
-                    const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w[j]));
+                    // a bfloat16 value is the binary32 number with the same upper 16 bits
+                    const float2 f = FMT == 2 ? __half22float2(*reinterpret_cast<const __half2*>(&w[j]))
+                                              : make_float2(__uint_as_float(w[j] << 16), __uint_as_float(w[j] & 0xffff0000u));
                     v[2 * j] = widen_f32(f.x);
                     v[2 * j + 1] = widen_f32(f.y);
                 }
@@ -156,6 +163,8 @@ widen_kernel(const void* __restrict__ src, int64_t cols, int64_t ld_src, double*
                 double x = 0.0;
                 if (c < cols) {
                     if (FMT == 2) x = widen_f16(static_cast<const uint16_t*>(src)[r * ld_src + c]);
+                    else if (FMT == 3)
+                        x = widen_f32(__uint_as_float((uint32_t)static_cast<const uint16_t*>(src)[r * ld_src + c] << 16));
                     else if (FMT == 1) x = (double)static_cast<const float*>(src)[r * ld_src + c];
                     else x = static_cast<const double*>(src)[r * ld_src + c];
                 }
@@ -197,6 +206,10 @@ lrc_status launch_round(const double* src, int64_t rows, int64_t cols, int64_t l
             round_pack_kernel<1><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total,
                                                             vec_src, (ld_dst % 4) == 0);
             break;
+        case LRC_BF16:
+            round_pack_kernel<3><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total,
+                                                            vec_src, (ld_dst % 8) == 0);
+            break;
         default:
             round_pack_kernel<2><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total,
                                                             vec_src, (ld_dst % 8) == 0);
@@ -220,6 +233,9 @@ lrc_status launch_widen(const void* src, lrc_fmt fmt, int64_t rows, int64_t cols
             break;
         case LRC_F32:
             widen_kernel<1><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total, vec_src, vec_dst);
+            break;
+        case LRC_BF16:
+            widen_kernel<3><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total, vec_src, vec_dst);
             break;
         default:
             widen_kernel<2><<<grid, kThreads, 0, s>>>(src, cols, ld_src, dst, ld_dst, gpr, total, vec_src, vec_dst);

@@ -25,6 +25,7 @@
 //
 // All arithmetic is binary64 (CUDA-core DFMA); the sums are deterministic
 // (fixed per-CTA ranges, partials added in a fixed order).
+#include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
 #include <algorithm>
@@ -47,6 +48,7 @@ constexpr int kCombineBlocks = 304;
 __device__ __forceinline__ double wide(double v) { return v; }
 __device__ __forceinline__ double wide(float v) { return (double)v; }
 __device__ __forceinline__ double wide(__half v) { return (double)__half2float(v); }
+__device__ __forceinline__ double wide(__nv_bfloat16 v) { return (double)__bfloat162float(v); }
 
 // ---- operand packing --------------------------------------------------------
 // P (L x 2k, row pitch 2k) from the row-major L x k factors X (binary64) and
@@ -712,6 +714,7 @@ lrc_status run_lowrank_eta(const double* U, const double* S, const double* Vt, c
         case LRC_F32: return lowrank_eta_t<float>(U, S, Vt, Uh, Sh, Vht, m, n, k, eta_out, norm_out, s);
         case LRC_F16:
         case LRC_F16_O16: return lowrank_eta_t<__half>(U, S, Vt, Uh, Sh, Vht, m, n, k, eta_out, norm_out, s);
+        case LRC_BF16: return lowrank_eta_t<__nv_bfloat16>(U, S, Vt, Uh, Sh, Vht, m, n, k, eta_out, norm_out, s);
     }
     set_error("unknown format");
     return LRC_ERR_INVALID_ARG;
@@ -724,6 +727,7 @@ lrc_status run_tt_eta(const TTShape& sh, const void* const* hats, lrc_fmt fmt, d
         case LRC_F32: return tt_eta_t<float>(sh, hats, eta_out, norm_out, s);
         case LRC_F16:
         case LRC_F16_O16: return tt_eta_t<__half>(sh, hats, eta_out, norm_out, s);
+        case LRC_BF16: return tt_eta_t<__nv_bfloat16>(sh, hats, eta_out, norm_out, s);
     }
     set_error("unknown format");
     return LRC_ERR_INVALID_ARG;

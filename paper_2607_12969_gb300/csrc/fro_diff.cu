@@ -53,13 +53,22 @@ __device__ __forceinline__ void load8(const void* p, int64_t g, double v[kGroup]
             v[4 * j + 2] = t.z;
             v[4 * j + 3] = t.w;
         }
-    } else {
+    } else if (F == 2) {
         const uint4 t = __ldcs(reinterpret_cast<const uint4*>(p) + g);
         const uint32_t w[4] = {t.x, t.y, t.z, t.w};
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             v[2 * j] = widen_h((uint16_t)(w[j] & 0xffffu));
             v[2 * j + 1] = widen_h((uint16_t)(w[j] >> 16));
+        }
+    } else {
+        // bfloat16: the binary32 number with the same upper 16 bits
+        const uint4 t = __ldcs(reinterpret_cast<const uint4*>(p) + g);
+        const uint32_t w[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            v[2 * j] = (double)__uint_as_float(w[j] << 16);
+            v[2 * j + 1] = (double)__uint_as_float(w[j] & 0xffff0000u);
         }
     }
 }
@@ -68,6 +77,7 @@ template <int F>
 __device__ __forceinline__ double load1(const void* p, int64_t i) {
     if (F == 0) return static_cast<const double*>(p)[i];
     if (F == 1) return (double)static_cast<const float*>(p)[i];
+    if (F == 3) return (double)__uint_as_float((uint32_t)static_cast<const uint16_t*>(p)[i] << 16);
     return widen_h(static_cast<const uint16_t*>(p)[i]);
 }
 
@@ -232,7 +242,7 @@ fro_final_kernel(const double* __restrict__ partial, int nblocks, double* __rest
     }
 }
 
-int fcode(lrc_fmt f) { return f == LRC_F64 ? 0 : (f == LRC_F32 ? 1 : 2); }
+int fcode(lrc_fmt f) { return f == LRC_F64 ? 0 : (f == LRC_F32 ? 1 : (f == LRC_BF16 ? 3 : 2)); }
 
 template <int FA, bool NORM>
 void launch_partial_n(int fb, int grid, const void* A, const void* B, int64_t count, double* partial,
@@ -241,6 +251,7 @@ void launch_partial_n(int fb, int grid, const void* A, const void* B, int64_t co
         case 0: fro_partial_kernel<FA, 0, NORM><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
         case 1: fro_partial_kernel<FA, 1, NORM><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
         case 2: fro_partial_kernel<FA, 2, NORM><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
+        case 3: fro_partial_kernel<FA, 3, NORM><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
         default: fro_partial_kernel<FA, -1, NORM><<<grid, kThreads, 0, s>>>(A, B, count, partial); break;
     }
 }
@@ -286,6 +297,7 @@ lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, in
     switch (a) {
         case 0: launch_partial<0>(b, grid, A, B, count, partial, s, norm); break;
         case 1: launch_partial<1>(b, grid, A, B, count, partial, s, norm); break;
+        case 3: launch_partial<3>(b, grid, A, B, count, partial, s, norm); break;
         default: launch_partial<2>(b, grid, A, B, count, partial, s, norm); break;
     }
     lrc_status st = after_launch("fro_partial_kernel");
@@ -360,6 +372,7 @@ lrc_status run_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fm
     switch (a) {
         case 0: launch_partial<0>(b, grid, A, B, count, partial, s, norm); break;
         case 1: launch_partial<1>(b, grid, A, B, count, partial, s, norm); break;
+        case 3: launch_partial<3>(b, grid, A, B, count, partial, s, norm); break;
         default: launch_partial<2>(b, grid, A, B, count, partial, s, norm); break;
     }
     lrc_status st = after_launch("fro_partial_kernel (no-alloc)");

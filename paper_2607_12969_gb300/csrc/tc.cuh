@@ -234,6 +234,9 @@ __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.
 __host__ __device__ constexpr uint32_t idesc_f16_f32(uint32_t M, uint32_t N) {
     return (1u << 4) | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
+// OR'ed into the descriptor above: A and B are bfloat16 (format code 1 at
+// bits 7-9 and 10-12) instead of binary16
+constexpr uint32_t kIdescBF16 = (1u << 7) | (1u << 10);
 
 // Shared-memory matrix descriptor (sm_100 family, version bits 46-48 = 1).
 //   swizzle: 0 = none (canonical 8-row x 16-byte core matrices), 2 = 128-byte
@@ -271,6 +274,20 @@ __device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
     const __half2 h = __floats2half2_rn(lo, hi);
     return *reinterpret_cast<const uint32_t*>(&h);
 }
+
+// Two binary32 values rounded to nearest even into bfloat16, lo in the low half.
+__device__ __forceinline__ uint32_t pack_bf162(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+__device__ __forceinline__ uint16_t to_bf16_bits(float x) {
+    uint16_t h;
+    asm("cvt.rn.bf16.f32 %0, %1;" : "=h"(h) : "f"(x));
+    return h;
+}
+// A bfloat16 value is the binary32 number with the same upper 16 bits.
+__device__ __forceinline__ float bf16_bits_to_float(uint32_t h) { return __uint_as_float(h << 16); }
 
 }  // namespace tc
 }  // namespace lrc

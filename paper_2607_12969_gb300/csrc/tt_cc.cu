@@ -15,7 +15,9 @@
 // Element types: binary64 cores with binary64 arithmetic, and binary16 cores
 // with binary32 arithmetic and a binary32 or binary16 output (the latter
 // rounded once per entry) for the shapes the tensor-core kernels do not take.
-// binary32 cores take the product chain of tt_chain.cu.
+// binary32 cores take the product chain of tt_chain.cu.  bfloat16 cores
+// (LRC_BF16) take the binary16 form with a bfloat16 output.
+#include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
 #include "common.cuh"
@@ -27,11 +29,13 @@ constexpr int kThreads = 256;
 constexpr int kTM = 4, kTN = 4;
 
 __device__ __forceinline__ float to_acc(__half x) { return __half2float(x); }
+__device__ __forceinline__ float to_acc(__nv_bfloat16 x) { return __bfloat162float(x); }
 __device__ __forceinline__ float to_acc(float x) { return x; }
 __device__ __forceinline__ double to_acc(double x) { return x; }
 __device__ __forceinline__ void store_out(float* p, float v) { *p = v; }
 __device__ __forceinline__ void store_out(double* p, double v) { *p = v; }
 __device__ __forceinline__ void store_out(__half* p, float v) { *p = __float2half_rn(v); }
+__device__ __forceinline__ void store_out(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
 
 template <typename TIn>
 struct TTParams {
@@ -206,6 +210,9 @@ lrc_status launch_tt_cc(const TTShape& sh, lrc_fmt fmt, void* out, cudaStream_t 
             return launch_tt_cc_t<double, double, double>(sh, static_cast<double*>(out), s, "tt_cc_kernel<f64>");
         case LRC_F16:
             return launch_tt_cc_t<float, __half, float>(sh, static_cast<float*>(out), s, "tt_cc_kernel<f16,o32>");
+        case LRC_BF16:
+            return launch_tt_cc_t<float, __nv_bfloat16, __nv_bfloat16>(sh, static_cast<__nv_bfloat16*>(out), s,
+                                                                      "tt_cc_kernel<bf16>");
         default:
             return launch_tt_cc_t<float, __half, __half>(sh, static_cast<__half*>(out), s, "tt_cc_kernel<f16,o16>");
     }

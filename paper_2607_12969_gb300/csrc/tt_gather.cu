@@ -8,7 +8,10 @@
 // the slice coalesced and add v_a (broadcast by a shuffle) times it.  The
 // last core is a column, reduced across the warp with a fixed butterfly.
 // Cores stay in L2; nothing but the indices and the outputs touches HBM.
+#include <cuda_bf16.h>
 #include <cuda_fp16.h>
+
+#include <type_traits>
 
 #include <algorithm>
 
@@ -33,6 +36,10 @@ template <>
 __device__ __forceinline__ float ld_core<float>(const float* p) { return __ldg(p); }
 template <>
 __device__ __forceinline__ float ld_core<__half>(const __half* p) { return __half2float(__ldg(p)); }
+template <>
+__device__ __forceinline__ float ld_core<__nv_bfloat16>(const __nv_bfloat16* p) {
+    return __uint_as_float((uint32_t)__ldg(reinterpret_cast<const unsigned short*>(p)) << 16);
+}
 
 __device__ __forceinline__ double ld_core64(const double* p) { return __ldg(p); }
 
@@ -47,7 +54,9 @@ __device__ __forceinline__ A load_elem(const T* p) {
 
 template <typename O, typename A>
 __device__ __forceinline__ O store_cast(A v) {
-    if constexpr (sizeof(O) == 2) {
+    if constexpr (std::is_same_v<O, __nv_bfloat16>) {
+        return __float2bfloat16_rn((float)v);
+    } else if constexpr (sizeof(O) == 2) {
         return __float2half_rn((float)v);
     } else {
         return (O)v;
@@ -62,6 +71,10 @@ template <>
 __device__ __forceinline__ float quiet_nan<float>() { return __int_as_float(0x7fc00000); }
 template <>
 __device__ __forceinline__ __half quiet_nan<__half>() { return __ushort_as_half((unsigned short)0x7e00); }
+template <>
+__device__ __forceinline__ __nv_bfloat16 quiet_nan<__nv_bfloat16>() {
+    return __ushort_as_bfloat16((unsigned short)0x7fc0);
+}
 
 // T: core element type, A: arithmetic type, O: output type, S: slots per lane
 // (ranks up to 32 S).
@@ -196,6 +209,7 @@ lrc_status launch_tt_gather(const TTShape& sh, lrc_fmt fmt, const int64_t* idx, 
         case LRC_F32: return launch_typed<float, float, float>(g, rmax, idx, count, out, s);
         case LRC_F16: return launch_typed<__half, float, float>(g, rmax, idx, count, out, s);
         case LRC_F16_O16: return launch_typed<__half, float, __half>(g, rmax, idx, count, out, s);
+        case LRC_BF16: return launch_typed<__nv_bfloat16, float, __nv_bfloat16>(g, rmax, idx, count, out, s);
     }
     set_error("unknown format");
     return LRC_ERR_INVALID_ARG;

@@ -26,7 +26,13 @@
 // [2^14, 2^15) before rounding, so lo stays a normal binary16 number; the
 // product's epilogue multiplies each output entry by the inverse scales
 // (exact).
+// bfloat16 cores (LRC_BF16) take the same chain with bfloat16 operand images
+// rounded once (the format's method-precision workspace) and a bfloat16
+// tensor-core product.
+#include <cuda_bf16.h>
 #include <cuda_fp16.h>
+
+#include <type_traits>
 
 #include "common.cuh"
 #include "tc.cuh"
@@ -63,6 +69,14 @@ __device__ __forceinline__ __half part_value(float y, bool lo) {
     return lo ? __float2half_rn(y - __half2float(hi)) : hi;
 }
 
+// Encoding of one operand-image element: binary16 parts, or one bfloat16
+// rounding (the bfloat16 chain has a single part).
+template <bool BF>
+__device__ __forceinline__ uint16_t image_bits(float y, bool lo) {
+    if constexpr (BF) return tc::to_bf16_bits(y);
+    else return __half_as_ushort(part_value(y, lo));
+}
+
 __device__ __forceinline__ float block_max(float v, float* sh) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
@@ -87,7 +101,7 @@ struct SideArgs {
     Parts pw, pu;
     int scale_w, scale_u;
     unsigned char* Wimg;      // ceil(P / 128) images of 128 x kp
-    __half* Uimg;             // Q rows of kp
+    uint16_t* Uimg;           // Q rows of kp
     float* Zout;              // binary32 mode: Z (P x r) and S (r x Q), row-major
     float* Sout;
     int* esc_w;               // [ceil(P / kUnit)]
@@ -95,6 +109,9 @@ struct SideArgs {
 };
 
 __device__ __forceinline__ float core_at(const __half* g, int64_t i) { return __half2float(__ldg(g + i)); }
+__device__ __forceinline__ float core_at(const __nv_bfloat16* g, int64_t i) {
+    return tc::bf16_bits_to_float(__ldg(reinterpret_cast<const unsigned short*>(g) + i));
+}
 __device__ __forceinline__ float core_at(const float* g, int64_t i) { return __ldg(g + i); }
 
 // Copies count core elements to shared memory, dst[didx(e)] = G[sidx(e)],
@@ -138,7 +155,17 @@ __device__ __forceinline__ const float* stage_core(const SideArgs& a, int l, flo
         for (int u = 0; u < 4; ++u) {
             const int64_t i = v0 + u * (int64_t)blockDim.x + threadIdx.x;
             if (i < nv) {
-                if constexpr (sizeof(TC) == 2) {
+                if constexpr (std::is_same_v<TC, __nv_bfloat16>) {
+                    const uint32_t q[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+                    float f[8];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        f[2 * j] = __uint_as_float(q[j] << 16);
+                        f[2 * j + 1] = __uint_as_float(q[j] & 0xffff0000u);
+                    }
+                    reinterpret_cast<float4*>(gs + i * 8)[0] = make_float4(f[0], f[1], f[2], f[3]);
+                    reinterpret_cast<float4*>(gs + i * 8)[1] = make_float4(f[4], f[5], f[6], f[7]);
+                } else if constexpr (sizeof(TC) == 2) {
                     const __half2* h = reinterpret_cast<const __half2*>(&w[u]);
                     const float2 f0 = __half22float2(h[0]), f1 = __half22float2(h[1]);
                     const float2 f2 = __half22float2(h[2]), f3 = __half22float2(h[3]);
@@ -253,6 +280,7 @@ __device__ float* right_cols(const SideArgs& a, int64_t q0, int64_t qend, float*
 template <typename TC, bool IMG>
 __global__ void __launch_bounds__(256)
 tt_side_kernel(const SideArgs a) {
+    constexpr bool BF = std::is_same_v<TC, __nv_bfloat16>;
     extern __shared__ float sbuf[];
     __shared__ float red[8];
     tc::pdl_wait();
@@ -287,11 +315,11 @@ tt_side_kernel(const SideArgs a) {
             const int row = i % kUnit, c0 = (i / kUnit) * 8;
             const int p = c0 / a.rp, a0 = c0 - p * a.rp;
             const bool lo = (a.pw.lomask >> p) & 1;
-            __align__(16) __half h[8];
+            __align__(16) uint16_t h[8];
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
                 const int k = a0 + j;
-                h[j] = (k < a.r && row < nrow) ? part_value(z[row * a.ldb + k] * f, lo) : __float2half_rn(0.0f);
+                h[j] = (k < a.r && row < nrow) ? image_bits<BF>(z[row * a.ldb + k] * f, lo) : (uint16_t)0;
             }
             *reinterpret_cast<uint4*>(tile + tc::w_image_off((uint32_t)(ro + row), (uint32_t)c0)) =
                 *reinterpret_cast<const uint4*>(h);
@@ -327,11 +355,11 @@ tt_side_kernel(const SideArgs a) {
             const int p = c0 / a.rp, a0 = c0 - p * a.rp;
             const bool lo = (a.pu.lomask >> p) & 1;
             const float* col = sc + (base + q) * a.ldb;
-            __align__(16) __half h[8];
+            __align__(16) uint16_t h[8];
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
                 const int k = a0 + j;
-                h[j] = (k < a.r) ? part_value(col[k] * f, lo) : __float2half_rn(0.0f);
+                h[j] = (k < a.r) ? image_bits<BF>(col[k] * f, lo) : (uint16_t)0;
             }
             *reinterpret_cast<uint4*>(a.Uimg + (q0 + q) * kp + c0) = *reinterpret_cast<const uint4*>(h);
         }
@@ -392,6 +420,7 @@ namespace {
 template <typename TC>
 lrc_status launch_split_t(const TTShape& sh, bool out16, void* out, cudaStream_t s, bool* handled) {
     constexpr bool kExactCores = sizeof(TC) == 2;
+    constexpr bool kBF = std::is_same_v<TC, __nv_bfloat16>;
     *handled = false;
     const int d = sh.d;
     if (d > 16) return LRC_OK;
@@ -434,7 +463,7 @@ lrc_status launch_split_t(const TTShape& sh, bool out16, void* out, cudaStream_t
     if (st != LRC_OK) return st;
     unsigned char* ws = static_cast<unsigned char*>(wsp);
     a.Wimg = ws;
-    a.Uimg = reinterpret_cast<__half*>(ws + w_bytes);
+    a.Uimg = reinterpret_cast<uint16_t*>(ws + w_bytes);
     a.esc_w = reinterpret_cast<int*>(ws + w_bytes + u_bytes);
     a.esc_u = a.esc_w + a.wunits;
     cudaError_t e = cudaFuncSetAttribute(tt_side_kernel<TC, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -443,7 +472,7 @@ lrc_status launch_split_t(const TTShape& sh, bool out16, void* out, cudaStream_t
     e = launch_pdl(tt_side_kernel<TC, true>, dim3((unsigned)(a.wunits + uunits)), dim3(256), smem, s, a);
     if (e != cudaSuccess) return cuda_fail(e, "tt_side_kernel launch");
     if ((st = after_launch("tt_side_kernel")) != LRC_OK) return st;
-    return launch_y_product(a.Wimg, kp, a.Uimg, kp, a.Q, a.P, out16, out, a.esc_w, a.esc_u, s);
+    return launch_y_product(a.Wimg, kp, a.Uimg, kp, a.Q, a.P, out16, out, a.esc_w, a.esc_u, s, false, kBF);
 }
 
 }  // namespace
@@ -454,6 +483,13 @@ lrc_status launch_tt_split_f16(const TTShape& sh, bool out16, void* out, cudaStr
 
 lrc_status launch_tt_split_f32tc(const TTShape& sh, float* out, cudaStream_t s, bool* handled) {
     return launch_split_t<float>(sh, false, out, s, handled);
+}
+
+lrc_status launch_tt_bf16(const TTShape& sh, void* out, cudaStream_t s) {
+    bool handled = false;
+    lrc_status st = launch_split_t<__nv_bfloat16>(sh, true, out, s, &handled);
+    if (handled) return st;
+    return launch_tt_cc(sh, LRC_BF16, out, s);
 }
 
 lrc_status launch_tt_side_f32(const TTShape& sh, float* out, cudaStream_t s, bool* handled) {

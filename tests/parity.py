@@ -5,8 +5,11 @@ import numpy as np
 import oracle
 
 # relative Frobenius tolerances per path
-TOL = {"f64": 1e-12, "f32": 1e-5, "f16": 1e-5, "f16_o16": 2e-3, "f32tc": 1e-5}
-BITS_DTYPE = {"f64": np.float64, "f32": np.uint32, "f16": np.uint16}
+# bf16: 4 u with u = 2^-8, the multiple of the unit roundoff the FP16-output
+# bar uses (2e-3 ~ 4 x 2^-11): W and the output are each rounded once to
+# bfloat16, a relative Frobenius error of at most about 2u
+TOL = {"f64": 1e-12, "f32": 1e-5, "f16": 1e-5, "f16_o16": 2e-3, "f32tc": 1e-5, "bf16": 4 * 2.0 ** -8}
+BITS_DTYPE = {"f64": np.float64, "f32": np.uint32, "f16": np.uint16, "bf16": np.uint16}
 
 
 def base_fmt(fmt: str) -> str:
@@ -33,7 +36,15 @@ def packed(lrc, a64: np.ndarray, fmt: str, dev):
 
 
 def bits(t, fmt: str) -> np.ndarray:
+    import torch
+    if t.dtype == torch.bfloat16:            # numpy has no bfloat16: read the encodings
+        t = t.view(torch.int16)
     return t.cpu().numpy().view(BITS_DTYPE[base_fmt(fmt)])
+
+
+def host64(t) -> np.ndarray:
+    """FP64 copy of a device tensor of any storage format (exact widening)."""
+    return t.double().cpu().numpy()
 
 
 def oracle_inputs(U, s, Vt, X, fmt):

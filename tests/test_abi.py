@@ -54,8 +54,10 @@ def test_validation_rejects_before_launch(L):
     assert st == -1
     st = L.lrc_apply(16, 16, 16, 16, 16, 4, 4, 2, 1, 7, None)
     assert st == -1
-    st = L.lrc_apply(16, 16, 16, 16, 16, 4, 4, 2, 1, 5, None)       # one past LRC_F32_TC
+    st = L.lrc_apply(16, 16, 16, 16, 16, 4, 4, 2, 1, 6, None)       # one past LRC_BF16
     assert st == -1
+    st = L.lrc_apply(17, 16, 16, 16, 16, 4, 4, 2, 1, 5, None)       # LRC_BF16 is a format: checks go on
+    assert st == -2
     st = L.lrc_apply(17, 16, 16, 16, 16, 4, 4, 2, 1, 4, None)       # LRC_F32_TC is a format: checks go on
     assert st == -2
     st = L.lrc_apply(17, 16, 16, 16, 16, 4, 4, 2, 1, 0, None)      # misaligned U
