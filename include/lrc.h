@@ -126,7 +126,8 @@ LRC_API lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows,
  *
  * Element types: LRC_F64 -> U, S, Vt, X, Y binary64; LRC_F32 -> all
  * binary32; LRC_F16 -> U, S, Vt, X binary16 and Y binary32; LRC_F16_O16 ->
- * all binary16 (the intermediate is rounded to binary16 as well).  Pad
+ * all binary16 (the intermediate is rounded to binary16 as well); LRC_BF16
+ * -> all bfloat16 (intermediate too), on the tensor-core path at every b.  Pad
  * columns of U, Vt and X are never read.  All five pointers must be 16-byte
  * aligned.  k may exceed min(m, n).  Asynchronous on `stream`.
  *
@@ -145,6 +146,34 @@ LRC_API lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows,
 LRC_API lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X, void* Y,
                      int64_t m, int64_t n, int64_t k, int64_t b, lrc_fmt fmt,
                      lrc_stream_t stream);
+
+/*
+ * lrc_apply_batched -- `count` independent applies of lrc_apply in one call:
+ * problem p applies its own rank-k[p] factors U[p], S[p], Vt[p] of an
+ * m[p] x n[p] matrix to its own b[p] queries X[p], writing Y[p].  The paper
+ * times its matrix applies aggregated over a set of matrices (Sec. 4.4, ten
+ * matrices per measurement); this is that aggregate as one call.
+ *
+ *   U, S, Vt, X, Y   HOST arrays of `count` DEVICE pointers, each with the
+ *                    layout, element type and alignment of lrc_apply
+ *   m, n, k, b       HOST arrays of `count` sizes
+ *   fmt              one format for every problem
+ *
+ * LRC_F16, LRC_F16_O16 and LRC_BF16: the problems share the tensor-core
+ * kernels' launches -- one launch per phase for up to 16 problems (the
+ * multiprocessors are divided among the problems in proportion to their
+ * work; larger counts take one set of launches per 16), and every batch size
+ * takes the tensor-core path.  Other formats: the problems are launched one
+ * after another as lrc_apply would.  Results equal lrc_apply's on each
+ * problem up to the summation order of the split reduction (same tolerance).
+ * 0 <= count <= 4096.  Every problem is validated before anything is
+ * launched; the message of a failure names the problem.  Workspace: the
+ * stream's library workspace, the sum of the problems' (see lrc_apply).
+ * Asynchronous on `stream`.
+ */
+LRC_API lrc_status lrc_apply_batched(int count, const void* const* U, const void* const* S, const void* const* Vt,
+                                     const void* const* X, void* const* Y, const int64_t* m, const int64_t* n,
+                                     const int64_t* k, const int64_t* b, lrc_fmt fmt, lrc_stream_t stream);
 
 /*
  * tt_reconstruct -- dense Tensor-Train reconstruction (Sec. 5.1:

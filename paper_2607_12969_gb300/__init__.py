@@ -55,6 +55,8 @@ def load() -> ctypes.CDLL:
     L.lrc_widen_factors.restype = i32
     L.lrc_apply.argtypes = [vp, vp, vp, vp, vp, i64, i64, i64, i64, i32, vp]
     L.lrc_apply.restype = i32
+    L.lrc_apply_batched.argtypes = [i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, i32, vp]
+    L.lrc_apply_batched.restype = i32
     L.tt_reconstruct.argtypes = [vp, vp, vp, i32, i32, vp, vp]
     L.tt_reconstruct.restype = i32
     L.lrc_fro_diff.argtypes = [vp, i32, vp, i32, i64, vp, vp, vp]
@@ -212,6 +214,32 @@ def lrc_apply(U, S, Vt, X, Y, m: int, n: int, k: int, b: int, fmt, stream=None):
         _need(Y, "Y", output_dtype(fmt), b * m, stream=stream)
     _check(load().lrc_apply(_ptr(U), _ptr(S), _ptr(Vt), _ptr(X), _ptr(Y), m, n, k, b, _fmt(fmt),
                             _stream(stream)))
+
+
+def lrc_apply_batched(U: Sequence, S: Sequence, Vt: Sequence, X: Sequence, Y: Sequence, m: Sequence[int],
+                      n: Sequence[int], k: Sequence[int], b: Sequence[int], fmt, stream=None):
+    """Several independent applies in one call: problem p is
+    lrc_apply(U[p], S[p], Vt[p], X[p], Y[p], m[p], n[p], k[p], b[p], fmt)."""
+    count = len(U)
+    if not all(len(a) == count for a in (S, Vt, X, Y, m, n, k, b)):
+        raise ValueError("every argument needs one entry per problem")
+    st, ot = storage_dtype(fmt), output_dtype(fmt)
+    for p in range(count):
+        mp, np_, kp, bp = int(m[p]), int(n[p]), int(k[p]), int(b[p])
+        if mp > 0 and np_ > 0 and kp > 0 and bp > 0:
+            ldk, ldn = lrc_packed_ld(kp), lrc_packed_ld(np_)
+            _need(U[p], f"U[{p}]", st, _extent(mp, kp, ldk), stream=stream)
+            _need(S[p], f"S[{p}]", st, kp, stream=stream)
+            _need(Vt[p], f"Vt[{p}]", st, _extent(kp, np_, ldn), stream=stream)
+            _need(X[p], f"X[{p}]", st, _extent(bp, np_, ldn), stream=stream)
+            _need(Y[p], f"Y[{p}]", ot, bp * mp, stream=stream)
+    arr = lambda ts: (ctypes.c_void_p * max(count, 1))(*[_ptr(t) for t in ts])  # noqa: E731
+    i64s = lambda xs: (ctypes.c_int64 * max(count, 1))(*[int(x) for x in xs])   # noqa: E731
+    pu, ps, pv, px, py = arr(U), arr(S), arr(Vt), arr(X), arr(Y)
+    am, an, ak, ab = i64s(m), i64s(n), i64s(k), i64s(b)
+    c = lambda a: ctypes.cast(a, ctypes.c_void_p)   # noqa: E731
+    _check(load().lrc_apply_batched(count, c(pu), c(ps), c(pv), c(px), c(py), c(am), c(an), c(ak), c(ab),
+                                    _fmt(fmt), _stream(stream)))
 
 
 def _need_cores(cores, dims, ranks, fmt, stream=None) -> bool:

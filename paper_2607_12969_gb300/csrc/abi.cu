@@ -134,10 +134,14 @@ lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows, int64_t
     return launch_widen(src, fmt, rows, cols, ld_src, dst, ld_dst, as_stream(stream));
 }
 
-lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X, void* Y,
-                     int64_t m, int64_t n, int64_t k, int64_t b, lrc_fmt fmt,
-                     lrc_stream_t stream) {
-    if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+}  // extern "C"
+
+namespace {
+
+// Checks of one apply (sizes, overflow, pointers, alignment) before anything
+// is launched.
+lrc_status check_apply(const void* U, const void* S, const void* Vt, const void* X, const void* Y, int64_t m,
+                       int64_t n, int64_t k, int64_t b) {
     if (m <= 0 || n <= 0 || k <= 0 || b <= 0)
         return invalid("sizes must be positive (m=%lld n=%lld k=%lld b=%lld)", (long long)m,
                        (long long)n, (long long)k, (long long)b);
@@ -153,24 +157,82 @@ lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X
     if (!aligned16(Vt)) return misaligned("Vt");
     if (!aligned16(X)) return misaligned("X");
     if (!aligned16(Y)) return misaligned("Y");
-    cudaStream_t s = as_stream(stream);
-    if (apply_skinny_takes(plain_fmt(fmt), b, k))
-        return launch_apply_skinny(U, S, Vt, X, Y, m, n, k, b, plain_fmt(fmt), s);
+    return LRC_OK;
+}
+
+lrc_status dispatch_apply(const ApplyProblem& p, lrc_fmt fmt, cudaStream_t s) {
+    if (apply_skinny_takes(plain_fmt(fmt), p.b, p.k))
+        return launch_apply_skinny(p.U, p.S, p.Vt, p.X, p.Y, p.m, p.n, p.k, p.b, plain_fmt(fmt), s);
     switch (fmt) {
         case LRC_F64:
-            return launch_apply_f64((const double*)U, (const double*)S, (const double*)Vt,
-                                    (const double*)X, (double*)Y, m, n, k, b, s);
+            return launch_apply_f64((const double*)p.U, (const double*)p.S, (const double*)p.Vt, (const double*)p.X,
+                                    (double*)p.Y, p.m, p.n, p.k, p.b, s);
         case LRC_F32:
         case LRC_F32_TC:
-            return launch_apply_f32((const float*)U, (const float*)S, (const float*)Vt,
-                                    (const float*)X, (float*)Y, m, n, k, b, fmt == LRC_F32_TC, s);
+            return launch_apply_f32((const float*)p.U, (const float*)p.S, (const float*)p.Vt, (const float*)p.X,
+                                    (float*)p.Y, p.m, p.n, p.k, p.b, fmt == LRC_F32_TC, s);
         case LRC_F16:
         case LRC_F16_O16:
-            return launch_apply_f16(U, S, Vt, X, Y, m, n, k, b, fmt == LRC_F16_O16, s);
+            return launch_apply_f16(p.U, p.S, p.Vt, p.X, p.Y, p.m, p.n, p.k, p.b, fmt == LRC_F16_O16, s);
         case LRC_BF16:
-            return launch_apply_f16(U, S, Vt, X, Y, m, n, k, b, true, s, true);
+            return launch_apply_f16(p.U, p.S, p.Vt, p.X, p.Y, p.m, p.n, p.k, p.b, true, s, true);
     }
     return invalid("unknown format");
+}
+
+}  // namespace
+
+extern "C" {
+
+lrc_status lrc_apply(const void* U, const void* S, const void* Vt, const void* X, void* Y,
+                     int64_t m, int64_t n, int64_t k, int64_t b, lrc_fmt fmt,
+                     lrc_stream_t stream) {
+    if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    lrc_status st = check_apply(U, S, Vt, X, Y, m, n, k, b);
+    if (st != LRC_OK) return st;
+    return dispatch_apply(ApplyProblem{U, S, Vt, X, Y, m, n, k, b}, fmt, as_stream(stream));
+}
+
+lrc_status lrc_apply_batched(int count, const void* const* U, const void* const* S, const void* const* Vt,
+                             const void* const* X, void* const* Y, const int64_t* m, const int64_t* n,
+                             const int64_t* k, const int64_t* b, lrc_fmt fmt, lrc_stream_t stream) {
+    if (!valid_fmt(fmt)) return invalid("unknown format %d", (int)fmt);
+    if (count < 0 || count > 4096) return invalid("count must be in [0, 4096] (got %d)", count);
+    if (count == 0) return LRC_OK;
+    if (!U || !S || !Vt || !X || !Y || !m || !n || !k || !b) return invalid("null array");
+    for (int p = 0; p < count; ++p) {
+        lrc_status st = check_apply(U[p], S[p], Vt[p], X[p], Y[p], m[p], n[p], k[p], b[p]);
+        if (st != LRC_OK) {
+            char msg[256];
+            snprintf(msg, sizeof msg, "%s", lrc_last_error());
+            set_error("problem %d: %s", p, msg);
+            return st;
+        }
+        if ((fmt == LRC_F16 || fmt == LRC_F16_O16 || fmt == LRC_BF16) && k[p] > 512) {
+            set_error("problem %d: binary16 / bfloat16 ranks up to 512 (got %lld)", p, (long long)k[p]);
+            return LRC_ERR_UNSUPPORTED;
+        }
+    }
+    cudaStream_t s = as_stream(stream);
+    ApplyProblem pr[64];
+    if (fmt == LRC_F16 || fmt == LRC_F16_O16 || fmt == LRC_BF16) {
+        // tensor-core formats: one launch per phase for every group of problems
+        const int gmax = apply_f16_group_max();
+        for (int p0 = 0; p0 < count; p0 += gmax) {
+            const int c = count - p0 < gmax ? count - p0 : gmax;
+            for (int i = 0; i < c; ++i)
+                pr[i] = ApplyProblem{U[p0 + i], S[p0 + i], Vt[p0 + i], X[p0 + i], Y[p0 + i],
+                                     m[p0 + i], n[p0 + i], k[p0 + i], b[p0 + i]};
+            lrc_status st = launch_apply_f16_group(pr, c, fmt != LRC_F16, fmt == LRC_BF16, s);
+            if (st != LRC_OK) return st;
+        }
+        return LRC_OK;
+    }
+    for (int p = 0; p < count; ++p) {
+        lrc_status st = dispatch_apply(ApplyProblem{U[p], S[p], Vt[p], X[p], Y[p], m[p], n[p], k[p], b[p]}, fmt, s);
+        if (st != LRC_OK) return st;
+    }
+    return LRC_OK;
 }
 
 lrc_status tt_reconstruct(const void* const* cores, const int64_t* dims, const int64_t* ranks,

@@ -109,9 +109,9 @@ __device__ __forceinline__ bool next_chunk(int64_t& q, int64_t qbeg, int64_t qen
     return true;
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
-apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_v,
-                const __grid_constant__ CUtensorMap tm_xp, const __grid_constant__ CUtensorMap tm_vp, const W1Args a) {
+// Phase 1 of one problem, run by CTA `cta` of the `ncta` CTAs given to it.
+__device__ __forceinline__ void w1_body(const CUtensorMap* tm_x, const CUtensorMap* tm_v, const CUtensorMap* tm_xp,
+                                        const CUtensorMap* tm_vp, const W1Args& a, int64_t cta, int64_t ncta) {
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = align1024(smem_raw);
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + a.bar_off);
@@ -123,8 +123,8 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
     volatile int* abort = reinterpret_cast<int*>(tmem_slot + 1);
     unsigned int* err = &g_err_apply_tc;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t qbeg = a.Q * blockIdx.x / gridDim.x;
-    const int64_t qend = a.Q * (blockIdx.x + 1) / gridDim.x;
+    const int64_t qbeg = a.Q * cta / ncta;
+    const int64_t qend = a.Q * (cta + 1) / ncta;
     pdl_trigger();                 // the reduction kernel may be scheduled now; it waits for this grid
 
     if (threadIdx.x == 0) {
@@ -139,10 +139,10 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
         mbar_init(mma_done, 1);
         *abort = 0;
         fence_barrier_init();
-        tma_prefetch_desc(&tm_x);
-        tma_prefetch_desc(&tm_v);
-        tma_prefetch_desc(&tm_xp);
-        tma_prefetch_desc(&tm_vp);
+        tma_prefetch_desc(tm_x);
+        tma_prefetch_desc(tm_v);
+        tma_prefetch_desc(tm_xp);
+        tma_prefetch_desc(tm_vp);
     }
     if (warp == 1) tmem_alloc(tmem_slot, a.tmem_cols);
     tc_fence_before();
@@ -183,8 +183,8 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
                         for (int64_t pg = seg_first ? g0 : g0 + 2; pg <= g0 + 2; ++pg) {
                             const int64_t pkb = pg * kPfBlocks;
                             if (rbase + pkb >= seg_end) break;
-                            if (pf_x) tma_prefetch_2d(&tm_xp, (int32_t)(pkb * BK), (int32_t)(bt * BM));
-                            if (pf_v) tma_prefetch_2d(&tm_vp, (int32_t)(pkb * BK), grp * a.kgp);
+                            if (pf_x) tma_prefetch_2d(tm_xp, (int32_t)(pkb * BK), (int32_t)(bt * BM));
+                            if (pf_v) tma_prefetch_2d(tm_vp, (int32_t)(pkb * BK), grp * a.kgp);
                         }
                     }
                     const int slot = it % a.stages;
@@ -193,8 +193,8 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
                     mbar_arrive_expect_tx(&full[slot], (uint32_t)nb * (kXBytes + vbox));
                     for (int u = 0; u < nb; ++u) {
                         const int32_t kx = (int32_t)((qs + u - rbase) * BK);
-                        tma_load_2d(sp + (size_t)u * kXBytes, &tm_x, kx, (int32_t)(bt * BM), &full[slot]);
-                        tma_load_2d(sp + (size_t)kStageBlocks * kXBytes + (size_t)u * vbox, &tm_v, kx, grp * a.kgp,
+                        tma_load_2d(sp + (size_t)u * kXBytes, tm_x, kx, (int32_t)(bt * BM), &full[slot]);
+                        tma_load_2d(sp + (size_t)kStageBlocks * kXBytes + (size_t)u * vbox, tm_v, kx, grp * a.kgp,
                                     &full[slot]);
                     }
                 }
@@ -270,7 +270,7 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
             const int64_t bt = row - (int64_t)grp * a.btiles;
             const int kgw = min(a.kgp, a.kp - grp * a.kgp);
             const bool valid = bt * BM + r < a.b;
-            float* prow = a.P + ((size_t)(blockIdx.x + row) * a.kgp) * BM + r;
+            float* prow = a.P + ((size_t)(cta + row) * a.kgp) * BM + r;
             // every condition is decided once per 32 columns: the stores below
             // are straight-line code (a branch per element costs far more than
             // the store itself)
@@ -321,6 +321,34 @@ apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant_
     }
 }
 
+__global__ void __launch_bounds__(kThreads, 1)
+apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_v,
+                const __grid_constant__ CUtensorMap tm_xp, const __grid_constant__ CUtensorMap tm_vp, const W1Args a) {
+    w1_body(&tm_x, &tm_v, &tm_xp, &tm_vp, a, blockIdx.x, gridDim.x);
+}
+
+// Several problems in one launch: CTA blocks [cta_off[p], cta_off[p + 1]) run
+// problem p with its own arguments and tensor maps.
+constexpr int kMaxGroup = 16;
+struct GroupW1 {
+    CUtensorMap tm[kMaxGroup][4];    // X, V^T, X prefetch, V^T prefetch
+    W1Args args[kMaxGroup];
+    int cta_off[kMaxGroup + 1];
+    int count;
+};
+
+__device__ __forceinline__ int group_of(const int* off, int count, int64_t blk) {
+    int p = 0;
+    while (p + 1 < count && blk >= off[p + 1]) ++p;
+    return p;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) apply_w1_group_kernel(const __grid_constant__ GroupW1 g) {
+    const int p = group_of(g.cta_off, g.count, blockIdx.x);
+    w1_body(&g.tm[p][0], &g.tm[p][1], &g.tm[p][2], &g.tm[p][3], g.args[p], blockIdx.x - g.cta_off[p],
+            g.cta_off[p + 1] - g.cta_off[p]);
+}
+
 // ================================================================ reduction
 struct W2Args {
     int64_t b, btiles, nkb, Q;
@@ -364,12 +392,9 @@ __device__ __forceinline__ void put_w8(const W2Args& a, int64_t bt, int r, int c
 
 // One thread per (row tile, 8 columns, row): the partials of the entry are
 // added in CTA order, kBatch partials' loads in flight at a time.
-__global__ void __launch_bounds__(256)
-apply_w2_kernel(const W2Args a) {
-    pdl_trigger();
-    pdl_wait();                    // partials of the phase-1 grid
+__device__ __forceinline__ void w2_body(const W2Args& a, int64_t blk) {
     const int cg8 = a.kp / 8;
-    const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t e = blk * blockDim.x + threadIdx.x;
     if (e >= a.btiles * cg8 * BM) return;
     const int r = (int)(e % BM);
     const int64_t t = e / BM;
@@ -416,15 +441,12 @@ apply_w2_kernel(const W2Args a) {
 // partials' loads in flight at a time; warp 0 then adds the 16 warp sums in
 // warp order -- the same order on every run.
 constexpr int kW2Slices = 16;
-__global__ void __launch_bounds__(32 * kW2Slices)
-apply_w2_slice_kernel(const W2Args a) {
+__device__ __forceinline__ void w2_slice_body(const W2Args& a, int64_t blk) {
     __shared__ float red[kW2Slices][8][33];
-    pdl_trigger();
-    pdl_wait();                    // partials of the phase-1 grid
     const int cg8 = a.kp / 8;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t cg = blockIdx.x % cg8;
-    const int64_t t = blockIdx.x / cg8;
+    const int64_t cg = blk % cg8;
+    const int64_t t = blk / cg8;
     const int rb = (int)(t & 3);
     const int64_t bt = t >> 2;
     const int col0 = (int)cg * 8;
@@ -484,6 +506,37 @@ apply_w2_slice_kernel(const W2Args a) {
     put_w8(a, bt, r, col0, w);
 }
 
+__global__ void __launch_bounds__(256)
+apply_w2_kernel(const W2Args a) {
+    pdl_trigger();
+    pdl_wait();                    // partials of the phase-1 grid
+    w2_body(a, blockIdx.x);
+}
+
+__global__ void __launch_bounds__(32 * kW2Slices)
+apply_w2_slice_kernel(const W2Args a) {
+    pdl_trigger();
+    pdl_wait();
+    w2_slice_body(a, blockIdx.x);
+}
+
+struct GroupW2 {
+    W2Args args[kMaxGroup];
+    int blk_off[kMaxGroup + 1];
+    int count;
+};
+
+// SLICE: the sliced reduction (many partials per entry) for every problem of
+// the launch, else the plain one
+template <bool SLICE>
+__global__ void __launch_bounds__(SLICE ? 32 * kW2Slices : 256) apply_w2_group_kernel(const __grid_constant__ GroupW2 g) {
+    pdl_trigger();
+    pdl_wait();
+    const int p = group_of(g.blk_off, g.count, blockIdx.x);
+    if constexpr (SLICE) w2_slice_body(g.args[p], blockIdx.x - g.blk_off[p]);
+    else w2_body(g.args[p], blockIdx.x - g.blk_off[p]);
+}
+
 // ================================================================ phase 2
 struct YArgs {
     int64_t m, b, T;
@@ -505,8 +558,9 @@ struct YArgs {
     const int* esc_u;
 };
 
-__global__ void __launch_bounds__(kThreadsY, 1)
-apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__ CUtensorMap tm_y, const YArgs a) {
+// Phase 2 of one problem, run by CTA `cta` of the `ncta` CTAs given to it.
+__device__ __forceinline__ void y_body(const CUtensorMap* tm_u, const CUtensorMap* tm_y, const YArgs& a, int64_t cta,
+                                       int64_t ncta) {
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = align1024(smem_raw);
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + a.bar_off);
@@ -520,8 +574,8 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
     volatile int* abort = reinterpret_cast<int*>(tmem_slot + 1);
     unsigned int* err = &g_err_apply_tc;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t tbeg = a.T * blockIdx.x / gridDim.x;
-    const int64_t tend = a.T * (blockIdx.x + 1) / gridDim.x;
+    const int64_t tbeg = a.T * cta / ncta;
+    const int64_t tend = a.T * (cta + 1) / ncta;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < a.stages; ++i) {
@@ -537,8 +591,8 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
         mbar_init(mma_done, 1);
         *abort = 0;
         fence_barrier_init();
-        tma_prefetch_desc(&tm_u);
-        tma_prefetch_desc(&tm_y);
+        tma_prefetch_desc(tm_u);
+        tma_prefetch_desc(tm_y);
     }
     if (warp == 1) tmem_alloc(tmem_slot, a.tmem_cols);
     tc_fence_before();
@@ -570,7 +624,7 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
                     const int slot = it % a.stages;
                     if (!(ok = mbar_wait(&empty[slot], ((it / a.stages) & 1) ^ 1, abort, err, 1u))) break;
                     mbar_arrive_expect_tx(&full[slot], a.u_bytes);
-                    tma_load_2d(smem + (size_t)slot * a.slot_bytes, &tm_u, kc * BK, (int32_t)(mt * a.n2),
+                    tma_load_2d(smem + (size_t)slot * a.slot_bytes, tm_u, kc * BK, (int32_t)(mt * a.n2),
                                 &full[slot]);
                 }
             }
@@ -710,7 +764,7 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
                     fence_proxy_async_smem();
                     named_bar_sync(2 + half, 128);      // all four slices are written
                     if (issuer) {
-                        if (col0 < a.m) tma_store_2d(&tm_y, (int32_t)col0, (int32_t)row0, box);
+                        if (col0 < a.m) tma_store_2d(tm_y, (int32_t)col0, (int32_t)row0, box);
                         bulk_commit();      // one group per chunk, even empty: the staging reuse counts on it
                     }
                 } else {
@@ -744,6 +798,23 @@ apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__
         tc_fence_after();
         tmem_dealloc(tmem, a.tmem_cols);
     }
+}
+
+__global__ void __launch_bounds__(kThreadsY, 1)
+apply_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__ CUtensorMap tm_y, const YArgs a) {
+    y_body(&tm_u, &tm_y, a, blockIdx.x, gridDim.x);
+}
+
+struct GroupY {
+    CUtensorMap tm[kMaxGroup][2];    // U, Y
+    YArgs args[kMaxGroup];
+    int cta_off[kMaxGroup + 1];
+    int count;
+};
+
+__global__ void __launch_bounds__(kThreadsY, 1) apply_y_group_kernel(const __grid_constant__ GroupY g) {
+    const int p = group_of(g.cta_off, g.count, blockIdx.x);
+    y_body(&g.tm[p][0], &g.tm[p][1], g.args[p], blockIdx.x - g.cta_off[p], g.cta_off[p + 1] - g.cta_off[p]);
 }
 
 // ---------------------------------------------------------------- host side
@@ -881,10 +952,23 @@ lrc_status launch_y(const CUtensorMap& tu, const CUtensorMap& ty, const YArgs& a
 
 }  // namespace
 
-lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y, int64_t m,
-                            int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s, bool bf16) {
-    lrc_status st = get_encoder();
-    if (st != LRC_OK) return st;
+namespace {
+
+// The three launches of one binary16 / bfloat16 apply, planned in two
+// stages: the shapes (column groups, ring depths, tile widths), then -- once
+// the phase-1 and phase-2 CTA counts and the workspace are known -- the
+// pointers, the reduction's layout and the tensor maps.
+struct F16Plan {
+    W1Args a1{};
+    W2Args a2{};
+    YArgs a3{};
+    size_t smem1 = 0, smem3 = 0;
+    int64_t P1 = 0, P3 = 0, w2_blocks = 0;
+    bool slice = false;
+    CUtensorMap tx, tv, txp, tvp, tu, ty;
+};
+
+lrc_status plan_f16_shape(int64_t m, int64_t n, int64_t k, int64_t b, bool out16, bool bf16, F16Plan& pl) {
     if (bf16 && !out16) {
         set_error("bfloat16 apply: the output is bfloat16");
         return LRC_ERR_UNSUPPORTED;
@@ -894,13 +978,12 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
         set_error("binary16 apply supports rank up to 512 (got %lld)", (long long)k);
         return LRC_ERR_UNSUPPORTED;
     }
-    const int sms = sm_count();
     const int64_t btiles = (b + BM - 1) / BM;
     const int planes = out16 ? 1 : 2;
     const uint32_t tile_bytes = (uint32_t)BM * (uint32_t)kp * 2u;
 
     // ---- phase-1 plan: column groups, ring depth, running sum
-    W1Args a1{};
+    W1Args& a1 = pl.a1;
     a1.b = b;
     a1.btiles = btiles;
     a1.nkb = (n + BK - 1) / BK;
@@ -913,7 +996,6 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
     a1.chunk_blocks = out16 ? (int)(a1.nkb < 0x7fffffff ? a1.nkb : 0x7fffffff) : kChunkBlocks;
     const bool use_sum = a1.chunk_blocks < a1.nkb;
     a1.slot_bytes = (uint32_t)round_up((size_t)kStageBlocks * (kXBytes + (size_t)a1.kgp * 128), 1024);
-    size_t smem1 = 0;
     for (int stages = 6; stages >= 2; --stages) {
         size_t off = (size_t)stages * a1.slot_bytes;
         off = round_up(off, 8);
@@ -922,11 +1004,11 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
         if (off + 1024 <= kSmemMax) {
             a1.stages = stages;
             a1.bar_off = (uint32_t)bar_off;
-            smem1 = off + 1024;
+            pl.smem1 = off + 1024;
             break;
         }
     }
-    if (!smem1) {
+    if (!pl.smem1) {
         set_error("binary16 apply: rank %lld does not fit in shared memory", (long long)k);
         return LRC_ERR_UNSUPPORTED;
     }
@@ -939,76 +1021,191 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
         set_error("binary16 apply: rank %lld does not fit in tensor memory", (long long)k);
         return LRC_ERR_UNSUPPORTED;
     }
-    const int64_t P1 = a1.Q < sms ? a1.Q : sms;
 
     // ---- phase-2 plan: tile width, ring depth
-    YArgs a3{};
-    size_t smem3 = 0;
-    if ((st = plan_y(a3, smem3, m, b, kp, planes, out16, false)) != LRC_OK) return st;
-    a3.tile_bytes = tile_bytes;
+    lrc_status st = plan_y(pl.a3, pl.smem3, m, b, kp, planes, out16, false);
+    if (st != LRC_OK) return st;
+    pl.a3.tile_bytes = tile_bytes;
+    pl.a3.bf16 = bf16 ? 1 : 0;
+    pl.a3.idesc_ab = bf16 ? kIdescBF16 : 0u;
+    return LRC_OK;
+}
+
+// Workspace of the call for P1 phase-1 CTAs: W images, then the partials.
+size_t f16_ws_images(const F16Plan& pl) {
+    const int planes = pl.a3.planes;
+    return round_up((size_t)pl.a1.btiles * planes * pl.a3.tile_bytes, 256);
+}
+size_t f16_ws_bytes(const F16Plan& pl, int64_t P1) {
+    return f16_ws_images(pl) +
+           round_up((size_t)(pl.a1.btiles * pl.a1.G + P1) * pl.a1.kgp * BM * sizeof(float), 256);
+}
+
+lrc_status plan_f16_finish(F16Plan& pl, const void* U, const void* S, const void* Vt, const void* X, void* Y,
+                           int64_t m, int64_t n, int64_t k, int64_t b, bool out16, bool bf16, int64_t P1,
+                           int64_t P3, unsigned char* ws) {
+    W1Args& a1 = pl.a1;
+    YArgs& a3 = pl.a3;
+    pl.P1 = P1;
+    pl.P3 = P3;
+    a1.P = reinterpret_cast<float*>(ws + f16_ws_images(pl));
+    a3.W = ws;
     a3.Y = Y;
-    a3.bf16 = bf16 ? 1 : 0;
-    a3.idesc_ab = bf16 ? kIdescBF16 : 0u;
-    const int64_t P3 = a3.T < sms ? a3.T : sms;
-
-    // ---- workspace: W images, then the phase-1 partials
-    const size_t w_bytes_total = round_up((size_t)btiles * planes * tile_bytes, 256);
-    const size_t p_bytes = (size_t)(btiles * a1.G + P1) * a1.kgp * BM * sizeof(float);
-    void* ws = nullptr;
-    if ((st = stream_workspace(s, w_bytes_total + p_bytes, &ws)) != LRC_OK) return st;
-    unsigned char* Wimg = static_cast<unsigned char*>(ws);
-    a1.P = reinterpret_cast<float*>(Wimg + w_bytes_total);
-    a3.W = Wimg;
-
-    const int64_t ldn = lrc_packed_ld(n), ldk = lrc_packed_ld(k);
-    CUtensorMap tx, tv, tu, ty, txp, tvp;
-    const CUtensorMapDataType dt = t16(bf16);
-    if ((st = make_map(&tx, dt, X, n, b, ldn * 2, BK, BM, "X")) != LRC_OK) return st;
-    if ((st = make_map(&tv, dt, Vt, n, k, ldn * 2, BK, (uint32_t)a1.kgp, "Vt")) != LRC_OK) return st;
-    if ((st = make_map(&txp, dt, X, n, b, ldn * 2, kPfBlocks * BK, BM, "X prefetch", CU_TENSOR_MAP_SWIZZLE_NONE)) !=
-        LRC_OK)
-        return st;
-    if ((st = make_map(&tvp, dt, Vt, n, k, ldn * 2, kPfBlocks * BK, (uint32_t)a1.kgp, "Vt prefetch",
-                       CU_TENSOR_MAP_SWIZZLE_NONE)) != LRC_OK)
-        return st;
-    if ((st = make_map(&tu, dt, U, k, m, ldk * 2, BK, (uint32_t)a3.n2, "U")) != LRC_OK) return st;
-    if ((st = make_y_map(&ty, a3, Y, m, b, out16)) != LRC_OK) return st;
-
-    cudaError_t e = cudaFuncSetAttribute(apply_w1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
-    if (e != cudaSuccess) return cuda_fail(e, "apply_w1_kernel smem attribute");
-    apply_w1_kernel<<<(unsigned)P1, kThreads, smem1, s>>>(tx, tv, txp, tvp, a1);
-    if ((st = after_launch("apply_w1_kernel")) != LRC_OK) return st;
-
-    W2Args a2{};
+    W2Args& a2 = pl.a2;
     a2.b = b;
-    a2.btiles = btiles;
+    a2.btiles = a1.btiles;
     a2.nkb = a1.nkb;
     a2.Q = a1.Q;
     a2.P1 = (int)P1;
     a2.G = a1.G;
     a2.kgp = a1.kgp;
-    a2.kp = kp;
+    a2.kp = a1.kp;
     a2.k = (int)k;
-    a2.planes = planes;
-    a2.tile_bytes = tile_bytes;
+    a2.planes = a3.planes;
+    a2.tile_bytes = a3.tile_bytes;
     a2.P = a1.P;
     a2.S = static_cast<const uint16_t*>(S);
     a2.bf16 = bf16 ? 1 : 0;
-    a2.W = Wimg;
-    const int64_t n2items = btiles * (kp / 8) * BM;
+    a2.W = ws;
+    const int kp = a1.kp;
     const int64_t max_parts = (a1.nkb * P1 + a1.Q - 1) / a1.Q + 1;     // CTAs sharing one row, at most
-    if (max_parts >= 16) {
-        e = launch_pdl(apply_w2_slice_kernel, dim3((unsigned)(btiles * 4 * (kp / 8))), dim3(32 * kW2Slices), 0, s,
-                       a2);
+    pl.slice = max_parts >= 16;
+    pl.w2_blocks = pl.slice ? a1.btiles * 4 * (kp / 8) : (a1.btiles * (kp / 8) * BM + 255) / 256;
+
+    const int64_t ldn = lrc_packed_ld(n), ldk = lrc_packed_ld(k);
+    const CUtensorMapDataType dt = t16(bf16);
+    lrc_status st;
+    if ((st = make_map(&pl.tx, dt, X, n, b, ldn * 2, BK, BM, "X")) != LRC_OK) return st;
+    if ((st = make_map(&pl.tv, dt, Vt, n, k, ldn * 2, BK, (uint32_t)a1.kgp, "Vt")) != LRC_OK) return st;
+    if ((st = make_map(&pl.txp, dt, X, n, b, ldn * 2, kPfBlocks * BK, BM, "X prefetch", CU_TENSOR_MAP_SWIZZLE_NONE)) !=
+        LRC_OK)
+        return st;
+    if ((st = make_map(&pl.tvp, dt, Vt, n, k, ldn * 2, kPfBlocks * BK, (uint32_t)a1.kgp, "Vt prefetch",
+                       CU_TENSOR_MAP_SWIZZLE_NONE)) != LRC_OK)
+        return st;
+    if ((st = make_map(&pl.tu, dt, U, k, m, ldk * 2, BK, (uint32_t)a3.n2, "U")) != LRC_OK) return st;
+    if ((st = make_y_map(&pl.ty, a3, Y, m, b, out16)) != LRC_OK) return st;
+    if (!a3.tma_store) pl.ty = pl.tu;          // unused by the kernel
+    return LRC_OK;
+}
+
+}  // namespace
+
+lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y, int64_t m,
+                            int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s, bool bf16) {
+    lrc_status st = get_encoder();
+    if (st != LRC_OK) return st;
+    F16Plan pl;
+    if ((st = plan_f16_shape(m, n, k, b, out16, bf16, pl)) != LRC_OK) return st;
+    const int sms = sm_count();
+    const int64_t P1 = pl.a1.Q < sms ? pl.a1.Q : sms;
+    const int64_t P3 = pl.a3.T < sms ? pl.a3.T : sms;
+    void* ws = nullptr;
+    if ((st = stream_workspace(s, f16_ws_bytes(pl, P1), &ws)) != LRC_OK) return st;
+    if ((st = plan_f16_finish(pl, U, S, Vt, X, Y, m, n, k, b, out16, bf16, P1, P3, static_cast<unsigned char*>(ws))) !=
+        LRC_OK)
+        return st;
+
+    cudaError_t e = cudaFuncSetAttribute(apply_w1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem1);
+    if (e != cudaSuccess) return cuda_fail(e, "apply_w1_kernel smem attribute");
+    apply_w1_kernel<<<(unsigned)P1, kThreads, pl.smem1, s>>>(pl.tx, pl.tv, pl.txp, pl.tvp, pl.a1);
+    if ((st = after_launch("apply_w1_kernel")) != LRC_OK) return st;
+    if (pl.slice) {
+        e = launch_pdl(apply_w2_slice_kernel, dim3((unsigned)pl.w2_blocks), dim3(32 * kW2Slices), 0, s, pl.a2);
         if (e != cudaSuccess) return cuda_fail(e, "apply_w2_slice_kernel launch");
         if ((st = after_launch("apply_w2_slice_kernel")) != LRC_OK) return st;
     } else {
-        e = launch_pdl(apply_w2_kernel, dim3((unsigned)((n2items + 255) / 256)), dim3(256), 0, s, a2);
+        e = launch_pdl(apply_w2_kernel, dim3((unsigned)pl.w2_blocks), dim3(256), 0, s, pl.a2);
         if (e != cudaSuccess) return cuda_fail(e, "apply_w2_kernel launch");
         if ((st = after_launch("apply_w2_kernel")) != LRC_OK) return st;
     }
+    return launch_y(pl.tu, pl.ty, pl.a3, pl.smem3, P3, s);
+}
 
-    return launch_y(tu, ty, a3, smem3, P3, s);
+int apply_f16_group_max() { return kMaxGroup; }
+
+lrc_status launch_apply_f16_group(const ApplyProblem* pr, int count, bool out16, bool bf16, cudaStream_t s) {
+    if (count < 1 || count > kMaxGroup) {
+        set_error("grouped binary16 apply: 1 to %d problems per launch (got %d)", kMaxGroup, count);
+        return LRC_ERR_INVALID_ARG;
+    }
+    lrc_status st = get_encoder();
+    if (st != LRC_OK) return st;
+    static thread_local F16Plan pls[kMaxGroup];
+    int64_t qsum = 0, tsum = 0;
+    for (int p = 0; p < count; ++p) {
+        pls[p] = F16Plan{};
+        if ((st = plan_f16_shape(pr[p].m, pr[p].n, pr[p].k, pr[p].b, out16, bf16, pls[p])) != LRC_OK) return st;
+        qsum += pls[p].a1.Q;
+        tsum += pls[p].a3.T;
+    }
+    // CTAs in proportion to each problem's share of the units (at least one,
+    // at most one per unit), about one SM's worth in all
+    const int sms = sm_count();
+    int64_t P1[kMaxGroup], P3[kMaxGroup];
+    size_t ws_bytes = 0;
+    for (int p = 0; p < count; ++p) {
+        int64_t c1 = sms * pls[p].a1.Q / qsum, c3 = sms * pls[p].a3.T / tsum;
+        c1 = c1 < 1 ? 1 : (c1 > pls[p].a1.Q ? pls[p].a1.Q : c1);
+        c3 = c3 < 1 ? 1 : (c3 > pls[p].a3.T ? pls[p].a3.T : c3);
+        P1[p] = c1;
+        P3[p] = c3;
+        ws_bytes += f16_ws_bytes(pls[p], c1);
+    }
+    void* wsp = nullptr;
+    if ((st = stream_workspace(s, ws_bytes, &wsp)) != LRC_OK) return st;
+    unsigned char* ws = static_cast<unsigned char*>(wsp);
+    static thread_local GroupW1 g1;
+    static thread_local GroupW2 g2[2];
+    static thread_local GroupY g3;
+    g1.count = g3.count = count;
+    g1.cta_off[0] = g3.cta_off[0] = 0;
+    g2[0].count = g2[1].count = 0;
+    g2[0].blk_off[0] = g2[1].blk_off[0] = 0;
+    size_t smem1 = 0, smem3 = 0;
+    for (int p = 0; p < count; ++p) {
+        F16Plan& pl = pls[p];
+        if ((st = plan_f16_finish(pl, pr[p].U, pr[p].S, pr[p].Vt, pr[p].X, pr[p].Y, pr[p].m, pr[p].n, pr[p].k, pr[p].b,
+                                  out16, bf16, P1[p], P3[p], ws)) != LRC_OK)
+            return st;
+        ws += f16_ws_bytes(pl, P1[p]);
+        g1.tm[p][0] = pl.tx;
+        g1.tm[p][1] = pl.tv;
+        g1.tm[p][2] = pl.txp;
+        g1.tm[p][3] = pl.tvp;
+        g1.args[p] = pl.a1;
+        g1.cta_off[p + 1] = g1.cta_off[p] + (int)P1[p];
+        GroupW2& w = g2[pl.slice ? 1 : 0];
+        w.args[w.count] = pl.a2;
+        w.blk_off[w.count + 1] = w.blk_off[w.count] + (int)pl.w2_blocks;
+        ++w.count;
+        g3.tm[p][0] = pl.tu;
+        g3.tm[p][1] = pl.ty;
+        g3.args[p] = pl.a3;
+        g3.cta_off[p + 1] = g3.cta_off[p] + (int)P3[p];
+        smem1 = pl.smem1 > smem1 ? pl.smem1 : smem1;
+        smem3 = pl.smem3 > smem3 ? pl.smem3 : smem3;
+    }
+    cudaError_t e = cudaFuncSetAttribute(apply_w1_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
+    if (e != cudaSuccess) return cuda_fail(e, "apply_w1_group_kernel smem attribute");
+    apply_w1_group_kernel<<<(unsigned)g1.cta_off[count], kThreads, smem1, s>>>(g1);
+    if ((st = after_launch("apply_w1_group_kernel")) != LRC_OK) return st;
+    if (g2[0].count) {
+        e = launch_pdl(apply_w2_group_kernel<false>, dim3((unsigned)g2[0].blk_off[g2[0].count]), dim3(256), 0, s, g2[0]);
+        if (e != cudaSuccess) return cuda_fail(e, "apply_w2_group_kernel launch");
+        if ((st = after_launch("apply_w2_group_kernel")) != LRC_OK) return st;
+    }
+    if (g2[1].count) {
+        e = launch_pdl(apply_w2_group_kernel<true>, dim3((unsigned)g2[1].blk_off[g2[1].count]), dim3(32 * kW2Slices), 0,
+                       s, g2[1]);
+        if (e != cudaSuccess) return cuda_fail(e, "apply_w2_group_kernel launch");
+        if ((st = after_launch("apply_w2_group_kernel")) != LRC_OK) return st;
+    }
+    e = cudaFuncSetAttribute(apply_y_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem3);
+    if (e != cudaSuccess) return cuda_fail(e, "apply_y_group_kernel smem attribute");
+    e = launch_pdl(apply_y_group_kernel, dim3((unsigned)g3.cta_off[count]), dim3(kThreadsY), smem3, s, g3);
+    if (e != cudaSuccess) return cuda_fail(e, "apply_y_group_kernel launch");
+    return after_launch("apply_y_group_kernel");
 }
 
 lrc_status encode_map_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, int64_t cols, int64_t rows,

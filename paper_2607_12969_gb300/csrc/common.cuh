@@ -97,6 +97,19 @@ lrc_status launch_apply_split_f64(const double* U, const double* S, const double
                                   int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
 lrc_status launch_apply_split_f32(const float* U, const float* S, const float* Vt, const float* X, float* Y,
                                   int64_t m, int64_t n, int64_t k, int64_t b, cudaStream_t s);
+// One apply of a batch (lrc_apply_batched); layouts of lrc_apply.
+struct ApplyProblem {
+    const void* U;
+    const void* S;
+    const void* Vt;
+    const void* X;
+    void* Y;
+    int64_t m, n, k, b;
+};
+// Up to apply_f16_group_max() binary16 / bfloat16 problems in one launch per
+// phase (apply_tc.cu); every problem is validated by the caller.
+int apply_f16_group_max();
+lrc_status launch_apply_f16_group(const ApplyProblem* pr, int count, bool out16, bool bf16, cudaStream_t s);
 // bf16: bfloat16 operands and output (out16 must be set)
 lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y,
                             int64_t m, int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s,
