@@ -28,10 +28,12 @@ replica with its own query batches: weak scaling, no collective).
 The FP64 baseline (rank k), the compensated calls and torch.matmul (the
 paper's own method, cuBLAS) are then timed in randomised paired blocks, as in
 the paper's Sec. 3.4 protocol: speedup = median over blocks of the paired
-ratio t(FP64, k) / t(fmt, k').
+ratio t(FP64, k) / t(fmt, k').  The blocks also hold the paper's aggregate
+over a set of matrices (ten square matrices of sizes 400..1138, rank 40 in
+FP64 and 41 compensated, 8192 queries each, one lrc_apply_batched call).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-  python bench.py --case {apply,tt,round,fro,eta_matrix,eta_tt,eta_dense,gather,peaks} ...
+  python bench.py --case {apply,tt,round,fro,eta_matrix,eta_tt,eta_dense,gather,peaks,batched} ...
 """
 from __future__ import annotations
 
@@ -113,7 +115,11 @@ def rank_set(fmt: str) -> str:
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from
 # one ncu capture of the call type's kernels as they stand; an entry is
 # removed when its kernels change.
-MEASURED_TRAFFIC: dict = {}
+MEASURED_TRAFFIC: dict = {
+    # eta_matrix@sweep (lrc_lowrank_eta, m = n = 16384, k' = 272, binary16):
+    # all six kernels of one call, profiles/eta_matrix_lowrank_16384x16384_k272.md
+    "eta_matrix@sweep": 1_858_600_000,
+}
 
 
 def work_round(rows, cols, ld, fmt):
@@ -346,6 +352,57 @@ class TTWL:
             self.results[f"eta_{s}"] = res["eta"]
 
 
+class BatchWL:
+    """The paper's aggregate over a set of matrices (Sec. 4.4): ten square
+    matrices of seeded sizes in [400, 1138] (the sizes of the paper's
+    matrices; sigma_j = j^-1.5 stands in for their spectra), rank 40 in FP64
+    and 41 compensated, 8192 queries each, applied by one lrc_apply_batched
+    call per format."""
+    name = "batch10"
+    COUNT, B, K, KP = 10, 8192, 40, 41
+
+    def __init__(self, lrc, torch, dev):
+        rng = np.random.default_rng(4242)
+        self.sizes = [int(v) for v in rng.integers(400, 1139, size=self.COUNT)]
+        ld = lrc.lrc_packed_ld
+        self.ops = {f: [] for f in ("f64",) + STORE + ("bf16",)}
+        self.Y = {f: [] for f in ("f64",) + COMP + ("bf16",)}
+        for p, n in enumerate(self.sizes):
+            q1 = W.orthonormal_columns(n, self.KP, 50_000 + p)
+            q2 = W.orthonormal_columns(n, self.KP, 60_000 + p)
+            sig = W.spectrum("alg1.5", self.KP)
+            X = torch.from_numpy(W.gaussian((self.B, n), 70_000 + p)).to(dev)
+            Q1, Q2t = torch.from_numpy(q1).to(dev), torch.from_numpy(np.ascontiguousarray(q2.T)).to(dev)
+            s = torch.from_numpy(sig[None, :].copy()).to(dev)
+            for f in ("f64",) + STORE + ("bf16",):
+                k = self.K if f == "f64" else self.KP
+                dt = lrc.storage_dtype(f)
+                U = torch.empty((n, ld(k)), dtype=dt, device=dev)
+                S = torch.empty((1, ld(k)), dtype=dt, device=dev)
+                Vt = torch.empty((k, ld(n)), dtype=dt, device=dev)
+                Xr = torch.empty((self.B, ld(n)), dtype=dt, device=dev)
+                lrc.lrc_round_factors(Q1, n, k, self.KP, U, U.shape[1], f)
+                lrc.lrc_round_factors(s, 1, k, self.KP, S, S.shape[1], f)
+                lrc.lrc_round_factors(Q2t, k, n, n, Vt, Vt.shape[1], f)
+                lrc.lrc_round_factors(X, self.B, n, n, Xr, Xr.shape[1], f)
+                self.ops[f].append((U, S, Vt, Xr))
+            for f in ("f64",) + COMP + ("bf16",):
+                self.Y[f].append(torch.empty((self.B, n), dtype=lrc.output_dtype(f), device=dev))
+
+    def call(self, lrc, fmt):
+        ops = self.ops[store_of(fmt)]
+        k = self.K if fmt == "f64" else self.KP
+        c = self.COUNT
+        lrc.lrc_apply_batched([o[0] for o in ops], [o[1] for o in ops], [o[2] for o in ops], [o[3] for o in ops],
+                              self.Y[fmt], self.sizes, self.sizes, [k] * c, [self.B] * c, fmt)
+
+    def work(self, fmt):
+        k = self.K if fmt == "f64" else self.KP
+        ws = [work_apply(n, n, k, self.B, fmt) for n in self.sizes]
+        w = {"bytes": sum(x["bytes"] for x in ws), "flops": sum(x["flops"] for x in ws), "alu": ALU[fmt]}
+        return w
+
+
 class Step:
     """One pass of the rank-compensated path over every workload."""
 
@@ -442,6 +499,7 @@ class Paired:
 
     def __init__(self, lrc, torch, dev, step):
         self.calls = []       # (workload, method, impl, fn)
+        self.works = {}       # (workload, method) -> algorithmic work of this library's call
         ld = lrc.lrc_packed_ld
         self.keep = []
         for wl in step.mats:
@@ -455,6 +513,9 @@ class Paired:
             Vt64 = d["Q2t"][:k]
             Y64 = torch.empty((b, m), dtype=torch.float64, device=dev)
             self.keep += [U64, S64, Y64]
+            self.works[(wl.name, "f64")] = work_apply(m, n, k, b, "f64")
+            for f in COMP:
+                self.works[(wl.name, f)] = work_apply(m, n, wl.kp[store_of(f)], b, f)
             self.calls.append((wl.name, "f64", "ours", lambda U64=U64, S64=S64, Vt64=Vt64, Y64=Y64, d=d, m=m, n=n,
                                k=k, b=b: lrc.lrc_apply(U64, S64, Vt64, d["X"], Y64, m, n, k, b, "f64")))
             for f in COMP:
@@ -472,6 +533,25 @@ class Paired:
                 self.keep += [Wt, Yt]
                 self.calls.append((wl.name, f, "torch", lambda U=U, S=S, Vt=Vt, X=X, kk=kk, Wt=Wt, Yt=Yt, n=n:
                                    torch_apply(torch, X, Vt, S, U, kk, n, Wt, Yt)))
+        # the paper's ten-matrix aggregate: lrc_apply_batched, and torch.matmul problem by problem
+        self.batch = BatchWL(lrc, torch, dev)
+        bw = self.batch
+        for f in ("f64",) + COMP:
+            self.works[(bw.name, f)] = bw.work(f)
+            self.calls.append((bw.name, f, "ours", lambda f=f: bw.call(lrc, f)))
+        for f in ("f64", "f32", "f16_o16"):
+            kk = bw.K if f == "f64" else bw.KP
+            bufs = []
+            for (U, S, Vt, X), n in zip(bw.ops[store_of(f)], bw.sizes):
+                Wt = torch.empty((bw.B, kk), dtype=U.dtype, device=dev)
+                Yt = torch.empty((bw.B, n), dtype=U.dtype, device=dev)
+                bufs.append((U, S, Vt, X, n, Wt, Yt))
+            self.keep.append(bufs)
+
+            def tb(bufs=bufs, kk=kk):
+                for U, S, Vt, X, n, Wt, Yt in bufs:
+                    torch_apply(torch, X, Vt, S, U, kk, n, Wt, Yt)
+            self.calls.append((bw.name, f, "torch", tb))
         for wl in step.tts:
             cfg = wl.cfg
             c64 = [torch.from_numpy(c).to(dev) for c in wl.host["f64"]]
@@ -484,6 +564,9 @@ class Paired:
                 turn["i"] += 1
                 lrc.tt_reconstruct(c64, cfg.dims, r64, "f64", outs64[turn["i"] % len(outs64)])
             self.calls.append((wl.name, "f64", "ours", tt64))
+            self.works[(wl.name, "f64")] = work_tt(cfg.dims, r64, "f64")
+            for f in COMP:
+                self.works[(wl.name, f)] = work_tt(cfg.dims, cfg.ranks[store_of(f)], f)
             for f in COMP:
                 s = store_of(f)
 
@@ -866,6 +949,10 @@ def run_case(args):
         out = torch.empty(args.count, dtype=lrc.output_dtype(fmt), device=dev)
         call = lambda: lrc.tt_gather(cores, cfg.dims, ranks, fmt, idx, out)  # noqa: E731
         work = work_gather(cfg.dims, ranks, fmt, args.count)
+    elif args.case == "batched":
+        bw = BatchWL(lrc, torch, dev)
+        call = lambda: bw.call(lrc, fmt)  # noqa: E731
+        work = bw.work(fmt)
     elif args.case == "fro":
         a = torch.randn(args.count, dtype=torch.float64, device=dev)
         b2 = torch.randn(args.count, dtype=torch.float64, device=dev)
@@ -915,7 +1002,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--case", choices=["apply", "tt", "fro", "round", "eta_matrix", "eta_tt", "eta_dense",
-                                       "gather", "peaks"], default=None,
+                                       "gather", "peaks", "batched"], default=None,
                     help="time one call type instead of the step (profiling captures)")
     ap.add_argument("--fmt", default="f16")
     ap.add_argument("--m", type=int, default=16384)
@@ -991,9 +1078,11 @@ def main():
     paired = Paired(lrc, torch, dev, step)
     paired.run(torch, 1)                          # warm-up block
     ptimes = paired.run(torch, max(args.blocks, 1))
-    kind_of = {n: "apply" for n in MATRIX_WL}
+    kind_of = {n: "apply" for n in MATRIX_WL + ("batch10",)}
     kind_of.update({n: "tt" for n in TT_WL})
     speed, vs_torch, paired_ms, torch_ms = paired_report(ptimes, kind_of)
+    paired_frac = {f"{kind_of[w]}_{f}@{w}": roofline_time(wk) / (paired_ms[f"{kind_of[w]}_{f}@{w}"] * 1e-3)
+                   for (w, f), wk in paired.works.items()}
     del paired
     torch.cuda.empty_cache()
 
@@ -1101,6 +1190,7 @@ def main():
                                  "per call behind a GPU-side wait; median of paired per-block ratios "
                                  "t(FP64, rank k) / t(fmt, rank k')"),
             "fp64_baseline_ms": fp64_base,
+            "paired_roofline_frac": paired_frac,
             "torch_matmul_ms": torch_ms,
             "speedup_vs_torch_matmul": vs_torch,
             "latency_us_tiny": latency_us,

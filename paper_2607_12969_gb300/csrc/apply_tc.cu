@@ -734,7 +734,7 @@ __device__ __forceinline__ void y_body(const CUtensorMap* tm_u, const CUtensorMa
                         for (int j = 32; j < 64; ++j) v[j] = __float_as_uint(__fmul_rn(__uint_as_float(v[j]), f1));
                     }
                 }
-                if (a.tma_store) {
+                {
                     uint32_t packed[32];
                     if (a.out16 && a.bf16) {
 #pragma unroll
@@ -750,7 +750,7 @@ __device__ __forceinline__ void y_body(const CUtensorMap* tm_u, const CUtensorMa
                     }
                     unsigned char* box = hstage + (size_t)(chunk & (a.ydepth - 1)) * (128 * 128);
                     unsigned char* sb = box + (size_t)g * (32 * 128);
-                    if (chunk >= a.ydepth && issuer) {
+                    if (a.tma_store && chunk >= a.ydepth && issuer) {
                         if (a.ydepth == 2) bulk_wait_read<1>();
                         else bulk_wait_read<0>();
                     }
@@ -761,25 +761,36 @@ __device__ __forceinline__ void y_body(const CUtensorMap* tm_u, const CUtensorMa
                         *reinterpret_cast<uint4*>(sb + off) =
                             make_uint4(packed[4 * j], packed[4 * j + 1], packed[4 * j + 2], packed[4 * j + 3]);
                     }
-                    fence_proxy_async_smem();
-                    named_bar_sync(2 + half, 128);      // all four slices are written
-                    if (issuer) {
-                        if (col0 < a.m) tma_store_2d(tm_y, (int32_t)col0, (int32_t)row0, box);
-                        bulk_commit();      // one group per chunk, even empty: the staging reuse counts on it
-                    }
-                } else {
-                    const int64_t grow = row0 + r;
-                    if (grow < a.b) {
-                        if (a.out16) {
-                            uint16_t* yrow = static_cast<uint16_t*>(a.Y) + grow * a.m;
-                            for (int j = 0; j < 64; ++j)
-                                if (col0 + j < a.m)
-                                    yrow[col0 + j] = a.bf16 ? to_bf16_bits(__uint_as_float(v[j]))
-                                                            : __half_as_ushort(__float2half_rn(__uint_as_float(v[j])));
-                        } else {
-                            float* yrow = static_cast<float*>(a.Y) + grow * a.m;
-                            for (int j = 0; j < 32; ++j)
-                                if (col0 + j < a.m) yrow[col0 + j] = __uint_as_float(v[j]);
+                    if (a.tma_store) {
+                        fence_proxy_async_smem();
+                        named_bar_sync(2 + half, 128);      // all four slices are written
+                        if (issuer) {
+                            if (col0 < a.m) tma_store_2d(tm_y, (int32_t)col0, (int32_t)row0, box);
+                            bulk_commit();      // one group per chunk, even empty: the staging reuse counts on it
+                        }
+                    } else {
+                        // Rows whose pitch is not a multiple of 16 bytes (no TMA store): the
+                        // warp writes its own 32 staged rows one at a time, lane l the row's
+                        // bytes 4l..4l+3 -- one coalesced 128-byte run per row.
+                        __syncwarp();
+                        const int nvalid = (int)(a.m - col0 < ecols ? a.m - col0 : ecols);   // columns inside Y
+                        for (int rr = 0; rr < 32; ++rr) {
+                            const int64_t grow = row0 + g * 32 + rr;
+                            if (grow >= a.b) break;
+                            const uint32_t w = *reinterpret_cast<const uint32_t*>(
+                                sb + rr * 128 + (((lane >> 2) ^ (rr & 7)) * 16) + (lane & 3) * 4);
+                            if (a.out16) {
+                                uint16_t* y = static_cast<uint16_t*>(a.Y) + grow * a.m + col0 + 2 * lane;
+                                const int c = 2 * lane;
+                                if (c + 1 < nvalid && ((reinterpret_cast<uintptr_t>(y) & 3u) == 0)) {
+                                    *reinterpret_cast<uint32_t*>(y) = w;
+                                } else {
+                                    if (c < nvalid) y[0] = (uint16_t)(w & 0xffffu);
+                                    if (c + 1 < nvalid) y[1] = (uint16_t)(w >> 16);
+                                }
+                            } else if (lane < nvalid) {
+                                *(static_cast<uint32_t*>(a.Y) + grow * a.m + col0 + lane) = w;
+                            }
                         }
                     }
                 }
