@@ -7,7 +7,9 @@ code: the only module both use is ``workloads`` (seeded inputs, no method
 arithmetic).
 
 Every function cites the passage of the paper it follows; the C source
-(``oracle.c``) holds the arithmetic.  Inputs that the GPU sees in FP32/FP16
+(``oracle.c``) holds the arithmetic of the hot path.  The factorization side
+(TT-SVD, left-orthogonalization) takes LAPACK's SVD and QR, through numpy, as
+the primitive of each step of the paper's algorithm.  Inputs that the GPU sees in FP32/FP16
 are given to the oracle as the oracle's own rounding of the FP64 data,
 decoded back to FP64 exactly, so both sides evaluate the same rounded
 factors.
@@ -278,3 +280,51 @@ def tt_storage_bits(dims: Sequence[int], ranks: Sequence[int], fmt: str) -> floa
 def tt_storage_ratio(dims, ranks_base, ranks_aug, fmt: str) -> float:
     """Exact TT storage ratio from the core dimensions (Sec. 6.1)."""
     return tt_storage_bits(dims, ranks_aug, fmt) / tt_storage_bits(dims, ranks_base, "f64")
+
+
+# --------------------------------------------------------------------------
+# factorization side: TT-SVD and left-orthogonalization (Sec. 5, Sec. 6.1)
+# --------------------------------------------------------------------------
+
+def tt_svd(T: np.ndarray, ranks: Sequence[int]):
+    """TT-SVD (Sec. 5: the sequential truncated SVDs of Oseledets' algorithm;
+    Alg. alg:tt_compensation steps 1-2).  The remainder C starts as T; at bond
+    l it is reshaped to (r_{l-1} n_l) x (rest), its SVD U s V^T is truncated
+    to r_l = min(ranks[l], len(s)) terms, core l is U[:, :r_l] and the next
+    remainder is diag(s[:r_l]) V^T[:r_l].  The library SVD (LAPACK) is the
+    step's primitive.  Returns (cores, delta2): delta2[l - 1] = sum of the
+    discarded s_j^2 at bond l (summed from the smallest up).  The error of
+    the result is ||T - T_R||_F^2 = sum(delta2) (the discarded parts of the
+    successive steps are orthogonal)."""
+    import math
+    A = _f64(T)
+    dims = A.shape
+    d = len(dims)
+    C = A.reshape(-1)
+    rp = 1
+    cores, delta2 = [], []
+    for l in range(d - 1):
+        C = C.reshape(rp * dims[l], -1)
+        U, s, Vt = np.linalg.svd(C, full_matrices=False)
+        r = min(int(ranks[l + 1]), s.size)
+        delta2.append(math.fsum((s[r:] ** 2)[::-1]))
+        cores.append(np.ascontiguousarray(U[:, :r].reshape(rp, dims[l], r)))
+        C = s[:r, None] * Vt[:r]
+        rp = r
+    cores.append(np.ascontiguousarray(C.reshape(rp, dims[-1], 1)))
+    return cores, delta2
+
+
+def tt_left_orthogonalize(cores: Sequence[np.ndarray]):
+    """Left-orthogonal gauge (Sec. 6.1): for l = 1..d-1 the unfolding
+    (r_{l-1} n_l) x r_l of core l is factored Q R (LAPACK QR), core l becomes
+    Q and R multiplies core l + 1 from the left.  The tensor is unchanged."""
+    cs = [_f64(c).copy() for c in cores]
+    for l in range(len(cs) - 1):
+        r0, n, r1 = cs[l].shape
+        Q, R = np.linalg.qr(cs[l].reshape(r0 * n, r1))
+        k = Q.shape[1]
+        cs[l] = np.ascontiguousarray(Q.reshape(r0, n, k))
+        nxt = cs[l + 1]
+        cs[l + 1] = np.ascontiguousarray((R @ nxt.reshape(nxt.shape[0], -1)).reshape(k, nxt.shape[1], nxt.shape[2]))
+    return cs

@@ -287,3 +287,20 @@ def sample_indices(count: int, total: int, seed: int) -> np.ndarray:
     if count >= total:
         return np.arange(total, dtype=np.int64)
     return np.sort(rng.choice(total, size=count, replace=False)).astype(np.int64)
+
+
+# ---------------------------------------------------------------------------
+# the paper's closed-form three-way tensors (Sec. 7.2), C order, 1-based i, j, k
+# ---------------------------------------------------------------------------
+
+def hilbert_3d(n: int = 100) -> np.ndarray:
+    """T(i, j, k) = 1 / (i + j + k - 2)."""
+    i = np.arange(1, n + 1, dtype=np.float64)
+    return 1.0 / (i[:, None, None] + i[None, :, None] + i[None, None, :] - 2.0)
+
+
+def decay_3d(n: int = 60) -> np.ndarray:
+    """T(i, j, k) = 1 / (1 + |i - j| + |j - k| + |i - k|)."""
+    i = np.arange(1, n + 1, dtype=np.float64)
+    a, b, c = i[:, None, None], i[None, :, None], i[None, None, :]
+    return 1.0 / (1.0 + np.abs(a - b) + np.abs(b - c) + np.abs(a - c))
