@@ -375,6 +375,53 @@ LRC_API lrc_status lrc_device_status(lrc_stream_t stream);
 LRC_API lrc_status lrc_selftest_wait_timeout(int64_t limit_ns, lrc_stream_t stream);
 
 /*
+ * lrc_tt_svd -- TT-SVD of a dense tensor on the GPU (Sec. 5: Oseledets'
+ * sequential truncated SVDs; Alg. alg:tt_compensation steps 1-2, the FP64
+ * baseline T_R and the augmented T_{R+delta}), in binary64.
+ *
+ *   T       device, the dense tensor, prod(dims) binary64 entries, C order
+ *           (i_1 slowest), 8-byte aligned; not modified
+ *   dims, ranks, d  as in tt_reconstruct: the ranks to truncate to, with
+ *           ranks[0] = ranks[d] = 1 and every ranks[l] at most the smaller
+ *           side of unfolding l, min(ranks[l-1] dims[l-1], dims[l] ... dims[d-1]),
+ *           which must itself be at most 1024
+ *   cores   HOST array of d DEVICE pointers, core l receives
+ *           ranks[l] x dims[l] x ranks[l+1] binary64 values (C order)
+ *   delta2_out   host, may be NULL: d - 1 values, the sum of the discarded
+ *           squared singular values at each bond; ||T - T_R||_F^2 is their sum
+ *           (the discarded parts of the sequential steps are orthogonal)
+ *   spectra_out  host, may be NULL: every singular value of every unfolding
+ *           remainder, bond after bond, each bond's in descending order
+ *           (min(rows, cols) values per bond) -- the local spectra of the
+ *           certificate's diagnostics
+ *
+ * Each bond's SVD is a one-sided Jacobi SVD of the tall side of the
+ * remainder (column pairs rotated until orthogonal to sqrt(L) units of
+ * roundoff; at most 40 sweeps, else LRC_ERR_UNSUPPORTED), so small singular
+ * values are accurate to about u times the largest.  The cores 1..d-1 are
+ * left-orthonormal.  d = 2 is the truncated SVD of a dims[0] x dims[1]
+ * matrix: cores[0] = U_k, cores[1] = diag(s_k) V_k^T, spectra_out = all
+ * singular values.  Scratch: the stream's library workspace, about
+ * 16 prod(dims) bytes.  SYNCHRONISES `stream`.
+ */
+LRC_API lrc_status lrc_tt_svd(const double* T, const int64_t* dims, const int64_t* ranks, int d,
+                              double* const* cores, double* delta2_out, double* spectra_out,
+                              lrc_stream_t stream);
+
+/*
+ * lrc_tt_left_orthogonalize -- the left-orthogonal gauge (Sec. 6.1), in
+ * place, binary64: for l = 1..d-1 the unfolding (r_{l-1} n_l) x r_l of core
+ * l is factored Q R' (Q with orthonormal columns, from a one-sided Jacobi
+ * SVD: Q = U, R' = diag(s) V^T), core l becomes Q and core l + 1 becomes
+ * R' core l + 1.  The tensor is unchanged (to rounding) and ||G_d||_F =
+ * ||T||_F.  Requires r_l <= r_{l-1} n_l and r_l <= 1024; a zero singular
+ * value leaves a zero column in Q (still exact).  cores: HOST array of d
+ * DEVICE pointers (binary64, layout of tt_reconstruct).  SYNCHRONISES `stream`.
+ */
+LRC_API lrc_status lrc_tt_left_orthogonalize(double* const* cores, const int64_t* dims, const int64_t* ranks, int d,
+                                             lrc_stream_t stream);
+
+/*
  * lrc_probe_peak -- measured rate of one arithmetic unit of this GPU, the
  * denominator of the roofline fractions of the binary32 and binary64 paths
  * (their products run on the CUDA cores' FMA units or on the binary64 tensor

@@ -84,6 +84,10 @@ def load() -> ctypes.CDLL:
     L.lrc_shutdown.restype = i32
     L.lrc_device_status.argtypes = [vp]
     L.lrc_device_status.restype = i32
+    L.lrc_tt_svd.argtypes = [vp, vp, vp, i32, vp, vp, vp, vp]
+    L.lrc_tt_svd.restype = i32
+    L.lrc_tt_left_orthogonalize.argtypes = [vp, vp, vp, i32, vp]
+    L.lrc_tt_left_orthogonalize.restype = i32
     L.lrc_probe_peak.argtypes = [i32, i64, vp, vp]
     L.lrc_probe_peak.restype = i32
     L.lrc_selftest_wait_timeout.argtypes = [i64, vp]
@@ -393,6 +397,51 @@ def lrc_device_status(stream=None) -> int:
     """Synchronises the stream; returns the lrc_status (0, or -6 if a bounded
     device wait gave up since the last call).  Does not raise."""
     return int(load().lrc_device_status(_stream(stream)))
+
+
+def lrc_tt_svd(T, dims: Sequence[int], ranks: Sequence[int], cores: Sequence, stream=None,
+               want_spectra: bool = False):
+    """TT-SVD of the dense binary64 tensor T into `cores` (preallocated
+    binary64 tensors of shapes ranks[l] x dims[l] x ranks[l+1]).  Returns
+    (delta2, spectra): the discarded squared singular values per bond and,
+    if asked, every bond's singular values (a list of arrays)."""
+    import numpy as np
+    import torch
+    d = len(dims)
+    if len(cores) != d or len(ranks) != d + 1:
+        raise ValueError("cores needs d entries and ranks d + 1")
+    _need(T, "T", torch.float64, np_prod(dims), stream=stream)
+    _need_cores(cores, dims, ranks, "f64", stream)
+    sizes, rest = [], np_prod(dims)
+    for l in range(d - 1):
+        rest //= int(dims[l])
+        sizes.append(min(int(ranks[l]) * int(dims[l]), rest))
+    delta2 = (ctypes.c_double * max(d - 1, 1))()
+    spec = (ctypes.c_double * max(sum(sizes), 1))() if want_spectra else None
+    ptrs = (ctypes.c_void_p * d)(*[c.data_ptr() for c in cores])
+    dd = (ctypes.c_int64 * d)(*[int(x) for x in dims])
+    rr = (ctypes.c_int64 * (d + 1))(*[int(x) for x in ranks])
+    _check(load().lrc_tt_svd(_ptr(T), ctypes.cast(dd, ctypes.c_void_p), ctypes.cast(rr, ctypes.c_void_p), d,
+                             ctypes.cast(ptrs, ctypes.c_void_p), ctypes.cast(delta2, ctypes.c_void_p),
+                             ctypes.cast(spec, ctypes.c_void_p) if spec is not None else None, _stream(stream)))
+    spectra = None
+    if spec is not None:
+        flat, spectra, o = np.array(spec[:]), [], 0
+        for n in sizes:
+            spectra.append(flat[o:o + n])
+            o += n
+    return [delta2[i] for i in range(d - 1)], spectra
+
+
+def lrc_tt_left_orthogonalize(cores: Sequence, dims: Sequence[int], ranks: Sequence[int], stream=None) -> None:
+    """Left-orthogonal gauge of binary64 cores, in place."""
+    d = len(cores)
+    _need_cores(cores, dims, ranks, "f64", stream)
+    ptrs = (ctypes.c_void_p * d)(*[c.data_ptr() for c in cores])
+    dd = (ctypes.c_int64 * d)(*[int(x) for x in dims])
+    rr = (ctypes.c_int64 * (d + 1))(*[int(x) for x in ranks])
+    _check(load().lrc_tt_left_orthogonalize(ctypes.cast(ptrs, ctypes.c_void_p), ctypes.cast(dd, ctypes.c_void_p),
+                                            ctypes.cast(rr, ctypes.c_void_p), d, _stream(stream)))
 
 
 PROBE_KINDS = {"ffma": 0, "ffma2": 1, "dfma": 2, "dmma": 3}

@@ -444,6 +444,48 @@ lrc_status lrc_selftest_wait_timeout(int64_t limit_ns, lrc_stream_t stream) {
     return launch_wait_timeout_probe(limit_ns, as_stream(stream));
 }
 
+lrc_status lrc_tt_svd(const double* T, const int64_t* dims, const int64_t* ranks, int d, double* const* cores,
+                      double* delta2_out, double* spectra_out, lrc_stream_t stream) {
+    TTShape sh;
+    lrc_status st = tt_shape((const void* const*)cores, dims, ranks, d, 8, "cores", &sh);
+    if (st != LRC_OK) return st;
+    if (!T) return invalid("null T");
+    if ((reinterpret_cast<uintptr_t>(T) & 7u) != 0) return misaligned("T");
+    int64_t rest = sh.numel;
+    for (int l = 0; l < d - 1; ++l) {
+        rest /= dims[l];
+        const int64_t rows = ranks[l] * dims[l], p = rows < rest ? rows : rest;
+        if (ranks[l + 1] > p)
+            return invalid("ranks[%d] = %lld exceeds the smaller side (%lld) of unfolding %d", l + 1,
+                           (long long)ranks[l + 1], (long long)p, l + 1);
+        if (p > factor_max_cols()) {
+            set_error("TT-SVD: unfolding %d's smaller side is %lld; at most %d", l + 1, (long long)p,
+                      factor_max_cols());
+            return LRC_ERR_UNSUPPORTED;
+        }
+    }
+    int64_t t;
+    if (!mul_ok(sh.numel, 16, &t)) return invalid("tensor too large");
+    return run_tt_svd(T, sh, cores, delta2_out, spectra_out, as_stream(stream));
+}
+
+lrc_status lrc_tt_left_orthogonalize(double* const* cores, const int64_t* dims, const int64_t* ranks, int d,
+                                     lrc_stream_t stream) {
+    TTShape sh;
+    lrc_status st = tt_shape((const void* const*)cores, dims, ranks, d, 8, "cores", &sh);
+    if (st != LRC_OK) return st;
+    for (int l = 0; l < d - 1; ++l) {
+        if (ranks[l + 1] > ranks[l] * dims[l])
+            return invalid("ranks[%d] = %lld exceeds ranks[%d] * dims[%d] = %lld", l + 1, (long long)ranks[l + 1], l,
+                           l, (long long)(ranks[l] * dims[l]));
+        if (ranks[l + 1] > factor_max_cols()) {
+            set_error("left-orthogonalization: rank %lld above %d", (long long)ranks[l + 1], factor_max_cols());
+            return LRC_ERR_UNSUPPORTED;
+        }
+    }
+    return run_tt_left_orthogonalize(sh, cores, as_stream(stream));
+}
+
 lrc_status lrc_probe_peak(int kind, int64_t iters, double* flops_out, lrc_stream_t stream) {
     if (kind < 0 || kind > 3) return invalid("kind must be 0..3");
     if (iters < 1 || iters > (1LL << 30)) return invalid("iters must be in [1, 2^30]");

@@ -227,6 +227,13 @@ lrc_status run_lowrank_eta(const double* U, const double* S, const double* Vt, c
 lrc_status run_tt_eta(const TTShape& sh, const void* const* hats, lrc_fmt fmt, double* eta_out, double* norm_out,
                       cudaStream_t s);
 
+// Factorization side (factor.cu), binary64; synchronise s.  The caller has
+// checked the shapes (every rank at most the smaller side of its unfolding).
+int factor_max_cols();
+lrc_status run_tt_svd(const double* T, const TTShape& sh, double* const* cores, double* delta2_out,
+                      double* spectra_out, cudaStream_t s);
+lrc_status run_tt_left_orthogonalize(const TTShape& sh, double* const* cores, cudaStream_t s);
+
 // Measured rate of one arithmetic unit (peak_probe.cu); synchronises s.
 lrc_status run_probe_peak(int kind, int64_t iters, double* flops_out, cudaStream_t s);
 
