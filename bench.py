@@ -33,7 +33,7 @@ over a set of matrices (ten square matrices of sizes 400..1138, rank 40 in
 FP64 and 41 compensated, 8192 queries each, one lrc_apply_batched call).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-  python bench.py --case {apply,tt,round,fro,eta_matrix,eta_tt,eta_dense,gather,peaks,batched} ...
+  python bench.py --case {apply,tt,round,fro,eta_matrix,eta_tt,eta_dense,gather,peaks,batched,ttsvd} ...
 """
 from __future__ import annotations
 
@@ -949,6 +949,24 @@ def run_case(args):
         out = torch.empty(args.count, dtype=lrc.output_dtype(fmt), device=dev)
         call = lambda: lrc.tt_gather(cores, cfg.dims, ranks, fmt, idx, out)  # noqa: E731
         work = work_gather(cfg.dims, ranks, fmt, args.count)
+    elif args.case == "ttsvd":
+        # TT-SVD of a dense tensor: the paper's hilbert_3d (--tt hilbert) or
+        # decay_3d (--tt decay) at uniform rank --k, or a TT workload's dense
+        # FP64 tensor at its binary16 rank set (--tt tt3 ...)
+        if args.tt in ("hilbert", "decay"):
+            T = W.hilbert_3d(100) if args.tt == "hilbert" else W.decay_3d(60)
+            dims, ranks = T.shape, (1, args.k, args.k, 1)
+            Td = torch.from_numpy(T.reshape(-1)).to(dev)
+        else:
+            cfg = W.TT_CONFIGS[args.tt]
+            dims, ranks = cfg.dims, cfg.ranks["f16"]
+            c64 = [torch.from_numpy(c).to(dev) for c in W.tt_cores(cfg, "f16")]
+            Td = torch.empty(int(np.prod(dims)), dtype=torch.float64, device=dev)
+            lrc.tt_reconstruct(c64, dims, ranks, "f64", Td)
+        outc = [torch.empty((ranks[l], dims[l], ranks[l + 1]), dtype=torch.float64, device=dev)
+                for l in range(len(dims))]
+        call = lambda: lrc.lrc_tt_svd(Td, dims, ranks, outc)  # noqa: E731
+        work = {"bytes": Td.numel() * 8, "flops": 0, "alu": None}
     elif args.case == "batched":
         bw = BatchWL(lrc, torch, dev)
         call = lambda: bw.call(lrc, fmt)  # noqa: E731
@@ -1002,7 +1020,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--case", choices=["apply", "tt", "fro", "round", "eta_matrix", "eta_tt", "eta_dense",
-                                       "gather", "peaks", "batched"], default=None,
+                                       "gather", "peaks", "batched", "ttsvd"], default=None,
                     help="time one call type instead of the step (profiling captures)")
     ap.add_argument("--fmt", default="f16")
     ap.add_argument("--m", type=int, default=16384)

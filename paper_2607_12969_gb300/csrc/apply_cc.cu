@@ -507,7 +507,9 @@ lrc_status launch_apply_f32(const float* U, const float* S, const float* Vt, con
     int64_t splits = (2 * resident + tiles1 - 1) / tiles1;
     const int64_t min_splits = (n + kMaxChunk - 1) / kMaxChunk;
     if (splits < min_splits) splits = min_splits;
-    const int64_t max_splits = (n + 255) / 256;
+    // at least 64 terms per partial: a product with few tiles (small b and k)
+    // gets enough CTAs that no CTA walks a long serial chain of K slabs
+    const int64_t max_splits = (n + 63) / 64;
     if (splits > max_splits) splits = max_splits > min_splits ? max_splits : min_splits;
     if (splits < 1) splits = 1;
     // the product rounds each split's K range up to its 16-wide slabs
