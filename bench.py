@@ -889,8 +889,19 @@ def run_case(args):
         mk = lambda a: lrc.round_matrix(torch.from_numpy(a if a.ndim == 2 else a[None, :]).to(dev), fmt)  # noqa: E731
         U, S, V, Xd = mk(f.U), mk(f.s), mk(f.Vt), mk(X)
         Y = torch.empty((b, m), dtype=lrc.output_dtype(fmt), device=dev)
-        call = lambda: lrc.lrc_apply(U, S, V, Xd, Y, m, n, k, b, fmt)  # noqa: E731
         work = work_apply(m, n, k, b, fmt)
+        # --rotate: copies of every operand and output, used in turn, so that
+        # no call finds its inputs in L2 (cold, HBM-judged); else every call
+        # after the first reads them from L2 when they fit (warm)
+        sets = [(U, S, V, Xd, Y)]
+        if args.rotate:
+            sets += [tuple(t.clone() for t in sets[0]) for _ in range(rotation(work["bytes"]) - 1)]
+        turn = {"i": 0}
+
+        def call():
+            turn["i"] += 1
+            Uc, Sc, Vc, Xc, Yc = sets[turn["i"] % len(sets)]
+            lrc.lrc_apply(Uc, Sc, Vc, Xc, Yc, m, n, k, b, fmt)
     elif args.case == "tt":
         cfg = W.TT_CONFIGS[args.tt]
         cores = [torch.from_numpy(c).to(dev).to(lrc.storage_dtype(fmt)).contiguous() for c in W.tt_cores(cfg, base)]
@@ -1028,7 +1039,8 @@ def main():
     ap.add_argument("--b", type=int, default=2048)
     ap.add_argument("--k", type=int, default=144)
     ap.add_argument("--tt", default="tt3")
-    ap.add_argument("--rotate", action="store_true", help="TT case: rotate outputs over more than 2 x L2")
+    ap.add_argument("--rotate", action="store_true",
+                    help="TT case: rotate outputs, apply case: rotate operands and outputs, over more than 2 x L2")
     ap.add_argument("--count", type=int, default=1 << 26)
     ap.add_argument("--reps", type=int, default=3)
     args = ap.parse_args()

@@ -7,20 +7,25 @@
 // is set by how many bytes each SM has in flight.  Every operand tile is
 // therefore one set of TMA copies issued at the start of its CTA (2-D boxes,
 // zero-filled outside the arrays, so the arithmetic needs no bounds tests).
-// Three launches on the caller's stream:
+// Two launches on the caller's stream, chained by programmatic dependent
+// launch:
 //   skinny_w1_kernel  grid (n-chunk, block of 32 rows of V^T): the chunk of X
 //                     (at most 16 rows) and of the 32 rows of V^T land in
 //                     shared memory; each warp takes 4 rows of V^T, each lane
 //                     keeps the b partial dot products of every row over its
 //                     16-byte columns, a recursive halving adds them across
-//                     the warp.  One partial W per chunk.
-//   skinny_w2_kernel  W = (sum of the chunks' partials) diag(s), a warp per
-//                     entry; for binary16 output W is rounded to binary16 (the
-//                     method-precision workspace of Sec. 3.4).
+//                     the warp.  One partial W per chunk.  The last CTA of a
+//                     row block to finish (an arrival counter) adds the
+//                     chunks' partials in chunk order, scales by diag(s) and
+//                     writes that block of W; for binary16 output W is
+//                     rounded to binary16 (the method-precision workspace of
+//                     Sec. 3.4).  The CTAs let the second kernel start as
+//                     soon as their copies are issued.
 //   skinny_y_kernel   a CTA per 64 rows of U (32 for binary64): the rows are
-//                     requested before the wait for the previous kernel, W
-//                     (b x k) follows as one bulk copy; groups of 8 lanes
-//                     take 4 rows (2) each, a lane every 8th column.
+//                     requested at once, so they stream while the first
+//                     kernel still runs; after the wait for it W (b x k)
+//                     follows as one bulk copy; groups of 8 lanes take 4
+//                     rows (2) each, a lane every 8th column.
 // Arithmetic: binary64 FMAs for binary64, binary32 FMAs otherwise (binary16
 // factors widened exactly; Sec. 3.4: FP16 products accumulate in FP32).  The
 // summation order is fixed: results are reproducible on a device.
@@ -130,8 +135,11 @@ __device__ __forceinline__ void store_out(double* p, double v) { *p = v; }
 __device__ __forceinline__ void store_out(float* p, float v) { *p = v; }
 __device__ __forceinline__ void store_out(__half* p, float v) { *p = __float2half_rn(v); }
 
+// The dynamic shared-memory base rounded up to 128 bytes by an offset (not
+// through an integer), so that the compiler still sees a shared-memory
+// pointer and emits shared loads rather than generic ones.
 __device__ __forceinline__ unsigned char* align128(unsigned char* p) {
-    return reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 127) & ~static_cast<uintptr_t>(127));
+    return p + ((128u - (tc::smem_u32(p) & 127u)) & 127u);
 }
 
 // Waits for copy group q of the CTA's nq (all threads).  On a timeout thread
@@ -176,6 +184,55 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
 }
 
 // ---------------------------------------------------------------- phase 1
+// The fold of the last CTA of a row block: W[c][j] = s_j * sum over chunks ch
+// of Wp[ch][c][j] for the block's rows j (BR of them) and every query c.
+// Each entry takes G lanes (G = 256 / entries, a power of two, at most 32);
+// lane g adds the chunks of its contiguous G-th of the range in chunk order,
+// with 16 loads in flight, and a butterfly over the G lanes adds the G sums
+// (every lane ends with the same value, in an order fixed by G: the result
+// does not depend on which CTA finished last).
+template <typename T, int BR>
+__device__ __forceinline__ void fold_chunks(const T* __restrict__ Wp, int nchunks, int b, int k, int jb,
+                                            const T* s_blk, int round16, int kv, T* __restrict__ W) {
+    constexpr int kBatch = 16;
+    const int E = BR * b;
+    int G = 1;
+    while (G < 32 && 2 * G * E <= kThreadsS) G *= 2;
+    const int64_t bk = (int64_t)b * k;
+    for (int t = threadIdx.x; t < ((E * G + 31) & ~31); t += kThreadsS) {
+        const int e = t / G, g = t - e * G;
+        const int c = e / BR, j = jb + (e - c * BR);
+        const bool live = e < E && j < k;
+        const int ch0 = (int)((int64_t)nchunks * g / G), ch1 = (int)((int64_t)nchunks * (g + 1) / G);
+        const T* src = Wp + (int64_t)c * k + j;
+        T sum = T(0);
+        if (live) {
+            for (int ch = ch0; ch < ch1; ch += kBatch) {
+                T v[kBatch];
+#pragma unroll
+                for (int i = 0; i < kBatch; ++i) v[i] = (ch + i < ch1) ? __ldcg(src + (ch + i) * bk) : T(0);
+#pragma unroll
+                for (int i = 0; i < kBatch; ++i) sum += v[i];
+            }
+        }
+        for (int o = G / 2; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+        if (live && g == 0) {
+            sum *= s_blk[j - jb];
+            if (round16) sum = (T)__half2float(__float2half_rn((float)sum));
+            W[(int64_t)c * kv + j] = sum;
+        }
+    }
+}
+
+// Arrival at a counter: release of this thread's (and, after a CTA barrier,
+// the CTA's) earlier writes, acquire of the writes released by the earlier
+// arrivals.
+__device__ __forceinline__ unsigned int arrive_acq_rel(unsigned int* p) {
+    unsigned int old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(p) : "memory");
+    return old;
+}
+
 // Shared memory: [X boxes: nbox x B x kBox][V^T boxes: nbox x 8 RW x kBox]
 // [a barrier per box pair][abort flag]; column i of the chunk is box i / kBox,
 // offset i % kBox.  The boxes are multiplied in order as they land.  RW rows
@@ -183,7 +240,8 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
 template <typename TS, typename T, int B, int RW>
 __global__ void __launch_bounds__(kThreadsS, 2)
 skinny_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_v, int k, int b,
-                 int L, T* __restrict__ Wp) {
+                 int L, T* __restrict__ Wp, unsigned int* __restrict__ cnt, const TS* __restrict__ S, int kv,
+                 int round16, T* __restrict__ W) {
     constexpr int EV = EVof<TS>::v;
     constexpr int BR = kWarps * RW;              // rows of V^T per CTA
     extern __shared__ unsigned char smem_raw[];
@@ -197,6 +255,10 @@ skinny_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
     const int64_t chunk = blockIdx.x;
     const int32_t i0 = (int32_t)(chunk * L);
     const int jb = (int)blockIdx.y * BR;
+    __shared__ int last_cta;
+    __shared__ T s_blk[BR];          // s_j of the block's rows, for the fold
+    tc::pdl_wait();                  // X, V^T, s and the workspace are the previous kernels'
+    if (threadIdx.x < BR) s_blk[threadIdx.x] = jb + (int)threadIdx.x < k ? to_t<T>(S[jb + threadIdx.x]) : T(0);
     if (threadIdx.x == 0) {
         for (int q = 0; q < nbox; ++q) tc::mbar_init(&bar[q], 1);
         *abort = 0;
@@ -207,6 +269,7 @@ skinny_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
             tc::tma_load_2d(xs + (size_t)q * B * kBox, &tm_x, i0 + q * kBox, 0, &bar[q]);
         }
     }
+    tc::pdl_trigger();               // the second product streams U meanwhile
     __syncthreads();
     const int jl = warp * RW;                 // first local row of the warp
     T acc[RW * B];                            // acc[r * B + c]: row jl + r, query c
@@ -231,7 +294,6 @@ skinny_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
             }
         }
     }
-    tc::pdl_trigger();
     constexpr int N = RW * B;
     halving_sum<T, N, 32>(acc, lane);
     if (halving_writer<N, 32>(lane)) {
@@ -243,48 +305,39 @@ skinny_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
             if (c < b && j < k) Wp[(chunk * b + c) * k + j] = acc[t];
         }
     }
-}
-
-// ---------------------------------------------------------------- phase 1b
-// A warp per entry of W ([b][kv], zero in the columns k..kv-1): lane l adds
-// chunks l, l + 32, ... in order, a fixed butterfly adds the lane sums (the
-// same order on every run).
-template <typename TS, typename T>
-__global__ void __launch_bounds__(256)
-skinny_w2_kernel(const T* __restrict__ Wp, int nchunks, int b, int k, int kv, const TS* __restrict__ S, int round16,
-                 T* __restrict__ W) {
-    tc::pdl_wait();                  // partials of the phase-1 grid
-    tc::pdl_trigger();
-    const int lane = threadIdx.x & 31;
-    const int64_t e = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    if (e >= (int64_t)b * kv) return;
-    const int c = (int)(e / kv), j = (int)(e - (int64_t)c * kv);
-    T acc = T(0);
-    if (j < k) {
-        const int64_t bk = (int64_t)b * k;
-        for (int ch = lane; ch < nchunks; ch += 32) acc += Wp[(int64_t)ch * bk + (int64_t)c * k + j];
-        acc = warp_sum(acc);
-        acc *= to_t<T>(S[j]);
-        if (round16) acc = (T)__half2float(__float2half_rn((float)acc));
-    }
-    if (lane == 0) W[e] = acc;
+    // the last CTA of this row block adds the partials of every chunk
+    __syncthreads();
+    if (threadIdx.x == 0) last_cta = arrive_acq_rel(&cnt[blockIdx.y]) == gridDim.x - 1;
+    __syncthreads();
+    if (!last_cta) return;
+    fold_chunks<T, BR>(Wp, (int)gridDim.x, b, k, jb, s_blk, round16, kv, W);
+    if (blockIdx.y == gridDim.y - 1)             // the zero columns k .. kv-1 of W
+        for (int e = threadIdx.x; e < b * (kv - k); e += kThreadsS) {
+            const int c = e / (kv - k);
+            W[(int64_t)c * kv + k + (e - c * (kv - k))] = T(0);
+        }
+    if (threadIdx.x == 0) cnt[blockIdx.y] = 0u;
 }
 
 // ---------------------------------------------------------------- phase 2
-// A CTA of kYWarps warps owns 16 RPG rows of U: each warp's four groups of 8
-// lanes take RPG rows each, and a lane covers every 8th 16-byte column of
-// its rows (a short reduction: the rank is only a few hundred).  Shared
-// memory: [U: nkb boxes of 16 RPG rows x kbw][W: B x kv][barrier of U]
-// [barrier of W][abort flag]; column j of U is box j / kbw, offset j % kbw;
-// kv = nkb * kbw.
-constexpr int kYWarps = 4;
-constexpr int kYGroup = 8;
-template <typename TS, typename T, typename TOut, int B, int RPG>
-__global__ void __launch_bounds__(32 * kYWarps)
+// A CTA owns 16 RPG rows of U, in groups of G lanes (G = 8, or 32 for at
+// most 4 queries, where the work per row is short and a longer reduction
+// across lanes costs less than a longer loop): each group takes RPG rows, a
+// lane covers every G-th 16-byte column of its rows (the rank is only a few
+// hundred); G / 2 warps.  Shared memory: [U: nkb boxes of 16 RPG rows x kbw]
+// [W: B x kv][barrier of U][barrier of W][abort flag]; column j of U is box
+// j / kbw, offset j % kbw; kv = nkb * kbw.  One thread waits for the copies
+// (the CTA may be resident while the first kernel still runs: the other
+// warps sleep at the CTA barrier instead of polling).
+template <int G>
+constexpr int y_warps() { return G / 2; }
+template <typename TS, typename T, typename TOut, int B, int RPG, int G>
+__global__ void __launch_bounds__(32 * y_warps<G>())
 skinny_y_kernel(const __grid_constant__ CUtensorMap tm_u, const T* __restrict__ W, int64_t m, int b, int nkb,
-                int kbw, TOut* __restrict__ Y) {
+                int kbw, unsigned int* __restrict__ cnt, int ncnt, TOut* __restrict__ Y) {
     constexpr int EV = EVof<TS>::v;
-    constexpr int RC = kYWarps * (32 / kYGroup) * RPG;     // rows of the CTA
+    constexpr int NT = 32 * y_warps<G>();
+    constexpr int RC = y_warps<G>() * (32 / G) * RPG;       // rows of the CTA (16 RPG)
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = align128(smem_raw);
     const int kv = nkb * kbw;
@@ -295,6 +348,8 @@ skinny_y_kernel(const __grid_constant__ CUtensorMap tm_u, const T* __restrict__ 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t rb = (int64_t)blockIdx.x * RC;
     const uint32_t w_bytes = (uint32_t)((size_t)b * kv * sizeof(T));
+    // rows b..B-1 of W are zero (disjoint from the bulk copy of rows 0..b-1)
+    for (int e = b * kv + threadIdx.x; e < B * kv; e += NT) ws[e] = T(0);
     if (threadIdx.x == 0) {
         tc::mbar_init(&bar[0], 1);
         tc::mbar_init(&bar[1], 1);
@@ -303,22 +358,31 @@ skinny_y_kernel(const __grid_constant__ CUtensorMap tm_u, const T* __restrict__ 
         tc::mbar_arrive_expect_tx(&bar[0], (uint32_t)(nkb * RC * kbw * (int)sizeof(TS)));
         for (int q = 0; q < nkb; ++q)
             tc::tma_load_2d(us + (size_t)q * RC * kbw, &tm_u, q * kbw, (int32_t)rb, &bar[0]);
-        tc::pdl_wait();              // W of the reduction kernel
+        tc::pdl_wait();              // W of the first kernel
+        // leave the first kernel's counters at zero for the next call, also
+        // after an aborted first kernel whose CTAs did not all arrive
+        if (blockIdx.x == 0)
+            for (int i = 0; i < ncnt; ++i) cnt[i] = 0u;
         tc::mbar_arrive_expect_tx(&bar[1], w_bytes);
         bulk_load(ws, W, w_bytes, &bar[1]);
+        if (!(tc::mbar_wait(&bar[1], 0, abort, &g_err_skinny, 2u) &&
+              tc::mbar_wait(&bar[0], 0, abort, &g_err_skinny, 2u))) {
+            // no copy may still be landing when the CTA exits
+            volatile int no_abort = 0;
+            for (int i = 0; i < 2; ++i) tc::mbar_wait(&bar[i], 0, &no_abort, &g_err_skinny, 2u, 100000000ull);
+            *abort = 1;
+        }
     }
-    // rows b..B-1 of W are zero
-    for (int e = b * kv + threadIdx.x; e < B * kv; e += 32 * kYWarps) ws[e] = T(0);
+    tc::pdl_trigger();               // the next call's first kernel may set up
     __syncthreads();
-    if (!wait_tiles(bar, 1, 2, abort, 2u)) return;
-    if (!wait_tiles(bar, 0, 2, abort, 2u)) return;
-    const int sl = lane & (kYGroup - 1);
-    const int rl = (warp * (32 / kYGroup) + (lane / kYGroup)) * RPG;
+    if (*abort) return;
+    const int sl = lane & (G - 1);
+    const int rl = (warp * (32 / G) + (lane / G)) * RPG;
     constexpr int N = RPG * B;
     T acc[N];                                    // acc[r * B + c]: row rl + r, query c
 #pragma unroll
     for (int i = 0; i < N; ++i) acc[i] = T(0);
-    for (int v = sl; v < kv / EV; v += kYGroup) {
+    for (int v = sl; v < kv / EV; v += G) {
         const int j = v * EV, q = j / kbw, o = j - q * kbw;
         T uu[RPG][EV];
 #pragma unroll
@@ -333,17 +397,21 @@ skinny_y_kernel(const __grid_constant__ CUtensorMap tm_u, const T* __restrict__ 
                 for (int e = 0; e < EV; ++e) acc[r * B + c] = fma(wv[e], uu[r][e], acc[r * B + c]);
         }
     }
-    halving_sum<T, N, kYGroup>(acc, lane);
+    halving_sum<T, N, G>(acc, lane);
     const int64_t r0 = rb + rl;
-    if (halving_writer<N, kYGroup>(lane)) {
-        const int base = halving_index<N, kYGroup>(lane);
+    if (halving_writer<N, G>(lane)) {
+        const int base = halving_index<N, G>(lane);
 #pragma unroll
-        for (int t = 0; t < (N >= kYGroup ? N / kYGroup : 1); ++t) {
+        for (int t = 0; t < (N >= G ? N / G : 1); ++t) {
             const int idx = base + t, r = idx / B, c = idx - r * B;
             if (c < b && r0 + r < m) store_out(Y + (int64_t)c * m + r0 + r, acc[t]);
         }
     }
 }
+
+// lanes per row group of the second product (binary64 stays at 8: its
+// multiply-adds, not the latency of the chain, bound it)
+constexpr int y_group(int B, int64_t e) { return (B <= 4 && e < 8) ? 32 : 8; }
 
 template <typename TS>
 constexpr int y_rpg() { return sizeof(TS) == 8 ? 2 : 4; }
@@ -389,7 +457,7 @@ SkinnyPlan plan_skinny(int64_t m, int64_t n, int64_t k, int B, int64_t e, int64_
     p.kv = p.nkb * p.kbw;
     p.smem1 = (size_t)(L / kBox) * (B + br) * kBox * e + 8 * (size_t)(L / kBox + 1) + 128;
     // second product: CTAs of 16 RPG rows of U
-    const int64_t rc = (int64_t)kYWarps * (32 / kYGroup) * (e == 8 ? 2 : 4);
+    const int64_t rc = 16 * (int64_t)(e == 8 ? 2 : 4);
     p.yblocks = (m + rc - 1) / rc;
     p.smem3 = (size_t)p.nkb * rc * p.kbw * e + (size_t)B * p.kv * et + 24 + 128;
     return p;
@@ -412,6 +480,8 @@ lrc_status launch_skinny_b(const TS* U, const TS* S, const TS* Vt, const TS* X, 
     void* ws = nullptr;
     lrc_status st = stream_workspace(s, part_bytes + w_bytes, &ws);
     if (st != LRC_OK) return st;
+    unsigned int* cnt = nullptr;
+    if ((st = stream_counters(s, &cnt)) != LRC_OK) return st;
     T* Wp = static_cast<T*>(ws);
     T* Wd = reinterpret_cast<T*>(static_cast<unsigned char*>(ws) + part_bytes);
 
@@ -420,25 +490,23 @@ lrc_status launch_skinny_b(const TS* U, const TS* S, const TS* Vt, const TS* X, 
     constexpr int RW = w1_rows(B, (int64_t)sizeof(TS));
     if ((st = encode_map_2d(&tv, map_type<TS>(), Vt, n, k, ldn * e, kBox, kWarps * RW, false, "Vt")) != LRC_OK)
         return st;
-    constexpr int kRowsY = kYWarps * (32 / kYGroup) * y_rpg<TS>();
+    constexpr int kRowsY = 16 * y_rpg<TS>();
     if ((st = encode_map_2d(&tu, map_type<TS>(), U, k, m, ldk * e, (uint32_t)p.kbw, kRowsY, false, "U")) != LRC_OK)
         return st;
 
     cudaError_t ce = cudaFuncSetAttribute(skinny_w1_kernel<TS, T, B, RW>,
                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem1);
     if (ce != cudaSuccess) return cuda_fail(ce, "skinny_w1_kernel smem attribute");
-    skinny_w1_kernel<TS, T, B, RW><<<dim3((unsigned)p.nchunks, (unsigned)p.jblocks), kThreadsS, p.smem1, s>>>(
-        tx, tv, (int)k, (int)b, (int)p.L, Wp);
+    ce = launch_pdl(skinny_w1_kernel<TS, T, B, RW>, dim3((unsigned)p.nchunks, (unsigned)p.jblocks), dim3(kThreadsS),
+                    p.smem1, s, tx, tv, (int)k, (int)b, (int)p.L, Wp, cnt, S, (int)p.kv, round16 ? 1 : 0, Wd);
+    if (ce != cudaSuccess) return cuda_fail(ce, "skinny_w1_kernel launch");
     if ((st = after_launch("skinny_w1_kernel")) != LRC_OK) return st;
-    ce = launch_pdl(skinny_w2_kernel<TS, T>, dim3((unsigned)((b * p.kv * 32 + 255) / 256)), dim3(256), 0, s,
-                    (const T*)Wp, (int)p.nchunks, (int)b, (int)k, (int)p.kv, S, round16 ? 1 : 0, Wd);
-    if (ce != cudaSuccess) return cuda_fail(ce, "skinny_w2_kernel launch");
-    if ((st = after_launch("skinny_w2_kernel")) != LRC_OK) return st;
-    auto ykernel = skinny_y_kernel<TS, T, TOut, B, y_rpg<TS>()>;
+    constexpr int G = y_group(B, (int64_t)sizeof(TS));
+    auto ykernel = skinny_y_kernel<TS, T, TOut, B, y_rpg<TS>(), G>;
     ce = cudaFuncSetAttribute(ykernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem3);
     if (ce != cudaSuccess) return cuda_fail(ce, "skinny_y_kernel smem attribute");
-    ce = launch_pdl(ykernel, dim3((unsigned)p.yblocks), dim3(32 * kYWarps), p.smem3, s, tu, (const T*)Wd, m, (int)b,
-                    (int)p.nkb, (int)p.kbw, Y);
+    ce = launch_pdl(ykernel, dim3((unsigned)p.yblocks), dim3(32 * y_warps<G>()), p.smem3, s, tu, (const T*)Wd, m, (int)b,
+                    (int)p.nkb, (int)p.kbw, cnt, (int)p.jblocks, Y);
     if (ce != cudaSuccess) return cuda_fail(ce, "skinny_y_kernel launch");
     return after_launch("skinny_y_kernel");
 }

@@ -210,6 +210,10 @@ lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, in
 void release_scratch();
 // Per-(device, stream) workspace, grown on demand; freed by release_workspaces().
 lrc_status stream_workspace(cudaStream_t s, size_t bytes, void** out);
+// Per-(device, stream) arrival counters, zero between kernels: kStreamCounters
+// of them, made (and zeroed in stream order) on first use.
+constexpr int kStreamCounters = 1024;
+lrc_status stream_counters(cudaStream_t s, unsigned int** out);
 void release_workspaces();
 lrc_status run_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
                                 double* diff_out, double* normA_out, cudaStream_t s);

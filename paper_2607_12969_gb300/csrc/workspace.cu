@@ -4,6 +4,10 @@
 // the old buffer) before the old buffer is freed.  Calls on different
 // streams get different buffers, so they may run concurrently; calls on one
 // stream are ordered by the stream.  lrc_shutdown() frees every buffer.
+//
+// Beside it each (device, stream) has a small buffer of arrival counters for
+// kernels whose last CTA finishes a reduction: zeroed once when it is made
+// (in stream order), and left at zero by every kernel that uses it.
 #include <map>
 #include <mutex>
 #include <utility>
@@ -21,6 +25,7 @@ struct Buf {
 
 std::mutex g_ws_mu;
 std::map<std::pair<int, cudaStream_t>, Buf> g_ws;
+std::map<std::pair<int, cudaStream_t>, Buf> g_cnt;
 
 }  // namespace
 
@@ -52,17 +57,46 @@ lrc_status stream_workspace(cudaStream_t s, size_t bytes, void** out) {
     return LRC_OK;
 }
 
+lrc_status stream_counters(cudaStream_t s, unsigned int** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    std::lock_guard<std::mutex> lock(g_ws_mu);
+    Buf& b = g_cnt[std::make_pair(dev, s)];
+    if (!b.ptr) {
+        const size_t bytes = sizeof(unsigned int) * kStreamCounters;
+        e = cudaMalloc(&b.ptr, bytes);
+        if (e != cudaSuccess) {
+            b.ptr = nullptr;
+            cudaGetLastError();
+            set_error("counter allocation failed: %s", cudaGetErrorString(e));
+            return LRC_ERR_NOMEM;
+        }
+        e = cudaMemsetAsync(b.ptr, 0, bytes, s);
+        if (e != cudaSuccess) {
+            cudaFree(b.ptr);
+            b.ptr = nullptr;
+            return cuda_fail(e, "cudaMemsetAsync (counters)");
+        }
+        b.bytes = bytes;
+    }
+    *out = static_cast<unsigned int*>(b.ptr);
+    return LRC_OK;
+}
+
 void release_workspaces() {
     std::lock_guard<std::mutex> lock(g_ws_mu);
     int prev = -1;
     cudaGetDevice(&prev);
-    for (auto& kv : g_ws) {
-        if (kv.second.ptr) {
-            cudaSetDevice(kv.first.first);
-            cudaFree(kv.second.ptr);
+    for (auto* m : {&g_ws, &g_cnt}) {
+        for (auto& kv : *m) {
+            if (kv.second.ptr) {
+                cudaSetDevice(kv.first.first);
+                cudaFree(kv.second.ptr);
+            }
         }
+        m->clear();
     }
-    g_ws.clear();
     if (prev >= 0) cudaSetDevice(prev);
 }
 
