@@ -66,7 +66,7 @@ struct Bars {
     uint64_t *a1_full, *a1_empty;
     uint64_t *b1_full, *b1_empty;      // [2]
     uint64_t *d1_full, *d1_empty;      // [2]
-    uint64_t *a2_full, *a2_empty;      // [2]
+    uint64_t *a2_full, *a2_unused;     // [2]
     uint64_t *d2_full, *acc_empty;     // [2]
     uint64_t *mma_done;
     uint64_t *b2_full;
@@ -83,7 +83,7 @@ __device__ __forceinline__ Bars carve(unsigned char* smem, const T3Args& a) {
     B.b1_empty = p + 5;
     B.d1_full = p + 7;
     B.a2_full = p + 9;
-    B.a2_empty = p + 11;
+    B.a2_unused = p + 11;
     B.d2_full = p + 13;
     B.acc_empty = p + 15;
     B.mma_done = p + 17;
@@ -108,6 +108,26 @@ __device__ __forceinline__ void unit_coords(const T3Args& a, int64_t u, int64_t&
     i = rest / a.sn;
     h = (int)(rest - i * a.sn);
 }
+
+// Coordinates of consecutive units without divisions (the single-thread
+// roles walk their units in order; a 64-bit division costs them hundreds of
+// cycles a unit).
+struct UnitWalk {
+    int64_t qt, i;
+    int h;
+    __device__ __forceinline__ void start(const T3Args& a, int64_t u) { unit_coords(a, u, qt, i, h); }
+    // does the unit after this one start another i_1 tile?
+    __device__ __forceinline__ bool last_of_tile(const T3Args& a) const { return h + 1 == a.sn && i + 1 == a.n2; }
+    __device__ __forceinline__ void next(const T3Args& a) {
+        if (++h == a.sn) {
+            h = 0;
+            if (++i == a.n2) {
+                i = 0;
+                ++qt;
+            }
+        }
+    }
+};
 
 // Operand images: the rows of G_1 of every 128-row i_1 tile, G_2(i_2)^T for
 // every i_2 (row b, column a = G_2[a, i_2, b]) and G_3^T (row c, column
@@ -192,7 +212,6 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
             mbar_init(&B.b1_empty[q], 1);
             mbar_init(&B.d1_full[q], 1);
             mbar_init(&B.a2_full[q], 128);
-            mbar_init(&B.a2_empty[q], 1);
             mbar_init(&B.d2_full[q], 1);
             mbar_init(&B.acc_empty[q], 128);
         }
@@ -219,10 +238,10 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
             int64_t prev_qt = -1;
             int builds = 0;
             int64_t j = 0;
-            for (; j < nunits; ++j) {
-                int64_t qt, i;
-                int h;
-                unit_coords(a, ubeg + j, qt, i, h);
+            UnitWalk w;
+            w.start(a, ubeg);
+            for (; j < nunits; ++j, w.next(a)) {
+                const int64_t qt = w.qt, i = w.i;
                 if (qt != prev_qt) {
                     if (builds > 0 && !mbar_wait(B.a1_empty, (uint32_t)((builds - 1) & 1), abort, err, 1u)) break;
                     mbar_arrive_expect_tx(B.a1_full, a.a1_bytes);
@@ -231,7 +250,10 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
                     ++builds;
                 }
                 const int slot = (int)(j & 1);
-                if (!mbar_wait(&B.b1_empty[slot], (uint32_t)((j >> 1) & 1) ^ 1u, abort, err, 1u)) break;
+                // slot free once stage 1 of unit j - 2 has read it: with two D1
+                // buffers that is D1's own completion (one commit less a unit)
+                uint64_t* freed = a.nd1 == 2 ? &B.d1_full[slot] : &B.b1_empty[slot];
+                if (!mbar_wait(freed, (uint32_t)((j >> 1) & 1) ^ 1u, abort, err, 1u)) break;
                 mbar_arrive_expect_tx(&B.b1_full[slot], a.b1_bytes);
                 bulk_load(smem + a.off_b1 + (size_t)slot * a.b1_bytes, a.b1img + (size_t)i * a.b1_bytes, a.b1_bytes,
                           &B.b1_full[slot]);
@@ -253,10 +275,13 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
             const uint32_t b2s = smem_u32(smem + a.off_b2);
             int64_t cur_qt = -1;
             int qcount = 0;
+            UnitWalk w1, w2;          // units of the next stage 1 and stage 2 (both in order)
+            w1.start(a, ubeg);
+            w2.start(a, ubeg);
             auto stage1 = [&](int64_t j) -> bool {
-                int64_t qt, i;
-                int h;
-                unit_coords(a, ubeg + j, qt, i, h);
+                const int64_t qt = w1.qt;
+                const bool last = (j + 1 == nunits) || w1.last_of_tile(a);
+                w1.next(a);
                 const int buf = (int)(j & 1);
                 if (qt != cur_qt) {
                     if (!mbar_wait(B.a1_full, (uint32_t)(qcount & 1), abort, err, 2u)) return false;
@@ -278,23 +303,15 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
                 const uint32_t d1col = tmem + 2u * (uint32_t)a.n2h + (uint32_t)(db * a.r2p);
                 for (int ks = 0; ks < a.r1p / 16; ++ks)
                     mma_f16(d1col, ad + (uint64_t)ks * 256u, bd + (uint64_t)ks * bstep, idesc1, ks > 0);
-                mma_commit(&B.b1_empty[buf]);
+                if (a.nd1 == 1) mma_commit(&B.b1_empty[buf]);
                 mma_commit(&B.d1_full[db]);
                 // last unit of this i_1 tile: G_1 tile may be replaced once these MMAs finish
-                bool last = (j + 1 == nunits);
-                if (!last) {
-                    int64_t qn, in;
-                    int hn;
-                    unit_coords(a, ubeg + j + 1, qn, in, hn);
-                    last = (qn != qt);
-                }
                 if (last) mma_commit(B.a1_empty);
                 return true;
             };
             auto stage2 = [&](int64_t j) -> bool {
-                int64_t qt, i;
-                int h;
-                unit_coords(a, ubeg + j, qt, i, h);
+                const int h = w2.h;
+                w2.next(a);
                 const int buf = (int)(j & 1);
                 if (!mbar_wait(&B.a2_full[buf], (uint32_t)((j >> 1) & 1), abort, err, 2u)) return false;
                 if (!mbar_wait(&B.acc_empty[buf], (uint32_t)((j >> 1) & 1) ^ 1u, abort, err, 2u)) return false;
@@ -311,8 +328,7 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
                     mma_f16(tmem + (uint32_t)buf * a.n2h, hd + (uint64_t)ks * 256u, bdesc, idesc2, ks > 0);
                     if (!a.out16) mma_f16(tmem + (uint32_t)buf * a.n2h, ld + (uint64_t)ks * 256u, bdesc, idesc2, 1u);
                 }
-                mma_commit(&B.a2_empty[buf]);
-                mma_commit(&B.d2_full[buf]);
+                mma_commit(&B.d2_full[buf]);          // also frees the A2 slot for unit j + 2
                 return true;
             };
             // stage 1 runs nd1 units ahead of stage 2: with one D1 buffer the next
@@ -346,7 +362,8 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
             tmem_ld_wait();
             tc_fence_before();
             mbar_arrive(&B.d1_empty[db]);          // D1 is in registers: the next stage 1 may overwrite it
-            if (!group_wait(&B.a2_empty[buf], (uint32_t)((j >> 1) & 1) ^ 1u, abort, err, 4u, 2, 128)) break;
+            // A2 slot free once stage 2 of unit j - 2 has completed
+            if (!group_wait(&B.d2_full[buf], (uint32_t)((j >> 1) & 1) ^ 1u, abort, err, 4u, 2, 128)) break;
             unsigned char* ahi = smem + a.off_a2 + (size_t)buf * 2 * a.a2_bytes;
             unsigned char* alo = ahi + a.a2_bytes;
 #pragma unroll
@@ -377,10 +394,11 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
         const uint32_t lane_base = (uint32_t)(g * 32) << 16;
         unsigned char* wstage = smem + a.off_stage + (size_t)g * (2 * 32 * 128);
         int chunk = 0;
-        for (int64_t j = 0; j < nunits; ++j) {
-            int64_t qt, i;
-            int h;
-            unit_coords(a, ubeg + j, qt, i, h);
+        UnitWalk w;
+        w.start(a, ubeg);
+        for (int64_t j = 0; j < nunits; ++j, w.next(a)) {
+            const int64_t qt = w.qt, i = w.i;
+            const int h = w.h;
             const int buf = (int)(j & 1);
             if (!group_wait(&B.d2_full[buf], (uint32_t)((j >> 1) & 1), abort, err, 8u, 1, 128)) break;
             tc_fence_after();
