@@ -18,8 +18,15 @@
 // buffers after them; the converters release D1 as soon as it is in their
 // registers, so stage 1 of the next unit overlaps this unit's conversion and
 // stage 2.  Warp roles:
-//   0..3 epilogue, 4..7 converters, 8 MMA issuer (one thread), 9 loader (one
-//   thread).  A small image kernel first writes every operand the tensor
+//   0..3 epilogue, and 11..14 too when the plan takes two epilogue warps per
+//   tensor-memory lane quarter (alternate 128-byte column chunks; otherwise
+//   they idle), 4..7 converters, 8 stage-2 MMA issuer
+//   (one thread; it also
+//   owns the tensor memory), 9 loader (one thread), 10 stage-1 MMA issuer (one
+//   thread).  The two stages' MMAs are issued from two threads: their chains
+//   are independent (stage 1 waits for a free D1 and its operands, stage 2
+//   for A2 and a free accumulator), and a single issuer spent more time on
+//   instruction issue and commits than the epilogue takes to drain a unit.  A small image kernel first writes every operand the tensor
 //   cores read from the cores -- the G_1 rows of each i_1 tile, G_2(i_2)^T
 //   for every i_2, G_3^T -- in its shared-memory layout; the loader moves
 //   them with bulk copies (the main kernel is launched dependent on the
@@ -41,7 +48,8 @@ namespace {
 using namespace tc;
 
 constexpr int BM = 128;
-constexpr int kThreads = 320;
+constexpr int kThreads = 480;
+constexpr int kEpiWarpsMax = 8;    // warps 0..3 and 11..14
 
 struct T3Args {
     int64_t n1, n2;
@@ -49,6 +57,7 @@ struct T3Args {
     int n2h, sn;                   // n_3 slice per unit, number of slices
     int64_t units;                 // (i_1 tile, i_2, n_3 slice) units
     int cw, out16;
+    int nep;                       // epilogue warps per lane quarter (1 or 2)
     int nd1;                       // D1 buffers (TMEM columns 2 n2h .. 2 n2h + nd1 r2p)
     uint32_t tmem_cols;
     uint32_t off_a1, off_b1, off_a2, off_b2, off_stage, off_bar;
@@ -66,7 +75,7 @@ struct Bars {
     uint64_t *a1_full, *a1_empty;
     uint64_t *b1_full, *b1_empty;      // [2]
     uint64_t *d1_full, *d1_empty;      // [2]
-    uint64_t *a2_full, *a2_unused;     // [2]
+    uint64_t *a2_full, *mma_done1;     // [2], [1]: stage-1 issuer's MMAs complete
     uint64_t *d2_full, *acc_empty;     // [2]
     uint64_t *mma_done;
     uint64_t *b2_full;
@@ -83,7 +92,7 @@ __device__ __forceinline__ Bars carve(unsigned char* smem, const T3Args& a) {
     B.b1_empty = p + 5;
     B.d1_full = p + 7;
     B.a2_full = p + 9;
-    B.a2_unused = p + 11;
+    B.mma_done1 = p + 11;
     B.d2_full = p + 13;
     B.acc_empty = p + 15;
     B.mma_done = p + 17;
@@ -213,9 +222,10 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
             mbar_init(&B.d1_full[q], 1);
             mbar_init(&B.a2_full[q], 128);
             mbar_init(&B.d2_full[q], 1);
-            mbar_init(&B.acc_empty[q], 128);
+            mbar_init(&B.acc_empty[q], 128 * a.nep);
         }
         mbar_init(B.mma_done, 1);
+        mbar_init(B.mma_done1, 1);
         mbar_init(B.b2_full, 1);
         for (int q = 0; q < 2; ++q) mbar_init(&B.d1_empty[q], 128);
         *B.abort = 0;
@@ -265,10 +275,11 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
             for (int64_t q = (j - 2 > 0 ? j - 2 : 0); q < j && q < nunits; ++q)
                 mbar_wait(&B.b1_full[q & 1], (uint32_t)((q >> 1) & 1), &no_abort, err, 0u, 100000000ull);
         }
-    } else if (warp == 8) {
-        // ------------------------------------------------------------ MMA issuer
+    } else if (warp == 8 || warp == 10) {
+        // ------------------------------------------------------------ MMA issuers
+        // warp 10: stage 1 of every unit; warp 8: stage 2 of every unit
         if (lane == 0) {
-            bool ok = mbar_wait(B.b2_full, 0, abort, err, 2u);
+            bool ok = true;
             const uint32_t idesc1 = idesc_f16_f32(BM, (uint32_t)a.r2p);
             const uint32_t idesc2 = idesc_f16_f32(BM, (uint32_t)a.n2h);
             const uint32_t a1s = smem_u32(smem + a.off_a1);
@@ -289,9 +300,9 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
                     ++qcount;
                 }
                 // D1 has its own columns: it waits only for the converters of unit j - nd1
-                const int db = (int)(j % a.nd1);
-                if (j >= a.nd1 &&
-                    !mbar_wait(&B.d1_empty[db], (uint32_t)(((j / a.nd1) - 1) & 1), abort, err, 2u))
+                const int db = a.nd1 == 2 ? (int)(j & 1) : 0;
+                const int64_t dphase = a.nd1 == 2 ? (j >> 1) : j;
+                if (j >= a.nd1 && !mbar_wait(&B.d1_empty[db], (uint32_t)((dphase - 1) & 1), abort, err, 2u))
                     return false;
                 if (!mbar_wait(&B.b1_full[buf], (uint32_t)((j >> 1) & 1), abort, err, 2u)) return false;
                 tc_fence_after();
@@ -331,29 +342,30 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
                 mma_commit(&B.d2_full[buf]);          // also frees the A2 slot for unit j + 2
                 return true;
             };
-            // stage 1 runs nd1 units ahead of stage 2: with one D1 buffer the next
-            // stage 1 goes as soon as the converters have read D1 (before this
-            // unit's stage 2), with two it follows this unit's stage 2
-            for (int64_t u = 0; u < a.nd1 && u < nunits && ok; ++u) ok = stage1(u);
-            for (int64_t j = 0; j < nunits && ok; ++j) {
-                const int64_t u = j + a.nd1;
-                if (a.nd1 == 1 && u < nunits && !(ok = stage1(u))) break;
-                if (!(ok = stage2(j))) break;
-                if (a.nd1 == 2 && u < nunits) ok = stage1(u);
+            uint64_t* done = B.mma_done;
+            if (warp == 10) {
+                // stage 1 runs up to nd1 units ahead of the converters
+                for (int64_t j = 0; j < nunits && ok; ++j) ok = stage1(j);
+                done = B.mma_done1;
+            } else {
+                ok = mbar_wait(B.b2_full, 0, abort, err, 2u);
+                for (int64_t j = 0; j < nunits && ok; ++j) ok = stage2(j);
             }
-            mma_commit(B.mma_done);
+            // this thread's MMAs complete before the tensor memory is released
+            mma_commit(done);
             volatile int no_abort = 0;
-            mbar_wait(B.mma_done, 0, &no_abort, err, 2u, 100000000ull);
+            mbar_wait(done, 0, &no_abort, err, 2u, 100000000ull);
         }
-    } else if (warp >= 4) {
+    } else if (warp >= 4 && warp < 8) {
         // ------------------------------------------------------------ converters (warps 4..7)
         const int g = warp & 3;
         const int r = g * 32 + lane;
         const uint32_t lane_base = (uint32_t)(g * 32) << 16;
         for (int64_t j = 0; j < nunits; ++j) {
             const int buf = (int)(j & 1);
-            const int db = (int)(j % a.nd1);
-            if (!group_wait(&B.d1_full[db], (uint32_t)((j / a.nd1) & 1), abort, err, 4u, 2, 128)) break;
+            const int db = a.nd1 == 2 ? (int)(j & 1) : 0;
+            const int64_t dphase = a.nd1 == 2 ? (j >> 1) : j;
+            if (!group_wait(&B.d1_full[db], (uint32_t)(dphase & 1), abort, err, 4u, 2, 128)) break;
             tc_fence_after();
             uint32_t v[64];
             const uint32_t tcol = tmem + lane_base + 2u * (uint32_t)a.n2h + (uint32_t)(db * a.r2p);
@@ -385,14 +397,16 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
             tc_fence_before();
             mbar_arrive(&B.a2_full[buf]);
         }
-    } else {
+    } else if (warp < 4 || a.nep == 2) {
         // ------------------------------------------------------------ epilogue
-        // each warp drains its own 32 rows through its own staging pair and
-        // issues its own 32-row TMA stores: no barrier across the four warps
+        // each warp drains its own 32 rows (its lane quarter) on every other
+        // column chunk through its own staging pair and issues its own 32-row
+        // TMA stores: no barrier across the eight warps
         const int g = warp & 3;
+        const int hh = warp >= 11 ? 1 : 0;
         const int r = g * 32 + lane;
         const uint32_t lane_base = (uint32_t)(g * 32) << 16;
-        unsigned char* wstage = smem + a.off_stage + (size_t)g * (2 * 32 * 128);
+        unsigned char* wstage = smem + a.off_stage + (size_t)(hh * 4 + g) * (2 * 32 * 128);
         int chunk = 0;
         UnitWalk w;
         w.start(a, ubeg);
@@ -400,9 +414,9 @@ tt3_f16_tc_kernel(const __grid_constant__ CUtensorMap tm_out, const T3Args a) {
             const int64_t qt = w.qt, i = w.i;
             const int h = w.h;
             const int buf = (int)(j & 1);
-            if (!group_wait(&B.d2_full[buf], (uint32_t)((j >> 1) & 1), abort, err, 8u, 1, 128)) break;
+            if (!group_wait(&B.d2_full[buf], (uint32_t)((j >> 1) & 1), abort, err, 8u, 1, 128 * a.nep)) break;
             tc_fence_after();
-            for (int cc = 0; cc < a.n2h; cc += a.cw, ++chunk) {
+            for (int cc = hh * a.cw; cc < a.n2h; cc += a.nep * a.cw, ++chunk) {
                 uint32_t v[64];
                 const uint32_t tcol = tmem + lane_base + (uint32_t)buf * a.n2h + (uint32_t)cc;
                 tmem_ld32(tcol, *reinterpret_cast<uint32_t(*)[32]>(&v[0]));
@@ -521,8 +535,14 @@ bool tt3_f16_tc_plan(const TTShape& sh, bool out16, T3Args* out_args, size_t* sm
     a.off_b2 = off;
     off += a.b2_bytes;
     off = (off + 1023) / 1024 * 1024;
+    // two epilogue warps per lane quarter when a unit has a chunk for each:
+    // measured faster for binary16 output (the conversion bounds that
+    // epilogue: 512^2 x 224 37.4 -> 32.1 us) and for binary32 units of at
+    // most 128 columns (256^3: 20.7 -> 19.5 us); binary32 units of 224
+    // columns, already at the store rate, measured slower (49.5 -> 52.0 us)
+    a.nep = (a.n2h >= 2 * a.cw && (out16 || a.n2h <= 128)) ? 2 : 1;
     a.off_stage = off;
-    off += 2 * BM * 128;
+    off += (uint32_t)(4 * a.nep) * 2 * 32 * 128;
     off = (off + 7) / 8 * 8;
     a.off_bar = off;
     off += 21 * 8 + 16;
