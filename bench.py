@@ -837,10 +837,40 @@ def run_oracle_timing(steps: int, warmup: int, threads: int | None = None):
 # single-call mode (the commands the ncu captures in profiles/ run)
 # ---------------------------------------------------------------------------
 
+def memory_rates(torch, dev, reps, nbytes=4 << 30):
+    """HBM rates of plain streams over `nbytes` (far above the 129 MB L2, so
+    what is still in L2 when the timing stops is a few percent): a pure
+    write (fill), a pure read (sum) and a copy of half the bytes each way,
+    CUDA events, best of `reps`.  Returns GB/s by kind."""
+    x = torch.empty(nbytes // 4, dtype=torch.float32, device=dev)
+    y = torch.empty(nbytes // 8, dtype=torch.float32, device=dev)
+    x.fill_(1.0)
+    half = x[: nbytes // 8]
+    ops = {"write": (lambda: x.fill_(2.0), nbytes), "read": (lambda: x.sum(), nbytes),
+           "copy": (lambda: y.copy_(half), nbytes)}
+    out = {}
+    for name, (fn, moved) in ops.items():
+        fn()
+        torch.cuda.synchronize()
+        best = None
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            fn()
+            e1.record()
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1)
+            best = ms if best is None else min(best, ms)
+        out[name] = moved / (best * 1e-3) / 1e9
+    del x, y
+    return out
+
+
 def run_peaks(lrc, torch, dev, reps):
     """Measured arithmetic rates: the library's FMA-chain probes and
-    torch.matmul (cuBLAS) per dtype at 8192^3."""
-    out = {}
+    torch.matmul (cuBLAS) per dtype at 8192^3; HBM write, read and copy
+    rates of plain streams."""
+    out = {f"hbm_{k}_gbs": v for k, v in memory_rates(torch, dev, reps).items()}
     for kind in ("ffma", "ffma2", "dfma", "dmma"):
         iters = 1 << 22 if kind.startswith("ffma") else 1 << 17
         out[f"probe_{kind}_tflops"] = max(lrc.lrc_probe_peak(kind, iters) for _ in range(reps)) / 1e12
