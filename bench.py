@@ -429,9 +429,10 @@ class Step:
     def run(self, record=False, on_outputs=None, wait_inputs=None):
         """One pass.  wait_inputs(workload), if given, is called before a
         workload's first call (the end-to-end run makes the stream wait for
-        that workload's input copies there); on_outputs, if given, once the
-        apply and TT outputs are enqueued (the eta and certificate work that
-        follows reads none of them)."""
+        that workload's input copies there); on_outputs(workload), if given,
+        once that workload's apply or TT outputs are enqueued (the end-to-end
+        run reads them back from there on while the later workloads and the
+        eta and certificate work, which reads none of them, run)."""
         self.record = record
         lrc = self.lrc
         order = [self.mats[1]] + self.tts + [self.mats[0], self.mats[2]]
@@ -439,8 +440,8 @@ class Step:
             if wait_inputs is not None:
                 wait_inputs(wl)
             wl.calls(lrc, self)
-        if on_outputs is not None:
-            on_outputs()
+            if on_outputs is not None:
+                on_outputs(wl)
         for wl in self.mats + self.tts:
             wl.eta_calls(lrc, self)
 
@@ -1182,16 +1183,17 @@ def main():
     def wait_inputs(wl):
         main_stream.wait_event(ready[wl.name])
 
-    def read_back():
-        # outputs come back on a second copy stream while the eta work runs
+    def read_back(wl):
+        # a workload's outputs come back on a second copy stream as soon as
+        # its calls are done, while the later workloads and the eta work run
         done = torch.cuda.Event()
         done.record()
         d2h_stream.wait_event(done)
         with torch.cuda.stream(d2h_stream):
-            for wl in step.mats:
+            if isinstance(wl, MatrixWL):
                 for f, y in wl.Y.items():
                     outs[wl.name][f].copy_(y, non_blocking=True)
-            for wl in step.tts:
+            else:
                 for f, o in wl.last_outputs().items():
                     outs[wl.name][f].copy_(o, non_blocking=True)
 
