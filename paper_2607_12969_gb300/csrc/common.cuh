@@ -214,6 +214,11 @@ lrc_status stream_workspace(cudaStream_t s, size_t bytes, void** out);
 // of them, made (and zeroed in stream order) on first use.
 constexpr int kStreamCounters = 1024;
 lrc_status stream_counters(cudaStream_t s, unsigned int** out);
+// Per-(device, stream) slot of kResultSlots doubles in mapped pinned host
+// memory: `dev` is the address kernels write, `host` the one the host reads
+// once the stream has synchronised.
+constexpr int kResultSlots = 8;
+lrc_status stream_result_slot(cudaStream_t s, double** host, double** dev);
 void release_workspaces();
 lrc_status run_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
                                 double* diff_out, double* normA_out, cudaStream_t s);

@@ -547,11 +547,17 @@ lrc_status pack_cols(const double* X, int64_t ldx, const void* Xh, int64_t ldh, 
     return after_launch("eta_pack_cols_kernel");
 }
 
-lrc_status read_result(const double* res, double* eta_out, double* norm_out, cudaStream_t s) {
-    double host[2];
-    cudaError_t e = cudaMemcpyAsync(host, res, sizeof host, cudaMemcpyDeviceToHost, s);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (eta result)");
-    e = cudaStreamSynchronize(s);
+// The last step of an eta: eta_finish_kernel adds the block sums in order
+// and writes (eta, norm) into the stream's mapped result slot; the host reads
+// them once the stream has synchronised (no copy-engine transfer).
+lrc_status finish_eta(const double* cpart, int nparts, double* eta_out, double* norm_out, cudaStream_t s) {
+    double* host = nullptr;
+    double* dev = nullptr;
+    lrc_status st = stream_result_slot(s, &host, &dev);
+    if (st != LRC_OK) return st;
+    eta_finish_kernel<<<1, 32, 0, s>>>(cpart, nparts, dev);
+    if ((st = after_launch("eta_finish_kernel")) != LRC_OK) return st;
+    const cudaError_t e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize (eta)");
     *eta_out = host[0];
     if (norm_out) *norm_out = host[1];
@@ -583,7 +589,7 @@ lrc_status lowrank_eta_t(const double* U, const double* S, const double* Vt, con
     const size_t o_pu = c.take((size_t)m * w * 8), o_pv = c.take((size_t)n * w * 8);
     const size_t o_gu = c.take((size_t)w * w * 8), o_gv = c.take((size_t)w * w * 8);
     const size_t o_part = c.take((size_t)gram_slots(sp, 2) * 8);
-    const size_t o_cp = c.take((size_t)2 * kCombineBlocks * 8), o_res = c.take(16);
+    const size_t o_cp = c.take((size_t)2 * kCombineBlocks * 8);
     void* ws = nullptr;
     lrc_status st = stream_workspace(s, c.off, &ws);
     if (st != LRC_OK) return st;
@@ -593,7 +599,6 @@ lrc_status lowrank_eta_t(const double* U, const double* S, const double* Vt, con
     double* Gu = (double*)(base + o_gu);
     double* Gv = (double*)(base + o_gv);
     double* cpart = (double*)(base + o_cp);
-    double* res = (double*)(base + o_res);
     sp[0].A = sp[0].B = Pu;
     sp[0].C = Gu;
     sp[1].A = sp[1].B = Pv;
@@ -605,9 +610,7 @@ lrc_status lowrank_eta_t(const double* U, const double* S, const double* Vt, con
     const int cb = std::min(kCombineBlocks, kk);
     eta_lowrank_combine_kernel<T><<<cb, 256, 0, s>>>(Gu, Gv, S, (const T*)Sh, kk, cpart);
     if ((st = after_launch("eta_lowrank_combine_kernel")) != LRC_OK) return st;
-    eta_finish_kernel<<<1, 32, 0, s>>>(cpart, cb, res);
-    if ((st = after_launch("eta_finish_kernel")) != LRC_OK) return st;
-    return read_result(res, eta_out, norm_out, s);
+    return finish_eta(cpart, cb, eta_out, norm_out, s);
 }
 
 // The three products of one interior level (D-columns: CD, X_D; Z-columns:
@@ -649,7 +652,7 @@ lrc_status tt_eta_t(const TTShape& sh, const void* const* hats, double* eta_out,
     const size_t o_pk = c.take((size_t)pack_max * 8), o_lev = c.take((size_t)lev_max * 8);
     const size_t o_m0 = c.take((size_t)4 * rmax * rmax * 8), o_m1 = c.take((size_t)4 * rmax * rmax * 8);
     const size_t o_part = c.take((size_t)slots * 8);
-    const size_t o_cp = c.take((size_t)2 * kCombineBlocks * 8), o_res = c.take(16);
+    const size_t o_cp = c.take((size_t)2 * kCombineBlocks * 8);
     void* ws = nullptr;
     lrc_status st = stream_workspace(s, c.off, &ws);
     if (st != LRC_OK) return st;
@@ -660,7 +663,6 @@ lrc_status tt_eta_t(const TTShape& sh, const void* const* hats, double* eta_out,
     double* Mnext = (double*)(base + o_m1);
     double* part = (double*)(base + o_part);
     double* cpart = (double*)(base + o_cp);
-    double* res = (double*)(base + o_res);
 
     // level 1: M_1 = [dG_1, Gh_1]^T [dG_1, Gh_1]  (G_1 is n_1 x r_1)
     if ((st = pack_rows<T>((const double*)sh.cores[0], r1, hats[0], r1, n1, r1, 0, Pk, s)) != LRC_OK) return st;
@@ -699,9 +701,7 @@ lrc_status tt_eta_t(const TTShape& sh, const void* const* hats, double* eta_out,
     const int cb = std::min(kCombineBlocks, rl);
     eta_tt_combine_kernel<<<cb, 256, 0, s>>>(Mcur, Mnext, rl, cpart);
     if ((st = after_launch("eta_tt_combine_kernel")) != LRC_OK) return st;
-    eta_finish_kernel<<<1, 32, 0, s>>>(cpart, cb, res);
-    if ((st = after_launch("eta_finish_kernel")) != LRC_OK) return st;
-    return read_result(res, eta_out, norm_out, s);
+    return finish_eta(cpart, cb, eta_out, norm_out, s);
 }
 
 }  // namespace

@@ -302,13 +302,14 @@ lrc_status run_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, in
     }
     lrc_status st = after_launch("fro_partial_kernel");
     if (st != LRC_OK) return st;
-    double* result = partial + 2 * kMaxBlocks;
+    // the two results go straight to the stream's mapped host slot (no
+    // copy-engine transfer behind other copies)
+    double* host = nullptr;
+    double* result = nullptr;
+    if ((st = stream_result_slot(s, &host, &result)) != LRC_OK) return st;
     fro_final_kernel<<<1, 1024, 0, s>>>(partial, grid, result);
     st = after_launch("fro_final_kernel");
     if (st != LRC_OK) return st;
-    double host[2];
-    e = cudaMemcpyAsync(host, result, sizeof host, cudaMemcpyDeviceToHost, s);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (fro_diff result)");
     e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize (fro_diff)");
     *diff_out = host[0];

@@ -7,7 +7,11 @@
 //
 // Beside it each (device, stream) has a small buffer of arrival counters for
 // kernels whose last CTA finishes a reduction: zeroed once when it is made
-// (in stream order), and left at zero by every kernel that uses it.
+// (in stream order), and left at zero by every kernel that uses it; and a
+// result slot in mapped pinned host memory, which the finishing kernel of a
+// scalar reduction writes directly (the host reads it after the stream has
+// synchronised), so a scalar result never queues behind bulk copies on the
+// copy engines.
 #include <map>
 #include <mutex>
 #include <utility>
@@ -26,6 +30,11 @@ struct Buf {
 std::mutex g_ws_mu;
 std::map<std::pair<int, cudaStream_t>, Buf> g_ws;
 std::map<std::pair<int, cudaStream_t>, Buf> g_cnt;
+struct Slot {
+    double* host = nullptr;
+    double* dev = nullptr;
+};
+std::map<std::pair<int, cudaStream_t>, Slot> g_slot;
 
 }  // namespace
 
@@ -84,6 +93,34 @@ lrc_status stream_counters(cudaStream_t s, unsigned int** out) {
     return LRC_OK;
 }
 
+lrc_status stream_result_slot(cudaStream_t s, double** host, double** dev) {
+    int d = 0;
+    cudaError_t e = cudaGetDevice(&d);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    std::lock_guard<std::mutex> lock(g_ws_mu);
+    Slot& sl = g_slot[std::make_pair(d, s)];
+    if (!sl.host) {
+        void* h = nullptr;
+        e = cudaHostAlloc(&h, sizeof(double) * kResultSlots, cudaHostAllocMapped);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            set_error("result slot allocation failed: %s", cudaGetErrorString(e));
+            return LRC_ERR_NOMEM;
+        }
+        void* dp = nullptr;
+        e = cudaHostGetDevicePointer(&dp, h, 0);
+        if (e != cudaSuccess) {
+            cudaFreeHost(h);
+            return cuda_fail(e, "cudaHostGetDevicePointer (result slot)");
+        }
+        sl.host = static_cast<double*>(h);
+        sl.dev = static_cast<double*>(dp);
+    }
+    *host = sl.host;
+    *dev = sl.dev;
+    return LRC_OK;
+}
+
 void release_workspaces() {
     std::lock_guard<std::mutex> lock(g_ws_mu);
     int prev = -1;
@@ -97,6 +134,9 @@ void release_workspaces() {
         }
         m->clear();
     }
+    for (auto& kv : g_slot)
+        if (kv.second.host) cudaFreeHost(kv.second.host);
+    g_slot.clear();
     if (prev >= 0) cudaSetDevice(prev);
 }
 
