@@ -138,8 +138,12 @@ LRC_API lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows,
  * workspace owned by the library: one buffer per (device, stream),
  * allocated on first use and reallocated -- after synchronizing `stream` --
  * when a larger problem arrives, freed by lrc_shutdown().  Calls on
- * different streams use different buffers.  Binary16 ranks: up to 320 for
- * LRC_F16 and 512 for LRC_F16_O16, else LRC_ERR_UNSUPPORTED.
+ * different streams use different buffers.  Batches of at most 16 queries
+ * (4 for binary16) on the CUDA cores add their per-chunk partial sums in the
+ * same workspace and keep a per-stream buffer of 1024 arrival counters
+ * (zeroed once when made, left at zero by every call, freed by
+ * lrc_shutdown()).  Binary16 ranks: up to 320 for LRC_F16 and 512 for
+ * LRC_F16_O16, else LRC_ERR_UNSUPPORTED.
  */
 /* LRC_F32_TC: as LRC_F32, with the second product (W U^T) on the tensor
  * cores when b > 32 and k <= 192; otherwise the LRC_F32 kernels. */
@@ -248,7 +252,11 @@ LRC_API lrc_status tt_gather(const void* const* cores, const int64_t* dims, cons
  * fixed order, so repeated calls on the same data give identical bits.
  * Uses library-held device scratch (allocated on first use per device,
  * released by lrc_shutdown), so concurrent calls on different streams of
- * the same device must not overlap.  SYNCHRONISES `stream`.
+ * the same device must not overlap.  The two results are written by the
+ * final kernel into a per-stream slot of mapped pinned host memory
+ * (allocated on first use, released by lrc_shutdown) and read once the
+ * stream has synchronised, so they never wait behind other copies on the
+ * copy engines.  SYNCHRONISES `stream`.
  */
 LRC_API lrc_status lrc_fro_diff(const void* A, lrc_fmt fa, const void* B, lrc_fmt fb, int64_t count,
                         double* diff_out, double* normA_out, lrc_stream_t stream);
@@ -304,7 +312,8 @@ LRC_API lrc_status lrc_fro_diff_noalloc(const void* A, lrc_fmt fa, const void* B
  * relative to ||A||.  Work: about 2 (m + n) k (2k + 1) binary64 flops.
  * All arithmetic binary64; deterministic on a device.  k <= 4096.  Pointers
  * 16-byte aligned.  Scratch: the stream's library workspace (see
- * lrc_apply), 16 (m + n) k bytes plus O(k^2).  SYNCHRONISES `stream`.
+ * lrc_apply), 16 (m + n) k bytes plus O(k^2); the results come back through
+ * the stream's mapped host slot (see lrc_fro_diff).  SYNCHRONISES `stream`.
  */
 LRC_API lrc_status lrc_lowrank_eta(const double* U, const double* S, const double* Vt,
                                    const void* Uh, const void* Sh, const void* Vht, lrc_fmt fmt,
@@ -333,8 +342,9 @@ LRC_API lrc_status lrc_lowrank_eta(const double* U, const double* S, const doubl
  * Work: about sum over interior cores of 8 r_{l-1} n_l r_l (2 r_{l-1} +
  * r_l) binary64 flops.  Deterministic on a device.  Cores aligned to their
  * element size.  Scratch: the stream's workspace, two buffers of
- * 4 r_{l-1} n_l r_l binary64 for the largest interior core plus O(r^2).
- * SYNCHRONISES `stream`.
+ * 4 r_{l-1} n_l r_l binary64 for the largest interior core plus O(r^2); the
+ * results come back through the stream's mapped host slot (see
+ * lrc_fro_diff).  SYNCHRONISES `stream`.
  */
 LRC_API lrc_status lrc_tt_eta(const double* const* cores, const void* const* cores_hat,
                               const int64_t* dims, const int64_t* ranks, int d, lrc_fmt fmt,
