@@ -265,12 +265,15 @@ class MatrixWL:
         self.Y = {f: T((b, m), lrc.output_dtype(f)) for f in COMP}
         self.results = {}
 
-    def calls(self, lrc, step):
-        """Rounding (a1) and applies (a2-a4) of this workload."""
+    def calls(self, lrc, step, on_output=None):
+        """Rounding (a1) and applies (a2-a4) of this workload, one storage
+        format at a time, binary16 first: the FP32 apply, the longest call,
+        runs last.  on_output(workload, fmt), if given, after each apply (the
+        end-to-end run reads that output back from there on)."""
         cfg, d = self.cfg, self.d
         m, n, b = cfg.m, cfg.n, cfg.b
         kmax = d["Q1"].shape[1]
-        for s in STORE:
+        for s in sorted(STORE, key=lambda x: x == "f32"):
             F, k = self.fac[s], self.kp[s]
             step.timed(f"round@{self.name}", work_round(m, k, F["U64"].shape[1], "f64"),
                        lambda: lrc.lrc_round_factors(d["Q1"], m, k, kmax, F["U64"], F["U64"].shape[1], "f64"))
@@ -282,10 +285,11 @@ class MatrixWL:
                        lambda: lrc.lrc_round_factors(d["Q2t"], k, n, n, F["Vt"], F["Vt"].shape[1], s))
             step.timed(f"round@{self.name}", work_round(b, n, F["X"].shape[1], s),
                        lambda: lrc.lrc_round_factors(d["X"], b, n, n, F["X"], F["X"].shape[1], s))
-        for f in COMP:
-            F, k = self.fac[store_of(f)], self.kp[store_of(f)]
-            step.timed(f"apply_{f}@{self.name}", work_apply(m, n, k, b, f),
-                       lambda: lrc.lrc_apply(F["U"], F["S"], F["Vt"], F["X"], self.Y[f], m, n, k, b, f))
+            for f in (f for f in COMP if store_of(f) == s):
+                step.timed(f"apply_{f}@{self.name}", work_apply(m, n, k, b, f),
+                           lambda: lrc.lrc_apply(F["U"], F["S"], F["Vt"], F["X"], self.Y[f], m, n, k, b, f))
+                if on_output is not None:
+                    on_output(self, f)
 
     def eta_calls(self, lrc, step):
         """eta of each storage format (a6, fused route) and the certificate (a7)."""
@@ -325,7 +329,9 @@ class TTWL:
         self.turn = 0
         self.results = {}
 
-    def calls(self, lrc, step):
+    def calls(self, lrc, step, on_output=None):
+        """Rounding (a1) and reconstructions (a5) of this workload;
+        on_output(workload, fmt), if given, after each reconstruction."""
         cfg = self.cfg
         for s in STORE:
             for src, dst in zip(self.c64[s], self.low[s]):
@@ -338,10 +344,9 @@ class TTWL:
             o = outs[self.turn % len(outs)]
             step.timed(f"tt_{f}@{self.name}", work_tt(cfg.dims, cfg.ranks[s], f),
                        lambda: lrc.tt_reconstruct(self.low[s], cfg.dims, cfg.ranks[s], f, o))
+            if on_output is not None:
+                on_output(self, f, o)
         self.turn += 1
-
-    def last_outputs(self):
-        return {f: self.out[f][(self.turn - 1) % len(self.out[f])] for f in COMP}
 
     def eta_calls(self, lrc, step):
         cfg = self.cfg
@@ -429,19 +434,17 @@ class Step:
     def run(self, record=False, on_outputs=None, wait_inputs=None):
         """One pass.  wait_inputs(workload), if given, is called before a
         workload's first call (the end-to-end run makes the stream wait for
-        that workload's input copies there); on_outputs(workload), if given,
-        once that workload's apply or TT outputs are enqueued (the end-to-end
-        run reads them back from there on while the later workloads and the
-        eta and certificate work, which reads none of them, run)."""
+        that workload's input copies there); on_outputs(workload, fmt[, out]),
+        if given, once an apply or TT output is enqueued (the end-to-end run
+        reads it back from there on while the later calls and the eta and
+        certificate work, which reads none of the outputs, run)."""
         self.record = record
         lrc = self.lrc
         order = [self.mats[1]] + self.tts + [self.mats[0], self.mats[2]]
         for wl in order:
             if wait_inputs is not None:
                 wait_inputs(wl)
-            wl.calls(lrc, self)
-            if on_outputs is not None:
-                on_outputs(wl)
+            wl.calls(lrc, self, on_output=on_outputs)
         for wl in self.mats + self.tts:
             wl.eta_calls(lrc, self)
 
@@ -1183,19 +1186,14 @@ def main():
     def wait_inputs(wl):
         main_stream.wait_event(ready[wl.name])
 
-    def read_back(wl):
-        # a workload's outputs come back on a second copy stream as soon as
-        # its calls are done, while the later workloads and the eta work run
+    def read_back(wl, f, out=None):
+        # each output comes back on a second copy stream as soon as its call
+        # is done, while the later calls and the eta work run
         done = torch.cuda.Event()
         done.record()
         d2h_stream.wait_event(done)
         with torch.cuda.stream(d2h_stream):
-            if isinstance(wl, MatrixWL):
-                for f, y in wl.Y.items():
-                    outs[wl.name][f].copy_(y, non_blocking=True)
-            else:
-                for f, o in wl.last_outputs().items():
-                    outs[wl.name][f].copy_(o, non_blocking=True)
+            outs[wl.name][f].copy_(wl.Y[f] if out is None else out, non_blocking=True)
 
     def e2e_once():
         copy_inputs()
