@@ -24,8 +24,9 @@
 //   skinny_y_kernel   a CTA per 64 rows of U (32 for binary64): the rows are
 //                     requested at once, so they stream while the first
 //                     kernel still runs; after the wait for it W (b x k)
-//                     follows as one bulk copy; groups of 8 lanes take 4
-//                     rows (2) each, a lane every 8th column.
+//                     follows as one bulk copy; groups of G lanes (8, or 32
+//                     for at most 4 queries in 2- and 4-byte formats) take 4
+//                     rows (2) each, a lane every G-th 16-byte column.
 // Arithmetic: binary64 FMAs for binary64, binary32 FMAs otherwise (binary16
 // factors widened exactly; Sec. 3.4: FP16 products accumulate in FP32).  The
 // summation order is fixed: results are reproducible on a device.
