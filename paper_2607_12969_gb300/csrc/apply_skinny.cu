@@ -471,7 +471,7 @@ lrc_status launch_skinny_b(const TS* U, const TS* S, const TS* Vt, const TS* X, 
     const int64_t e = (int64_t)sizeof(TS);
     const SkinnyPlan p = plan_skinny(m, n, k, B, e, (int64_t)sizeof(T));
     int64_t t;
-    if (!mul_ok(p.nchunks * b, k, &t) || p.nchunks > 65535 || p.jblocks > 65535 || n > INT32_MAX ||
+    if (!mul_ok(p.nchunks * b, k, &t) || p.nchunks > 65535 || p.jblocks > kStreamCounters || n > INT32_MAX ||
         m > INT32_MAX || p.smem1 > kSmemMaxS || p.smem3 > kSmemMaxS) {
         set_error("small-batch apply: problem outside the kernel");
         return LRC_ERR_UNSUPPORTED;
