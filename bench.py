@@ -265,13 +265,13 @@ class MatrixWL:
         self.Y = {f: T((b, m), lrc.output_dtype(f)) for f in COMP}
         self.results = {}
 
-    def calls(self, lrc, step, on_output=None):
-        """Rounding (a1) and applies (a2-a4) of this workload, one storage
-        format at a time, binary16 first: the FP32 apply, the longest call,
-        runs last.  on_output(workload, fmt), if given, after each apply (the
-        end-to-end run reads that output back from there on)."""
+    QUERIES = ("X",)           # host inputs that only the applies read; the rest are the factors
+
+    def factor_calls(self, lrc, step):
+        """Rounding (a1) of the factors: the FP64 pack of U (the eta input)
+        and U, s, V^T in each storage format."""
         cfg, d = self.cfg, self.d
-        m, n, b = cfg.m, cfg.n, cfg.b
+        m, n = cfg.m, cfg.n
         kmax = d["Q1"].shape[1]
         for s in sorted(STORE, key=lambda x: x == "f32"):
             F, k = self.fac[s], self.kp[s]
@@ -283,6 +283,16 @@ class MatrixWL:
                        lambda: lrc.lrc_round_factors(d["s"], 1, k, kmax, F["S"], F["S"].shape[1], s))
             step.timed(f"round@{self.name}", work_round(k, n, F["Vt"].shape[1], s),
                        lambda: lrc.lrc_round_factors(d["Q2t"], k, n, n, F["Vt"], F["Vt"].shape[1], s))
+
+    def query_calls(self, lrc, step, on_output=None):
+        """Rounding (a1) of the query batch and the applies (a2-a4), one
+        storage format at a time, binary16 first: the FP32 apply, the longest
+        call, runs last.  on_output(workload, fmt), if given, after each apply
+        (the end-to-end run reads that output back from there on)."""
+        cfg, d = self.cfg, self.d
+        m, n, b = cfg.m, cfg.n, cfg.b
+        for s in sorted(STORE, key=lambda x: x == "f32"):
+            F, k = self.fac[s], self.kp[s]
             step.timed(f"round@{self.name}", work_round(b, n, F["X"].shape[1], s),
                        lambda: lrc.lrc_round_factors(d["X"], b, n, n, F["X"], F["X"].shape[1], s))
             for f in (f for f in COMP if store_of(f) == s):
@@ -432,20 +442,31 @@ class Step:
             fn()
 
     def run(self, record=False, on_outputs=None, wait_inputs=None):
-        """One pass.  wait_inputs(workload), if given, is called before a
-        workload's first call (the end-to-end run makes the stream wait for
-        that workload's input copies there); on_outputs(workload, fmt[, out]),
-        if given, once an apply or TT output is enqueued (the end-to-end run
-        reads it back from there on while the later calls and the eta and
-        certificate work, which reads none of the outputs, run)."""
+        """One pass.  wait_inputs(workload, part), if given, is called before
+        the calls that read a workload's inputs ("factors", "queries" or
+        "cores"; the end-to-end run makes the stream wait for those input
+        copies there); on_outputs(workload, fmt[, out]), if given, once an
+        apply or TT output is enqueued (the end-to-end run reads it back from
+        there on while the later calls and the eta and certificate work,
+        which reads none of the outputs, run).  A matrix workload's eta and
+        certificate depend on its factors only, so they run before its query
+        batch is read: in the end-to-end run they overlap the transfer of
+        the queries (4.3 GB for the b = 32768 workload)."""
         self.record = record
         lrc = self.lrc
+        wait = wait_inputs if wait_inputs is not None else (lambda wl, part: None)
         order = [self.mats[1]] + self.tts + [self.mats[0], self.mats[2]]
         for wl in order:
-            if wait_inputs is not None:
-                wait_inputs(wl)
-            wl.calls(lrc, self, on_output=on_outputs)
-        for wl in self.mats + self.tts:
+            if isinstance(wl, MatrixWL):
+                wait(wl, "factors")
+                wl.factor_calls(lrc, self)
+                wl.eta_calls(lrc, self)
+                wait(wl, "queries")
+                wl.query_calls(lrc, self, on_output=on_outputs)
+            else:
+                wait(wl, "cores")
+                wl.calls(lrc, self, on_output=on_outputs)
+        for wl in self.tts:
             wl.eta_calls(lrc, self)
 
     def results(self):
@@ -1173,18 +1194,24 @@ def main():
         with torch.cuda.stream(h2d_stream):
             for wl in [step.mats[1]] + step.tts + [step.mats[0], step.mats[2]]:
                 if isinstance(wl, MatrixWL):
-                    for k, h in pin[wl.name].items():
-                        wl.d[k].copy_(h, non_blocking=True)
+                    # the factors first (the eta work needs only them), then the queries
+                    for part, keys in (("factors", [k for k in pin[wl.name] if k not in wl.QUERIES]),
+                                       ("queries", list(wl.QUERIES))):
+                        for k in keys:
+                            wl.d[k].copy_(pin[wl.name][k], non_blocking=True)
+                        ev = torch.cuda.Event()
+                        ev.record()
+                        ready[(wl.name, part)] = ev
                 else:
                     for s in STORE:
                         for dd, h in zip(wl.c64[s], pin[wl.name][s]):
                             dd.copy_(h, non_blocking=True)
-                ev = torch.cuda.Event()
-                ev.record()
-                ready[wl.name] = ev
+                    ev = torch.cuda.Event()
+                    ev.record()
+                    ready[(wl.name, "cores")] = ev
 
-    def wait_inputs(wl):
-        main_stream.wait_event(ready[wl.name])
+    def wait_inputs(wl, part):
+        main_stream.wait_event(ready[(wl.name, part)])
 
     def read_back(wl, f, out=None):
         # each output comes back on a second copy stream as soon as its call
