@@ -25,6 +25,15 @@
  *  - The library never traps and has no CPU fallback: it needs an sm_103a
  *    GPU.  Device scratch is allocated only where an entry point says so
  *    (library workspaces, allocated on first use and reused).
+ *  - Stream order holds as for any kernel: work the caller enqueues after a
+ *    call starts after the call's kernels have completed.  Inside a call the
+ *    kernels are chained by programmatic dependent launch, and the last
+ *    kernel of a call may let the next kernel of the stream begin its
+ *    prologue early; that only affects a caller's own kernel launched with
+ *    the programmatic-serialization attribute, which (as CUDA requires of
+ *    such a kernel) must execute griddepcontrol.wait before it reads the
+ *    call's outputs.  Every library kernel launched that way waits before
+ *    it touches memory written by an earlier kernel.
  */
 #ifndef LRC_H
 #define LRC_H
