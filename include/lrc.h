@@ -32,8 +32,10 @@
  *    prologue early; that only affects a caller's own kernel launched with
  *    the programmatic-serialization attribute, which (as CUDA requires of
  *    such a kernel) must execute griddepcontrol.wait before it reads the
- *    call's outputs.  Every library kernel launched that way waits before
- *    it touches memory written by an earlier kernel.
+ *    call's outputs.  A library kernel launched that way reads memory an
+ *    earlier kernel of the stream may have written only after its
+ *    griddepcontrol.wait, or after a kernel of its own call that has
+ *    already waited for everything before the call.
  */
 #ifndef LRC_H
 #define LRC_H
