@@ -66,7 +66,6 @@ constexpr int kEpiWarpsY = 8;
 constexpr int kThreadsY = 64 + 32 * kEpiWarpsY;
 constexpr uint32_t kXBytes = BM * BK * 2;    // one X box
 constexpr int kChunkBlocks = 8;              // k-blocks per accumulation chunk (FP32 output)
-constexpr int kPfBlocks = 4;                 // k-blocks per L2 prefetch box (512-byte rows)
 constexpr int kStageBlocks = 2;              // k-blocks per phase-1 ring stage
 
 __device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
@@ -110,8 +109,8 @@ __device__ __forceinline__ bool next_chunk(int64_t& q, int64_t qbeg, int64_t qen
 }
 
 // Phase 1 of one problem, run by CTA `cta` of the `ncta` CTAs given to it.
-__device__ __forceinline__ void w1_body(const CUtensorMap* tm_x, const CUtensorMap* tm_v, const CUtensorMap* tm_xp,
-                                        const CUtensorMap* tm_vp, const W1Args& a, int64_t cta, int64_t ncta) {
+__device__ __forceinline__ void w1_body(const CUtensorMap* tm_x, const CUtensorMap* tm_v, const W1Args& a, int64_t cta,
+                                        int64_t ncta) {
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = align1024(smem_raw);
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + a.bar_off);
@@ -141,8 +140,6 @@ __device__ __forceinline__ void w1_body(const CUtensorMap* tm_x, const CUtensorM
         fence_barrier_init();
         tma_prefetch_desc(tm_x);
         tma_prefetch_desc(tm_v);
-        tma_prefetch_desc(tm_xp);
-        tma_prefetch_desc(tm_vp);
     }
     if (warp == 1) tmem_alloc(tmem_slot, a.tmem_cols);
     tc_fence_before();
@@ -164,29 +161,8 @@ __device__ __forceinline__ void w1_body(const CUtensorMap* tm_x, const CUtensorM
                 const int grp = (int)(row / a.btiles);
                 const int64_t bt = row - (int64_t)grp * a.btiles;
                 const int64_t rbase = row * a.nkb;
-                const int64_t seg_end = rbase + a.nkb < qend ? rbase + a.nkb : qend;
                 for (int64_t qs = q0; qs < q1; qs += kStageBlocks, ++it) {
                     const int nb = (q1 - qs >= kStageBlocks) ? kStageBlocks : (int)(q1 - qs);
-                    // L2 prefetch of X and V^T in 512-byte-wide rows (four k-blocks),
-                    // up to two groups ahead, so that the operand boxes (128-byte
-                    // rows) hit L2.  Only first touches are prefetched: X by the
-                    // CTAs of column group 0 (those of the other groups read the
-                    // same tile side by side), V^T on the first row tile (it stays
-                    // in L2 for the others) -- a prefetch of a resident line still
-                    // costs an L2 transaction, and L2 is this kernel's busiest unit.
-                    const bool pf_x = grp == 0, pf_v = bt == 0;
-                    for (int u = 0; u < nb && (pf_x || pf_v); ++u) {
-                        const int64_t kb = qs + u - rbase;
-                        const bool seg_first = (qs + u == qbeg) || (kb == 0);
-                        if (!seg_first && (kb & (kPfBlocks - 1)) != 0) continue;
-                        const int64_t g0 = kb / kPfBlocks;
-                        for (int64_t pg = seg_first ? g0 : g0 + 2; pg <= g0 + 2; ++pg) {
-                            const int64_t pkb = pg * kPfBlocks;
-                            if (rbase + pkb >= seg_end) break;
-                            if (pf_x) tma_prefetch_2d(tm_xp, (int32_t)(pkb * BK), (int32_t)(bt * BM));
-                            if (pf_v) tma_prefetch_2d(tm_vp, (int32_t)(pkb * BK), grp * a.kgp);
-                        }
-                    }
                     const int slot = it % a.stages;
                     if (!(ok = mbar_wait(&empty[slot], ((it / a.stages) & 1) ^ 1, abort, err, 1u))) break;
                     unsigned char* sp = smem + (size_t)slot * a.slot_bytes;
@@ -323,15 +299,15 @@ __device__ __forceinline__ void w1_body(const CUtensorMap* tm_x, const CUtensorM
 
 __global__ void __launch_bounds__(kThreads, 1)
 apply_w1_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_v,
-                const __grid_constant__ CUtensorMap tm_xp, const __grid_constant__ CUtensorMap tm_vp, const W1Args a) {
-    w1_body(&tm_x, &tm_v, &tm_xp, &tm_vp, a, blockIdx.x, gridDim.x);
+                const W1Args a) {
+    w1_body(&tm_x, &tm_v, a, blockIdx.x, gridDim.x);
 }
 
 // Several problems in one launch: CTA blocks [cta_off[p], cta_off[p + 1]) run
 // problem p with its own arguments and tensor maps.
 constexpr int kMaxGroup = 16;
 struct GroupW1 {
-    CUtensorMap tm[kMaxGroup][4];    // X, V^T, X prefetch, V^T prefetch
+    CUtensorMap tm[kMaxGroup][2];    // X, V^T
     W1Args args[kMaxGroup];
     int cta_off[kMaxGroup + 1];
     int count;
@@ -345,8 +321,7 @@ __device__ __forceinline__ int group_of(const int* off, int count, int64_t blk) 
 
 __global__ void __launch_bounds__(kThreads, 1) apply_w1_group_kernel(const __grid_constant__ GroupW1 g) {
     const int p = group_of(g.cta_off, g.count, blockIdx.x);
-    w1_body(&g.tm[p][0], &g.tm[p][1], &g.tm[p][2], &g.tm[p][3], g.args[p], blockIdx.x - g.cta_off[p],
-            g.cta_off[p + 1] - g.cta_off[p]);
+    w1_body(&g.tm[p][0], &g.tm[p][1], g.args[p], blockIdx.x - g.cta_off[p], g.cta_off[p + 1] - g.cta_off[p]);
 }
 
 // ================================================================ reduction
@@ -410,7 +385,7 @@ __device__ __forceinline__ void w2_body(const W2Args& a, int64_t blk) {
         const int64_t ur = (int64_t)grp * a.btiles + bt;
         const int64_t cf = cta_of(ur * a.nkb, a.Q, a.P1);
         const int64_t cl = cta_of(ur * a.nkb + a.nkb - 1, a.Q, a.P1);
-        constexpr int kBatch = 8;
+        constexpr int kBatch = 4;
         const size_t pstride = (size_t)a.kgp * BM;
         const float* p0 = a.P + ((size_t)(cf + ur) * a.kgp + j0) * BM + r;
         const int64_t np = cl - cf + 1;
@@ -506,7 +481,9 @@ __device__ __forceinline__ void w2_slice_body(const W2Args& a, int64_t blk) {
     put_w8(a, bt, r, col0, w);
 }
 
-__global__ void __launch_bounds__(256)
+// Four CTAs a SM (at most 64 registers a thread): the 576 CTAs of a
+// b = 8192, k' = 144 reduction run in one wave.
+__global__ void __launch_bounds__(256, 4)
 apply_w2_kernel(const W2Args a) {
     pdl_trigger();
     pdl_wait();                    // partials of the phase-1 grid
@@ -976,7 +953,7 @@ struct F16Plan {
     size_t smem1 = 0, smem3 = 0;
     int64_t P1 = 0, P3 = 0, w2_blocks = 0;
     bool slice = false;
-    CUtensorMap tx, tv, txp, tvp, tu, ty;
+    CUtensorMap tx, tv, tu, ty;
 };
 
 lrc_status plan_f16_shape(int64_t m, int64_t n, int64_t k, int64_t b, bool out16, bool bf16, F16Plan& pl) {
@@ -1088,12 +1065,6 @@ lrc_status plan_f16_finish(F16Plan& pl, const void* U, const void* S, const void
     lrc_status st;
     if ((st = make_map(&pl.tx, dt, X, n, b, ldn * 2, BK, BM, "X")) != LRC_OK) return st;
     if ((st = make_map(&pl.tv, dt, Vt, n, k, ldn * 2, BK, (uint32_t)a1.kgp, "Vt")) != LRC_OK) return st;
-    if ((st = make_map(&pl.txp, dt, X, n, b, ldn * 2, kPfBlocks * BK, BM, "X prefetch", CU_TENSOR_MAP_SWIZZLE_NONE)) !=
-        LRC_OK)
-        return st;
-    if ((st = make_map(&pl.tvp, dt, Vt, n, k, ldn * 2, kPfBlocks * BK, (uint32_t)a1.kgp, "Vt prefetch",
-                       CU_TENSOR_MAP_SWIZZLE_NONE)) != LRC_OK)
-        return st;
     if ((st = make_map(&pl.tu, dt, U, k, m, ldk * 2, BK, (uint32_t)a3.n2, "U")) != LRC_OK) return st;
     if ((st = make_y_map(&pl.ty, a3, Y, m, b, out16)) != LRC_OK) return st;
     if (!a3.tma_store) pl.ty = pl.tu;          // unused by the kernel
@@ -1119,7 +1090,7 @@ lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const 
 
     cudaError_t e = cudaFuncSetAttribute(apply_w1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem1);
     if (e != cudaSuccess) return cuda_fail(e, "apply_w1_kernel smem attribute");
-    apply_w1_kernel<<<(unsigned)P1, kThreads, pl.smem1, s>>>(pl.tx, pl.tv, pl.txp, pl.tvp, pl.a1);
+    apply_w1_kernel<<<(unsigned)P1, kThreads, pl.smem1, s>>>(pl.tx, pl.tv, pl.a1);
     if ((st = after_launch("apply_w1_kernel")) != LRC_OK) return st;
     if (pl.slice) {
         e = launch_pdl(apply_w2_slice_kernel, dim3((unsigned)pl.w2_blocks), dim3(32 * kW2Slices), 0, s, pl.a2);
@@ -1182,8 +1153,6 @@ lrc_status launch_apply_f16_group(const ApplyProblem* pr, int count, bool out16,
         ws += f16_ws_bytes(pl, P1[p]);
         g1.tm[p][0] = pl.tx;
         g1.tm[p][1] = pl.tv;
-        g1.tm[p][2] = pl.txp;
-        g1.tm[p][3] = pl.tvp;
         g1.args[p] = pl.a1;
         g1.cta_off[p + 1] = g1.cta_off[p] + (int)P1[p];
         GroupW2& w = g2[pl.slice ? 1 : 0];
