@@ -161,7 +161,7 @@ lrc_status check_apply(const void* U, const void* S, const void* Vt, const void*
 }
 
 lrc_status dispatch_apply(const ApplyProblem& p, lrc_fmt fmt, cudaStream_t s) {
-    if (apply_skinny_takes(plain_fmt(fmt), p.b, p.k))
+    if (apply_skinny_takes(plain_fmt(fmt), p.m, p.n, p.k, p.b))
         return launch_apply_skinny(p.U, p.S, p.Vt, p.X, p.Y, p.m, p.n, p.k, p.b, plain_fmt(fmt), s);
     switch (fmt) {
         case LRC_F64:

@@ -1,6 +1,7 @@
-// apply_skinny.cu -- low-rank apply for batches of at most 16 queries, every
-// format, on the CUDA cores (Sec. 4.4, Eq. gpu_matrix_apply:
-// Y = [(X V) diag(s)] U^T).
+// apply_skinny.cu -- low-rank apply for small batches (Sec. 4.4, Eq.
+// gpu_matrix_apply: Y = [(X V) diag(s)] U^T): at most 16 queries in every
+// format on the CUDA cores, and up to 64 queries in binary16 and bfloat16 on
+// the tensor cores (the second half of the file).
 //
 // With a handful of queries the apply streams the two factors once and does
 // b multiply-adds per factor element: two matrix-vector streams whose speed
@@ -31,6 +32,8 @@
 // factors widened exactly; Sec. 3.4: FP16 products accumulate in FP32).  The
 // summation order is fixed: results are reproducible on a device.
 #include <cuda_fp16.h>
+
+#include <algorithm>
 
 #include "common.cuh"
 #include "tc.cuh"
@@ -410,6 +413,369 @@ skinny_y_kernel(const __grid_constant__ CUtensorMap tm_u, const T* __restrict__ 
     }
 }
 
+// ---------------------------------------------------------------- 16-bit storage on the tensor cores
+// Batches of 2..64 queries in binary16 (1..64 for binary16 output and in
+// bfloat16): the b multiply-adds per factor element would bound the
+// CUDA-core loops, so both products run as tcgen05 MMAs whose N is the query
+// count padded to NB (16, 32 or 64; twice that in the second product for
+// FP32 output, whose hi and lo planes of W sit side by side along N) and
+// whose M is 128 ranks (first product) or 128 rows of U (second).
+//   skinny_tc_w_kernel  grid (chunk of n, tile of 128 ranks) in clusters of
+//                       kTcCluster chunks.  The CTA copies its chunk of V^T
+//                       (128 ranks x cb k-blocks) and of X (the b rows,
+//                       zero-filled to NB) at once, multiplies
+//                       W^T = V^T X^T into one tensor-memory accumulator
+//                       (at most 8 k-blocks: the accumulation length of the
+//                       chunked FP32 accumulation) and stages it in shared
+//                       memory; every CTA of the cluster then adds, for an
+//                       eighth of the entries, the kTcCluster partials in
+//                       rank order through distributed shared memory and
+//                       writes that part of the cluster partial.  The last
+//                       cluster of a rank tile to arrive (a counter) adds
+//                       the cluster partials in cluster order, scales by
+//                       diag(s) and writes W as the second product's operand
+//                       planes: hi and lo binary16 for FP32 output (w = hi +
+//                       lo to about 22 bits), one rounding for 16-bit
+//                       output.
+//   skinny_tc_y_kernel  a CTA per 128 rows of U: the U tile is requested
+//                       before the wait for the first kernel (U is an input
+//                       of the call), W after it; D = U_tile W^T holds the
+//                       tile's outputs for every query (FP32 output: the hi
+//                       and lo halves of D added in binary32), and each
+//                       query's 128 outputs are one coalesced run of stores.
+// Fixed summation orders (tensor core within a chunk, cluster rank, cluster
+// index): results are reproducible on a device.
+constexpr int kTcK = 64;                         // 16-bit elements per 128-byte swizzled row
+constexpr int kTcM = 128;                        // MMA rows
+constexpr int kTcCluster = 8;                    // chunks of n per cluster
+constexpr int kTcMaxChunks = 64;                 // chunks of n per rank tile, at most
+constexpr int kTcMaxBatch = 64;                  // queries, at most
+constexpr int kTcThreadsW = 512;
+constexpr int kTcThreadsY = 128;
+constexpr uint32_t kTcABytes = kTcM * kTcK * 2;  // one 128-row operand box
+
+__device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
+    return p + ((1024u - (tc::smem_u32(p) & 1023u)) & 1023u);
+}
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// Every thread of every CTA of the cluster: shared-memory writes before it
+// are visible to the cluster's reads after it.
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// 16 bytes of the shared memory of cluster CTA `rank` at the offset of the
+// local shared address `addr`.
+__device__ __forceinline__ float4 ld_cluster4(uint32_t addr, uint32_t rank) {
+    uint32_t ra;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(addr), "r"(rank));
+    float4 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(ra)
+                 : "memory");
+    return v;
+}
+
+__device__ __forceinline__ float4 add4(float4 a, float4 b) {
+    return make_float4(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y), __fadd_rn(a.z, b.z), __fadd_rn(a.w, b.w));
+}
+
+struct TcWArgs {
+    int k, kp, b, nkb, cb, nclusters;
+    int planes;               // W planes: 2 (hi and lo, FP32 output) or 1
+    int bf16;                 // bfloat16 storage and W
+    uint32_t idesc;           // MMA instruction descriptor
+    uint32_t bar_off;         // barriers after the tile / fold region
+    const uint16_t* S;
+    float* P;                 // cluster partials [rank tile][cluster][NB queries][128 ranks]
+    uint16_t* W;              // W planes [plane][b][kp]
+    unsigned int* cnt;        // an arrival counter per rank tile
+};
+
+// Shared memory: [region: cb V^T boxes, cb X boxes; later the staged partial
+// (NB x 128 binary32, [query][rank])][cb + 1 barriers][tensor-memory address]
+// [abort flag].
+template <int NB>
+__global__ void __launch_bounds__(kTcThreadsW, 1)
+skinny_tc_w_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_x, const TcWArgs a) {
+    constexpr uint32_t kXBytes = NB * kTcK * 2;
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* smem = align1024(smem_raw);
+    unsigned char* vs = smem;
+    unsigned char* xs = smem + (size_t)a.cb * kTcABytes;
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + a.bar_off);
+    uint64_t* mma_done = full + a.cb;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+    volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    __shared__ int last_cluster;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int chunk = blockIdx.x, rt = blockIdx.y;
+    const int kb0 = chunk * a.cb;
+    const int nb = a.nkb - kb0 < a.cb ? (a.nkb - kb0 > 0 ? a.nkb - kb0 : 0) : a.cb;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < a.cb + 1; ++i) tc::mbar_init(&full[i], 1);
+        *abort = 0;
+        tc::fence_barrier_init();
+        tc::tma_prefetch_desc(&tm_v);
+        tc::tma_prefetch_desc(&tm_x);
+    }
+    constexpr uint32_t kCols = NB < 32 ? 32u : (uint32_t)NB;
+    if (warp == 1) tc::tmem_alloc(tmem_slot, kCols);
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    tc::pdl_wait();                  // X, V^T, s and the workspace are the previous kernels'
+    if (threadIdx.x == 0)
+        for (int i = 0; i < nb; ++i) {
+            tc::mbar_arrive_expect_tx(&full[i], kTcABytes + kXBytes);
+            const int32_t x = (kb0 + i) * kTcK;
+            tc::tma_load_2d(vs + (size_t)i * kTcABytes, &tm_v, x, rt * kTcM, &full[i]);
+            tc::tma_load_2d(xs + (size_t)i * kXBytes, &tm_x, x, 0, &full[i]);
+        }
+    tc::pdl_trigger();               // the second product streams U meanwhile
+    if (threadIdx.x == 0) {
+        int i = 0;
+        for (; i < nb; ++i) {
+            if (!tc::mbar_wait(&full[i], 0, abort, &g_err_skinny, 8u)) break;
+            tc::tc_fence_after();
+            const uint64_t dv = tc::desc_sw128(tc::smem_u32(vs + (size_t)i * kTcABytes));
+            const uint64_t dx = tc::desc_sw128(tc::smem_u32(xs + (size_t)i * kXBytes));
+#pragma unroll
+            for (int kk = 0; kk < kTcK / 16; ++kk)
+                tc::mma_f16(tmem, dv + 2 * kk, dx + 2 * kk, a.idesc, (i | kk) != 0 ? 1u : 0u);
+        }
+        tc::mma_commit(mma_done);    // also after a give-up: the MMAs issued finish first
+        volatile int no_abort = 0;
+        tc::mbar_wait(mma_done, 0, &no_abort, &g_err_skinny, 8u, 100000000ull);
+        for (int j = i; j < nb; ++j)  // copies still landing
+            tc::mbar_wait(&full[j], 0, &no_abort, &g_err_skinny, 8u, 100000000ull);
+    }
+    __syncwarp();
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    // the partial, staged as [query][rank] (the operand boxes are no longer read)
+    float* stage = reinterpret_cast<float*>(smem);
+    if (warp < 4) {
+        const int r = warp * 32 + lane;
+#pragma unroll
+        for (int c0 = 0; c0 < NB; c0 += 32) {
+            uint32_t v[32];
+            tc::tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+            tc::tmem_ld_wait();
+#pragma unroll
+            for (int q = 0; q < (NB < 32 ? NB : 32); ++q)
+                stage[(c0 + q) * kTcM + r] = nb > 0 ? __uint_as_float(v[q]) : 0.0f;
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, kCols);
+    }
+    __syncwarp();
+    cluster_sync();                  // every partial of the cluster is staged
+    // The cluster partial: CTA j of the cluster adds, for its eighth of the
+    // (query, 4 ranks) entries, the kTcCluster staged partials in rank order.
+    const int cl = chunk / kTcCluster;
+    const int crank = (int)cluster_ctarank();
+    const int n4 = a.b * (kTcM / 4);
+    float4* cp = reinterpret_cast<float4*>(a.P + ((size_t)rt * a.nclusters + cl) * NB * kTcM);
+    for (int e = n4 * crank / kTcCluster + (int)threadIdx.x; e < n4 * (crank + 1) / kTcCluster;
+         e += kTcThreadsW) {
+        {
+            const uint32_t addr = tc::smem_u32(stage) + 16u * (uint32_t)e;
+            float4 v[kTcCluster];
+#pragma unroll
+            for (int r = 0; r < kTcCluster; ++r) v[r] = ld_cluster4(addr, (uint32_t)r);
+            float4 sum = v[0];
+#pragma unroll
+            for (int r = 1; r < kTcCluster; ++r) sum = add4(sum, v[r]);
+            cp[e] = sum;
+        }
+    }
+    __syncwarp();
+    cluster_sync();                  // the staged partials stay until every CTA has read them
+    if (crank != 0) return;
+    // the cluster's first CTA arrives for the cluster (the cluster barrier
+    // ordered the other CTAs' partial stores before this release)
+    if (threadIdx.x == 0) last_cluster = arrive_acq_rel(&a.cnt[rt]) == (unsigned)(a.nclusters - 1);
+    __syncthreads();
+    if (!last_cluster) return;
+    // The rank tile's cluster partials added in cluster order, scaled by
+    // diag(s), written as W.  Thread t takes ranks 4 (t % 32) .. + 3 of
+    // queries t / 32, t / 32 + 16, ...
+    const int ranks = a.kp - rt * kTcM < kTcM ? a.kp - rt * kTcM : kTcM;
+    const int r4 = (int)(threadIdx.x & 31) * 4;
+    if (r4 >= ranks) return;                       // ranks is a multiple of 16
+    const int j0 = rt * kTcM + r4;
+    float sj[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int j = j0 + i;
+        sj[i] = 0.0f;
+        if (j < a.k) sj[i] = a.bf16 ? tc::bf16_bits_to_float(a.S[j]) : __half2float(__ushort_as_half(a.S[j]));
+    }
+    const float4* src = reinterpret_cast<const float4*>(a.P + (size_t)rt * a.nclusters * NB * kTcM);
+    constexpr int kC4 = NB * kTcM / 4;             // float4 per cluster partial
+    const size_t plane = (size_t)a.b * a.kp;
+    for (int q = (int)(threadIdx.x >> 5); q < a.b; q += kTcThreadsW / 32) {
+        const int e = q * (kTcM / 4) + (r4 >> 2);
+        float4 v[kTcMaxChunks / kTcCluster];
+#pragma unroll
+        for (int c = 0; c < kTcMaxChunks / kTcCluster; ++c)
+            v[c] = c < a.nclusters ? __ldcg(src + (size_t)c * kC4 + e) : make_float4(0.f, 0.f, 0.f, 0.f);
+        float4 sum = v[0];
+#pragma unroll
+        for (int c = 1; c < kTcMaxChunks / kTcCluster; ++c)
+            if (c < a.nclusters) sum = add4(sum, v[c]);
+        const float w[4] = {__fmul_rn(sum.x, sj[0]), __fmul_rn(sum.y, sj[1]), __fmul_rn(sum.z, sj[2]),
+                            __fmul_rn(sum.w, sj[3])};
+        uint16_t hi[4], lo[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (a.bf16) {
+                hi[i] = tc::to_bf16_bits(w[i]);
+            } else {
+                const __half h = __float2half_rn(w[i]);
+                hi[i] = __half_as_ushort(h);
+                lo[i] = __half_as_ushort(__float2half_rn(w[i] - __half2float(h)));
+            }
+        }
+        uint16_t* dst = a.W + (size_t)q * a.kp + j0;     // 8-byte aligned: j0 and kp are multiples of 4
+        *reinterpret_cast<uint2*>(dst) = make_uint2(hi[0] | ((uint32_t)hi[1] << 16), hi[2] | ((uint32_t)hi[3] << 16));
+        if (a.planes == 2)
+            *reinterpret_cast<uint2*>(dst + plane) =
+                make_uint2(lo[0] | ((uint32_t)lo[1] << 16), lo[2] | ((uint32_t)lo[3] << 16));
+    }
+}
+
+struct TcYArgs {
+    int64_t m;
+    int b, kp, kc, planes, rtiles;
+    int out16, bf16;          // 16-bit output (bfloat16 when bf16)
+    uint32_t idesc;
+    unsigned int* cnt;        // the first kernel's counters, left at zero for the next call
+    void* Y;
+};
+
+// Shared memory: [U: kc boxes of 128 rows][W: kc x planes boxes of NB rows,
+// the lo box of a k-block right after its hi box, so that the two form one
+// B operand of planes x NB rows: D = [U W_hi^T | U W_lo^T]]
+// [3 barriers][tensor-memory address][abort flag].
+template <int NB>
+__global__ void __launch_bounds__(kTcThreadsY, 1)
+skinny_tc_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__ CUtensorMap tm_w0,
+                   const __grid_constant__ CUtensorMap tm_w1, const TcYArgs a) {
+    constexpr uint32_t kWBytes = NB * kTcK * 2;
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* smem = align1024(smem_raw);
+    unsigned char* us = smem;
+    unsigned char* ws = smem + (size_t)a.kc * kTcABytes;
+    uint64_t* bar = reinterpret_cast<uint64_t*>(ws + (size_t)a.planes * a.kc * kWBytes);   // U, W, MMA
+    const uint32_t tcols = a.planes * NB <= 32 ? 32u : (uint32_t)(a.planes * NB);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + 3);
+    volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t row0 = (int64_t)blockIdx.x * kTcM;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
+        *abort = 0;
+        tc::fence_barrier_init();
+        tc::tma_prefetch_desc(&tm_u);
+        tc::tma_prefetch_desc(&tm_w0);
+        tc::tma_prefetch_desc(&tm_w1);
+        tc::mbar_arrive_expect_tx(&bar[0], (uint32_t)a.kc * kTcABytes);
+        for (int i = 0; i < a.kc; ++i) tc::tma_load_2d(us + (size_t)i * kTcABytes, &tm_u, i * kTcK, (int32_t)row0, &bar[0]);
+    }
+    if (warp == 1) tc::tmem_alloc(tmem_slot, tcols);
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    tc::pdl_trigger();               // the next call's first kernel may set up
+    if (threadIdx.x == 0) {
+        tc::pdl_wait();              // W of the first kernel
+        if (blockIdx.x == 0)         // also after an aborted first kernel
+            for (int i = 0; i < a.rtiles; ++i) a.cnt[i] = 0u;
+        tc::mbar_arrive_expect_tx(&bar[1], (uint32_t)(a.planes * a.kc) * kWBytes);
+        for (int p = 0; p < a.planes; ++p)
+            for (int i = 0; i < a.kc; ++i)
+                tc::tma_load_2d(ws + (size_t)(i * a.planes + p) * kWBytes, p ? &tm_w1 : &tm_w0, i * kTcK, 0, &bar[1]);
+        const bool ok = tc::mbar_wait(&bar[0], 0, abort, &g_err_skinny, 32u) &&
+                        tc::mbar_wait(&bar[1], 0, abort, &g_err_skinny, 32u);
+        if (ok) {
+            tc::tc_fence_after();
+            for (int i = 0; i < a.kc; ++i) {
+                const uint64_t du = tc::desc_sw128(tc::smem_u32(us + (size_t)i * kTcABytes));
+                const uint64_t dw = tc::desc_sw128(tc::smem_u32(ws + (size_t)i * a.planes * kWBytes));
+#pragma unroll
+                for (int kk = 0; kk < kTcK / 16; ++kk) {
+                    if ((i * kTcK + kk * 16) >= a.kp) break;
+                    tc::mma_f16(tmem, du + 2 * kk, dw + 2 * kk, a.idesc, (i | kk) != 0 ? 1u : 0u);
+                }
+            }
+        }
+        tc::mma_commit(&bar[2]);
+        volatile int no_abort = 0;
+        tc::mbar_wait(&bar[2], 0, &no_abort, &g_err_skinny, 32u, 100000000ull);
+        if (!ok)                     // no copy may still be landing when the CTA exits
+            for (int i = 0; i < 2; ++i) tc::mbar_wait(&bar[i], 0, &no_abort, &g_err_skinny, 32u, 100000000ull);
+    }
+    __syncwarp();
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    if (!*abort) {
+        // columns 0..NB-1: U W_hi^T (or U W^T); NB..2 NB-1: U W_lo^T; 32 queries at a time
+        const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
+        const int64_t row = row0 + warp * 32 + lane;
+#pragma unroll 1
+        for (int c0 = 0; c0 < NB && c0 < a.b; c0 += 32) {
+        uint32_t v[32], vl[32];
+        tc::tmem_ld32(tl + (uint32_t)c0, v);
+        if constexpr (NB >= 32)
+            if (a.planes == 2) tc::tmem_ld32(tl + (uint32_t)(NB + c0), vl);
+        tc::tmem_ld_wait();
+        if (row < a.m) {
+#pragma unroll
+            for (int qq = 0; qq < (NB < 32 ? NB : 32); ++qq) {
+                const int q = c0 + qq;
+                if (q >= a.b) break;
+                float y = __uint_as_float(v[qq]);
+                if (a.planes == 2) {
+                    if constexpr (NB >= 32) y = __fadd_rn(y, __uint_as_float(vl[qq]));
+                    else y = __fadd_rn(y, __uint_as_float(v[NB + qq]));
+                }
+                if (!a.out16) {
+                    static_cast<float*>(a.Y)[(int64_t)q * a.m + row] = y;
+                } else {
+                    const uint16_t h = a.bf16 ? tc::to_bf16_bits(y) : __half_as_ushort(__float2half_rn(y));
+                    static_cast<uint16_t*>(a.Y)[(int64_t)q * a.m + row] = h;
+                }
+            }
+        }
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, tcols);
+    }
+}
+
 // lanes per row group of the second product (binary64 stays at 8: its
 // multiply-adds, not the latency of the chain, bound it)
 constexpr int y_group(int B, int64_t e) { return (B <= 4 && e < 8) ? 32 : 8; }
@@ -524,15 +890,143 @@ lrc_status launch_skinny_t(const TS* U, const TS* S, const TS* Vt, const TS* X, 
     return LRC_ERR_UNSUPPORTED;
 }
 
+// Plan of the tensor-core variant: k-blocks per chunk (at most 8, at most
+// kTcMaxChunks chunks), clusters, shared memory of both kernels.
+struct TcPlan {
+    int kp, kc, rtiles, nkb, cb, nchunks, nclusters, planes;
+    size_t region, smem1, smem3;
+};
+
+TcPlan plan_skinny_tc(int64_t n, int64_t k, int64_t b, int NB, bool fp32_out) {
+    TcPlan p{};
+    p.kp = (int)((k + 15) / 16 * 16);
+    p.kc = (p.kp + kTcK - 1) / kTcK;
+    p.rtiles = (p.kp + kTcM - 1) / kTcM;
+    p.nkb = (int)((n + kTcK - 1) / kTcK);
+    p.cb = (p.nkb + kTcMaxChunks - 1) / kTcMaxChunks;
+    if (p.cb < 1) p.cb = 1;
+    p.nchunks = (p.nkb + p.cb - 1) / p.cb;
+    p.nclusters = (p.nchunks + kTcCluster - 1) / kTcCluster;
+    p.planes = fp32_out ? 2 : 1;
+    size_t region = (size_t)p.cb * (kTcABytes + (size_t)NB * kTcK * 2);
+    region = std::max(region, (size_t)NB * kTcM * 4);                       // the staged partial
+    p.region = (region + 15) / 16 * 16;
+    p.smem1 = 1024 + p.region + 8 * (size_t)(p.cb + 1) + 16;
+    p.smem3 = 1024 + (size_t)p.kc * kTcABytes + (size_t)p.planes * p.kc * NB * kTcK * 2 + 3 * 8 + 16;
+    return p;
+}
+
+// MMA width (queries) for b queries
+int tc_width(int64_t b) { return b <= 16 ? 16 : (b <= 32 ? 32 : 64); }
+
+bool skinny_tc_takes(lrc_fmt fmt, int64_t m, int64_t n, int64_t k, int64_t b) {
+    if (fmt != LRC_F16 && fmt != LRC_F16_O16 && fmt != LRC_BF16) return false;
+    // one binary16 query with FP32 output stays on the CUDA cores (about 0.5 us faster there)
+    const int64_t bmin = fmt == LRC_F16 ? 2 : 1;
+    if (b < bmin || b > kTcMaxBatch || k < 1 || k > 512 || n < 1 || m < 1 || m > INT32_MAX) return false;
+    if ((n + kTcK - 1) / kTcK > 8 * kTcMaxChunks) return false;     // at most 8 k-blocks per chunk
+    const TcPlan p = plan_skinny_tc(n, k, b, tc_width(b), fmt == LRC_F16);
+    return p.smem1 <= kSmemMaxS && p.smem3 <= kSmemMaxS;
+}
+
+template <int NB>
+lrc_status launch_skinny_tc_nb(const void* U, const void* S, const void* Vt, const void* X, void* Y, int64_t m,
+                               int64_t n, int64_t k, int64_t b, lrc_fmt fmt, cudaStream_t s) {
+    const bool bf16 = fmt == LRC_BF16;
+    const TcPlan p = plan_skinny_tc(n, k, b, NB, fmt == LRC_F16);
+    const size_t part_bytes = ((size_t)p.rtiles * p.nclusters * NB * kTcM * 4 + 255) / 256 * 256;
+    const size_t w_bytes = (size_t)p.planes * b * p.kp * 2;
+    void* ws = nullptr;
+    lrc_status st = stream_workspace(s, part_bytes + w_bytes, &ws);
+    if (st != LRC_OK) return st;
+    unsigned int* cnt = nullptr;
+    if ((st = stream_counters(s, &cnt)) != LRC_OK) return st;
+    float* P = static_cast<float*>(ws);
+    uint16_t* W = reinterpret_cast<uint16_t*>(static_cast<unsigned char*>(ws) + part_bytes);
+
+    const CUtensorMapDataType dt = bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+    const int64_t ldn = lrc_packed_ld(n), ldk = lrc_packed_ld(k);
+    CUtensorMap tv, tx, tu, tw0, tw1;
+    if ((st = encode_map_2d(&tv, dt, Vt, n, k, ldn * 2, kTcK, kTcM, true, "Vt")) != LRC_OK) return st;
+    if ((st = encode_map_2d(&tx, dt, X, n, b, ldn * 2, kTcK, NB, true, "X")) != LRC_OK) return st;
+    if ((st = encode_map_2d(&tu, dt, U, k, m, ldk * 2, kTcK, kTcM, true, "U")) != LRC_OK) return st;
+    if ((st = encode_map_2d(&tw0, dt, W, p.kp, b, (int64_t)p.kp * 2, kTcK, NB, true, "W")) != LRC_OK) return st;
+    tw1 = tw0;
+    if (p.planes == 2 &&
+        (st = encode_map_2d(&tw1, dt, W + (size_t)b * p.kp, p.kp, b, (int64_t)p.kp * 2, kTcK, NB, true, "W lo")) !=
+            LRC_OK)
+        return st;
+    const uint32_t ab = bf16 ? tc::kIdescBF16 : 0u;
+
+    TcWArgs a1{};
+    a1.k = (int)k;
+    a1.kp = p.kp;
+    a1.b = (int)b;
+    a1.nkb = p.nkb;
+    a1.cb = p.cb;
+    a1.nclusters = p.nclusters;
+    a1.planes = p.planes;
+    a1.bf16 = bf16 ? 1 : 0;
+    a1.idesc = tc::idesc_f16_f32(kTcM, NB) | ab;
+    a1.bar_off = (uint32_t)p.region;
+    a1.S = static_cast<const uint16_t*>(S);
+    a1.P = P;
+    a1.W = W;
+    a1.cnt = cnt;
+    cudaError_t ce = cudaFuncSetAttribute(skinny_tc_w_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)p.smem1);
+    if (ce != cudaSuccess) return cuda_fail(ce, "skinny_tc_w_kernel smem attribute");
+    {
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3((unsigned)(p.nclusters * kTcCluster), (unsigned)p.rtiles);
+        cfg.blockDim = dim3(kTcThreadsW);
+        cfg.dynamicSmemBytes = p.smem1;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[2];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = kTcCluster;
+        attr[1].val.clusterDim.y = 1;
+        attr[1].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 2;
+        ce = cudaLaunchKernelEx(&cfg, skinny_tc_w_kernel<NB>, tv, tx, a1);
+    }
+    if (ce != cudaSuccess) return cuda_fail(ce, "skinny_tc_w_kernel launch");
+    if ((st = after_launch("skinny_tc_w_kernel")) != LRC_OK) return st;
+
+    TcYArgs a3{};
+    a3.m = m;
+    a3.b = (int)b;
+    a3.kp = p.kp;
+    a3.kc = p.kc;
+    a3.planes = p.planes;
+    a3.rtiles = p.rtiles;
+    a3.out16 = fmt == LRC_F16 ? 0 : 1;
+    a3.bf16 = bf16 ? 1 : 0;
+    a3.idesc = tc::idesc_f16_f32(kTcM, (uint32_t)(p.planes * NB)) | ab;
+    a3.cnt = cnt;
+    a3.Y = Y;
+    ce = cudaFuncSetAttribute(skinny_tc_y_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem3);
+    if (ce != cudaSuccess) return cuda_fail(ce, "skinny_tc_y_kernel smem attribute");
+    ce = launch_pdl(skinny_tc_y_kernel<NB>, dim3((unsigned)((m + kTcM - 1) / kTcM)), dim3(kTcThreadsY), p.smem3, s, tu,
+                    tw0, tw1, a3);
+    if (ce != cudaSuccess) return cuda_fail(ce, "skinny_tc_y_kernel launch");
+    return after_launch("skinny_tc_y_kernel");
+}
+
 int64_t max_batch(lrc_fmt fmt) { return fmt == LRC_F16 || fmt == LRC_F16_O16 ? 4 : 16; }
 
 }  // namespace
 
-// Batches this path takes: up to 16 queries for binary32 and binary64, up
-// to 4 for binary16 (whose tensor-core path is faster from 16 queries on);
-// ranks whose tiles fit in shared memory.
-bool apply_skinny_takes(lrc_fmt fmt, int64_t b, int64_t k) {
-    if (fmt == LRC_BF16) return false;    // bfloat16 takes the tensor-core path at every batch size
+// Batches this path takes: up to 16 queries for binary32 and binary64 and
+// up to 4 for binary16 on the CUDA cores, ranks whose tiles fit in shared
+// memory; 5..32 queries in binary16 and up to 32 in bfloat16 on the tensor
+// cores (rank at most 512, n at most 32768).
+bool apply_skinny_takes(lrc_fmt fmt, int64_t m, int64_t n, int64_t k, int64_t b) {
+    if (skinny_tc_takes(fmt, m, n, k, b)) return true;
+    if (fmt == LRC_BF16) return false;
     if (b < 1 || b > max_batch(fmt) || k < 1 || k > 1024) return false;
     const int B = b <= 1 ? 1 : (b <= 4 ? 4 : (b <= 8 ? 8 : 16));
     const int64_t e = storage_bytes(fmt);
@@ -542,9 +1036,16 @@ bool apply_skinny_takes(lrc_fmt fmt, int64_t b, int64_t k) {
 
 lrc_status launch_apply_skinny(const void* U, const void* S, const void* Vt, const void* X, void* Y, int64_t m,
                                int64_t n, int64_t k, int64_t b, lrc_fmt fmt, cudaStream_t s) {
-    if (!apply_skinny_takes(fmt, b, k)) {
+    if (!apply_skinny_takes(fmt, m, n, k, b)) {
         set_error("small-batch apply: b = %lld, k = %lld outside the kernel", (long long)b, (long long)k);
         return LRC_ERR_UNSUPPORTED;
+    }
+    if (skinny_tc_takes(fmt, m, n, k, b)) {
+        switch (tc_width(b)) {
+            case 16: return launch_skinny_tc_nb<16>(U, S, Vt, X, Y, m, n, k, b, fmt, s);
+            case 32: return launch_skinny_tc_nb<32>(U, S, Vt, X, Y, m, n, k, b, fmt, s);
+            default: return launch_skinny_tc_nb<64>(U, S, Vt, X, Y, m, n, k, b, fmt, s);
+        }
     }
     switch (fmt) {
         case LRC_F64:
