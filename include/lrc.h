@@ -153,10 +153,10 @@ LRC_API lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows,
  * per-chunk partial sums in the same workspace and keep a per-stream buffer
  * of 1024 arrival counters (zeroed once when made, left at zero by every
  * call, freed by lrc_shutdown()): at most 16 queries in binary64 and
- * binary32 and 4 in binary16 on the CUDA cores, and up to 64 queries in
- * binary16 (from 2 for LRC_F16) and bfloat16 as two tensor-core products
- * when n <= 32768 and k <= 512 (the second product's tiles must fit in
- * shared memory).  Binary16 ranks: up to 320 for LRC_F16 and 512 for
+ * binary32 on the CUDA cores (binary16 too when the tensor-core products
+ * do not take the shape), and up to 64 queries in binary16 and bfloat16 as
+ * two tensor-core products when n <= 32768 and k <= 512 (the second
+ * product's tiles must fit in shared memory).  Binary16 ranks: up to 320 for LRC_F16 and 512 for
  * LRC_F16_O16, else LRC_ERR_UNSUPPORTED.
  */
 /* LRC_F32_TC: as LRC_F32, with the second product (W U^T) on the tensor

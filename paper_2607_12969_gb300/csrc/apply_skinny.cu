@@ -414,9 +414,9 @@ skinny_y_kernel(const __grid_constant__ CUtensorMap tm_u, const T* __restrict__ 
 }
 
 // ---------------------------------------------------------------- 16-bit storage on the tensor cores
-// Batches of 2..64 queries in binary16 (1..64 for binary16 output and in
-// bfloat16): the b multiply-adds per factor element would bound the
-// CUDA-core loops, so both products run as tcgen05 MMAs whose N is the query
+// Batches of at most 64 queries in binary16 and bfloat16: the b
+// multiply-adds per factor element would bound the CUDA-core loops, so both
+// products run as tcgen05 MMAs whose N is the query
 // count padded to NB (16, 32 or 64; twice that in the second product for
 // FP32 output, whose hi and lo planes of W sit side by side along N) and
 // whose M is 128 ranks (first product) or 128 rows of U (second).
@@ -436,10 +436,13 @@ skinny_y_kernel(const __grid_constant__ CUtensorMap tm_u, const T* __restrict__ 
 //                       diag(s) and writes W as the second product's operand
 //                       planes: hi and lo binary16 for FP32 output (w = hi +
 //                       lo to about 22 bits), one rounding for 16-bit
-//                       output.
+//                       output, laid out as the second product's shared
+//                       memory image (k-blocks of NB rows x 128 bytes in the
+//                       128-byte swizzle, the lo box after the hi box).
 //   skinny_tc_y_kernel  a CTA per 128 rows of U: the U tile is requested
 //                       before the wait for the first kernel (U is an input
-//                       of the call), W after it; D = U_tile W^T holds the
+//                       of the call), W after it (one bulk copy of the
+//                       image); D = U_tile W^T holds the
 //                       tile's outputs for every query (FP32 output: the hi
 //                       and lo halves of D added in binary32), and each
 //                       query's 128 outputs are one coalesced run of stores.
@@ -495,7 +498,7 @@ struct TcWArgs {
     uint32_t bar_off;         // barriers after the tile / fold region
     const uint16_t* S;
     float* P;                 // cluster partials [rank tile][cluster][NB queries][128 ranks]
-    uint16_t* W;              // W planes [plane][b][kp]
+    unsigned char* W;         // W image: [k-block][plane][NB rows x 128 bytes, 128-byte swizzle]
     unsigned int* cnt;        // an arrival counter per rank tile
 };
 
@@ -628,7 +631,9 @@ skinny_tc_w_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_consta
     }
     const float4* src = reinterpret_cast<const float4*>(a.P + (size_t)rt * a.nclusters * NB * kTcM);
     constexpr int kC4 = NB * kTcM / 4;             // float4 per cluster partial
-    const size_t plane = (size_t)a.b * a.kp;
+    constexpr uint32_t kBox = NB * 128;            // bytes of one W box
+    // the 4 ranks j0.. lie in 16-byte chunk (j0 % 64) / 8 of a 128-byte row of k-block j0 / 64
+    const int kblk = j0 >> 6, ch = (j0 & 63) >> 3, within = (j0 & 7) * 2;
     for (int q = (int)(threadIdx.x >> 5); q < a.b; q += kTcThreadsW / 32) {
         const int e = q * (kTcM / 4) + (r4 >> 2);
         float4 v[kTcMaxChunks / kTcCluster];
@@ -652,10 +657,10 @@ skinny_tc_w_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_consta
                 lo[i] = __half_as_ushort(__float2half_rn(w[i] - __half2float(h)));
             }
         }
-        uint16_t* dst = a.W + (size_t)q * a.kp + j0;     // 8-byte aligned: j0 and kp are multiples of 4
+        unsigned char* dst = a.W + ((size_t)kblk * a.planes * NB + q) * 128 + ((ch ^ (q & 7)) << 4) + within;
         *reinterpret_cast<uint2*>(dst) = make_uint2(hi[0] | ((uint32_t)hi[1] << 16), hi[2] | ((uint32_t)hi[3] << 16));
         if (a.planes == 2)
-            *reinterpret_cast<uint2*>(dst + plane) =
+            *reinterpret_cast<uint2*>(dst + kBox) =
                 make_uint2(lo[0] | ((uint32_t)lo[1] << 16), lo[2] | ((uint32_t)lo[3] << 16));
     }
 }
@@ -666,6 +671,7 @@ struct TcYArgs {
     int out16, bf16;          // 16-bit output (bfloat16 when bf16)
     uint32_t idesc;
     unsigned int* cnt;        // the first kernel's counters, left at zero for the next call
+    const unsigned char* W;   // the first kernel's W image (rows b..NB-1 unused: their D columns are not stored)
     void* Y;
 };
 
@@ -675,8 +681,7 @@ struct TcYArgs {
 // [3 barriers][tensor-memory address][abort flag].
 template <int NB>
 __global__ void __launch_bounds__(kTcThreadsY, 1)
-skinny_tc_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_constant__ CUtensorMap tm_w0,
-                   const __grid_constant__ CUtensorMap tm_w1, const TcYArgs a) {
+skinny_tc_y_kernel(const __grid_constant__ CUtensorMap tm_u, const TcYArgs a) {
     constexpr uint32_t kWBytes = NB * kTcK * 2;
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = align1024(smem_raw);
@@ -693,8 +698,6 @@ skinny_tc_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_consta
         *abort = 0;
         tc::fence_barrier_init();
         tc::tma_prefetch_desc(&tm_u);
-        tc::tma_prefetch_desc(&tm_w0);
-        tc::tma_prefetch_desc(&tm_w1);
         tc::mbar_arrive_expect_tx(&bar[0], (uint32_t)a.kc * kTcABytes);
         for (int i = 0; i < a.kc; ++i) tc::tma_load_2d(us + (size_t)i * kTcABytes, &tm_u, i * kTcK, (int32_t)row0, &bar[0]);
     }
@@ -708,10 +711,9 @@ skinny_tc_y_kernel(const __grid_constant__ CUtensorMap tm_u, const __grid_consta
         tc::pdl_wait();              // W of the first kernel
         if (blockIdx.x == 0)         // also after an aborted first kernel
             for (int i = 0; i < a.rtiles; ++i) a.cnt[i] = 0u;
-        tc::mbar_arrive_expect_tx(&bar[1], (uint32_t)(a.planes * a.kc) * kWBytes);
-        for (int p = 0; p < a.planes; ++p)
-            for (int i = 0; i < a.kc; ++i)
-                tc::tma_load_2d(ws + (size_t)(i * a.planes + p) * kWBytes, p ? &tm_w1 : &tm_w0, i * kTcK, 0, &bar[1]);
+        const uint32_t w_bytes = (uint32_t)(a.planes * a.kc) * kWBytes;
+        tc::mbar_arrive_expect_tx(&bar[1], w_bytes);
+        tc::bulk_load(ws, a.W, w_bytes, &bar[1]);
         const bool ok = tc::mbar_wait(&bar[0], 0, abort, &g_err_skinny, 32u) &&
                         tc::mbar_wait(&bar[1], 0, abort, &g_err_skinny, 32u);
         if (ok) {
@@ -921,9 +923,7 @@ int tc_width(int64_t b) { return b <= 16 ? 16 : (b <= 32 ? 32 : 64); }
 
 bool skinny_tc_takes(lrc_fmt fmt, int64_t m, int64_t n, int64_t k, int64_t b) {
     if (fmt != LRC_F16 && fmt != LRC_F16_O16 && fmt != LRC_BF16) return false;
-    // one binary16 query with FP32 output stays on the CUDA cores (about 0.5 us faster there)
-    const int64_t bmin = fmt == LRC_F16 ? 2 : 1;
-    if (b < bmin || b > kTcMaxBatch || k < 1 || k > 512 || n < 1 || m < 1 || m > INT32_MAX) return false;
+    if (b < 1 || b > kTcMaxBatch || k < 1 || k > 512 || n < 1 || m < 1 || m > INT32_MAX) return false;
     if ((n + kTcK - 1) / kTcK > 8 * kTcMaxChunks) return false;     // at most 8 k-blocks per chunk
     const TcPlan p = plan_skinny_tc(n, k, b, tc_width(b), fmt == LRC_F16);
     return p.smem1 <= kSmemMaxS && p.smem3 <= kSmemMaxS;
@@ -935,27 +935,21 @@ lrc_status launch_skinny_tc_nb(const void* U, const void* S, const void* Vt, con
     const bool bf16 = fmt == LRC_BF16;
     const TcPlan p = plan_skinny_tc(n, k, b, NB, fmt == LRC_F16);
     const size_t part_bytes = ((size_t)p.rtiles * p.nclusters * NB * kTcM * 4 + 255) / 256 * 256;
-    const size_t w_bytes = (size_t)p.planes * b * p.kp * 2;
+    const size_t w_bytes = (size_t)p.planes * p.kc * NB * 128;     // the W image
     void* ws = nullptr;
     lrc_status st = stream_workspace(s, part_bytes + w_bytes, &ws);
     if (st != LRC_OK) return st;
     unsigned int* cnt = nullptr;
     if ((st = stream_counters(s, &cnt)) != LRC_OK) return st;
     float* P = static_cast<float*>(ws);
-    uint16_t* W = reinterpret_cast<uint16_t*>(static_cast<unsigned char*>(ws) + part_bytes);
+    unsigned char* W = static_cast<unsigned char*>(ws) + part_bytes;
 
     const CUtensorMapDataType dt = bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
     const int64_t ldn = lrc_packed_ld(n), ldk = lrc_packed_ld(k);
-    CUtensorMap tv, tx, tu, tw0, tw1;
+    CUtensorMap tv, tx, tu;
     if ((st = encode_map_2d(&tv, dt, Vt, n, k, ldn * 2, kTcK, kTcM, true, "Vt")) != LRC_OK) return st;
     if ((st = encode_map_2d(&tx, dt, X, n, b, ldn * 2, kTcK, NB, true, "X")) != LRC_OK) return st;
     if ((st = encode_map_2d(&tu, dt, U, k, m, ldk * 2, kTcK, kTcM, true, "U")) != LRC_OK) return st;
-    if ((st = encode_map_2d(&tw0, dt, W, p.kp, b, (int64_t)p.kp * 2, kTcK, NB, true, "W")) != LRC_OK) return st;
-    tw1 = tw0;
-    if (p.planes == 2 &&
-        (st = encode_map_2d(&tw1, dt, W + (size_t)b * p.kp, p.kp, b, (int64_t)p.kp * 2, kTcK, NB, true, "W lo")) !=
-            LRC_OK)
-        return st;
     const uint32_t ab = bf16 ? tc::kIdescBF16 : 0u;
 
     TcWArgs a1{};
@@ -1007,11 +1001,12 @@ lrc_status launch_skinny_tc_nb(const void* U, const void* S, const void* Vt, con
     a3.bf16 = bf16 ? 1 : 0;
     a3.idesc = tc::idesc_f16_f32(kTcM, (uint32_t)(p.planes * NB)) | ab;
     a3.cnt = cnt;
+    a3.W = W;
     a3.Y = Y;
     ce = cudaFuncSetAttribute(skinny_tc_y_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem3);
     if (ce != cudaSuccess) return cuda_fail(ce, "skinny_tc_y_kernel smem attribute");
     ce = launch_pdl(skinny_tc_y_kernel<NB>, dim3((unsigned)((m + kTcM - 1) / kTcM)), dim3(kTcThreadsY), p.smem3, s, tu,
-                    tw0, tw1, a3);
+                    a3);
     if (ce != cudaSuccess) return cuda_fail(ce, "skinny_tc_y_kernel launch");
     return after_launch("skinny_tc_y_kernel");
 }
@@ -1020,10 +1015,10 @@ int64_t max_batch(lrc_fmt fmt) { return fmt == LRC_F16 || fmt == LRC_F16_O16 ? 4
 
 }  // namespace
 
-// Batches this path takes: up to 16 queries for binary32 and binary64 and
-// up to 4 for binary16 on the CUDA cores, ranks whose tiles fit in shared
-// memory; 5..32 queries in binary16 and up to 32 in bfloat16 on the tensor
-// cores (rank at most 512, n at most 32768).
+// Batches this path takes: up to 64 queries in binary16 and bfloat16 on the
+// tensor cores (rank at most 512, n at most 32768); otherwise up to 16
+// queries for binary32 and binary64 and up to 4 for binary16 on the CUDA
+// cores, ranks whose tiles fit in shared memory.
 bool apply_skinny_takes(lrc_fmt fmt, int64_t m, int64_t n, int64_t k, int64_t b) {
     if (skinny_tc_takes(fmt, m, n, k, b)) return true;
     if (fmt == LRC_BF16) return false;

@@ -114,10 +114,10 @@ lrc_status launch_apply_f16_group(const ApplyProblem* pr, int count, bool out16,
 lrc_status launch_apply_f16(const void* U, const void* S, const void* Vt, const void* X, void* Y,
                             int64_t m, int64_t n, int64_t k, int64_t b, bool out16, cudaStream_t s,
                             bool bf16 = false);
-// small batches (apply_skinny.cu): on the CUDA cores at most 16 queries in
-// binary32 and binary64 and 4 in binary16, ranks up to 1024 whose tiles fit
-// in shared memory; on the tensor cores 5..32 queries in binary16 and up to
-// 32 in bfloat16, rank at most 512, n at most 32768
+// small batches (apply_skinny.cu): on the tensor cores at most 64 queries in
+// binary16 and bfloat16, rank at most 512, n at most 32768; otherwise on the
+// CUDA cores at most 16 queries in binary32 and binary64 and 4 in binary16,
+// ranks up to 1024 whose tiles fit in shared memory
 bool apply_skinny_takes(lrc_fmt fmt, int64_t m, int64_t n, int64_t k, int64_t b);
 lrc_status launch_apply_skinny(const void* U, const void* S, const void* Vt, const void* X, void* Y, int64_t m,
                                int64_t n, int64_t k, int64_t b, lrc_fmt fmt, cudaStream_t s);
