@@ -516,7 +516,7 @@ __global__ void __launch_bounds__(SLICE ? 32 * kW2Slices : 256) apply_w2_group_k
 
 // ================================================================ phase 2
 struct YArgs {
-    int64_t m, b, T;
+    int64_t m, b, T, btiles;
     int kp, n2, kc2, mtiles, planes, stages;
     uint32_t u_bytes, slot_bytes, tile_bytes;
     uint32_t w_off, ystage_off, bar_off, tmem_cols;
@@ -524,6 +524,11 @@ struct YArgs {
     int bf16;                 // bfloat16 operands and output
     uint32_t idesc_ab;        // operand-format bits of the MMA descriptor
     int ydepth;               // staging buffers per epilogue warp (1 or 2): TMA stores in flight
+    // U resident (one plane of W): the CTA's units run column tile by column
+    // tile; the U tile of a column tile is loaded once and W streams through
+    // two buffers (the barriers full/empty[0..1]), so that each output tile
+    // reads a W tile (128 x k') instead of a U tile (n2 x k') from L2
+    int ures;
     const unsigned char* W;
     void* Y;
     // optional power-of-two scales of the operands, in groups of 32 rows of W
@@ -578,7 +583,79 @@ __device__ __forceinline__ void y_body(const CUtensorMap* tm_u, const CUtensorMa
     const uint32_t tmem = *tmem_slot;
     pdl_wait();                    // W images of the reduction kernel (the prologue above overlapped it)
 
-    if (warp == 0) {
+    if (warp == 0 && a.ures) {
+        // ------------------------------------------------------------ producer, U resident
+        if (lane == 0) {
+            int wl = 0, ul = 0;
+            int64_t cur_mt = -1;
+            bool ok = true;
+            for (int64_t t = tbeg; t < tend && ok; ++t) {
+                const int64_t mt = t / a.btiles;
+                const int64_t bt = t - mt * a.btiles;
+                if (mt != cur_mt) {
+                    // U of the new column tile, once the MMAs on the previous one are done
+                    if (!(ok = mbar_wait(w_empty, (ul & 1) ^ 1, abort, err, 1u))) break;
+                    mbar_arrive_expect_tx(w_full, (uint32_t)a.kc2 * a.u_bytes);
+                    for (int kc = 0; kc < a.kc2; ++kc)
+                        tma_load_2d(smem + (size_t)kc * a.u_bytes, tm_u, kc * BK, (int32_t)(mt * a.n2), w_full);
+                    ++ul;
+                    cur_mt = mt;
+                }
+                const int slot = wl & 1;
+                if (!(ok = mbar_wait(&empty[slot], ((wl >> 1) & 1) ^ 1, abort, err, 1u))) break;
+                mbar_arrive_expect_tx(&full[slot], a.tile_bytes);
+                bulk_load(smem + a.w_off + (size_t)slot * a.tile_bytes, a.W + (size_t)bt * a.tile_bytes, a.tile_bytes,
+                          &full[slot]);
+                ++wl;
+            }
+            if (!ok) {
+                volatile int no_abort = 0;
+                for (int j = wl - 2 > 0 ? wl - 2 : 0; j < wl; ++j)
+                    mbar_wait(&full[j & 1], (j >> 1) & 1, &no_abort, err, 0u, 100000000ull);
+                if (ul > 0) mbar_wait(w_full, (ul - 1) & 1, &no_abort, err, 0u, 100000000ull);
+            }
+        }
+    } else if (warp == 1 && a.ures) {
+        // ------------------------------------------------------------ MMA issuer, U resident
+        if (lane == 0) {
+            int wl = 0, ul = 0, tl = 0;
+            int64_t cur_mt = -1;
+            bool ok = true;
+            const uint32_t idesc2 = idesc_f16_f32(BM, (uint32_t)a.n2) | a.idesc_ab;
+            for (int64_t t = tbeg; t < tend && ok; ++t, ++tl) {
+                const int64_t mt = t / a.btiles;
+                if (mt != cur_mt) {
+                    if (ul > 0) mma_commit(w_empty);        // the previous U is free once these MMAs finish
+                    if (!(ok = mbar_wait(w_full, ul & 1, abort, err, 2u))) break;
+                    tc_fence_after();
+                    ++ul;
+                    cur_mt = mt;
+                }
+                const int ab = tl & 1;
+                if (!(ok = mbar_wait(&acc_empty[ab], ((tl >> 1) & 1) ^ 1, abort, err, 2u))) break;
+                const int slot = wl & 1;
+                if (!(ok = mbar_wait(&full[slot], (wl >> 1) & 1, abort, err, 2u))) break;
+                tc_fence_after();
+                const uint64_t whd = smem_desc(smem_u32(smem + a.w_off + (size_t)slot * a.tile_bytes), 2048, 128, 0);
+                const uint32_t dcol = tmem + (uint32_t)(ab * a.n2);
+                for (int kc = 0; kc < a.kc2; ++kc) {
+                    const uint64_t ud = desc_sw128(smem_u32(smem + (size_t)kc * a.u_bytes));
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk) {
+                        const int ks = kc * (BK / 16) + kk;
+                        if (ks * 16 >= a.kp) break;
+                        mma_f16(dcol, whd + (uint64_t)ks * 256u, ud + 2 * kk, idesc2, (kc | kk) != 0);
+                    }
+                }
+                mma_commit(&empty[slot]);
+                mma_commit(&acc_full[ab]);
+                ++wl;
+            }
+            mma_commit(mma_done);
+            volatile int no_abort = 0;
+            mbar_wait(mma_done, 0, &no_abort, err, 2u, 100000000ull);
+        }
+    } else if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
             int it = 0, wl = 0;
@@ -672,8 +749,15 @@ __device__ __forceinline__ void y_body(const CUtensorMap* tm_u, const CUtensorMa
         unsigned char* hstage = smem + a.ystage_off + (size_t)half * a.ydepth * (128 * 128);
         int chunk = 0, tl = 0;
         for (int64_t t = tbeg; t < tend; ++t, ++tl) {
-            const int64_t bt = t / a.mtiles;
-            const int mt = (int)(t - bt * a.mtiles);
+            int64_t bt;
+            int mt;
+            if (a.ures) {
+                mt = (int)(t / a.btiles);
+                bt = t - (int64_t)mt * a.btiles;
+            } else {
+                bt = t / a.mtiles;
+                mt = (int)(t - bt * a.mtiles);
+            }
             const int64_t row0 = bt * BM;
             const int ab = tl & 1;
             const bool scaled = a.esc_w != nullptr;
@@ -915,9 +999,40 @@ lrc_status plan_y(YArgs& a3, size_t& smem3, int64_t m, int64_t b, int kp, int pl
         return LRC_ERR_UNSUPPORTED;
     }
     a3.mtiles = (int)((m + a3.n2 - 1) / a3.n2);
+    a3.btiles = btiles;
     a3.T = btiles * a3.mtiles;
     a3.tmem_cols = pow2_cols(2u * (uint32_t)a3.n2);
+    a3.ures = 0;
     return LRC_OK;
+}
+
+// The U-resident layout of the product (one plane of W): U tile of kc2 boxes,
+// two W buffers, staging; false when it does not fit in shared memory, and
+// for a single k-block, where the U ring streams one box per output tile and
+// the per-tile W copy would only add latency (measured: k' = 48 and 64 were
+// 2-9 % slower U-resident, k' = 144 7 % faster).
+bool plan_y_ures(YArgs& a3, size_t& smem3, uint32_t tile_bytes) {
+    if (a3.planes != 1 || a3.kc2 < 2) return false;
+    for (int depth = 2; depth >= 1; --depth) {
+        size_t off = (size_t)a3.kc2 * a3.u_bytes;
+        const size_t w_off = off;
+        off += 2 * (size_t)tile_bytes;
+        off = round_up(off, 1024);
+        const size_t ystage_off = off;
+        off += (size_t)kEpiWarpsY * depth * 32 * 128;
+        const size_t bar_off = off;
+        off += (size_t)(2 * 2 + 7) * 8 + 16;
+        if (off + 1024 > kSmemMax) continue;
+        a3.ures = 1;
+        a3.stages = 2;
+        a3.ydepth = depth;
+        a3.w_off = (uint32_t)w_off;
+        a3.ystage_off = (uint32_t)ystage_off;
+        a3.bar_off = (uint32_t)bar_off;
+        smem3 = off + 1024;
+        return true;
+    }
+    return false;
 }
 
 CUtensorMapDataType t16(bool bf16) { return bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16; }
@@ -1013,6 +1128,9 @@ lrc_status plan_f16_shape(int64_t m, int64_t n, int64_t k, int64_t b, bool out16
     // ---- phase-2 plan: tile width, ring depth
     lrc_status st = plan_y(pl.a3, pl.smem3, m, b, kp, planes, out16, false);
     if (st != LRC_OK) return st;
+    // 16-bit output: a W tile (128 x k') per output tile instead of a U tile
+    // (n2 x k'), where the U tile fits in shared memory with two W buffers
+    plan_y_ures(pl.a3, pl.smem3, tile_bytes);
     pl.a3.tile_bytes = tile_bytes;
     pl.a3.bf16 = bf16 ? 1 : 0;
     pl.a3.idesc_ab = bf16 ? kIdescBF16 : 0u;
