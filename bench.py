@@ -1186,32 +1186,51 @@ def main():
     h2d_stream, d2h_stream = torch.cuda.Stream(), torch.cuda.Stream()
     main_stream = torch.cuda.current_stream()
     ready = {}
+    # two sets of device input buffers, alternating between steps: the inputs
+    # of step j + 1 come in while step j runs on the other set
+    dsets = {wl.name: [wl.d, {k: torch.empty_like(v) for k, v in wl.d.items()}] for wl in step.mats}
+    csets = {wl.name: [wl.c64, {s: [torch.empty_like(c) for c in wl.c64[s]] for s in STORE}] for wl in step.tts}
+    done_with = [None, None]          # per set: the main-stream event after the last step that read it
 
-    def copy_inputs():
-        # every workload's FP64 inputs on a copy stream, in the order the step
-        # uses them; the step waits for each workload's own copies only
-        h2d_stream.wait_stream(main_stream)
+    def copy_inputs(j):
+        # every workload's FP64 inputs of step j into set j % 2 on a copy
+        # stream, in the order the step uses them, once the step that last
+        # read that set is done; the step waits for each workload's own copies
+        idx = j % 2
+        if done_with[idx] is not None:
+            h2d_stream.wait_event(done_with[idx])
         with torch.cuda.stream(h2d_stream):
             for wl in [step.mats[1]] + step.tts + [step.mats[0], step.mats[2]]:
                 if isinstance(wl, MatrixWL):
                     # the factors first (the eta work needs only them), then the queries
+                    d = dsets[wl.name][idx]
                     for part, keys in (("factors", [k for k in pin[wl.name] if k not in wl.QUERIES]),
                                        ("queries", list(wl.QUERIES))):
                         for k in keys:
-                            wl.d[k].copy_(pin[wl.name][k], non_blocking=True)
+                            d[k].copy_(pin[wl.name][k], non_blocking=True)
                         ev = torch.cuda.Event()
                         ev.record()
-                        ready[(wl.name, part)] = ev
+                        ready[(wl.name, part, idx)] = ev
                 else:
+                    c = csets[wl.name][idx]
                     for s in STORE:
-                        for dd, h in zip(wl.c64[s], pin[wl.name][s]):
+                        for dd, h in zip(c[s], pin[wl.name][s]):
                             dd.copy_(h, non_blocking=True)
                     ev = torch.cuda.Event()
                     ev.record()
-                    ready[(wl.name, "cores")] = ev
+                    ready[(wl.name, "cores", idx)] = ev
+
+    copied = {}
+    cur = [0]
 
     def wait_inputs(wl, part):
-        main_stream.wait_event(ready[(wl.name, part)])
+        main_stream.wait_event(ready[(wl.name, part, cur[0])])
+        if part in ("queries", "cores"):
+            # the calls below rewrite this workload's outputs: the previous
+            # step's read-back of them has to be done
+            for key, ev in copied.items():
+                if key[0] == wl.name:
+                    main_stream.wait_event(ev)
 
     def read_back(wl, f, out=None):
         # each output comes back on a second copy stream as soon as its call
@@ -1221,21 +1240,44 @@ def main():
         d2h_stream.wait_event(done)
         with torch.cuda.stream(d2h_stream):
             outs[wl.name][f].copy_(wl.Y[f] if out is None else out, non_blocking=True)
+            ev = torch.cuda.Event()
+            ev.record()
+            copied[(wl.name, f)] = ev
 
-    def e2e_once():
-        copy_inputs()
+    def e2e_once(j, nsteps):
+        # Consecutive steps overlap: step j + 1's inputs are copied in (set
+        # (j + 1) % 2) while step j runs on set j % 2, and step j's outputs
+        # come back while step j + 1 runs; a call that rewrites an output
+        # waits for the previous read-back of it.  Every step of the run
+        # copies all of its own inputs in and all of its outputs out: no
+        # copy of a step outside [0, nsteps) is issued.
+        if j == 0:
+            copy_inputs(0)
+        if j + 1 < nsteps:
+            copy_inputs(j + 1)
+        cur[0] = j % 2
+        for wl in step.mats:
+            wl.d = dsets[wl.name][cur[0]]
+        for wl in step.tts:
+            wl.c64 = csets[wl.name][cur[0]]
         step.run(record=False, on_outputs=read_back, wait_inputs=wait_inputs)
-        main_stream.synchronize()
-        d2h_stream.synchronize()
+        ev = torch.cuda.Event()
+        ev.record()
+        done_with[cur[0]] = ev
 
-    e2e_once()
+    e2e_once(0, 1)                    # warm-up
     barrier(world)
     torch.cuda.synchronize()
+    done_with[:] = [None, None]
     t0 = time.perf_counter()
-    for _ in range(args.steps):
-        e2e_once()
+    for j in range(args.steps):
+        e2e_once(j, args.steps)
     torch.cuda.synchronize()
     e2e_ms = (time.perf_counter() - t0) * 1e3 / args.steps
+    for wl in step.mats:
+        wl.d = dsets[wl.name][0]
+    for wl in step.tts:
+        wl.c64 = csets[wl.name][0]
     e2e_ms_max = reduce_max(e2e_ms, world, dev)
     e2e_value = aggregate_value(rt_all, e2e_ms_max)
     st = lrc.lrc_device_status()
