@@ -197,3 +197,28 @@ def test_f32tc_wide_dynamic_range(lrc, cuda):
     # per-row relative error: every query row is judged against its own scale
     err = np.linalg.norm(got - want, axis=1) / np.linalg.norm(want, axis=1)
     assert err.max() <= 1e-5, err.max()
+
+
+@pytest.mark.parametrize("fmt", ["f16_o16", "bf16"])
+@pytest.mark.parametrize("m,n,k,b", [
+    (2000, 3000, 100, 777),    # two k-blocks, ragged m and b: U resident, W streamed
+    (5000, 2000, 160, 1300),   # three k-blocks; CTAs whose ranges cross column tiles
+    (300, 700, 129, 2000),     # a single column tile, many row tiles
+])
+def test_resident_u_product_vs_oracle(lrc, cuda, fmt, m, n, k, b):
+    """16-bit-output applies whose second product keeps U resident per
+    column tile (several k-blocks, one plane of W) match the oracle and are
+    reproducible bit for bit."""
+    f = W.random_factors(m, n, k, seed=m + 7 * k)
+    X = W.gaussian((b, n), b + 91)
+    Ud, Sd, Vd, Xd = (packed(lrc, a, fmt, cuda) for a in (f.U, f.s, f.Vt, X))
+    outs = []
+    for _ in range(2):
+        Y = torch.full((b, m), float("nan"), dtype=lrc.output_dtype(fmt), device=cuda)
+        lrc.lrc_apply(Ud, Sd, Vd, Xd, Y, m, n, k, b, fmt)
+        outs.append(Y)
+    assert lrc.lrc_device_status() == 0
+    assert torch.equal(outs[0].view(torch.int16), outs[1].view(torch.int16))
+    want = oracle.apply(*oracle_inputs(f.U, f.s, f.Vt, X, fmt))
+    err = rel_fro(outs[0].double().cpu().numpy(), want)
+    assert err <= TOL[fmt], (fmt, err)
