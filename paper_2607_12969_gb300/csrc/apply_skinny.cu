@@ -905,8 +905,13 @@ TcPlan plan_skinny_tc(int64_t n, int64_t k, int64_t b, int NB, bool fp32_out) {
     p.kc = (p.kp + kTcK - 1) / kTcK;
     p.rtiles = (p.kp + kTcM - 1) / kTcM;
     p.nkb = (int)((n + kTcK - 1) / kTcK);
-    p.cb = (p.nkb + kTcMaxChunks - 1) / kTcMaxChunks;
+    // fewer, longer chunks above 4 queries: the folds read chunks x b x 128
+    // entries a rank tile (m = n = 16384, k' = 272: b = 64 17.4 -> 15.3 us
+    // with 32 chunks instead of 64; b = 1 10.4 against 10.6 us)
+    const int want = b <= 4 ? kTcMaxChunks : kTcMaxChunks / 2;
+    p.cb = (p.nkb + want - 1) / want;
     if (p.cb < 1) p.cb = 1;
+    if (p.cb > 8) p.cb = (p.nkb + kTcMaxChunks - 1) / kTcMaxChunks;   // at most 8 k-blocks a chunk
     p.nchunks = (p.nkb + p.cb - 1) / p.cb;
     p.nclusters = (p.nchunks + kTcCluster - 1) / kTcCluster;
     p.planes = fp32_out ? 2 : 1;
