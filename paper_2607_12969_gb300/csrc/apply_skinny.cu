@@ -634,16 +634,9 @@ skinny_tc_w_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_consta
     constexpr uint32_t kBox = NB * 128;            // bytes of one W box
     // the 4 ranks j0.. lie in 16-byte chunk (j0 % 64) / 8 of a 128-byte row of k-block j0 / 64
     const int kblk = j0 >> 6, ch = (j0 & 63) >> 3, within = (j0 & 7) * 2;
-    for (int q = (int)(threadIdx.x >> 5); q < a.b; q += kTcThreadsW / 32) {
-        const int e = q * (kTcM / 4) + (r4 >> 2);
-        float4 v[kTcMaxChunks / kTcCluster];
-#pragma unroll
-        for (int c = 0; c < kTcMaxChunks / kTcCluster; ++c)
-            v[c] = c < a.nclusters ? __ldcg(src + (size_t)c * kC4 + e) : make_float4(0.f, 0.f, 0.f, 0.f);
-        float4 sum = v[0];
-#pragma unroll
-        for (int c = 1; c < kTcMaxChunks / kTcCluster; ++c)
-            if (c < a.nclusters) sum = add4(sum, v[c]);
+    // W entries (q, j0..j0+3) from the sum of the cluster partials: scale,
+    // round, store in the swizzled image
+    auto emit = [&](int q, float4 sum) {
         const float w[4] = {__fmul_rn(sum.x, sj[0]), __fmul_rn(sum.y, sj[1]), __fmul_rn(sum.z, sj[2]),
                             __fmul_rn(sum.w, sj[3])};
         uint16_t hi[4], lo[4];
@@ -662,6 +655,45 @@ skinny_tc_w_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_consta
         if (a.planes == 2)
             *reinterpret_cast<uint2*>(dst + kBox) =
                 make_uint2(lo[0] | ((uint32_t)lo[1] << 16), lo[2] | ((uint32_t)lo[3] << 16));
+    };
+    constexpr int kQStep = kTcThreadsW / 32;       // queries a pass of the CTA takes
+    const int q0 = (int)(threadIdx.x >> 5);
+    if (NB > kQStep && a.nclusters <= 4) {
+        // several queries a thread: every load of the thread in flight at once
+        constexpr int kQ = NB > kQStep ? NB / kQStep : 1;
+        float4 v[kQ][4];
+#pragma unroll
+        for (int i = 0; i < kQ; ++i)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const int q = q0 + i * kQStep;
+                v[i][c] = (q < a.b && c < a.nclusters)
+                              ? __ldcg(src + (size_t)c * kC4 + q * (kTcM / 4) + (r4 >> 2))
+                              : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+        for (int i = 0; i < kQ; ++i) {
+            const int q = q0 + i * kQStep;
+            if (q >= a.b) break;
+            float4 sum = v[i][0];
+#pragma unroll
+            for (int c = 1; c < 4; ++c)
+                if (c < a.nclusters) sum = add4(sum, v[i][c]);
+            emit(q, sum);
+        }
+        return;
+    }
+    for (int q = q0; q < a.b; q += kQStep) {
+        const int e = q * (kTcM / 4) + (r4 >> 2);
+        float4 v[kTcMaxChunks / kTcCluster];
+#pragma unroll
+        for (int c = 0; c < kTcMaxChunks / kTcCluster; ++c)
+            v[c] = c < a.nclusters ? __ldcg(src + (size_t)c * kC4 + e) : make_float4(0.f, 0.f, 0.f, 0.f);
+        float4 sum = v[0];
+#pragma unroll
+        for (int c = 1; c < kTcMaxChunks / kTcCluster; ++c)
+            if (c < a.nclusters) sum = add4(sum, v[c]);
+        emit(q, sum);
     }
 }
 
