@@ -490,6 +490,46 @@ __device__ __forceinline__ float4 add4(float4 a, float4 b) {
     return make_float4(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y), __fadd_rn(a.z, b.z), __fadd_rn(a.w, b.w));
 }
 
+struct TcWArgs;
+
+// W entries (q, j0..j0+3) = s_j * sum, rounded (hi and lo binary16 for FP32
+// output, one rounding otherwise) into the second product's swizzled image:
+// the 4 ranks lie in 16-byte chunk (j0 % 64) / 8 of a 128-byte row of
+// k-block j0 / 64, the lo box right after the hi box.
+template <int NB>
+__device__ __forceinline__ void emit_w(unsigned char* W, int planes, int bf16, int q, int j0, float4 sum,
+                                       const float (&sj)[4]) {
+    const float w[4] = {__fmul_rn(sum.x, sj[0]), __fmul_rn(sum.y, sj[1]), __fmul_rn(sum.z, sj[2]),
+                        __fmul_rn(sum.w, sj[3])};
+    uint16_t hi[4], lo[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        if (bf16) {
+            hi[i] = tc::to_bf16_bits(w[i]);
+        } else {
+            const __half h = __float2half_rn(w[i]);
+            hi[i] = __half_as_ushort(h);
+            lo[i] = __half_as_ushort(__float2half_rn(w[i] - __half2float(h)));
+        }
+    }
+    const int kblk = j0 >> 6, ch = (j0 & 63) >> 3, within = (j0 & 7) * 2;
+    unsigned char* dst = W + ((size_t)kblk * planes * NB + q) * 128 + ((ch ^ (q & 7)) << 4) + within;
+    *reinterpret_cast<uint2*>(dst) = make_uint2(hi[0] | ((uint32_t)hi[1] << 16), hi[2] | ((uint32_t)hi[3] << 16));
+    if (planes == 2)
+        *reinterpret_cast<uint2*>(dst + NB * 128) =
+            make_uint2(lo[0] | ((uint32_t)lo[1] << 16), lo[2] | ((uint32_t)lo[3] << 16));
+}
+
+// s_j for the 4 ranks j0..j0+3 (0 from rank k on)
+__device__ __forceinline__ void load_s4(const uint16_t* S, int k, int bf16, int j0, float (&sj)[4]) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int j = j0 + i;
+        sj[i] = 0.0f;
+        if (j < k) sj[i] = bf16 ? tc::bf16_bits_to_float(S[j]) : __half2float(__ushort_as_half(S[j]));
+    }
+}
+
 struct TcWArgs {
     int k, kp, b, nkb, cb, nclusters;
     int planes;               // W planes: 2 (hi and lo, FP32 output) or 1
@@ -590,26 +630,36 @@ skinny_tc_w_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_consta
     cluster_sync();                  // every partial of the cluster is staged
     // The cluster partial: CTA j of the cluster adds, for its eighth of the
     // (query, 4 ranks) entries, the kTcCluster staged partials in rank order.
+    // With a single cluster a rank tile (n up to 8 chunks) that sum is the
+    // whole reduction: the CTAs write their W entries themselves.
     const int cl = chunk / kTcCluster;
     const int crank = (int)cluster_ctarank();
     const int n4 = a.b * (kTcM / 4);
+    const int ranks = a.kp - rt * kTcM < kTcM ? a.kp - rt * kTcM : kTcM;
     float4* cp = reinterpret_cast<float4*>(a.P + ((size_t)rt * a.nclusters + cl) * NB * kTcM);
     for (int e = n4 * crank / kTcCluster + (int)threadIdx.x; e < n4 * (crank + 1) / kTcCluster;
          e += kTcThreadsW) {
-        {
-            const uint32_t addr = tc::smem_u32(stage) + 16u * (uint32_t)e;
-            float4 v[kTcCluster];
+        const uint32_t addr = tc::smem_u32(stage) + 16u * (uint32_t)e;
+        float4 v[kTcCluster];
 #pragma unroll
-            for (int r = 0; r < kTcCluster; ++r) v[r] = ld_cluster4(addr, (uint32_t)r);
-            float4 sum = v[0];
+        for (int r = 0; r < kTcCluster; ++r) v[r] = ld_cluster4(addr, (uint32_t)r);
+        float4 sum = v[0];
 #pragma unroll
-            for (int r = 1; r < kTcCluster; ++r) sum = add4(sum, v[r]);
+        for (int r = 1; r < kTcCluster; ++r) sum = add4(sum, v[r]);
+        if (a.nclusters > 1) {
             cp[e] = sum;
+        } else {
+            const int q = e / (kTcM / 4), r4 = (e - q * (kTcM / 4)) * 4;
+            if (r4 < ranks) {
+                float sj[4];
+                load_s4(a.S, a.k, a.bf16, rt * kTcM + r4, sj);
+                emit_w<NB>(a.W, a.planes, a.bf16, q, rt * kTcM + r4, sum, sj);
+            }
         }
     }
     __syncwarp();
     cluster_sync();                  // the staged partials stay until every CTA has read them
-    if (crank != 0) return;
+    if (crank != 0 || a.nclusters == 1) return;
     // the cluster's first CTA arrives for the cluster (the cluster barrier
     // ordered the other CTAs' partial stores before this release)
     if (threadIdx.x == 0) last_cluster = arrive_acq_rel(&a.cnt[rt]) == (unsigned)(a.nclusters - 1);
@@ -618,44 +668,14 @@ skinny_tc_w_kernel(const __grid_constant__ CUtensorMap tm_v, const __grid_consta
     // The rank tile's cluster partials added in cluster order, scaled by
     // diag(s), written as W.  Thread t takes ranks 4 (t % 32) .. + 3 of
     // queries t / 32, t / 32 + 16, ...
-    const int ranks = a.kp - rt * kTcM < kTcM ? a.kp - rt * kTcM : kTcM;
     const int r4 = (int)(threadIdx.x & 31) * 4;
     if (r4 >= ranks) return;                       // ranks is a multiple of 16
     const int j0 = rt * kTcM + r4;
     float sj[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int j = j0 + i;
-        sj[i] = 0.0f;
-        if (j < a.k) sj[i] = a.bf16 ? tc::bf16_bits_to_float(a.S[j]) : __half2float(__ushort_as_half(a.S[j]));
-    }
+    load_s4(a.S, a.k, a.bf16, j0, sj);
     const float4* src = reinterpret_cast<const float4*>(a.P + (size_t)rt * a.nclusters * NB * kTcM);
     constexpr int kC4 = NB * kTcM / 4;             // float4 per cluster partial
-    constexpr uint32_t kBox = NB * 128;            // bytes of one W box
-    // the 4 ranks j0.. lie in 16-byte chunk (j0 % 64) / 8 of a 128-byte row of k-block j0 / 64
-    const int kblk = j0 >> 6, ch = (j0 & 63) >> 3, within = (j0 & 7) * 2;
-    // W entries (q, j0..j0+3) from the sum of the cluster partials: scale,
-    // round, store in the swizzled image
-    auto emit = [&](int q, float4 sum) {
-        const float w[4] = {__fmul_rn(sum.x, sj[0]), __fmul_rn(sum.y, sj[1]), __fmul_rn(sum.z, sj[2]),
-                            __fmul_rn(sum.w, sj[3])};
-        uint16_t hi[4], lo[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            if (a.bf16) {
-                hi[i] = tc::to_bf16_bits(w[i]);
-            } else {
-                const __half h = __float2half_rn(w[i]);
-                hi[i] = __half_as_ushort(h);
-                lo[i] = __half_as_ushort(__float2half_rn(w[i] - __half2float(h)));
-            }
-        }
-        unsigned char* dst = a.W + ((size_t)kblk * a.planes * NB + q) * 128 + ((ch ^ (q & 7)) << 4) + within;
-        *reinterpret_cast<uint2*>(dst) = make_uint2(hi[0] | ((uint32_t)hi[1] << 16), hi[2] | ((uint32_t)hi[3] << 16));
-        if (a.planes == 2)
-            *reinterpret_cast<uint2*>(dst + kBox) =
-                make_uint2(lo[0] | ((uint32_t)lo[1] << 16), lo[2] | ((uint32_t)lo[3] << 16));
-    };
+    auto emit = [&](int q, float4 sum) { emit_w<NB>(a.W, a.planes, a.bf16, q, j0, sum, sj); };
     constexpr int kQStep = kTcThreadsW / 32;       // queries a pass of the CTA takes
     const int q0 = (int)(threadIdx.x >> 5);
     if (NB > kQStep && a.nclusters <= 4) {
