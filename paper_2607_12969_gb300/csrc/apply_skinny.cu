@@ -430,7 +430,8 @@ skinny_y_kernel(const __grid_constant__ CUtensorMap tm_u, const T* __restrict__ 
 //                       memory; every CTA of the cluster then adds, for an
 //                       eighth of the entries, the kTcCluster partials in
 //                       rank order through distributed shared memory and
-//                       writes that part of the cluster partial.  The last
+//                       writes that part of the cluster partial (W itself
+//                       when a rank tile has one cluster).  The last
 //                       cluster of a rank tile to arrive (a counter) adds
 //                       the cluster partials in cluster order, scales by
 //                       diag(s) and writes W as the second product's operand
@@ -489,8 +490,6 @@ __device__ __forceinline__ float4 ld_cluster4(uint32_t addr, uint32_t rank) {
 __device__ __forceinline__ float4 add4(float4 a, float4 b) {
     return make_float4(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y), __fadd_rn(a.z, b.z), __fadd_rn(a.w, b.w));
 }
-
-struct TcWArgs;
 
 // W entries (q, j0..j0+3) = s_j * sum, rounded (hi and lo binary16 for FP32
 // output, one rounding otherwise) into the second product's swizzled image:
