@@ -831,26 +831,40 @@ __device__ __forceinline__ void y_body(const CUtensorMap* tm_u, const CUtensorMa
                         }
                     } else {
                         // Rows whose pitch is not a multiple of 16 bytes (no TMA store): the
-                        // warp writes its own 32 staged rows one at a time, lane l the row's
-                        // bytes 4l..4l+3 -- one coalesced 128-byte run per row.
+                        // warp writes its own 32 staged rows, lane l the row's bytes
+                        // 4l..4l+3 -- one coalesced 128-byte run per row.  The 32 shared
+                        // loads come first, so that the stores do not each wait for one
+                        // (a load-store chain per row ran the ten-matrix batch's product
+                        // at about 1.2 TB/s).
                         __syncwarp();
                         const int nvalid = (int)(a.m - col0 < ecols ? a.m - col0 : ecols);   // columns inside Y
-                        for (int rr = 0; rr < 32; ++rr) {
-                            const int64_t grow = row0 + g * 32 + rr;
-                            if (grow >= a.b) break;
-                            const uint32_t w = *reinterpret_cast<const uint32_t*>(
+                        const int64_t rbase = row0 + g * 32;
+                        const int nrows = a.b - rbase >= 32 ? 32 : (a.b - rbase > 0 ? (int)(a.b - rbase) : 0);
+                        uint32_t wv[32];
+#pragma unroll
+                        for (int rr = 0; rr < 32; ++rr)
+                            wv[rr] = *reinterpret_cast<const uint32_t*>(
                                 sb + rr * 128 + (((lane >> 2) ^ (rr & 7)) * 16) + (lane & 3) * 4);
-                            if (a.out16) {
-                                uint16_t* y = static_cast<uint16_t*>(a.Y) + grow * a.m + col0 + 2 * lane;
-                                const int c = 2 * lane;
+                        if (a.out16) {
+                            const int c = 2 * lane;
+#pragma unroll
+                            for (int rr = 0; rr < 32; ++rr) {
+                                if (rr >= nrows) break;
+                                uint16_t* y = static_cast<uint16_t*>(a.Y) + (rbase + rr) * a.m + col0 + c;
+                                const uint32_t w = wv[rr];
                                 if (c + 1 < nvalid && ((reinterpret_cast<uintptr_t>(y) & 3u) == 0)) {
                                     *reinterpret_cast<uint32_t*>(y) = w;
                                 } else {
                                     if (c < nvalid) y[0] = (uint16_t)(w & 0xffffu);
                                     if (c + 1 < nvalid) y[1] = (uint16_t)(w >> 16);
                                 }
-                            } else if (lane < nvalid) {
-                                *(static_cast<uint32_t*>(a.Y) + grow * a.m + col0 + lane) = w;
+                            }
+                        } else if (lane < nvalid) {
+                            uint32_t* y = static_cast<uint32_t*>(a.Y) + rbase * a.m + col0 + lane;
+#pragma unroll
+                            for (int rr = 0; rr < 32; ++rr) {
+                                if (rr >= nrows) break;
+                                y[(int64_t)rr * a.m] = wv[rr];
                             }
                         }
                     }
