@@ -156,8 +156,10 @@ LRC_API lrc_status lrc_widen_factors(const void* src, lrc_fmt fmt, int64_t rows,
  * binary32 on the CUDA cores (binary16 too when the tensor-core products
  * do not take the shape), and up to 64 queries in binary16 and bfloat16 as
  * two tensor-core products when n <= 32768 and k <= 512 (the second
- * product's tiles must fit in shared memory).  Binary16 ranks: up to 320 for LRC_F16 and 512 for
- * LRC_F16_O16, else LRC_ERR_UNSUPPORTED.
+ * product's tiles must fit in shared memory).  Binary16 ranks: up to 512,
+ * and up to 320 for LRC_F16 where the small-batch tensor-core products do
+ * not take the call (more than 64 queries, n > 32768), else
+ * LRC_ERR_UNSUPPORTED.
  */
 /* LRC_F32_TC: as LRC_F32, with the second product (W U^T) on the tensor
  * cores when b > 32 and k <= 192; otherwise the LRC_F32 kernels. */
